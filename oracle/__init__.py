@@ -1,0 +1,7 @@
+"""fp64 CPU oracle of the LoRA-adapted linear layer.
+
+Test infrastructure only: the tests, the smoke check and the benchmark's CPU
+baseline arm are its only users; the CUDA library never imports it.
+"""
+from .lora_oracle import (lora_forward, lora_backward, lora_forward_rows,  # noqa: F401
+                          lora_backward_dx_rows, lora_adapter_grads, lora_step)

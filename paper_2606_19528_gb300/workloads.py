@@ -1,0 +1,107 @@
+"""Workload shapes: LoRA-adapted projections of 3B-class decoder layers.
+
+The fine-tuning method adapts the q and v projections with r = 16, alpha = 16
+(hyper-parameter table, "LoRA layers: q, v"); the workloads here adapt all
+seven projections of a decoder layer (q, k, v, o, gate, up, down), which is a
+superset of that setting.  Hidden sizes are those of Llama-3.2-3B
+(3072 -> 3072 / 1024 / 8192) and Qwen-2.5-3B (2048 -> 2048 / 256 / 11008),
+the two models of the paper's profiling setup.
+
+Projections that read the same decoder activation share one input buffer:
+q, k, v read the attention input; gate, up read the MLP input; o and down
+read their own.  `group` names that buffer.
+"""
+from __future__ import annotations
+
+from dataclasses import dataclass, field
+from typing import List
+
+
+@dataclass(frozen=True)
+class Proj:
+    name: str
+    d_in: int
+    d_out: int
+    group: int  # input-buffer id (projections with the same id share x)
+
+
+@dataclass
+class Workload:
+    name: str
+    cfg: int              # stream tag of the workload
+    T: int                # tokens
+    rank: int
+    alpha: float
+    projs: List[Proj] = field(default_factory=list)
+    layers: int = 1
+    zero_B: bool = False
+
+    @property
+    def scale(self) -> float:
+        return self.alpha / self.rank
+
+    def flops(self) -> float:
+        """Algorithmic FLOPs of one fwd+bwd over every projection and layer:
+        4TKN (the two base contractions) + 6Tr(K+N) (the rank-r products);
+        the frozen weight's gradient is never formed and not counted."""
+        T, r = self.T, self.rank
+        per = sum(4 * T * p.d_in * p.d_out + 6 * T * r * (p.d_in + p.d_out) for p in self.projs)
+        return float(per * self.layers)
+
+
+def llama_layer() -> List[Proj]:
+    h, kv, f = 3072, 1024, 8192
+    return [Proj("q", h, h, 0), Proj("k", h, kv, 0), Proj("v", h, kv, 0), Proj("o", h, h, 1),
+            Proj("gate", h, f, 2), Proj("up", h, f, 2), Proj("down", f, h, 3)]
+
+
+def qwen_layer() -> List[Proj]:
+    h, kv, f = 2048, 256, 11008
+    return [Proj("q", h, h, 0), Proj("k", h, kv, 0), Proj("v", h, kv, 0), Proj("o", h, h, 1),
+            Proj("gate", h, f, 2), Proj("up", h, f, 2), Proj("down", f, h, 3)]
+
+
+def single_small(zero_B: bool = False) -> Workload:
+    """One 256 -> 256 projection, T = 128, r = 8, alpha = 16 (and its B = 0 twin)."""
+    return Workload("single_T128_256x256_r8" + ("_B0" if zero_B else ""), 0, 128, 8, 16.0,
+                    [Proj("lin", 256, 256, 0)], zero_B=zero_B)
+
+
+def llama_q() -> Workload:
+    """Llama-3.2-3B-shaped q projection, T = 512, r = 16, alpha = 32."""
+    return Workload("llama3b_q_T512_r16", 1, 512, 16, 32.0, [Proj("q", 3072, 3072, 0)])
+
+
+def llama_layer_T2048() -> Workload:
+    """Seven projections of a Llama-3.2-3B-shaped layer, T = 2048, r = 16, alpha = 32."""
+    return Workload("llama3b_layer_T2048_r16", 2, 2048, 16, 32.0, llama_layer())
+
+
+def qwen_layer_T4096() -> Workload:
+    """Seven projections of a Qwen-2.5-3B-shaped layer, T = 4096, r = 64, alpha = 128."""
+    return Workload("qwen3b_layer_T4096_r64", 3, 4096, 64, 128.0, qwen_layer())
+
+
+SWEEP_RANKS = (4, 8, 16, 32, 64, 128)
+SWEEP_TOKENS = (256, 1024, 4096, 16384)
+
+
+def llama_sweep(T: int, r: int) -> Workload:
+    """Llama layer at (T, r) of the rank x token sweep; alpha = 2r keeps s = 2."""
+    return Workload(f"llama3b_layer_T{T}_r{r}", 4, T, r, 2.0 * r, llama_layer())
+
+
+def llama_stack28() -> Workload:
+    """28 Llama layers' projections, T = 1024, r = 16, alpha = 32, forward of
+    every layer first, then backward of every layer, from stored inputs."""
+    return Workload("llama3b_stack28_T1024_r16", 5, 1024, 16, 32.0, llama_layer(), layers=28)
+
+
+BY_NAME = {
+    "single": single_small,
+    "single_B0": lambda: single_small(True),
+    "llama_q": llama_q,
+    "llama_layer": llama_layer_T2048,
+    "qwen_layer": qwen_layer_T4096,
+    "llama_stack28": llama_stack28,
+}
