@@ -1,0 +1,147 @@
+/*
+ * lora.h -- C ABI of the GB300 (sm_103a) LoRA-adapted linear layer.
+ *
+ * The operation.  A frozen linear layer W is adapted by a trainable rank-r
+ * product, as in the LoRA fine-tuning the paper studies (Background,
+ * "Parameter-Efficient Fine-Tuning": low-rank decomposition matrices trained
+ * while the original weights stay frozen; rank r and alpha from the
+ * hyper-parameter table; s = alpha / r).  Token-major, row-major layout:
+ *
+ *   forward   su = s * x A^T                [T, r]   (saved for backward)
+ *             y  = x W^T + su B^T           [T, N]
+ *   backward  sv = s * dy B                 [T, r]   (internal)
+ *             dx = dy W + sv A              [T, K]
+ *             dB = dy^T su                  [N, r]   (= s dy^T x A^T)
+ *             dA = sv^T x                   [r, K]   (= s (dy B)^T x)
+ *
+ * y = x W^T and dx = dy W are Algorithm 1's y_base = W x and dx = W^T dy
+ * (column-vector form there).  W is frozen: no gradient of W is formed.
+ *
+ * Shapes: T tokens, K = d_in, N = d_out, r = rank.  x [T,K], W [N,K]
+ * (nn.Linear layout), A [r,K], B [N,r], y and dy [T,N], dx [T,K], su [T,r].
+ * Element types: every activation and parameter is bf16 (passed as its
+ * 16-bit pattern, `lora_bf16`); contractions accumulate in fp32; y, dx and su
+ * are rounded to bf16 (round to nearest even) once; dA and dB are fp32.
+ *
+ * Conventions shared by every entry point:
+ *  - every pointer is a CUDA device pointer on the current device, owned by
+ *    the caller, row-major and dense (leading dimension = row length), and
+ *    16-byte aligned; the library never allocates or frees memory;
+ *  - T, d_in and d_out are multiples of 8 (16-byte rows for the tensor-memory
+ *    accelerator), 1 <= rank <= 128, scale finite;
+ *  - calls are asynchronous on `stream` (a cudaStream_t; NULL = legacy
+ *    default stream); return LORA_OK once every kernel is enqueued;
+ *  - inputs may alias each other (e.g. q, k and v passing one x); outputs
+ *    must not alias any input or each other; W is never written;
+ *  - dA and dB are overwritten, not accumulated;
+ *  - `workspace` is scratch of at least the size the matching
+ *    *_workspace_size call reports, 256-byte aligned; its contents need no
+ *    initialisation and are garbage afterwards; calls that run concurrently
+ *    need separate workspaces;
+ *  - errors: a negative LORA_E* code is returned and nothing is enqueued
+ *    (argument errors), or kernels may already be enqueued (LORA_ECUDA).
+ *    Device-side bounded waits that expire set a status word readable with
+ *    lora_read_status (LORA_ETIMEOUT); they never trap.
+ */
+#ifndef LORA_GB300_H_
+#define LORA_GB300_H_
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef uint16_t lora_bf16; /* bit pattern of an IEEE bfloat16 */
+
+enum {
+  LORA_OK = 0,
+  LORA_EINVAL = -1,      /* bad shape, rank, scale, mode or count */
+  LORA_ENULL = -2,       /* a required pointer is NULL */
+  LORA_EALIGN = -3,      /* a pointer is not 16-byte aligned (workspace: 256) */
+  LORA_ECUDA = -4,       /* a CUDA runtime call or launch failed */
+  LORA_ETIMEOUT = -5,    /* a device-side bounded wait expired */
+  LORA_EWORKSPACE = -6,  /* workspace missing or smaller than required */
+  LORA_EDEVICE = -7      /* current device is not a compute capability 10.3 GPU */
+};
+
+enum { LORA_FWD = 1, LORA_BWD = 2, LORA_FWD_BWD = 3 };
+
+typedef struct lora_shape {
+  int64_t T;      /* tokens */
+  int64_t d_in;   /* K */
+  int64_t d_out;  /* N */
+  int64_t rank;   /* r */
+  float scale;    /* s = alpha / r */
+} lora_shape;
+
+/* Bytes of workspace that lora_linear_fwd (mode LORA_FWD), lora_linear_bwd
+ * (LORA_BWD) or both (LORA_FWD_BWD) need for `shape`.
+ * Returns LORA_OK, LORA_EINVAL or LORA_ENULL. */
+int lora_workspace_size(const lora_shape* shape, int mode, size_t* bytes);
+
+/* Forward of one LoRA linear: y = x W^T + s (x A^T) B^T.
+ * su [T,r] receives s x A^T for the backward; pass NULL for a forward that
+ * saves nothing (the no-grad forward of a checkpointed schedule).
+ * Reads x, W, A, B; writes y and su. */
+int lora_linear_fwd(const lora_shape* shape, const lora_bf16* x, const lora_bf16* W,
+                    const lora_bf16* A, const lora_bf16* B, lora_bf16* y, lora_bf16* su,
+                    void* workspace, size_t workspace_bytes, void* stream);
+
+/* Backward of one LoRA linear with W frozen.
+ * su is the forward's saved s x A^T.  dx may be NULL (no input gradient
+ * wanted); dA [r,K] and dB [N,r] are required.  Reads dy, x, W, A, B, su. */
+int lora_linear_bwd(const lora_shape* shape, const lora_bf16* dy, const lora_bf16* x,
+                    const lora_bf16* W, const lora_bf16* A, const lora_bf16* B,
+                    const lora_bf16* su, lora_bf16* dx, float* dA, float* dB,
+                    void* workspace, size_t workspace_bytes, void* stream);
+
+/* One adapted projection of a decoder layer (q, k, v, o, gate, up, down).
+ * Field meanings and rules as above; pointers a mode does not touch may be
+ * NULL (forward: x W A B y [su]; backward: dy x W A B su dA dB [dx]). */
+typedef struct lora_proj {
+  lora_shape shape;
+  const lora_bf16* x;
+  const lora_bf16* W;
+  const lora_bf16* A;
+  const lora_bf16* B;
+  const lora_bf16* dy;
+  lora_bf16* y;
+  lora_bf16* su;
+  lora_bf16* dx;
+  float* dA;
+  float* dB;
+} lora_proj;
+
+/* Workspace bytes for lora_stack_step over `projs` in `mode`. */
+int lora_stack_workspace_size(const lora_proj* projs, int n_proj, int mode, size_t* bytes);
+
+/* Forward and/or backward of n_proj independent projections (1..64), e.g.
+ * the seven adapted linears of one decoder layer.  Mode LORA_FWD_BWD runs
+ * every forward, then every backward.  Same semantics as n_proj calls of
+ * lora_linear_fwd / lora_linear_bwd, scheduled as one batch on `stream`. */
+int lora_stack_step(const lora_proj* projs, int n_proj, int mode, void* workspace,
+                    size_t workspace_bytes, void* stream);
+
+/* Waits for `stream`, then reads the device status word that bounded waits
+ * set when they expire: *status = LORA_OK or LORA_ETIMEOUT.  reset != 0
+ * clears it.  Returns LORA_OK or LORA_ECUDA. */
+int lora_read_status(void* stream, int* status, int reset);
+
+/* Limit, in nanoseconds of device time, of every bounded wait in the
+ * library's kernels (0 restores the default of 4 s).  For tests of the
+ * timeout path; affects launches made after the call.  Returns LORA_OK. */
+int lora_set_wait_limit_ns(int64_t ns);
+
+/* Static message for a LORA_* code. */
+const char* lora_strerror(int code);
+
+/* Library version, major * 10000 + minor * 100 + patch. */
+int lora_version(void);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* LORA_GB300_H_ */

@@ -1,0 +1,474 @@
+// C ABI of the LoRA linear (declared in include/lora.h): argument checks,
+// workspace planning, TMA descriptors and the launch sequence.
+//
+// forward  : su = s x A^T (row product)  ->  y = [x | su] . [W | B]^T (fused GEMM)
+// backward : sv = s dy B (row product), dB = dy^T su, dA = sv^T x (column
+//            products)  ->  dx = [dy | sv] . [W ; A] (fused GEMM)
+#include <math.h>
+#include <stdio.h>
+#include <string.h>
+
+#include <algorithm>
+#include <mutex>
+#include <vector>
+
+#include "common.cuh"
+#include "kernels.h"
+#include "lora.h"
+
+namespace lora {
+namespace {
+
+__device__ int g_status;  // first device-side error (kStatusTimeout), 0 if none
+
+constexpr int kMaxDevices = 64;
+constexpr long long kDefaultWaitNs = 4000000000ll;
+
+struct DeviceInfo {
+  bool ready = false;
+  bool supported = false;
+  int num_sms = 0;
+  int* status = nullptr;
+};
+
+std::mutex g_mu;
+DeviceInfo g_dev[kMaxDevices];
+long long g_wait_limit_ns = kDefaultWaitNs;
+
+typedef CUresult (*EncodeTiledFn)(CUtensorMap*, CUtensorMapDataType, cuuint32_t, void*, const cuuint64_t*,
+                                  const cuuint64_t*, const cuuint32_t*, const cuuint32_t*, CUtensorMapInterleave,
+                                  CUtensorMapSwizzle, CUtensorMapL2promotion, CUtensorMapFloatOOBfill);
+EncodeTiledFn g_encode = nullptr;
+
+int device_info(DeviceInfo** out) {
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= kMaxDevices) return LORA_ECUDA;
+  std::lock_guard<std::mutex> lk(g_mu);
+  DeviceInfo& d = g_dev[dev];
+  if (!d.ready) {
+    int major = 0, minor = 0, sms = 0;
+    if (cudaDeviceGetAttribute(&major, cudaDevAttrComputeCapabilityMajor, dev) != cudaSuccess ||
+        cudaDeviceGetAttribute(&minor, cudaDevAttrComputeCapabilityMinor, dev) != cudaSuccess ||
+        cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess)
+      return LORA_ECUDA;
+    d.supported = (major == 10 && minor == 3);
+    d.num_sms = sms;
+    if (d.supported) {
+      void* p = nullptr;
+      if (cudaGetSymbolAddress(&p, g_status) != cudaSuccess) return LORA_ECUDA;
+      d.status = static_cast<int*>(p);
+    }
+    if (!g_encode) {
+      cudaDriverEntryPointQueryResult q;
+      void* fn = nullptr;
+      if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &fn, 12000, cudaEnableDefault, &q) !=
+              cudaSuccess ||
+          q != cudaDriverEntryPointSuccess || fn == nullptr)
+        return LORA_ECUDA;
+      g_encode = reinterpret_cast<EncodeTiledFn>(fn);
+    }
+    d.ready = true;
+  }
+  if (!d.supported) return LORA_EDEVICE;
+  *out = &d;
+  return LORA_OK;
+}
+
+// 2-D bf16 tensor map over a row-major [outer, inner] matrix with row stride
+// `ld` elements, 128-byte swizzle, zero fill outside the matrix.
+int make_map(CUtensorMap* m, const void* ptr, uint64_t inner, uint64_t outer, uint64_t ld, uint32_t box_inner,
+             uint32_t box_outer) {
+  cuuint64_t dims[2] = {inner, outer};
+  cuuint64_t strides[1] = {ld * 2};
+  cuuint32_t box[2] = {box_inner, box_outer};
+  cuuint32_t estr[2] = {1, 1};
+  CUresult r = g_encode(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void*>(ptr), dims, strides, box, estr,
+                        CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+                        CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+  return r == CUDA_SUCCESS ? LORA_OK : LORA_ECUDA;
+}
+
+inline size_t up256(size_t x) { return (x + 255) & ~(size_t)255; }
+inline bool aligned16(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
+inline int cdiv(int64_t a, int64_t b) { return (int)((a + b - 1) / b); }
+
+int check_shape(const lora_shape* s) {
+  if (!s) return LORA_ENULL;
+  if (s->T < 8 || s->d_in < 8 || s->d_out < 8) return LORA_EINVAL;
+  if ((s->T % 8) || (s->d_in % 8) || (s->d_out % 8)) return LORA_EINVAL;
+  if (s->T > (1ll << 30) || s->d_in > (1ll << 20) || s->d_out > (1ll << 20)) return LORA_EINVAL;
+  if (s->rank < 1 || s->rank > 128) return LORA_EINVAL;
+  if (!isfinite(s->scale)) return LORA_EINVAL;
+  return LORA_OK;
+}
+
+// Workspace regions of one projection.
+struct Ws {
+  size_t su_pad = 0, b_pad = 0, sv = 0, part_u = 0, part_sv = 0, part_dB = 0, part_dA = 0;
+  size_t total = 0;
+  RowProjPlan pu{1, 1}, psv{1, 1};
+  ColProjPlan pdB{1, 1}, pdA{1, 1};
+};
+
+Ws plan_ws(const lora_shape& s, int mode, int num_sms) {
+  Ws w;
+  const int T = (int)s.T, K = (int)s.d_in, N = (int)s.d_out, r = (int)s.rank, r8 = rank_pad8(r);
+  const bool pad = (r % 8) != 0;
+  size_t off = 0;
+  auto take = [&](size_t bytes) {
+    const size_t o = off;
+    off += up256(bytes);
+    return o;
+  };
+  w.su_pad = take((size_t)T * r8 * 2);
+  if (pad) w.b_pad = take((size_t)N * r8 * 2);
+  if (mode & LORA_FWD) {
+    w.pu = plan_rowproj(T, K, num_sms);
+    if (w.pu.splits > 1) w.part_u = take((size_t)w.pu.splits * T * r * 4);
+  }
+  if (mode & LORA_BWD) {
+    w.sv = take((size_t)T * r8 * 2);
+    w.psv = plan_rowproj(T, N, num_sms);
+    if (w.psv.splits > 1) w.part_sv = take((size_t)w.psv.splits * T * r * 4);
+    w.pdB = plan_colproj(T, N, num_sms);
+    if (w.pdB.splits > 1) w.part_dB = take((size_t)w.pdB.splits * N * r * 4);
+    w.pdA = plan_colproj(T, K, num_sms);
+    if (w.pdA.splits > 1) w.part_dA = take((size_t)w.pdA.splits * K * r * 4);
+  }
+  w.total = off;
+  return w;
+}
+
+template <typename T>
+T* at(void* ws, size_t off) {
+  return reinterpret_cast<T*>(static_cast<uint8_t*>(ws) + off);
+}
+
+typedef __nv_bfloat16 bf;
+inline const bf* cb(const lora_bf16* p) { return reinterpret_cast<const bf*>(p); }
+inline bf* mb(lora_bf16* p) { return reinterpret_cast<bf*>(p); }
+
+// ------------------------------------------------------------------ forward
+// Rank-r part of the forward: su for the GEMM; returns the adapter operands.
+struct FwdOperands {
+  const bf* su;
+  int ld_su;
+  const bf* B;
+  int ld_b;
+};
+
+int fwd_rank_r(const lora_proj& p, void* ws, const Ws& w, cudaStream_t st, FwdOperands* o) {
+  const lora_shape& s = p.shape;
+  const int T = (int)s.T, K = (int)s.d_in, N = (int)s.d_out, r = (int)s.rank, r8 = rank_pad8(r);
+  const bool pad = (r % 8) != 0;
+  bf* su_gemm = (p.su && !pad) ? mb(p.su) : at<bf>(ws, w.su_pad);
+  const int ld_gemm = (p.su && !pad) ? r : r8;
+  bf* su_user2 = (p.su && pad) ? mb(p.su) : nullptr;
+  cudaError_t e = launch_rowproj(cb(p.x), K, cb(p.A), K, true, T, K, r, w.pu, at<float>(ws, w.part_u), su_gemm,
+                                 ld_gemm, su_user2, r, s.scale, st);
+  if (e != cudaSuccess) return LORA_ECUDA;
+  o->su = su_gemm;
+  o->ld_su = ld_gemm;
+  if (pad) {
+    if (launch_pad_cols(cb(p.B), N, r, at<bf>(ws, w.b_pad), r8, st) != cudaSuccess) return LORA_ECUDA;
+    o->B = at<bf>(ws, w.b_pad);
+    o->ld_b = r8;
+  } else {
+    o->B = cb(p.B);
+    o->ld_b = r;
+  }
+  return LORA_OK;
+}
+
+int add_fwd_problem(GemmBatch& b, const lora_proj& p, const FwdOperands& o) {
+  const lora_shape& s = p.shape;
+  const int i = b.num_problems;
+  const int64_t T = s.T, K = s.d_in, N = s.d_out, r = s.rank;
+  int rc;
+  if ((rc = make_map(&b.tmA[i], p.x, K, T, K, 64, 128)) != LORA_OK) return rc;
+  if ((rc = make_map(&b.tmA2[i], o.su, r, T, o.ld_su, 64, 128)) != LORA_OK) return rc;
+  if ((rc = make_map(&b.tmB[i], p.W, K, N, K, 64, 256)) != LORA_OK) return rc;
+  if ((rc = make_map(&b.tmB2[i], o.B, r, N, o.ld_b, 64, 256)) != LORA_OK) return rc;
+  GemmProblem& g = b.prob[i];
+  g.out = mb(p.y);
+  g.ldo = (int)N;
+  g.M = (int)T;
+  g.N = (int)N;
+  g.Kmain = (int)K;
+  g.r = (int)r;
+  g.num_n_tiles = cdiv(N, gemm_tile_n());
+  g.kb_main = cdiv(K, gemm_tile_k());
+  g.kb_total = g.kb_main + cdiv(r, gemm_tile_k());
+  g.tile_begin = b.total_tiles;
+  b.total_tiles += cdiv(T, gemm_tile_m()) * g.num_n_tiles;
+  b.num_problems++;
+  return LORA_OK;
+}
+
+// ------------------------------------------------------------------ backward
+struct BwdOperands {
+  const bf* sv;
+  int ld_sv;
+};
+
+int bwd_rank_r(const lora_proj& p, void* ws, const Ws& w, cudaStream_t st, BwdOperands* o) {
+  const lora_shape& s = p.shape;
+  const int T = (int)s.T, K = (int)s.d_in, N = (int)s.d_out, r = (int)s.rank, r8 = rank_pad8(r);
+  const bool pad = (r % 8) != 0;
+  const bf* su_in = cb(p.su);
+  int ld_su = r;
+  const bf* B_in = cb(p.B);
+  int ld_b = r;
+  if (pad) {
+    if (launch_pad_cols(cb(p.su), T, r, at<bf>(ws, w.su_pad), r8, st) != cudaSuccess) return LORA_ECUDA;
+    if (launch_pad_cols(cb(p.B), N, r, at<bf>(ws, w.b_pad), r8, st) != cudaSuccess) return LORA_ECUDA;
+    su_in = at<bf>(ws, w.su_pad);
+    ld_su = r8;
+    B_in = at<bf>(ws, w.b_pad);
+    ld_b = r8;
+  }
+  bf* sv = at<bf>(ws, w.sv);
+  if (launch_rowproj(cb(p.dy), N, B_in, ld_b, false, T, N, r, w.psv, at<float>(ws, w.part_sv), sv, r8, nullptr, 0,
+                     s.scale, st) != cudaSuccess)
+    return LORA_ECUDA;
+  if (launch_colproj(cb(p.dy), N, su_in, ld_su, T, N, r, w.pdB, at<float>(ws, w.part_dB), p.dB, true, st) !=
+      cudaSuccess)
+    return LORA_ECUDA;
+  if (launch_colproj(cb(p.x), K, sv, r8, T, K, r, w.pdA, at<float>(ws, w.part_dA), p.dA, false, st) != cudaSuccess)
+    return LORA_ECUDA;
+  o->sv = sv;
+  o->ld_sv = r8;
+  return LORA_OK;
+}
+
+int add_bwd_problem(GemmBatch& b, const lora_proj& p, const BwdOperands& o) {
+  const lora_shape& s = p.shape;
+  const int i = b.num_problems;
+  const int64_t T = s.T, K = s.d_in, N = s.d_out, r = s.rank;
+  int rc;
+  if ((rc = make_map(&b.tmA[i], p.dy, N, T, N, 64, 128)) != LORA_OK) return rc;
+  if ((rc = make_map(&b.tmA2[i], o.sv, r, T, o.ld_sv, 64, 128)) != LORA_OK) return rc;
+  // W [N, K] read MN-major: inner dimension K (the GEMM's output columns), rows = contraction
+  if ((rc = make_map(&b.tmB[i], p.W, K, N, K, 64, 64)) != LORA_OK) return rc;
+  if ((rc = make_map(&b.tmB2[i], p.A, K, r, K, 64, 64)) != LORA_OK) return rc;
+  GemmProblem& g = b.prob[i];
+  g.out = mb(p.dx);
+  g.ldo = (int)K;
+  g.M = (int)T;
+  g.N = (int)K;
+  g.Kmain = (int)N;
+  g.r = (int)r;
+  g.num_n_tiles = cdiv(K, gemm_tile_n());
+  g.kb_main = cdiv(N, gemm_tile_k());
+  g.kb_total = g.kb_main + cdiv(r, gemm_tile_k());
+  g.tile_begin = b.total_tiles;
+  b.total_tiles += cdiv(T, gemm_tile_m()) * g.num_n_tiles;
+  b.num_problems++;
+  return LORA_OK;
+}
+
+void init_batch(GemmBatch& b, const DeviceInfo* d) {
+  memset(&b, 0, sizeof(b));
+  b.status = d->status;
+  b.limit_ns = g_wait_limit_ns;
+}
+
+// ------------------------------------------------------------------ checks
+int check_fwd_ptrs(const lora_proj& p) {
+  if (!p.x || !p.W || !p.A || !p.B || !p.y) return LORA_ENULL;
+  const void* ps[] = {p.x, p.W, p.A, p.B, p.y, p.su};
+  for (const void* q : ps)
+    if (q && !aligned16(q)) return LORA_EALIGN;
+  return LORA_OK;
+}
+
+int check_bwd_ptrs(const lora_proj& p) {
+  if (!p.dy || !p.x || !p.W || !p.A || !p.B || !p.su || !p.dA || !p.dB) return LORA_ENULL;
+  const void* ps[] = {p.dy, p.x, p.W, p.A, p.B, p.su, p.dx, p.dA, p.dB};
+  for (const void* q : ps)
+    if (q && !aligned16(q)) return LORA_EALIGN;
+  return LORA_OK;
+}
+
+int check_ws(void* ws, size_t ws_bytes, size_t need) {
+  if (need == 0) return LORA_OK;
+  if (!ws || ws_bytes < need) return LORA_EWORKSPACE;
+  if (reinterpret_cast<uintptr_t>(ws) & 255u) return LORA_EALIGN;
+  return LORA_OK;
+}
+
+// Runs the given projections in `mode`; every argument already validated.
+int run_step(const lora_proj* projs, int n, int mode, void* ws, const std::vector<Ws>& plans,
+             const std::vector<size_t>& offs, DeviceInfo* d, cudaStream_t st) {
+  int rc;
+  if (mode & LORA_FWD) {
+    std::vector<FwdOperands> ops(n);
+    for (int i = 0; i < n; ++i)
+      if ((rc = fwd_rank_r(projs[i], at<uint8_t>(ws, offs[i]), plans[i], st, &ops[i])) != LORA_OK) return rc;
+    // heavier problems first so that the static tile walk ends balanced
+    std::vector<int> order(n);
+    for (int i = 0; i < n; ++i) order[i] = i;
+    std::stable_sort(order.begin(), order.end(),
+                     [&](int a, int b) { return projs[a].shape.d_in > projs[b].shape.d_in; });
+    for (int i0 = 0; i0 < n; i0 += kMaxProblems) {
+      GemmBatch b;
+      init_batch(b, d);
+      for (int i = i0; i < n && i < i0 + kMaxProblems; ++i)
+        if ((rc = add_fwd_problem(b, projs[order[i]], ops[order[i]])) != LORA_OK) return rc;
+      if (launch_fused_gemm(b, false, d->num_sms, st) != cudaSuccess) return LORA_ECUDA;
+    }
+  }
+  if (mode & LORA_BWD) {
+    std::vector<BwdOperands> ops(n);
+    for (int i = 0; i < n; ++i)
+      if ((rc = bwd_rank_r(projs[i], at<uint8_t>(ws, offs[i]), plans[i], st, &ops[i])) != LORA_OK) return rc;
+    std::vector<int> order;
+    for (int i = 0; i < n; ++i)
+      if (projs[i].dx) order.push_back(i);
+    std::stable_sort(order.begin(), order.end(),
+                     [&](int a, int b) { return projs[a].shape.d_out > projs[b].shape.d_out; });
+    for (size_t i0 = 0; i0 < order.size(); i0 += kMaxProblems) {
+      GemmBatch b;
+      init_batch(b, d);
+      for (size_t i = i0; i < order.size() && i < i0 + kMaxProblems; ++i)
+        if ((rc = add_bwd_problem(b, projs[order[i]], ops[order[i]])) != LORA_OK) return rc;
+      if (launch_fused_gemm(b, true, d->num_sms, st) != cudaSuccess) return LORA_ECUDA;
+    }
+  }
+  return LORA_OK;
+}
+
+int plan_all(const lora_proj* projs, int n, int mode, int num_sms, std::vector<Ws>* plans,
+             std::vector<size_t>* offs, size_t* total) {
+  size_t off = 0;
+  plans->resize(n);
+  offs->resize(n);
+  for (int i = 0; i < n; ++i) {
+    int rc = check_shape(&projs[i].shape);
+    if (rc != LORA_OK) return rc;
+    (*plans)[i] = plan_ws(projs[i].shape, mode, num_sms);
+    (*offs)[i] = off;
+    off += up256((*plans)[i].total);
+  }
+  *total = off;
+  return LORA_OK;
+}
+
+}  // namespace
+}  // namespace lora
+
+using namespace lora;
+
+extern "C" {
+
+int lora_version(void) { return 100; }
+
+const char* lora_strerror(int code) {
+  switch (code) {
+    case LORA_OK: return "ok";
+    case LORA_EINVAL: return "invalid shape, rank, scale, mode or count";
+    case LORA_ENULL: return "required pointer is NULL";
+    case LORA_EALIGN: return "pointer not 16-byte aligned (workspace: 256-byte)";
+    case LORA_ECUDA: return "CUDA runtime call or kernel launch failed";
+    case LORA_ETIMEOUT: return "a device-side bounded wait expired";
+    case LORA_EWORKSPACE: return "workspace missing or too small";
+    case LORA_EDEVICE: return "current device is not a compute capability 10.3 (GB300) GPU";
+    default: return "unknown error";
+  }
+}
+
+int lora_set_wait_limit_ns(int64_t ns) {
+  std::lock_guard<std::mutex> lk(g_mu);
+  g_wait_limit_ns = ns > 0 ? (long long)ns : kDefaultWaitNs;
+  return LORA_OK;
+}
+
+int lora_workspace_size(const lora_shape* shape, int mode, size_t* bytes) {
+  if (!shape || !bytes) return LORA_ENULL;
+  if (mode < LORA_FWD || mode > LORA_FWD_BWD) return LORA_EINVAL;
+  lora_proj p;
+  memset(&p, 0, sizeof(p));
+  p.shape = *shape;
+  return lora_stack_workspace_size(&p, 1, mode, bytes);
+}
+
+int lora_stack_workspace_size(const lora_proj* projs, int n_proj, int mode, size_t* bytes) {
+  if (!projs || !bytes) return LORA_ENULL;
+  if (n_proj < 1 || n_proj > 64 || mode < LORA_FWD || mode > LORA_FWD_BWD) return LORA_EINVAL;
+  DeviceInfo* d = nullptr;
+  int rc = device_info(&d);
+  if (rc != LORA_OK) return rc;
+  std::vector<Ws> plans;
+  std::vector<size_t> offs;
+  return plan_all(projs, n_proj, mode, d->num_sms, &plans, &offs, bytes);
+}
+
+int lora_stack_step(const lora_proj* projs, int n_proj, int mode, void* workspace, size_t workspace_bytes,
+                    void* stream) {
+  if (!projs) return LORA_ENULL;
+  if (n_proj < 1 || n_proj > 64 || mode < LORA_FWD || mode > LORA_FWD_BWD) return LORA_EINVAL;
+  DeviceInfo* d = nullptr;
+  int rc = device_info(&d);
+  if (rc != LORA_OK) return rc;
+  std::vector<Ws> plans;
+  std::vector<size_t> offs;
+  size_t need = 0;
+  if ((rc = plan_all(projs, n_proj, mode, d->num_sms, &plans, &offs, &need)) != LORA_OK) return rc;
+  for (int i = 0; i < n_proj; ++i) {
+    if ((mode & LORA_FWD) && (rc = check_fwd_ptrs(projs[i])) != LORA_OK) return rc;
+    if ((mode & LORA_BWD) && (rc = check_bwd_ptrs(projs[i])) != LORA_OK) return rc;
+    if (mode == LORA_FWD_BWD && !projs[i].su) return LORA_ENULL;  // the backward needs the saved su
+  }
+  if ((rc = check_ws(workspace, workspace_bytes, need)) != LORA_OK) return rc;
+  return run_step(projs, n_proj, mode, workspace, plans, offs, d, static_cast<cudaStream_t>(stream));
+}
+
+int lora_linear_fwd(const lora_shape* shape, const lora_bf16* x, const lora_bf16* W, const lora_bf16* A,
+                    const lora_bf16* B, lora_bf16* y, lora_bf16* su, void* workspace, size_t workspace_bytes,
+                    void* stream) {
+  if (!shape) return LORA_ENULL;
+  lora_proj p;
+  memset(&p, 0, sizeof(p));
+  p.shape = *shape;
+  p.x = x;
+  p.W = W;
+  p.A = A;
+  p.B = B;
+  p.y = y;
+  p.su = su;
+  return lora_stack_step(&p, 1, LORA_FWD, workspace, workspace_bytes, stream);
+}
+
+int lora_linear_bwd(const lora_shape* shape, const lora_bf16* dy, const lora_bf16* x, const lora_bf16* W,
+                    const lora_bf16* A, const lora_bf16* B, const lora_bf16* su, lora_bf16* dx, float* dA,
+                    float* dB, void* workspace, size_t workspace_bytes, void* stream) {
+  if (!shape) return LORA_ENULL;
+  lora_proj p;
+  memset(&p, 0, sizeof(p));
+  p.shape = *shape;
+  p.dy = dy;
+  p.x = x;
+  p.W = W;
+  p.A = A;
+  p.B = B;
+  p.su = const_cast<lora_bf16*>(su);  // read only in the backward
+  p.dx = dx;
+  p.dA = dA;
+  p.dB = dB;
+  return lora_stack_step(&p, 1, LORA_BWD, workspace, workspace_bytes, stream);
+}
+
+int lora_read_status(void* stream, int* status, int reset) {
+  if (!status) return LORA_ENULL;
+  if (cudaStreamSynchronize(static_cast<cudaStream_t>(stream)) != cudaSuccess) return LORA_ECUDA;
+  int v = 0;
+  if (cudaMemcpyFromSymbol(&v, g_status, sizeof(int)) != cudaSuccess) return LORA_ECUDA;
+  if (reset) {
+    const int z = 0;
+    if (cudaMemcpyToSymbol(g_status, &z, sizeof(int)) != cudaSuccess) return LORA_ECUDA;
+  }
+  *status = v ? LORA_ETIMEOUT : LORA_OK;
+  return LORA_OK;
+}
+
+}  // extern "C"

@@ -1,0 +1,164 @@
+"""Python binding of the C ABI in include/lora.h (argument marshalling only).
+
+Every function has the name and argument order of its C counterpart.  Device
+buffers may be passed as integers (device addresses) or as CUDA tensors of
+any object with `data_ptr()`; `stream` may be an integer cudaStream_t, an
+object with a `cuda_stream` attribute (a torch.cuda.Stream), or None for
+the caller's current torch stream.  A non-zero return code raises LoraError.
+The compute runs only in the CUDA library: if it is not built, loading
+fails with an error; there is no other code path.
+"""
+from __future__ import annotations
+
+import ctypes
+import os
+
+_LIB_PATH = os.path.join(os.path.dirname(os.path.abspath(__file__)), "_lib", "liblora_gb300.so")
+_lib = None
+
+LORA_OK = 0
+LORA_EINVAL = -1
+LORA_ENULL = -2
+LORA_EALIGN = -3
+LORA_ECUDA = -4
+LORA_ETIMEOUT = -5
+LORA_EWORKSPACE = -6
+LORA_EDEVICE = -7
+
+LORA_FWD = 1
+LORA_BWD = 2
+LORA_FWD_BWD = 3
+
+# every symbol that include/lora.h declares
+EXPORTS = ("lora_workspace_size", "lora_linear_fwd", "lora_linear_bwd", "lora_stack_workspace_size",
+           "lora_stack_step", "lora_read_status", "lora_set_wait_limit_ns", "lora_strerror", "lora_version")
+
+
+class LoraError(RuntimeError):
+    def __init__(self, code: int, where: str):
+        self.code = code
+        msg = library().lora_strerror(code).decode() if _lib is not None else str(code)
+        super().__init__(f"{where}: {msg} ({code})")
+
+
+class lora_shape(ctypes.Structure):
+    _fields_ = [("T", ctypes.c_int64), ("d_in", ctypes.c_int64), ("d_out", ctypes.c_int64),
+                ("rank", ctypes.c_int64), ("scale", ctypes.c_float)]
+
+
+class lora_proj(ctypes.Structure):
+    _fields_ = [("shape", lora_shape),
+                ("x", ctypes.c_void_p), ("W", ctypes.c_void_p), ("A", ctypes.c_void_p), ("B", ctypes.c_void_p),
+                ("dy", ctypes.c_void_p), ("y", ctypes.c_void_p), ("su", ctypes.c_void_p), ("dx", ctypes.c_void_p),
+                ("dA", ctypes.c_void_p), ("dB", ctypes.c_void_p)]
+
+
+def library(path: str = _LIB_PATH) -> ctypes.CDLL:
+    """Load the CUDA library (once).  Raises OSError if it has not been built."""
+    global _lib
+    if _lib is None:
+        if not os.path.exists(path):
+            raise OSError(f"CUDA library not built: {path} (run paper_2606_19528_gb300.build)")
+        lib = ctypes.CDLL(path)
+        vp, sz, i32, i64 = ctypes.c_void_p, ctypes.c_size_t, ctypes.c_int, ctypes.c_int64
+        P = ctypes.POINTER
+        lib.lora_workspace_size.argtypes = [P(lora_shape), i32, P(sz)]
+        lib.lora_linear_fwd.argtypes = [P(lora_shape), vp, vp, vp, vp, vp, vp, vp, sz, vp]
+        lib.lora_linear_bwd.argtypes = [P(lora_shape), vp, vp, vp, vp, vp, vp, vp, vp, vp, vp, sz, vp]
+        lib.lora_stack_workspace_size.argtypes = [P(lora_proj), i32, i32, P(sz)]
+        lib.lora_stack_step.argtypes = [P(lora_proj), i32, i32, vp, sz, vp]
+        lib.lora_read_status.argtypes = [vp, P(i32), i32]
+        lib.lora_set_wait_limit_ns.argtypes = [i64]
+        lib.lora_strerror.argtypes = [i32]
+        lib.lora_strerror.restype = ctypes.c_char_p
+        lib.lora_version.argtypes = []
+        for name in EXPORTS:
+            if name != "lora_strerror":
+                getattr(lib, name).restype = i32
+        _lib = lib
+    return _lib
+
+
+def _ptr(a):
+    if a is None:
+        return None
+    if isinstance(a, int):
+        return a
+    return a.data_ptr()
+
+
+def _stream(s):
+    if s is None:
+        import torch
+        return torch.cuda.current_stream().cuda_stream
+    if isinstance(s, int):
+        return s
+    return s.cuda_stream
+
+
+def _check(rc: int, where: str):
+    if rc != LORA_OK:
+        raise LoraError(rc, where)
+
+
+def make_shape(T, d_in, d_out, rank, scale) -> lora_shape:
+    return lora_shape(int(T), int(d_in), int(d_out), int(rank), float(scale))
+
+
+def make_proj(shape: lora_shape, x=None, W=None, A=None, B=None, dy=None, y=None, su=None, dx=None, dA=None,
+              dB=None) -> lora_proj:
+    return lora_proj(shape, _ptr(x), _ptr(W), _ptr(A), _ptr(B), _ptr(dy), _ptr(y), _ptr(su), _ptr(dx), _ptr(dA),
+                     _ptr(dB))
+
+
+def lora_workspace_size(shape: lora_shape, mode: int) -> int:
+    n = ctypes.c_size_t(0)
+    _check(library().lora_workspace_size(ctypes.byref(shape), mode, ctypes.byref(n)), "lora_workspace_size")
+    return n.value
+
+
+def lora_linear_fwd(shape, x, W, A, B, y, su, workspace, workspace_bytes, stream=None) -> None:
+    _check(library().lora_linear_fwd(ctypes.byref(shape), _ptr(x), _ptr(W), _ptr(A), _ptr(B), _ptr(y), _ptr(su),
+                                     _ptr(workspace), int(workspace_bytes), _stream(stream)), "lora_linear_fwd")
+
+
+def lora_linear_bwd(shape, dy, x, W, A, B, su, dx, dA, dB, workspace, workspace_bytes, stream=None) -> None:
+    _check(library().lora_linear_bwd(ctypes.byref(shape), _ptr(dy), _ptr(x), _ptr(W), _ptr(A), _ptr(B), _ptr(su),
+                                     _ptr(dx), _ptr(dA), _ptr(dB), _ptr(workspace), int(workspace_bytes),
+                                     _stream(stream)), "lora_linear_bwd")
+
+
+def _proj_array(projs):
+    arr = (lora_proj * len(projs))(*projs)
+    return arr
+
+
+def lora_stack_workspace_size(projs, mode: int) -> int:
+    arr = _proj_array(projs)
+    n = ctypes.c_size_t(0)
+    _check(library().lora_stack_workspace_size(arr, len(projs), mode, ctypes.byref(n)), "lora_stack_workspace_size")
+    return n.value
+
+
+def lora_stack_step(projs, mode: int, workspace, workspace_bytes, stream=None) -> None:
+    arr = _proj_array(projs)
+    _check(library().lora_stack_step(arr, len(projs), mode, _ptr(workspace), int(workspace_bytes),
+                                     _stream(stream)), "lora_stack_step")
+
+
+def lora_read_status(stream=None, reset: bool = True) -> int:
+    st = ctypes.c_int(0)
+    _check(library().lora_read_status(_stream(stream), ctypes.byref(st), 1 if reset else 0), "lora_read_status")
+    return st.value
+
+
+def lora_set_wait_limit_ns(ns: int) -> None:
+    _check(library().lora_set_wait_limit_ns(int(ns)), "lora_set_wait_limit_ns")
+
+
+def lora_strerror(code: int) -> str:
+    return library().lora_strerror(int(code)).decode()
+
+
+def lora_version() -> int:
+    return library().lora_version()

@@ -1,0 +1,284 @@
+"""GPU parity: the CUDA path, called through the C ABI, against the fp64 oracle
+on the same seeded bf16 inputs.  Tolerances: relative Frobenius error
+<= 5e-3 for y, su and dx, <= 1e-2 for dA and dB; exact where the arithmetic
+is exact (small integers, B = 0)."""
+import json
+import os
+
+import numpy as np
+import pytest
+import torch
+
+import oracle
+from paper_2606_19528_gb300 import lora, synth, workloads
+from tests import gpu_util as G
+
+pytestmark = pytest.mark.gpu
+
+GOLDEN = os.path.join(os.path.dirname(os.path.abspath(__file__)), "golden")
+
+
+def gen_proj(cfg, idx, layer, T, K, N, r, s, group=None, zero_B=False, seed=0):
+    x = synth.gen_x(seed, cfg, idx if group is None else group, layer, T, K)
+    W = synth.gen_W(seed, cfg, idx, layer, N, K)
+    A = synth.gen_A(seed, cfg, idx, layer, r, K)
+    B = synth.gen_B(seed, cfg, idx, layer, N, r, zero=zero_B)
+    dy = synth.gen_dy(seed, cfg, idx, layer, T, N)
+    return x, W, A, B, dy
+
+
+def check_full(p: G.DevProj, with_dx=True):
+    x, W, A, B, dy = (p.f64(k) for k in ("x", "W", "A", "B", "dy"))
+    y, u = oracle.lora_forward(x, W, A, B, p.s)
+    dx, dA, dB, _ = oracle.lora_backward(dy, x, W, A, B, p.s)
+    errs = {
+        "y": G.rel_fro(G.host_f64(p.y), y),
+        "su": G.rel_fro(G.host_f64(p.su), p.s * u),
+        "dA": G.rel_fro(G.host_f64(p.dA), dA),
+        "dB": G.rel_fro(G.host_f64(p.dB), dB),
+    }
+    if with_dx:
+        errs["dx"] = G.rel_fro(G.host_f64(p.dx), dx)
+    assert errs["y"] <= G.TOL_Y, errs
+    assert errs["su"] <= G.TOL_SU, errs
+    assert errs["dA"] <= G.TOL_GRAD, errs
+    assert errs["dB"] <= G.TOL_GRAD, errs
+    if with_dx:
+        assert errs["dx"] <= G.TOL_DX, errs
+    return errs
+
+
+def check_sampled(p: G.DevProj, rows, with_dx=True):
+    """Rows of y and dx computed one by one by the oracle; dA and dB in full."""
+    x, W, A, B, dy = (p.f64(k) for k in ("x", "W", "A", "B", "dy"))
+    y_rows = oracle.lora_forward_rows(rows, x, W, A, B, p.s)
+    dA, dB = oracle.lora_adapter_grads(dy, x, A, B, p.s)
+    su_rows = p.s * (x[rows] @ A.T)
+    errs = {
+        "y": G.rel_fro(G.host_f64(p.y)[rows], y_rows),
+        "su": G.rel_fro(G.host_f64(p.su)[rows], su_rows),
+        "dA": G.rel_fro(G.host_f64(p.dA), dA),
+        "dB": G.rel_fro(G.host_f64(p.dB), dB),
+    }
+    if with_dx:
+        dx_rows = oracle.lora_backward_dx_rows(rows, dy, W, A, B, p.s)
+        errs["dx"] = G.rel_fro(G.host_f64(p.dx)[rows], dx_rows)
+    for k, v in errs.items():
+        tol = G.TOL_GRAD if k in ("dA", "dB") else G.TOL_Y
+        assert v <= tol, (k, errs)
+    for t in (p.y, p.su, p.dA, p.dB) + ((p.dx,) if with_dx else ()):
+        assert not torch.isnan(t).any(), "an output element was never written"
+    return errs
+
+
+# --------------------------------------------------------------- exact cases
+
+def test_handworked_example_exact():
+    """The hand-worked integer example embedded in an 8 x 8 x 8 problem with
+    r = 1 (zero padding elsewhere): every result is exact in bf16 / fp32."""
+    with open(os.path.join(GOLDEN, "lora_handworked_T2_K3_N2_r1.json")) as f:
+        g = json.load(f)
+    T = K = N = 8
+    r = 1
+
+    def emb(name, rows, cols):
+        a = np.zeros((rows, cols))
+        v = np.array(g[name], dtype=np.float64)
+        a[:v.shape[0], :v.shape[1]] = v
+        return synth.to_bf16_bits(a)
+
+    p = G.DevProj(emb("x", T, K), emb("W", N, K), emb("A", r, K), emb("B", N, r), emb("dy", T, N), g["s"])
+    G.run_single(p)
+    got = {"y": G.host_f64(p.y), "su": G.host_f64(p.su), "dx": G.host_f64(p.dx), "dA": G.host_f64(p.dA),
+           "dB": G.host_f64(p.dB)}
+    want = {"y": g["y"], "su": (np.array(g["u"]) * g["s"]).tolist(), "dx": g["dx"], "dA": g["dA"], "dB": g["dB"]}
+    for k in want:
+        w = np.array(want[k], dtype=np.float64)
+        full = np.zeros_like(got[k])
+        full[:w.shape[0], :w.shape[1]] = w
+        assert np.array_equal(got[k], full), (k, got[k], full)
+
+
+def test_single_small_T128():
+    wl = workloads.single_small()
+    pr = wl.projs[0]
+    p = G.DevProj(*gen_proj(wl.cfg, 0, 0, wl.T, pr.d_in, pr.d_out, wl.rank, wl.scale), wl.scale)
+    G.run_single(p)
+    check_full(p)
+
+
+def test_init_invariant_B0():
+    """B = 0: dA is exactly zero, and y and dx do not depend on the rank of
+    the (all-zero) adapter slab: runs with r = 8 and r = 16 agree bit for bit."""
+    wl = workloads.single_small(zero_B=True)
+    pr = wl.projs[0]
+    outs = []
+    for r in (8, 16):
+        x, W, A, B, dy = gen_proj(wl.cfg, 0, 0, wl.T, pr.d_in, pr.d_out, r, wl.scale, zero_B=True)
+        p = G.DevProj(x, W, A, B, dy, 16.0 / r)
+        G.run_single(p)
+        assert not torch.any(p.dA != 0), "dA must be exactly 0 when B = 0"
+        check_full(p)
+        outs.append((p.y.clone(), p.dx.clone()))
+    assert torch.equal(outs[0][0].view(torch.int16), outs[1][0].view(torch.int16))
+    assert torch.equal(outs[0][1].view(torch.int16), outs[1][1].view(torch.int16))
+
+
+# --------------------------------------------------------------- ragged shapes
+
+RAGGED = [
+    # T, K, N, r : tails in every tile dimension, minimal sizes, padded ranks
+    (8, 8, 8, 1),
+    (136, 200, 264, 24),
+    (264, 72, 520, 4),
+    (128, 320, 136, 72),
+    (200, 136, 64, 128),
+    (72, 1032, 392, 16),
+    (384, 256, 768, 3),
+]
+
+
+@pytest.mark.parametrize("T,K,N,r", RAGGED, ids=[f"T{t}_K{k}_N{n}_r{r}" for t, k, n, r in RAGGED])
+def test_ragged_shapes(T, K, N, r):
+    s = 2.0
+    p = G.DevProj(*gen_proj(7, r, T, T, K, N, r, s), s)
+    G.run_single(p)
+    check_full(p)
+
+
+def test_forward_without_saved_su_and_backward_without_dx():
+    T, K, N, r, s = 256, 512, 384, 16, 2.0
+    bits = gen_proj(8, 0, 0, T, K, N, r, s)
+    p = G.DevProj(*bits, s)
+    G.run_single(p)
+    q = G.DevProj(*bits, s)
+    st = q.shape
+    ws = G.workspace(lora.lora_workspace_size(st, lora.LORA_FWD_BWD))
+    lora.lora_linear_fwd(st, q.x, q.W, q.A, q.B, q.y, None, ws, ws.numel())
+    lora.lora_linear_bwd(st, q.dy, q.x, q.W, q.A, q.B, p.su, None, q.dA, q.dB, ws, ws.numel())
+    torch.cuda.synchronize()
+    assert torch.equal(p.y.view(torch.int16), q.y.view(torch.int16))
+    assert torch.equal(p.dA, q.dA) and torch.equal(p.dB, q.dB)
+    assert torch.isnan(q.dx).all(), "dx = NULL must leave dx untouched"
+
+
+def test_deterministic():
+    T, K, N, r, s = 512, 1024, 768, 16, 2.0
+    bits = gen_proj(9, 0, 0, T, K, N, r, s)
+    a, b = G.DevProj(*bits, s), G.DevProj(*bits, s)
+    G.run_single(a)
+    G.run_single(b)
+    for n in ("y", "su", "dx"):
+        assert torch.equal(getattr(a, n).view(torch.int16), getattr(b, n).view(torch.int16)), n
+    assert torch.equal(a.dA, b.dA) and torch.equal(a.dB, b.dB)
+
+
+# --------------------------------------------------------------- workloads
+
+def test_llama_q_T512():
+    wl = workloads.llama_q()
+    pr = wl.projs[0]
+    p = G.DevProj(*gen_proj(wl.cfg, 0, 0, wl.T, pr.d_in, pr.d_out, wl.rank, wl.scale), wl.scale)
+    G.run_single(p)
+    check_full(p)
+
+
+def build_layer(wl, layer=0, seed=0):
+    xs = {}
+    ps = []
+    for i, pr in enumerate(wl.projs):
+        x, W, A, B, dy = gen_proj(wl.cfg, i, layer, wl.T, pr.d_in, pr.d_out, wl.rank, wl.scale, group=pr.group,
+                                  seed=seed)
+        share = xs.get(pr.group)
+        p = G.DevProj(x, W, A, B, dy, wl.scale, share_x=share)
+        xs.setdefault(pr.group, p.x)
+        ps.append(p)
+    return ps
+
+
+@pytest.mark.parametrize("name", ["llama_layer", "qwen_layer"])
+def test_layer_stack(name):
+    wl = workloads.BY_NAME[name]()
+    ps = build_layer(wl)
+    G.run_stack(ps)
+    rows = G.sample_rows(wl.T, 64, 11)
+    for p in ps:
+        check_sampled(p, rows)
+
+
+def test_stack_equals_single_calls():
+    """The grouped launch computes every tile exactly as a single call does."""
+    wl = workloads.llama_sweep(256, 16)
+    ps = build_layer(wl, seed=3)
+    G.run_stack(ps)
+    for i, pr in enumerate(wl.projs):
+        q = G.DevProj(*(ps[i].bits[k] for k in ("x", "W", "A", "B", "dy")), wl.scale)
+        G.run_single(q)
+        for n in ("y", "su", "dx"):
+            assert torch.equal(getattr(q, n).view(torch.int16), getattr(ps[i], n).view(torch.int16)), (pr.name, n)
+        assert torch.equal(q.dA, ps[i].dA) and torch.equal(q.dB, ps[i].dB), pr.name
+
+
+SWEEP = [(T, r) for T in workloads.SWEEP_TOKENS for r in workloads.SWEEP_RANKS]
+
+
+@pytest.mark.parametrize("T,r", SWEEP, ids=[f"T{T}_r{r}" for T, r in SWEEP])
+def test_rank_token_sweep(T, r):
+    wl = workloads.llama_sweep(T, r)
+    ps = build_layer(wl)
+    G.run_stack(ps)
+    rows = G.sample_rows(T, 32, T + r)
+    for p in ps:
+        check_sampled(p, rows)
+    del ps
+    torch.cuda.empty_cache()
+
+
+def test_stack28_forward_all_then_backward_all():
+    """28 layers: forward of every layer first (saving su), then backward of
+    every layer in reverse order from the stored inputs."""
+    wl = workloads.llama_stack28()
+    layers = [build_layer(wl, layer=l) for l in range(wl.layers)]
+    for ps in layers:
+        projs = [p.proj() for p in ps]
+        ws = G.workspace(lora.lora_stack_workspace_size(projs, lora.LORA_FWD))
+        lora.lora_stack_step(projs, lora.LORA_FWD, ws, ws.numel())
+    for ps in reversed(layers):
+        projs = [p.proj() for p in ps]
+        ws = G.workspace(lora.lora_stack_workspace_size(projs, lora.LORA_BWD))
+        lora.lora_stack_step(projs, lora.LORA_BWD, ws, ws.numel())
+    torch.cuda.synchronize()
+    assert lora.lora_read_status() == lora.LORA_OK
+    rows = G.sample_rows(wl.T, 8, 5)
+    for l, ps in enumerate(layers):
+        for p in ps:
+            check_sampled(p, rows)
+
+
+# --------------------------------------------------------------- argument errors on the device path
+
+def test_argument_errors():
+    T, K, N, r, s = 128, 256, 256, 8, 2.0
+    p = G.DevProj(*gen_proj(0, 0, 0, T, K, N, r, s), s)
+    st = p.shape
+    need = lora.lora_workspace_size(st, lora.LORA_FWD)
+    ws = G.workspace(need + 512)
+    with pytest.raises(lora.LoraError) as e:
+        lora.lora_linear_fwd(st, p.x, p.W, p.A, p.B, p.y, p.su, ws, need - 1)
+    assert e.value.code == lora.LORA_EWORKSPACE
+    with pytest.raises(lora.LoraError) as e:
+        lora.lora_linear_fwd(st, p.x.data_ptr() + 2, p.W, p.A, p.B, p.y, p.su, ws, need)
+    assert e.value.code == lora.LORA_EALIGN
+    with pytest.raises(lora.LoraError) as e:
+        lora.lora_linear_fwd(st, p.x, p.W, p.A, p.B, p.y, p.su, ws.data_ptr() + 16, need)
+    assert e.value.code == lora.LORA_EALIGN
+    for bad in (lora.make_shape(12, K, N, r, s), lora.make_shape(T, K, N, 0, s), lora.make_shape(T, K, N, 129, s),
+                lora.make_shape(T, K, N, r, float("inf"))):
+        with pytest.raises(lora.LoraError) as e:
+            lora.lora_linear_fwd(bad, p.x, p.W, p.A, p.B, p.y, p.su, ws, need)
+        assert e.value.code == lora.LORA_EINVAL
+    with pytest.raises(lora.LoraError) as e:
+        lora.lora_linear_bwd(st, p.dy, p.x, p.W, p.A, p.B, None, p.dx, p.dA, p.dB, ws, need)
+    assert e.value.code == lora.LORA_ENULL
+    torch.cuda.synchronize()
+    assert torch.isnan(p.y).all(), "a rejected call must enqueue nothing"
