@@ -1,0 +1,449 @@
+"""Benchmark of the LoRA-linear fwd+bwd hot path on GB300.
+
+    python bench.py [--gpus N] [--steps K] [--warmup W] [--impl gb300|reference]
+
+One step = forward then backward (lora_stack_step, LORA_FWD_BWD) of the seven
+LoRA-adapted projections of a Llama-3.2-3B-shaped decoder layer (q, k, v, o,
+gate, up, down; T = 2048 tokens, r = 16, alpha = 32), bf16 operands with fp32
+accumulation, on seeded synthetic inputs.  Metric: tokens/s of fwd+bwd, and
+the fraction of the GB300 dense-bf16 tensor peak it reaches.
+
+Multi-GPU (torchrun, one process per GPU): every rank runs its own replica
+on its own batch of T tokens (weak scaling, no collective on the data path);
+value = total tokens of all ranks / max-over-ranks time.
+
+--impl reference times the fp64 CPU oracle on this host's cores instead,
+each step a bounded token sample of the same workload.
+"""
+from __future__ import annotations
+
+import argparse
+import json
+import os
+import statistics
+import subprocess
+import sys
+import threading
+import time
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+if ROOT not in sys.path:
+    sys.path.insert(0, ROOT)
+
+import numpy as np  # noqa: E402
+
+from paper_2606_19528_gb300 import synth, workloads  # noqa: E402
+
+METRIC = "LoRA-linear fwd+bwd tokens/s and % of GB300 dense-BF16 tensor peak (1 GPU)"
+UNIT = "tokens/s"
+PEAKS_FILE = os.path.join(ROOT, "MEASURED_PEAKS.json")
+FALLBACK_PEAKS = {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "bf16_tflops_sustained": 1700.0}
+L2_FLUSH_BYTES = 256 << 20
+
+
+def load_peaks():
+    try:
+        with open(PEAKS_FILE) as f:
+            p = json.load(f)
+        return p, "measured"
+    except (OSError, ValueError):
+        return dict(FALLBACK_PEAKS), "fallback"
+
+
+# ----------------------------------------------------------------------------- inputs
+
+def gen_layer_bits(wl: workloads.Workload, seed: int = 0, T: int | None = None):
+    """bf16 bits of every projection's inputs (x shared per input group)."""
+    T = wl.T if T is None else T
+    xs = {}
+    out = []
+    for i, p in enumerate(wl.projs):
+        if p.group not in xs:
+            xs[p.group] = synth.gen_x(seed, wl.cfg, p.group, 0, T, p.d_in)
+        out.append({
+            "x": xs[p.group], "group": p.group,
+            "W": synth.gen_W(seed, wl.cfg, i, 0, p.d_out, p.d_in),
+            "A": synth.gen_A(seed, wl.cfg, i, 0, wl.rank, p.d_in),
+            "B": synth.gen_B(seed, wl.cfg, i, 0, p.d_out, wl.rank, zero=wl.zero_B),
+            "dy": synth.gen_dy(seed, wl.cfg, i, 0, T, p.d_out),
+        })
+    return out
+
+
+def gemm_flops(wl: workloads.Workload):
+    """Algorithmic FLOPs of the two fused contractions of one step."""
+    T, r = wl.T, wl.rank
+    fwd = sum(2 * T * (p.d_in + r) * p.d_out for p in wl.projs)
+    bwd = sum(2 * T * (p.d_out + r) * p.d_in for p in wl.projs)
+    return float(fwd), float(bwd)
+
+
+# ----------------------------------------------------------------------------- clocks
+
+class ClockSampler:
+    """nvidia-smi samples of SM clock and throttle reasons while running."""
+
+    FIELDS = ("clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+              "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+              "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+    NAMES = ("hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap")
+
+    def __init__(self, gpu_id: str, period_ms: int = 100):
+        self.cmd = ["nvidia-smi", "-i", gpu_id, f"--query-gpu={self.FIELDS}", "--format=csv,noheader,nounits",
+                    "-lms", str(period_ms)]
+        self.proc = None
+        self.lines = []
+        self.thread = None
+
+    def start(self):
+        try:
+            self.proc = subprocess.Popen(self.cmd, stdout=subprocess.PIPE, stderr=subprocess.DEVNULL, text=True)
+        except OSError:
+            self.proc = None
+            return
+        self.thread = threading.Thread(target=self._read, daemon=True)
+        self.thread.start()
+
+    def _read(self):
+        for line in self.proc.stdout:
+            self.lines.append(line.strip())
+
+    def stop(self):
+        if self.proc is None:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": [], "samples": 0, "note": "nvidia-smi unavailable"}
+        self.proc.terminate()
+        try:
+            self.proc.wait(timeout=5)
+        except subprocess.TimeoutExpired:
+            self.proc.kill()
+        self.thread.join(timeout=5)
+        sm, smax, power, reasons = [], [], [], set()
+        for ln in self.lines:
+            f = [c.strip() for c in ln.split(",")]
+            if len(f) < 8:
+                continue
+            try:
+                sm.append(float(f[0]))
+                smax.append(float(f[1]))
+                power.append(float(f[2]))
+            except ValueError:
+                continue
+            for name, v in zip(self.NAMES, f[4:8]):
+                if v.lower().startswith("active"):
+                    reasons.add(name)
+        return {"sm_mhz": statistics.median(sm) if sm else None, "sm_max_mhz": max(smax) if smax else None,
+                "reasons": sorted(reasons), "samples": len(sm),
+                "power_w_max": max(power) if power else None}
+
+
+# ----------------------------------------------------------------------------- CPU oracle timing
+
+def oracle_sample(wl: workloads.Workload, tokens: int, seed: int = 0):
+    """fp64 inputs of a `tokens`-token sample of the workload (outside timing)."""
+    bits = gen_layer_bits(wl, seed, T=tokens)
+    f = synth.bf16_bits_to_f64
+    return [{k: f(v) for k, v in p.items() if k != "group"} for p in bits]
+
+
+def time_oracle_step(sample, s: float):
+    import oracle
+    t0 = time.perf_counter()
+    c0 = time.process_time()
+    for p in sample:
+        oracle.lora_forward(p["x"], p["W"], p["A"], p["B"], s)
+        oracle.lora_backward(p["dy"], p["x"], p["W"], p["A"], p["B"], s)
+    return time.perf_counter() - t0, time.process_time() - c0
+
+
+def cpu_baseline(wl: workloads.Workload, budget_s: float = 15.0):
+    """The oracle as it stands on this host's cores, over a token sample sized
+    to about `budget_s` seconds of work; tokens/s of the full fwd+bwd."""
+    probe_T = 64
+    sample = oracle_sample(wl, probe_T)
+    time_oracle_step(sample, wl.scale)  # warm BLAS threads
+    wall, _ = time_oracle_step(sample, wl.scale)
+    T = int(min(wl.T, max(64, probe_T * budget_s / max(wall, 1e-3) / 2)))
+    T = max(8, T // 8 * 8)
+    sample = oracle_sample(wl, T)
+    walls, cpus = [], []
+    t_start = time.perf_counter()
+    while time.perf_counter() - t_start < budget_s / 2 or not walls:
+        w, c = time_oracle_step(sample, wl.scale)
+        walls.append(w)
+        cpus.append(c)
+    wall = sum(walls) / len(walls)
+    cores_used = max(1, round(sum(cpus) / sum(walls)))
+    return {"value": T / wall, "unit": UNIT, "cores": cores_used, "kind": "oracle",
+            "host_cpus": os.cpu_count(),
+            "sample": f"fp64 oracle (numpy BLAS) fwd+bwd of all {len(wl.projs)} projections on {T} of the "
+                      f"workload's {wl.T} tokens, {len(walls)} repetitions, mean {wall:.3f} s each"}
+
+
+def run_reference(args, wl):
+    """--impl reference: the oracle timed as the reference arm."""
+    rank = int(os.environ.get("RANK", "0"))
+    if rank != 0:
+        return 0
+    W, K = args.warmup, args.steps
+    probe = oracle_sample(wl, 32)
+    time_oracle_step(probe, wl.scale)
+    w32, _ = time_oracle_step(probe, wl.scale)
+    # tokens per step so that warmup + steps fit in about 90 s
+    per_step_budget = 90.0 / max(1, W + K)
+    T = int(32 * per_step_budget / max(w32, 1e-4))
+    T = max(8, min(wl.T, T // 8 * 8))
+    sample = oracle_sample(wl, T)
+    for _ in range(W):
+        time_oracle_step(sample, wl.scale)
+    walls, cpus = [], []
+    for _ in range(K):
+        w, c = time_oracle_step(sample, wl.scale)
+        walls.append(w)
+        cpus.append(c)
+    total = sum(walls)
+    value = T * K / total
+    cores = max(1, round(sum(cpus) / total))
+    line = {
+        "impl": "reference", "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": args.gpus,
+        "steps": K, "warmup": W, "ms_per_step": 1e3 * total / K, "higher_is_better": True,
+        "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic",
+        "config": {"workload": wl.name, "T": wl.T, "rank": wl.rank, "alpha": wl.alpha,
+                   "projections": [f"{p.name} {p.d_in}->{p.d_out}" for p in wl.projs],
+                   "sample_tokens_per_step": T},
+        "cpu_baseline": {"value": value, "unit": UNIT, "cores": cores, "kind": "oracle",
+                         "host_cpus": os.cpu_count(),
+                         "sample": f"{T} of {wl.T} tokens per step, all {len(wl.projs)} projections fwd+bwd"},
+        "e2e": {"value": value, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
+    }
+    print(json.dumps(line), flush=True)
+    return 0
+
+
+# ----------------------------------------------------------------------------- distributed helpers
+
+def dist_setup():
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    if world <= 1:
+        return None, 0, 1
+    import torch.distributed as dist
+    backend = "nccl" if os.environ.get("BENCH_DIST_BACKEND", "nccl") == "nccl" else "gloo"
+    dist.init_process_group(backend=backend)
+    return dist, dist.get_rank(), dist.get_world_size()
+
+
+def max_over_ranks(dist, value: float, device=None) -> float:
+    """Max of a host float over ranks (timing aggregation only, not the data path)."""
+    if dist is None:
+        return value
+    import torch
+    t = torch.tensor([value], dtype=torch.float64, device=device)
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return float(t.item())
+
+
+def barrier(dist, device=None):
+    if dist is not None:
+        if device is not None:
+            dist.barrier(device_ids=[device.index])
+        else:
+            dist.barrier()
+
+
+# ----------------------------------------------------------------------------- GPU arm
+
+class LayerOnDevice:
+    def __init__(self, wl, bits, torch, lora):
+        self.wl = wl
+        self.torch = torch
+        dev = torch.device("cuda")
+
+        def d(b):
+            return torch.from_numpy(np.ascontiguousarray(b).view(np.int16)).to(dev).view(torch.bfloat16)
+
+        T, r = wl.T, wl.rank
+        xs = {}
+        self.p = []
+        for pb, pr in zip(bits, wl.projs):
+            if pr.group not in xs:
+                xs[pr.group] = d(pb["x"])
+            e = {"x": xs[pr.group], "W": d(pb["W"]), "A": d(pb["A"]), "B": d(pb["B"]), "dy": d(pb["dy"]),
+                 "y": torch.empty(T, pr.d_out, dtype=torch.bfloat16, device=dev),
+                 "su": torch.empty(T, r, dtype=torch.bfloat16, device=dev),
+                 "dx": torch.empty(T, pr.d_in, dtype=torch.bfloat16, device=dev),
+                 "dA": torch.empty(r, pr.d_in, dtype=torch.float32, device=dev),
+                 "dB": torch.empty(pr.d_out, r, dtype=torch.float32, device=dev)}
+            self.p.append(e)
+        self.xs = xs
+        self.projs = [lora.make_proj(lora.make_shape(T, pr.d_in, pr.d_out, r, wl.scale), x=e["x"], W=e["W"],
+                                     A=e["A"], B=e["B"], dy=e["dy"], y=e["y"], su=e["su"], dx=e["dx"], dA=e["dA"],
+                                     dB=e["dB"]) for e, pr in zip(self.p, wl.projs)]
+        n = lora.lora_stack_workspace_size(self.projs, lora.LORA_FWD_BWD)
+        self.ws = torch.empty(max(n, 256), dtype=torch.uint8, device=dev)
+
+    def step(self, lora, stream):
+        lora.lora_stack_step(self.projs, lora.LORA_FWD_BWD, self.ws, self.ws.numel(), stream)
+
+
+def run_gpu(args, wl):
+    import torch
+
+    from paper_2606_19528_gb300 import lora
+
+    dist, rank, world = dist_setup()
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    torch.cuda.set_device(local)
+    device = torch.device("cuda", local)
+    lora.library()
+    peaks, peaks_src = load_peaks()
+
+    bits = gen_layer_bits(wl, seed=rank)
+    L = LayerOnDevice(wl, bits, torch, lora)
+    stream = torch.cuda.current_stream()
+    flush = torch.empty(L2_FLUSH_BYTES, dtype=torch.uint8, device=device)
+
+    W, K = max(3, args.warmup), args.steps
+    for _ in range(W):
+        L.step(lora, stream)
+    # a short profiled pass so that the event pool exists before the timed region
+    lora.lora_profile_begin()
+    L.step(lora, stream)
+    lora.lora_profile_end()
+    torch.cuda.synchronize()
+    assert lora.lora_read_status() == lora.LORA_OK
+
+    props = torch.cuda.get_device_properties(device)
+    gpu_id = str(getattr(props, "uuid", local))
+    if gpu_id and not gpu_id.startswith("GPU-") and len(gpu_id) == 36:
+        gpu_id = "GPU-" + gpu_id
+
+    # ---------------- timed region: device-resident inputs, L2 flushed between steps
+    ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in range(K)]
+    clocks = ClockSampler(gpu_id) if rank == 0 else None
+    barrier(dist, device)
+    torch.cuda.synchronize()
+    if clocks:
+        clocks.start()
+        time.sleep(0.3)
+    launches0 = lora.lora_launch_count()
+    lora.lora_profile_begin()
+    for i in range(K):
+        flush.zero_()
+        ev[i][0].record(stream)
+        L.step(lora, stream)
+        ev[i][1].record(stream)
+    torch.cuda.synchronize()
+    kern_ms, kern_launches = lora.lora_profile_end()
+    launches = lora.lora_launch_count() - launches0
+    barrier(dist, device)
+    clk = clocks.stop() if clocks else None
+    status = lora.lora_read_status()
+    step_ms_local = sum(a.elapsed_time(b) for a, b in ev) / K
+    step_ms = max_over_ranks(dist, step_ms_local, device)
+
+    # ---------------- end-to-end: host inputs (pinned) -> device -> step -> gradients back to host
+    e2e = None
+    if not args.no_e2e:
+        h_x = {g: torch.from_numpy(np.ascontiguousarray(b).view(np.int16)).pin_memory()
+               for g, b in ((pb["group"], pb["x"]) for pb in bits)}
+        h_dy = [torch.from_numpy(np.ascontiguousarray(pb["dy"]).view(np.int16)).pin_memory() for pb in bits]
+        h_dA = [torch.empty(e["dA"].shape, dtype=torch.float32).pin_memory() for e in L.p]
+        h_dB = [torch.empty(e["dB"].shape, dtype=torch.float32).pin_memory() for e in L.p]
+        h2d = sum(t.numel() * 2 for t in h_x.values()) + sum(t.numel() * 2 for t in h_dy)
+        d2h = sum(t.numel() * 4 for t in h_dA) + sum(t.numel() * 4 for t in h_dB)
+
+        def e2e_step():
+            for g, t in h_x.items():
+                L.xs[g].view(torch.int16).copy_(t, non_blocking=True)
+            for e, t in zip(L.p, h_dy):
+                e["dy"].view(torch.int16).copy_(t, non_blocking=True)
+            L.step(lora, stream)
+            for e, a, b in zip(L.p, h_dA, h_dB):
+                a.copy_(e["dA"], non_blocking=True)
+                b.copy_(e["dB"], non_blocking=True)
+
+        Ke = max(10, min(K, 200))
+        for _ in range(3):
+            e2e_step()
+        torch.cuda.synchronize()
+        barrier(dist, device)
+        e0 = torch.cuda.Event(enable_timing=True)
+        e1 = torch.cuda.Event(enable_timing=True)
+        e0.record(stream)
+        for _ in range(Ke):
+            e2e_step()
+        e1.record(stream)
+        torch.cuda.synchronize()
+        e2e_ms = max_over_ranks(dist, e0.elapsed_time(e1) / Ke, device)
+        e2e = {"value": world * wl.T / (e2e_ms / 1e3), "unit": UNIT, "h2d_bytes_per_step": h2d,
+               "d2h_bytes_per_step": d2h, "ms_per_step": e2e_ms, "steps": Ke,
+               "note": "x and dy copied from pinned host memory and dA, dB copied back to pinned host "
+                       "memory every step, all on the compute stream"}
+
+    if rank != 0:
+        if dist is not None:
+            dist.destroy_process_group()
+        return 0
+
+    flops = wl.flops()
+    tflops = flops / (step_ms / 1e3) / 1e12
+    f_fwd, f_bwd = gemm_flops(wl)
+    gemm_ms = (kern_ms["gemm_fwd"] + kern_ms["gemm_bwd"]) / K
+    gemm_tflops = (f_fwd + f_bwd) / (gemm_ms / 1e3) / 1e12
+    sustained = peaks.get("bf16_tflops_sustained", FALLBACK_PEAKS["bf16_tflops_sustained"])
+    burst = peaks.get("bf16_tflops", FALLBACK_PEAKS["bf16_tflops"])
+    per_kernel = {k: {"ms_per_step": kern_ms[k] / K, "launches_per_step": kern_launches[k] / K,
+                      "share": kern_ms[k] / max(1e-9, sum(kern_ms.values()))} for k in kern_ms}
+    line = {
+        "metric": METRIC, "value": world * wl.T / (step_ms / 1e3), "unit": UNIT, "n_gpus": world,
+        "steps": K, "warmup": W, "ms_per_step": step_ms, "higher_is_better": True, "scaling": "weak",
+        "vs_baseline": None, "dtype": "bf16", "data": "synthetic",
+        "config": {"workload": wl.name, "T": wl.T, "rank": wl.rank, "alpha": wl.alpha,
+                   "projections": [f"{p.name} {p.d_in}->{p.d_out}" for p in wl.projs],
+                   "step": "lora_stack_step(LORA_FWD_BWD): 7 forwards then 7 backwards",
+                   "flops_per_step": flops,
+                   "l2": "256 MiB buffer written between timed steps (outside the step events); "
+                         "inputs of one step (W 201 MB + x 71 MB + dy 113 MB) also exceed the 129 MB L2",
+                   "parallelism": f"{world} independent replica(s), no collective"},
+        "tflops": tflops,
+        "pct_of_bf16_peak": {"sustained": tflops / sustained, "burst": tflops / burst,
+                             "peak_tflops_sustained": sustained, "peak_tflops_burst": burst,
+                             "source": peaks_src},
+        "roofline": {"kernel": "fused_lora_gemm (fwd and bwd launches)", "bound": "tensor",
+                     "achieved": gemm_tflops, "peak": sustained, "unit": "TFLOP/s",
+                     "frac": gemm_tflops / sustained, "traffic": None,
+                     "peak_kind": f"bf16 sustained, of {peaks_src}",
+                     "frac_of_burst": gemm_tflops / burst,
+                     "flops_per_step": f_fwd + f_bwd, "ms_per_step": gemm_ms},
+        "kernels": per_kernel,
+        "gpu_launches": launches,
+        "clocks": clk,
+        "status": lora.lora_strerror(status),
+        "e2e": e2e,
+    }
+    if world == 1 and not args.no_cpu_baseline:
+        line["cpu_baseline"] = cpu_baseline(wl, budget_s=args.cpu_budget)
+    print(json.dumps(line), flush=True)
+    if dist is not None:
+        dist.destroy_process_group()
+    return 0
+
+
+def main(argv=None):
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=1000)
+    ap.add_argument("--warmup", type=int, default=20)
+    ap.add_argument("--impl", choices=("gb300", "reference"), default="gb300")
+    ap.add_argument("--workload", default="llama_layer", choices=sorted(workloads.BY_NAME))
+    ap.add_argument("--no-e2e", action="store_true")
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--cpu-budget", type=float, default=15.0)
+    args = ap.parse_args(argv)
+    wl = workloads.BY_NAME[args.workload]()
+    if args.impl == "reference":
+        return run_reference(args, wl)
+    return run_gpu(args, wl)
+
+
+if __name__ == "__main__":
+    sys.exit(main())

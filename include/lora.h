@@ -134,6 +134,29 @@ int lora_read_status(void* stream, int* status, int reset);
  * timeout path; affects launches made after the call.  Returns LORA_OK. */
 int lora_set_wait_limit_ns(int64_t ns);
 
+/* Kernel kinds of the profiling interface below. */
+enum {
+  LORA_KERNEL_GEMM_FWD = 0, /* fused [x | su] . [W | B]^T contraction */
+  LORA_KERNEL_GEMM_BWD = 1, /* fused [dy | sv] . [W ; A] contraction */
+  LORA_KERNEL_ROWPROJ = 2,  /* su = s x A^T, sv = s dy B (with their split reductions) */
+  LORA_KERNEL_COLPROJ = 3,  /* dB = dy^T su, dA = sv^T x (with their split reductions) */
+  LORA_KERNEL_PAD = 4,      /* zero-padded copies for ranks that are not multiples of 8 */
+  LORA_KERNEL_KINDS = 5
+};
+
+/* Number of kernels the library has enqueued since it was loaded (all
+ * devices).  A call rejected with an argument error enqueues none. */
+int64_t lora_launch_count(void);
+
+/* Device-time profiling: after lora_profile_begin, every launch group of
+ * the library is bracketed by CUDA events recorded on its stream.
+ * lora_profile_end waits for those events, writes the summed device time in
+ * milliseconds and the kernel launches per kind into ms[LORA_KERNEL_KINDS]
+ * and launches[LORA_KERNEL_KINDS] (either may be NULL), and stops recording.
+ * Returns LORA_OK, LORA_EINVAL (end without begin) or LORA_ECUDA. */
+int lora_profile_begin(void);
+int lora_profile_end(double* ms, int64_t* launches);
+
 /* Static message for a LORA_* code. */
 const char* lora_strerror(int code);
 

@@ -9,6 +9,7 @@
 #include <string.h>
 
 #include <algorithm>
+#include <atomic>
 #include <mutex>
 #include <vector>
 
@@ -34,6 +35,61 @@ struct DeviceInfo {
 std::mutex g_mu;
 DeviceInfo g_dev[kMaxDevices];
 long long g_wait_limit_ns = kDefaultWaitNs;
+
+// ------------------------------------------------------------------ launch count and profiling
+std::atomic<long long> g_launches{0};
+
+struct ProfRec {
+  int kind;
+  cudaEvent_t a, b;
+  long long launches;
+};
+
+struct Profiler {
+  bool on = false;
+  std::vector<cudaEvent_t> pool;  // events are reused across sessions
+  size_t next = 0;
+  std::vector<ProfRec> recs;
+  cudaEvent_t take() {
+    if (next == pool.size()) {
+      cudaEvent_t e = nullptr;
+      if (cudaEventCreate(&e) != cudaSuccess) return nullptr;
+      pool.push_back(e);
+    }
+    return pool[next++];
+  }
+};
+
+std::mutex g_prof_mu;
+Profiler g_prof;
+
+// Brackets one launch group with CUDA events while a profiling session is on.
+class ProfScope {
+ public:
+  ProfScope(int kind, cudaStream_t st) : kind_(kind), st_(st) {
+    std::lock_guard<std::mutex> lk(g_prof_mu);
+    if (!g_prof.on) return;
+    a_ = g_prof.take();
+    b_ = g_prof.take();
+    if (a_ && b_ && cudaEventRecord(a_, st_) == cudaSuccess) {
+      active_ = true;
+      l0_ = g_launches.load();
+    }
+  }
+  ~ProfScope() {
+    if (!active_) return;
+    std::lock_guard<std::mutex> lk(g_prof_mu);
+    if (g_prof.on && cudaEventRecord(b_, st_) == cudaSuccess)
+      g_prof.recs.push_back(ProfRec{kind_, a_, b_, g_launches.load() - l0_});
+  }
+
+ private:
+  int kind_;
+  cudaStream_t st_;
+  cudaEvent_t a_ = nullptr, b_ = nullptr;
+  bool active_ = false;
+  long long l0_ = 0;
+};
 
 typedef CUresult (*EncodeTiledFn)(CUtensorMap*, CUtensorMapDataType, cuuint32_t, void*, const cuuint64_t*,
                                   const cuuint64_t*, const cuuint32_t*, const cuuint32_t*, CUtensorMapInterleave,
@@ -164,12 +220,16 @@ int fwd_rank_r(const lora_proj& p, void* ws, const Ws& w, cudaStream_t st, FwdOp
   bf* su_gemm = (p.su && !pad) ? mb(p.su) : at<bf>(ws, w.su_pad);
   const int ld_gemm = (p.su && !pad) ? r : r8;
   bf* su_user2 = (p.su && pad) ? mb(p.su) : nullptr;
-  cudaError_t e = launch_rowproj(cb(p.x), K, cb(p.A), K, true, T, K, r, w.pu, at<float>(ws, w.part_u), su_gemm,
-                                 ld_gemm, su_user2, r, s.scale, st);
-  if (e != cudaSuccess) return LORA_ECUDA;
+  {
+    ProfScope ps(LORA_KERNEL_ROWPROJ, st);
+    if (launch_rowproj(cb(p.x), K, cb(p.A), K, true, T, K, r, w.pu, at<float>(ws, w.part_u), su_gemm, ld_gemm,
+                       su_user2, r, s.scale, st) != cudaSuccess)
+      return LORA_ECUDA;
+  }
   o->su = su_gemm;
   o->ld_su = ld_gemm;
   if (pad) {
+    ProfScope ps(LORA_KERNEL_PAD, st);
     if (launch_pad_cols(cb(p.B), N, r, at<bf>(ws, w.b_pad), r8, st) != cudaSuccess) return LORA_ECUDA;
     o->B = at<bf>(ws, w.b_pad);
     o->ld_b = r8;
@@ -220,6 +280,7 @@ int bwd_rank_r(const lora_proj& p, void* ws, const Ws& w, cudaStream_t st, BwdOp
   const bf* B_in = cb(p.B);
   int ld_b = r;
   if (pad) {
+    ProfScope ps(LORA_KERNEL_PAD, st);
     if (launch_pad_cols(cb(p.su), T, r, at<bf>(ws, w.su_pad), r8, st) != cudaSuccess) return LORA_ECUDA;
     if (launch_pad_cols(cb(p.B), N, r, at<bf>(ws, w.b_pad), r8, st) != cudaSuccess) return LORA_ECUDA;
     su_in = at<bf>(ws, w.su_pad);
@@ -228,14 +289,21 @@ int bwd_rank_r(const lora_proj& p, void* ws, const Ws& w, cudaStream_t st, BwdOp
     ld_b = r8;
   }
   bf* sv = at<bf>(ws, w.sv);
-  if (launch_rowproj(cb(p.dy), N, B_in, ld_b, false, T, N, r, w.psv, at<float>(ws, w.part_sv), sv, r8, nullptr, 0,
-                     s.scale, st) != cudaSuccess)
-    return LORA_ECUDA;
-  if (launch_colproj(cb(p.dy), N, su_in, ld_su, T, N, r, w.pdB, at<float>(ws, w.part_dB), p.dB, true, st) !=
-      cudaSuccess)
-    return LORA_ECUDA;
-  if (launch_colproj(cb(p.x), K, sv, r8, T, K, r, w.pdA, at<float>(ws, w.part_dA), p.dA, false, st) != cudaSuccess)
-    return LORA_ECUDA;
+  {
+    ProfScope ps(LORA_KERNEL_ROWPROJ, st);
+    if (launch_rowproj(cb(p.dy), N, B_in, ld_b, false, T, N, r, w.psv, at<float>(ws, w.part_sv), sv, r8, nullptr,
+                       0, s.scale, st) != cudaSuccess)
+      return LORA_ECUDA;
+  }
+  {
+    ProfScope ps(LORA_KERNEL_COLPROJ, st);
+    if (launch_colproj(cb(p.dy), N, su_in, ld_su, T, N, r, w.pdB, at<float>(ws, w.part_dB), p.dB, true, st) !=
+        cudaSuccess)
+      return LORA_ECUDA;
+    if (launch_colproj(cb(p.x), K, sv, r8, T, K, r, w.pdA, at<float>(ws, w.part_dA), p.dA, false, st) !=
+        cudaSuccess)
+      return LORA_ECUDA;
+  }
   o->sv = sv;
   o->ld_sv = r8;
   return LORA_OK;
@@ -315,6 +383,7 @@ int run_step(const lora_proj* projs, int n, int mode, void* ws, const std::vecto
       init_batch(b, d);
       for (int i = i0; i < n && i < i0 + kMaxProblems; ++i)
         if ((rc = add_fwd_problem(b, projs[order[i]], ops[order[i]])) != LORA_OK) return rc;
+      ProfScope ps(LORA_KERNEL_GEMM_FWD, st);
       if (launch_fused_gemm(b, false, d->num_sms, st) != cudaSuccess) return LORA_ECUDA;
     }
   }
@@ -332,6 +401,7 @@ int run_step(const lora_proj* projs, int n, int mode, void* ws, const std::vecto
       init_batch(b, d);
       for (size_t i = i0; i < order.size() && i < i0 + kMaxProblems; ++i)
         if ((rc = add_bwd_problem(b, projs[order[i]], ops[order[i]])) != LORA_OK) return rc;
+      ProfScope ps(LORA_KERNEL_GEMM_BWD, st);
       if (launch_fused_gemm(b, true, d->num_sms, st) != cudaSuccess) return LORA_ECUDA;
     }
   }
@@ -355,6 +425,9 @@ int plan_all(const lora_proj* projs, int n, int mode, int num_sms, std::vector<W
 }
 
 }  // namespace
+
+void note_launch() { g_launches.fetch_add(1, std::memory_order_relaxed); }
+
 }  // namespace lora
 
 using namespace lora;
@@ -456,6 +529,41 @@ int lora_linear_bwd(const lora_shape* shape, const lora_bf16* dy, const lora_bf1
   p.dA = dA;
   p.dB = dB;
   return lora_stack_step(&p, 1, LORA_BWD, workspace, workspace_bytes, stream);
+}
+
+int64_t lora_launch_count(void) { return (int64_t)g_launches.load(); }
+
+int lora_profile_begin(void) {
+  std::lock_guard<std::mutex> lk(g_prof_mu);
+  g_prof.recs.clear();
+  g_prof.next = 0;
+  g_prof.on = true;
+  return LORA_OK;
+}
+
+int lora_profile_end(double* ms, int64_t* launches) {
+  std::lock_guard<std::mutex> lk(g_prof_mu);
+  if (!g_prof.on) return LORA_EINVAL;
+  double acc[LORA_KERNEL_KINDS] = {0};
+  int64_t cnt[LORA_KERNEL_KINDS] = {0};
+  int rc = LORA_OK;
+  for (const ProfRec& r : g_prof.recs) {
+    float t = 0.f;
+    if (cudaEventSynchronize(r.b) != cudaSuccess || cudaEventElapsedTime(&t, r.a, r.b) != cudaSuccess) {
+      rc = LORA_ECUDA;
+      continue;
+    }
+    acc[r.kind] += t;
+    cnt[r.kind] += r.launches;
+  }
+  for (int k = 0; k < LORA_KERNEL_KINDS; ++k) {
+    if (ms) ms[k] = acc[k];
+    if (launches) launches[k] = cnt[k];
+  }
+  g_prof.recs.clear();
+  g_prof.next = 0;
+  g_prof.on = false;
+  return rc;
 }
 
 int lora_read_status(void* stream, int* status, int reset) {

@@ -274,6 +274,7 @@ cudaError_t launch_fused_gemm(const GemmBatch& batch, bool b_mn_major, int num_s
     fused_lora_gemm<true><<<grid, kThreads, kSmemBytes, stream>>>(batch);
   else
     fused_lora_gemm<false><<<grid, kThreads, kSmemBytes, stream>>>(batch);
+  note_launch();
   return cudaGetLastError();
 }
 

@@ -9,6 +9,9 @@
 
 namespace lora {
 
+// Counts one kernel launch (defined with the C ABI).
+void note_launch();
+
 // ---------------------------------------------------------------- fused GEMM
 constexpr int kMaxProblems = 8;
 

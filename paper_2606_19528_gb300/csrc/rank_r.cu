@@ -279,9 +279,14 @@ int grid_for(size_t n, int threads) {
   return (int)b;
 }
 
+// Raises the dynamic shared-memory limit of `kernel` once per process.
 template <typename K>
 cudaError_t set_smem(K kernel, int bytes) {
-  return cudaFuncSetAttribute(kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, bytes);
+  static bool done = false;  // one flag per kernel instantiation
+  if (done) return cudaSuccess;
+  cudaError_t e = cudaFuncSetAttribute(kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, bytes);
+  if (e == cudaSuccess) done = true;
+  return e;
 }
 
 template <int R>
@@ -295,16 +300,19 @@ cudaError_t rowproj_r(const __nv_bfloat16* X, int ldx, const __nv_bfloat16* Wm, 
     if ((e = set_smem(rowproj_kernel<R, true>, smem)) != cudaSuccess) return e;
     rowproj_kernel<R, true><<<grid, kThreads, smem, st>>>(X, ldx, Wm, ldw, T, C, r, plan.chunks_per_split, part,
                                                           out, ld_out, out2, ld_out2, scale);
+    note_launch();
   } else {
     if ((e = set_smem(rowproj_kernel<R, false>, smem)) != cudaSuccess) return e;
     rowproj_kernel<R, false><<<grid, kThreads, smem, st>>>(X, ldx, Wm, ldw, T, C, r, plan.chunks_per_split, part,
                                                            out, ld_out, out2, ld_out2, scale);
+    note_launch();
   }
   if ((e = cudaGetLastError()) != cudaSuccess) return e;
   if (plan.splits > 1) {
     const int ld = ld_out > ld_out2 ? ld_out : ld_out2;
     reduce_rows_kernel<<<grid_for((size_t)T * ld, 256), 256, 0, st>>>(part, plan.splits, T, r, out, ld_out, out2,
                                                                         ld_out2, scale);
+    note_launch();
     e = cudaGetLastError();
   }
   return e;
@@ -319,14 +327,17 @@ cudaError_t colproj_r(const __nv_bfloat16* X, int ldx, const __nv_bfloat16* S, i
   if (out_cr) {
     if ((e = set_smem(colproj_kernel<R, true>, smem)) != cudaSuccess) return e;
     colproj_kernel<R, true><<<grid, kThreads, smem, st>>>(X, ldx, S, lds, T, C, r, plan.chunks_per_split, part, out);
+    note_launch();
   } else {
     if ((e = set_smem(colproj_kernel<R, false>, smem)) != cudaSuccess) return e;
     colproj_kernel<R, false><<<grid, kThreads, smem, st>>>(X, ldx, S, lds, T, C, r, plan.chunks_per_split, part, out);
+    note_launch();
   }
   if ((e = cudaGetLastError()) != cudaSuccess) return e;
   if (plan.splits > 1) {
     const size_t n = (size_t)C * r;
     reduce_flat_kernel<<<grid_for(n, 256), 256, 0, st>>>(part, plan.splits, n, out);
+    note_launch();
     e = cudaGetLastError();
   }
   return e;
@@ -388,6 +399,7 @@ cudaError_t launch_pad_cols(const __nv_bfloat16* src, int rows, int r, __nv_bflo
                             cudaStream_t st) {
   const size_t n = (size_t)rows * ld_dst;
   pad_cols_kernel<<<grid_for(n, 256), 256, 0, st>>>(src, rows, r, dst, ld_dst);
+  note_launch();
   return cudaGetLastError();
 }
 

@@ -31,7 +31,16 @@ LORA_FWD_BWD = 3
 
 # every symbol that include/lora.h declares
 EXPORTS = ("lora_workspace_size", "lora_linear_fwd", "lora_linear_bwd", "lora_stack_workspace_size",
-           "lora_stack_step", "lora_read_status", "lora_set_wait_limit_ns", "lora_strerror", "lora_version")
+           "lora_stack_step", "lora_read_status", "lora_set_wait_limit_ns", "lora_launch_count",
+           "lora_profile_begin", "lora_profile_end", "lora_strerror", "lora_version")
+
+LORA_KERNEL_GEMM_FWD = 0
+LORA_KERNEL_GEMM_BWD = 1
+LORA_KERNEL_ROWPROJ = 2
+LORA_KERNEL_COLPROJ = 3
+LORA_KERNEL_PAD = 4
+LORA_KERNEL_KINDS = 5
+KERNEL_NAMES = ("gemm_fwd", "gemm_bwd", "rowproj", "colproj", "pad")
 
 
 class LoraError(RuntimeError):
@@ -69,12 +78,16 @@ def library(path: str = _LIB_PATH) -> ctypes.CDLL:
         lib.lora_stack_step.argtypes = [P(lora_proj), i32, i32, vp, sz, vp]
         lib.lora_read_status.argtypes = [vp, P(i32), i32]
         lib.lora_set_wait_limit_ns.argtypes = [i64]
+        lib.lora_launch_count.argtypes = []
+        lib.lora_profile_begin.argtypes = []
+        lib.lora_profile_end.argtypes = [P(ctypes.c_double), P(i64)]
         lib.lora_strerror.argtypes = [i32]
         lib.lora_strerror.restype = ctypes.c_char_p
         lib.lora_version.argtypes = []
         for name in EXPORTS:
             if name != "lora_strerror":
                 getattr(lib, name).restype = i32
+        lib.lora_launch_count.restype = i64
         _lib = lib
     return _lib
 
@@ -154,6 +167,23 @@ def lora_read_status(stream=None, reset: bool = True) -> int:
 
 def lora_set_wait_limit_ns(ns: int) -> None:
     _check(library().lora_set_wait_limit_ns(int(ns)), "lora_set_wait_limit_ns")
+
+
+def lora_launch_count() -> int:
+    return int(library().lora_launch_count())
+
+
+def lora_profile_begin() -> None:
+    _check(library().lora_profile_begin(), "lora_profile_begin")
+
+
+def lora_profile_end():
+    """Returns ({kind name: device ms}, {kind name: launches}) of the session."""
+    ms = (ctypes.c_double * LORA_KERNEL_KINDS)()
+    n = (ctypes.c_int64 * LORA_KERNEL_KINDS)()
+    _check(library().lora_profile_end(ms, n), "lora_profile_end")
+    return ({KERNEL_NAMES[k]: ms[k] for k in range(LORA_KERNEL_KINDS)},
+            {KERNEL_NAMES[k]: int(n[k]) for k in range(LORA_KERNEL_KINDS)})
 
 
 def lora_strerror(code: int) -> str:
