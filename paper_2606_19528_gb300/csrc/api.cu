@@ -23,6 +23,7 @@ namespace {
 __device__ int g_status;  // first device-side error (kStatusTimeout), 0 if none
 
 constexpr int kMaxDevices = 64;
+constexpr size_t kWsHeader = 256;  // 64 tile counters, one per fused-GEMM launch of a call
 constexpr long long kDefaultWaitNs = 4000000000ll;
 
 struct DeviceInfo {
@@ -160,16 +161,14 @@ int check_shape(const lora_shape* s) {
 
 // Workspace regions of one projection.
 struct Ws {
-  size_t su_pad = 0, b_pad = 0, sv = 0, part_u = 0, part_sv = 0, part_dB = 0, part_dA = 0;
+  size_t su_pad = 0, b_pad = 0, sv = 0;
   size_t total = 0;
-  RowProjPlan pu{1, 1}, psv{1, 1};
-  ColProjPlan pdB{1, 1}, pdA{1, 1};
 };
 
-Ws plan_ws(const lora_shape& s, int mode, int num_sms) {
+Ws plan_ws(const lora_shape& s, int mode) {
   Ws w;
-  const int T = (int)s.T, K = (int)s.d_in, N = (int)s.d_out, r = (int)s.rank, r8 = rank_pad8(r);
-  const bool pad = (r % 8) != 0;
+  const int64_t T = s.T, N = s.d_out, r8 = rank_pad8((int)s.rank);
+  const bool pad = (s.rank % 8) != 0;
   size_t off = 0;
   auto take = [&](size_t bytes) {
     const size_t o = off;
@@ -178,19 +177,7 @@ Ws plan_ws(const lora_shape& s, int mode, int num_sms) {
   };
   w.su_pad = take((size_t)T * r8 * 2);
   if (pad) w.b_pad = take((size_t)N * r8 * 2);
-  if (mode & LORA_FWD) {
-    w.pu = plan_rowproj(T, K, num_sms);
-    if (w.pu.splits > 1) w.part_u = take((size_t)w.pu.splits * T * r * 4);
-  }
-  if (mode & LORA_BWD) {
-    w.sv = take((size_t)T * r8 * 2);
-    w.psv = plan_rowproj(T, N, num_sms);
-    if (w.psv.splits > 1) w.part_sv = take((size_t)w.psv.splits * T * r * 4);
-    w.pdB = plan_colproj(T, N, num_sms);
-    if (w.pdB.splits > 1) w.part_dB = take((size_t)w.pdB.splits * N * r * 4);
-    w.pdA = plan_colproj(T, K, num_sms);
-    if (w.pdA.splits > 1) w.part_dA = take((size_t)w.pdA.splits * K * r * 4);
-  }
+  if (mode & LORA_BWD) w.sv = take((size_t)T * r8 * 2);
   w.total = off;
   return w;
 }
@@ -204,49 +191,140 @@ typedef __nv_bfloat16 bf;
 inline const bf* cb(const lora_bf16* p) { return reinterpret_cast<const bf*>(p); }
 inline bf* mb(lora_bf16* p) { return reinterpret_cast<bf*>(p); }
 
-// ------------------------------------------------------------------ forward
-// Rank-r part of the forward: su for the GEMM; returns the adapter operands.
-struct FwdOperands {
-  const bf* su;
-  int ld_su;
-  const bf* B;
+// Adapter operands of one projection's fused contraction.
+struct Operands {
+  const bf* s_in;  // su (forward) or sv (backward): [T, r], row stride ld_s
+  int ld_s;
+  const bf* B;     // forward: B [N, r], row stride ld_b
   int ld_b;
 };
 
-int fwd_rank_r(const lora_proj& p, void* ws, const Ws& w, cudaStream_t st, FwdOperands* o) {
-  const lora_shape& s = p.shape;
-  const int T = (int)s.T, K = (int)s.d_in, N = (int)s.d_out, r = (int)s.rank, r8 = rank_pad8(r);
-  const bool pad = (r % 8) != 0;
-  bf* su_gemm = (p.su && !pad) ? mb(p.su) : at<bf>(ws, w.su_pad);
-  const int ld_gemm = (p.su && !pad) ? r : r8;
-  bf* su_user2 = (p.su && pad) ? mb(p.su) : nullptr;
-  {
-    ProfScope ps(LORA_KERNEL_ROWPROJ, st);
-    if (launch_rowproj(cb(p.x), K, cb(p.A), K, true, T, K, r, w.pu, at<float>(ws, w.part_u), su_gemm, ld_gemm,
-                       su_user2, r, s.scale, st) != cudaSuccess)
-      return LORA_ECUDA;
+// Appends block (W, ldw, rw) -> (out, out2) to the row problem of activation X,
+// opening a new problem when X differs or the concatenated rank would pass 128.
+void add_row_block(std::vector<RowProb>& probs, const bf* X, int ldx, int T, int C, float scale, const bf* W,
+                   int ldw, int rw, bf* out, int ld_out, bf* out2, int ld_out2, bool fuse) {
+  RowProb* p = nullptr;
+  if (fuse) {
+    for (RowProb& q : probs) {
+      int used = 0;
+      for (int b = 0; b < q.nblk; ++b) used += rank_pad8(q.rw[b]);
+      if (q.X == X && q.T == T && q.C == C && q.ldx == ldx && q.scale == scale && q.nblk < kMaxRankBlocks &&
+          used + rank_pad8(rw) <= 128) {
+        p = &q;
+        break;
+      }
+    }
   }
-  o->su = su_gemm;
-  o->ld_su = ld_gemm;
-  if (pad) {
-    ProfScope ps(LORA_KERNEL_PAD, st);
-    if (launch_pad_cols(cb(p.B), N, r, at<bf>(ws, w.b_pad), r8, st) != cudaSuccess) return LORA_ECUDA;
-    o->B = at<bf>(ws, w.b_pad);
-    o->ld_b = r8;
-  } else {
-    o->B = cb(p.B);
-    o->ld_b = r;
+  if (!p) {
+    RowProb q;
+    memset(&q, 0, sizeof(q));
+    q.X = X;
+    q.ldx = ldx;
+    q.T = T;
+    q.C = C;
+    q.scale = scale;
+    probs.push_back(q);
+    p = &probs.back();
+  }
+  const int b = p->nblk++;
+  p->W[b] = W;
+  p->ldw[b] = ldw;
+  p->rw[b] = rw;
+  p->out[b] = out;
+  p->ld_out[b] = ld_out;
+  p->out2[b] = out2;
+  p->ld_out2[b] = ld_out2;
+}
+
+void add_col_block(std::vector<ColProb>& probs, const bf* X, int ldx, int T, int C, const bf* S, int lds, int rs,
+                   float* out, int out_cr, bool fuse) {
+  ColProb* p = nullptr;
+  if (fuse) {
+    for (ColProb& q : probs) {
+      int used = 0;
+      for (int b = 0; b < q.nblk; ++b) used += rank_pad8(q.rs[b]);
+      if (q.X == X && q.T == T && q.C == C && q.ldx == ldx && q.out_cr == out_cr && q.nblk < kMaxRankBlocks &&
+          used + rank_pad8(rs) <= 128) {
+        p = &q;
+        break;
+      }
+    }
+  }
+  if (!p) {
+    ColProb q;
+    memset(&q, 0, sizeof(q));
+    q.X = X;
+    q.ldx = ldx;
+    q.T = T;
+    q.C = C;
+    q.out_cr = out_cr;
+    probs.push_back(q);
+    p = &probs.back();
+  }
+  const int b = p->nblk++;
+  p->S[b] = S;
+  p->lds[b] = lds;
+  p->rs[b] = rs;
+  p->out[b] = out;
+}
+
+int launch_rows(std::vector<RowProb>& probs, bool w_rc, int num_sms, cudaStream_t st) {
+  const int tile = rank_tile();
+  for (size_t i0 = 0; i0 < probs.size(); i0 += kMaxRankProblems) {
+    RowBatch b;
+    memset(&b, 0, sizeof(b));
+    int rmax = 16, max_chunks = 1;
+    for (size_t i = i0; i < probs.size() && i < i0 + kMaxRankProblems; ++i) {
+      RowProb& p = probs[i];
+      int used = 0;
+      for (int k = 0; k < p.nblk; ++k) used += rank_pad8(p.rw[k]);
+      p.rpad = rank_pad16(used);
+      rmax = std::max(rmax, p.rpad);
+      max_chunks = std::max(max_chunks, cdiv(p.C, tile));
+      p.tile_begin = b.tiles;
+      b.tiles += cdiv(p.T, tile);
+      b.p[b.n++] = p;
+    }
+    b.splits = rank_splits(b.tiles, max_chunks, num_sms);
+    b.w_rc = w_rc ? 1 : 0;
+    for (int i = 0; i < b.n; ++i) b.p[i].cps = cdiv(cdiv(b.p[i].C, tile), b.splits);
+    if (launch_rowprod(b, rmax, st) != cudaSuccess) return LORA_ECUDA;
   }
   return LORA_OK;
 }
 
-int add_fwd_problem(GemmBatch& b, const lora_proj& p, const FwdOperands& o) {
+int launch_cols(std::vector<ColProb>& probs, int num_sms, cudaStream_t st) {
+  const int tile = rank_tile();
+  for (size_t i0 = 0; i0 < probs.size(); i0 += kMaxRankProblems) {
+    ColBatch b;
+    memset(&b, 0, sizeof(b));
+    int rmax = 16, max_chunks = 1;
+    for (size_t i = i0; i < probs.size() && i < i0 + kMaxRankProblems; ++i) {
+      ColProb& p = probs[i];
+      int used = 0;
+      for (int k = 0; k < p.nblk; ++k) used += rank_pad8(p.rs[k]);
+      p.rpad = rank_pad16(used);
+      rmax = std::max(rmax, p.rpad);
+      max_chunks = std::max(max_chunks, cdiv(p.T, tile));
+      p.tile_begin = b.tiles;
+      b.tiles += cdiv(p.C, tile);
+      b.p[b.n++] = p;
+    }
+    b.splits = rank_splits(b.tiles, max_chunks, num_sms);
+    for (int i = 0; i < b.n; ++i) b.p[i].cps = cdiv(cdiv(b.p[i].T, tile), b.splits);
+    if (launch_colprod(b, rmax, st) != cudaSuccess) return LORA_ECUDA;
+  }
+  return LORA_OK;
+}
+
+// ------------------------------------------------------------------ forward
+int add_fwd_problem(GemmBatch& b, const lora_proj& p, const Operands& o) {
   const lora_shape& s = p.shape;
   const int i = b.num_problems;
   const int64_t T = s.T, K = s.d_in, N = s.d_out, r = s.rank;
   int rc;
   if ((rc = make_map(&b.tmA[i], p.x, K, T, K, 64, 128)) != LORA_OK) return rc;
-  if ((rc = make_map(&b.tmA2[i], o.su, r, T, o.ld_su, 64, 128)) != LORA_OK) return rc;
+  if ((rc = make_map(&b.tmA2[i], o.s_in, r, T, o.ld_s, 64, 128)) != LORA_OK) return rc;
   if ((rc = make_map(&b.tmB[i], p.W, K, N, K, 64, 256)) != LORA_OK) return rc;
   if ((rc = make_map(&b.tmB2[i], o.B, r, N, o.ld_b, 64, 256)) != LORA_OK) return rc;
   GemmProblem& g = b.prob[i];
@@ -257,65 +335,24 @@ int add_fwd_problem(GemmBatch& b, const lora_proj& p, const FwdOperands& o) {
   g.Kmain = (int)K;
   g.r = (int)r;
   g.num_n_tiles = cdiv(N, gemm_tile_n());
+  g.num_m_tiles = cdiv(T, gemm_tile_m());
+  g.m_fast = N >= T ? 1 : 0;  // weight operand [N, K] at least as large as x [T, K]
   g.kb_main = cdiv(K, gemm_tile_k());
   g.kb_total = g.kb_main + cdiv(r, gemm_tile_k());
   g.tile_begin = b.total_tiles;
-  b.total_tiles += cdiv(T, gemm_tile_m()) * g.num_n_tiles;
+  b.total_tiles += g.num_m_tiles * g.num_n_tiles;
   b.num_problems++;
   return LORA_OK;
 }
 
 // ------------------------------------------------------------------ backward
-struct BwdOperands {
-  const bf* sv;
-  int ld_sv;
-};
-
-int bwd_rank_r(const lora_proj& p, void* ws, const Ws& w, cudaStream_t st, BwdOperands* o) {
-  const lora_shape& s = p.shape;
-  const int T = (int)s.T, K = (int)s.d_in, N = (int)s.d_out, r = (int)s.rank, r8 = rank_pad8(r);
-  const bool pad = (r % 8) != 0;
-  const bf* su_in = cb(p.su);
-  int ld_su = r;
-  const bf* B_in = cb(p.B);
-  int ld_b = r;
-  if (pad) {
-    ProfScope ps(LORA_KERNEL_PAD, st);
-    if (launch_pad_cols(cb(p.su), T, r, at<bf>(ws, w.su_pad), r8, st) != cudaSuccess) return LORA_ECUDA;
-    if (launch_pad_cols(cb(p.B), N, r, at<bf>(ws, w.b_pad), r8, st) != cudaSuccess) return LORA_ECUDA;
-    su_in = at<bf>(ws, w.su_pad);
-    ld_su = r8;
-    B_in = at<bf>(ws, w.b_pad);
-    ld_b = r8;
-  }
-  bf* sv = at<bf>(ws, w.sv);
-  {
-    ProfScope ps(LORA_KERNEL_ROWPROJ, st);
-    if (launch_rowproj(cb(p.dy), N, B_in, ld_b, false, T, N, r, w.psv, at<float>(ws, w.part_sv), sv, r8, nullptr,
-                       0, s.scale, st) != cudaSuccess)
-      return LORA_ECUDA;
-  }
-  {
-    ProfScope ps(LORA_KERNEL_COLPROJ, st);
-    if (launch_colproj(cb(p.dy), N, su_in, ld_su, T, N, r, w.pdB, at<float>(ws, w.part_dB), p.dB, true, st) !=
-        cudaSuccess)
-      return LORA_ECUDA;
-    if (launch_colproj(cb(p.x), K, sv, r8, T, K, r, w.pdA, at<float>(ws, w.part_dA), p.dA, false, st) !=
-        cudaSuccess)
-      return LORA_ECUDA;
-  }
-  o->sv = sv;
-  o->ld_sv = r8;
-  return LORA_OK;
-}
-
-int add_bwd_problem(GemmBatch& b, const lora_proj& p, const BwdOperands& o) {
+int add_bwd_problem(GemmBatch& b, const lora_proj& p, const Operands& o) {
   const lora_shape& s = p.shape;
   const int i = b.num_problems;
   const int64_t T = s.T, K = s.d_in, N = s.d_out, r = s.rank;
   int rc;
   if ((rc = make_map(&b.tmA[i], p.dy, N, T, N, 64, 128)) != LORA_OK) return rc;
-  if ((rc = make_map(&b.tmA2[i], o.sv, r, T, o.ld_sv, 64, 128)) != LORA_OK) return rc;
+  if ((rc = make_map(&b.tmA2[i], o.s_in, r, T, o.ld_s, 64, 128)) != LORA_OK) return rc;
   // W [N, K] read MN-major: inner dimension K (the GEMM's output columns), rows = contraction
   if ((rc = make_map(&b.tmB[i], p.W, K, N, K, 64, 64)) != LORA_OK) return rc;
   if ((rc = make_map(&b.tmB2[i], p.A, K, r, K, 64, 64)) != LORA_OK) return rc;
@@ -327,10 +364,12 @@ int add_bwd_problem(GemmBatch& b, const lora_proj& p, const BwdOperands& o) {
   g.Kmain = (int)N;
   g.r = (int)r;
   g.num_n_tiles = cdiv(K, gemm_tile_n());
+  g.num_m_tiles = cdiv(T, gemm_tile_m());
+  g.m_fast = K >= T ? 1 : 0;  // weight operand [N, K] at least as large as dy [T, N]
   g.kb_main = cdiv(N, gemm_tile_k());
   g.kb_total = g.kb_main + cdiv(r, gemm_tile_k());
   g.tile_begin = b.total_tiles;
-  b.total_tiles += cdiv(T, gemm_tile_m()) * g.num_n_tiles;
+  b.total_tiles += g.num_m_tiles * g.num_n_tiles;
   b.num_problems++;
   return LORA_OK;
 }
@@ -359,7 +398,6 @@ int check_bwd_ptrs(const lora_proj& p) {
 }
 
 int check_ws(void* ws, size_t ws_bytes, size_t need) {
-  if (need == 0) return LORA_OK;
   if (!ws || ws_bytes < need) return LORA_EWORKSPACE;
   if (reinterpret_cast<uintptr_t>(ws) & 255u) return LORA_EALIGN;
   return LORA_OK;
@@ -369,10 +407,42 @@ int check_ws(void* ws, size_t ws_bytes, size_t need) {
 int run_step(const lora_proj* projs, int n, int mode, void* ws, const std::vector<Ws>& plans,
              const std::vector<size_t>& offs, DeviceInfo* d, cudaStream_t st) {
   int rc;
+  auto W_ = [&](int i) { return at<uint8_t>(ws, offs[i]); };
+  // tile counters of the fused-GEMM launches live in the workspace header
+  int* counters = at<int>(ws, 0);
+  int next_counter = 0;
+  if (cudaMemsetAsync(counters, 0, kWsHeader, st) != cudaSuccess) return LORA_ECUDA;
   if (mode & LORA_FWD) {
-    std::vector<FwdOperands> ops(n);
-    for (int i = 0; i < n; ++i)
-      if ((rc = fwd_rank_r(projs[i], at<uint8_t>(ws, offs[i]), plans[i], st, &ops[i])) != LORA_OK) return rc;
+    std::vector<Operands> ops(n);
+    std::vector<RowProb> rows;
+    {
+      ProfScope ps(LORA_KERNEL_PAD, st);
+      for (int i = 0; i < n; ++i) {
+        const lora_proj& p = projs[i];
+        const int T = (int)p.shape.T, K = (int)p.shape.d_in, N = (int)p.shape.d_out, r = (int)p.shape.rank;
+        const int r8 = rank_pad8(r);
+        const bool pad = (r % 8) != 0;
+        bf* su_gemm = (p.su && !pad) ? mb(p.su) : at<bf>(W_(i), plans[i].su_pad);
+        const int ld_gemm = (p.su && !pad) ? r : r8;
+        bf* su_user2 = (p.su && pad) ? mb(p.su) : nullptr;
+        add_row_block(rows, cb(p.x), K, T, K, p.shape.scale, cb(p.A), K, r, su_gemm, ld_gemm, su_user2, r, true);
+        ops[i].s_in = su_gemm;
+        ops[i].ld_s = ld_gemm;
+        if (pad) {
+          if (launch_pad_cols(cb(p.B), N, r, at<bf>(W_(i), plans[i].b_pad), r8, st) != cudaSuccess)
+            return LORA_ECUDA;
+          ops[i].B = at<bf>(W_(i), plans[i].b_pad);
+          ops[i].ld_b = r8;
+        } else {
+          ops[i].B = cb(p.B);
+          ops[i].ld_b = r;
+        }
+      }
+    }
+    {
+      ProfScope ps(LORA_KERNEL_ROWPROJ, st);
+      if ((rc = launch_rows(rows, true, d->num_sms, st)) != LORA_OK) return rc;
+    }
     // heavier problems first so that the static tile walk ends balanced
     std::vector<int> order(n);
     for (int i = 0; i < n; ++i) order[i] = i;
@@ -381,6 +451,7 @@ int run_step(const lora_proj* projs, int n, int mode, void* ws, const std::vecto
     for (int i0 = 0; i0 < n; i0 += kMaxProblems) {
       GemmBatch b;
       init_batch(b, d);
+      b.tile_counter = counters + next_counter++;
       for (int i = i0; i < n && i < i0 + kMaxProblems; ++i)
         if ((rc = add_fwd_problem(b, projs[order[i]], ops[order[i]])) != LORA_OK) return rc;
       ProfScope ps(LORA_KERNEL_GEMM_FWD, st);
@@ -388,9 +459,54 @@ int run_step(const lora_proj* projs, int n, int mode, void* ws, const std::vecto
     }
   }
   if (mode & LORA_BWD) {
-    std::vector<BwdOperands> ops(n);
-    for (int i = 0; i < n; ++i)
-      if ((rc = bwd_rank_r(projs[i], at<uint8_t>(ws, offs[i]), plans[i], st, &ops[i])) != LORA_OK) return rc;
+    std::vector<Operands> ops(n);
+    std::vector<RowProb> rows;
+    std::vector<ColProb> cols;
+    std::vector<const bf*> su_in(n);
+    std::vector<int> ld_su(n);
+    {
+      ProfScope ps(LORA_KERNEL_PAD, st);
+      for (int i = 0; i < n; ++i) {
+        const lora_proj& p = projs[i];
+        const int T = (int)p.shape.T, N = (int)p.shape.d_out, r = (int)p.shape.rank, r8 = rank_pad8(r);
+        const bool pad = (r % 8) != 0;
+        const bf* B_in = cb(p.B);
+        int ld_b = r;
+        su_in[i] = cb(p.su);
+        ld_su[i] = r;
+        if (pad) {
+          if (launch_pad_cols(cb(p.su), T, r, at<bf>(W_(i), plans[i].su_pad), r8, st) != cudaSuccess ||
+              launch_pad_cols(cb(p.B), N, r, at<bf>(W_(i), plans[i].b_pad), r8, st) != cudaSuccess)
+            return LORA_ECUDA;
+          su_in[i] = at<bf>(W_(i), plans[i].su_pad);
+          ld_su[i] = r8;
+          B_in = at<bf>(W_(i), plans[i].b_pad);
+          ld_b = r8;
+        }
+        bf* sv = at<bf>(W_(i), plans[i].sv);
+        add_row_block(rows, cb(p.dy), N, T, N, p.shape.scale, B_in, ld_b, r, sv, r8, nullptr, 0, false);
+        ops[i].s_in = sv;
+        ops[i].ld_s = r8;
+      }
+    }
+    {
+      ProfScope ps(LORA_KERNEL_ROWPROJ, st);
+      if ((rc = launch_rows(rows, false, d->num_sms, st)) != LORA_OK) return rc;
+    }
+    for (int i = 0; i < n; ++i) {
+      const lora_proj& p = projs[i];
+      const int T = (int)p.shape.T, K = (int)p.shape.d_in, N = (int)p.shape.d_out, r = (int)p.shape.rank;
+      add_col_block(cols, cb(p.dy), N, T, N, su_in[i], ld_su[i], r, p.dB, 1, false);
+    }
+    for (int i = 0; i < n; ++i) {
+      const lora_proj& p = projs[i];
+      const int T = (int)p.shape.T, K = (int)p.shape.d_in, r = (int)p.shape.rank;
+      add_col_block(cols, cb(p.x), K, T, K, ops[i].s_in, ops[i].ld_s, r, p.dA, 0, true);
+    }
+    {
+      ProfScope ps(LORA_KERNEL_COLPROJ, st);
+      if ((rc = launch_cols(cols, d->num_sms, st)) != LORA_OK) return rc;
+    }
     std::vector<int> order;
     for (int i = 0; i < n; ++i)
       if (projs[i].dx) order.push_back(i);
@@ -399,6 +515,7 @@ int run_step(const lora_proj* projs, int n, int mode, void* ws, const std::vecto
     for (size_t i0 = 0; i0 < order.size(); i0 += kMaxProblems) {
       GemmBatch b;
       init_batch(b, d);
+      b.tile_counter = counters + next_counter++;
       for (size_t i = i0; i < order.size() && i < i0 + kMaxProblems; ++i)
         if ((rc = add_bwd_problem(b, projs[order[i]], ops[order[i]])) != LORA_OK) return rc;
       ProfScope ps(LORA_KERNEL_GEMM_BWD, st);
@@ -410,13 +527,13 @@ int run_step(const lora_proj* projs, int n, int mode, void* ws, const std::vecto
 
 int plan_all(const lora_proj* projs, int n, int mode, int num_sms, std::vector<Ws>* plans,
              std::vector<size_t>* offs, size_t* total) {
-  size_t off = 0;
+  size_t off = kWsHeader;
   plans->resize(n);
   offs->resize(n);
   for (int i = 0; i < n; ++i) {
     int rc = check_shape(&projs[i].shape);
     if (rc != LORA_OK) return rc;
-    (*plans)[i] = plan_ws(projs[i].shape, mode, num_sms);
+    (*plans)[i] = plan_ws(projs[i].shape, mode);
     (*offs)[i] = off;
     off += up256((*plans)[i].total);
   }

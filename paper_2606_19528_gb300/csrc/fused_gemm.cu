@@ -13,10 +13,14 @@
 // the second operand W [N, K] is contracted over its rows, i.e. it is read
 // MN-major straight from the frozen weight (no transposed copy of W).
 //
-// Structure: persistent CTAs (one per SM) walk a static tile list spanning
-// every problem of a batch (up to kMaxProblems projections), 128 x 256
-// output tiles, 64-deep contraction blocks.
-//   warp 0      TMA producer: 4-stage shared-memory ring, 128-byte swizzle
+// Structure: persistent CTAs (one per SM) take tiles from a tile list
+// spanning every problem of a batch (up to kMaxProblems projections, heavier
+// first) through a global atomic counter, so that tiles of unequal depth
+// balance across SMs; 128 x 256 output tiles, 64-deep contraction blocks.
+// Within a problem, consecutive tiles walk M when the weight operand is the
+// larger one, so each weight tile is read from DRAM once.
+//   warp 0      tile scheduler and TMA producer: 4-stage shared-memory ring,
+//               128-byte swizzle
 //   warp 1      tcgen05.mma issuer (one thread); owns the TMEM allocation
 //   warps 2..5  epilogue: TMEM -> registers -> bf16 -> global
 // Two 256-column fp32 accumulators in TMEM (512 columns) let the epilogue of
@@ -38,13 +42,17 @@ constexpr uint32_t kStageBytes = kAStage + kBStage;
 constexpr uint32_t kMnChunk = 64 * kBK * 2;        // one 64-wide MN chunk of B, 8 KB
 constexpr int kThreads = 192;
 constexpr uint32_t kTmemCols = 512;
+constexpr int kTileRing = 4;  // tile ids handed from the producer to the MMA and epilogue warps
 
 struct __align__(8) Ctl {
   uint64_t full[kStages];
   uint64_t empty[kStages];
   uint64_t tfull[2];
   uint64_t tempty[2];
+  uint64_t tile_full[kTileRing];
+  uint64_t tile_empty[kTileRing];
   uint64_t drain;
+  int tile_id[kTileRing];
   uint32_t tmem_base;
   int abort;
 };
@@ -54,10 +62,25 @@ constexpr size_t kSmemBytes = 1024 + (size_t)kStages * kStageBytes + sizeof(Ctl)
 __device__ __forceinline__ void decode_tile(const GemmBatch& b, int t, int& p, int& m0, int& n0) {
   p = 0;
   while (p + 1 < b.num_problems && t >= b.prob[p + 1].tile_begin) ++p;
-  const int local = t - b.prob[p].tile_begin;
-  const int nt = b.prob[p].num_n_tiles;
-  m0 = (local / nt) * kBM;
-  n0 = (local % nt) * kBN;
+  const GemmProblem& P = b.prob[p];
+  const int local = t - P.tile_begin;
+  if (P.m_fast) {
+    m0 = (local % P.num_m_tiles) * kBM;
+    n0 = (local / P.num_m_tiles) * kBN;
+  } else {
+    m0 = (local / P.num_n_tiles) * kBM;
+    n0 = (local % P.num_n_tiles) * kBN;
+  }
+}
+
+// Consumer side of the tile ring: the id of this role's it-th tile (-1: no more).
+__device__ __forceinline__ bool next_tile(Ctl* ctl, int it, const WaitCtl& wc, volatile int* abort, int* t) {
+  const int slot = it % kTileRing;
+  const uint32_t par = (uint32_t)((it / kTileRing) & 1);
+  if (!mbar_wait(smem_u32(&ctl->tile_full[slot]), par, wc, abort)) return false;
+  *t = *reinterpret_cast<volatile int*>(&ctl->tile_id[slot]);
+  mbar_arrive(smem_u32(&ctl->tile_empty[slot]));
+  return true;
 }
 
 template <bool kBMn>
@@ -80,6 +103,10 @@ __global__ void __launch_bounds__(kThreads, 1) fused_lora_gemm(const __grid_cons
     for (int a = 0; a < 2; ++a) {
       mbar_init(smem_u32(&ctl->tfull[a]), 1);
       mbar_init(smem_u32(&ctl->tempty[a]), 128);
+    }
+    for (int k = 0; k < kTileRing; ++k) {
+      mbar_init(smem_u32(&ctl->tile_full[k]), 1);
+      mbar_init(smem_u32(&ctl->tile_empty[k]), 1 + 128);  // MMA thread + epilogue threads
     }
     mbar_init(smem_u32(&ctl->drain), 1);
     ctl->abort = 0;
@@ -109,7 +136,16 @@ __global__ void __launch_bounds__(kThreads, 1) fused_lora_gemm(const __grid_cons
     if (lane == 0) {
       int stage = 0;
       uint32_t phase = 0;
-      for (int t = blockIdx.x; t < b.total_tiles; t += gridDim.x) {
+      for (int it = 0;; ++it) {
+        // fetch the next tile and hand its id to the other roles
+        const int slot = it % kTileRing;
+        if (!mbar_wait(smem_u32(&ctl->tile_empty[slot]), (uint32_t)(((it / kTileRing) & 1) ^ 1), wc, abort_flag))
+          break;
+        int t = atomicAdd(b.tile_counter, 1);
+        if (t >= b.total_tiles) t = -1;
+        ctl->tile_id[slot] = t;
+        mbar_arrive(smem_u32(&ctl->tile_full[slot]));
+        if (t < 0) break;
         int p, m0, n0;
         decode_tile(b, t, p, m0, n0);
         const GemmProblem& P = b.prob[p];
@@ -151,9 +187,10 @@ __global__ void __launch_bounds__(kThreads, 1) fused_lora_gemm(const __grid_cons
       constexpr uint32_t idesc = idesc_bf16_f32(kBM, kBN, 0, kBMn ? 1 : 0);
       int stage = 0;
       uint32_t phase = 0;
-      int it = 0;
       bool ok = true;
-      for (int t = blockIdx.x; t < b.total_tiles && ok; t += gridDim.x, ++it) {
+      for (int it = 0; ok; ++it) {
+        int t;
+        if (!next_tile(ctl, it, wc, abort_flag, &t) || t < 0) break;
         int p, m0, n0;
         decode_tile(b, t, p, m0, n0);
         const GemmProblem& P = b.prob[p];
@@ -194,8 +231,11 @@ __global__ void __launch_bounds__(kThreads, 1) fused_lora_gemm(const __grid_cons
   } else {
     // ------------------------------------------------------------ epilogue
     const int q = warp & 3;  // TMEM lane quadrant this warp may access
-    int it = 0;
-    for (int t = blockIdx.x; t < b.total_tiles; t += gridDim.x, ++it) {
+    for (int it = 0;; ++it) {
+      int t;
+      bool got = next_tile(ctl, it, wc, abort_flag, &t);
+      got = __all_sync(0xffffffffu, got);
+      if (!got || t < 0) break;
       int p, m0, n0;
       decode_tile(b, t, p, m0, n0);
       const GemmProblem& P = b.prob[p];

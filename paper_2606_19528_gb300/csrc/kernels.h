@@ -26,6 +26,8 @@ struct GemmProblem {
   int tile_begin;      // first index of this problem in the batch's tile list
   int kb_main;         // contraction blocks of the base part
   int kb_total;        // base + adapter blocks
+  int m_fast;          // 1: consecutive tiles walk M (the weight tile stays put)
+  int num_m_tiles;
 };
 
 // One launch: up to kMaxProblems independent fused contractions.
@@ -40,6 +42,7 @@ struct GemmBatch {
   GemmProblem prob[kMaxProblems];
   int num_problems;
   int total_tiles;
+  int* tile_counter;   // zero at launch; hands out tiles in list order
   int* status;
   long long limit_ns;
 };
@@ -51,36 +54,66 @@ int gemm_tile_n();
 int gemm_tile_k();
 
 // ---------------------------------------------------------------- rank-r kernels
-// Padded rank used by the rank-r kernels: r rounded up to a multiple of 16.
 inline int rank_pad16(int r) { return (r + 15) / 16 * 16; }
 inline int rank_pad8(int r) { return (r + 7) / 8 * 8; }
 
-// Row products  out[t, j] = scale * sum_c X[t, c] * Wv(j, c),  t < T, j < r.
-//   w_rc = true : Wv(j, c) = Wm[j * ldw + c]   (A of the adapter, [r, C])
-//   w_rc = false: Wv(j, c) = Wm[c * ldw + j]   (B of the adapter, [C, r]; ldw % 8 == 0)
-// The reduction over c is split across `splits` CTA columns; with splits > 1
-// fp32 partials go to `part` [splits, T, r] and reduce_rows finishes.
-struct RowProjPlan {
-  int splits;
-  int chunks_per_split;  // 64-wide column chunks per split
-};
-RowProjPlan plan_rowproj(int T, int C, int num_sms);
-cudaError_t launch_rowproj(const __nv_bfloat16* X, int ldx, const __nv_bfloat16* Wm, int ldw, bool w_rc,
-                           int T, int C, int r, const RowProjPlan& plan, float* part,
-                           __nv_bfloat16* out, int ld_out, __nv_bfloat16* out2, int ld_out2, float scale,
-                           cudaStream_t stream);
+constexpr int kMaxRankBlocks = 4;     // projections fused into one problem
+constexpr int kMaxRankProblems = 16;  // problems per launch
 
-// Column products  G[c, j] = sum_t X[t, c] * S[t, j],  c < C, j < r  (S: lds % 8 == 0).
-//   out_cr = true : out[c * r + j]   ([C, r], dB)
-//   out_cr = false: out[j * C + c]   ([r, C], dA)
-struct ColProjPlan {
-  int splits;
-  int chunks_per_split;  // 64-token chunks per split
+// Row product problem: out_b[t, j] = scale * sum_c X[t, c] * Wv_b(j, c) for
+// every block b (one projection each) sharing the activation X [T, C].
+//   w_rc launches: Wv_b(j, c) = W_b[j * ldw_b + c]   (A of the adapter, [r_b, C])
+//   otherwise:     Wv_0(j, c) = W_0[c * ldw_0 + j]   (B of the adapter, [C, r]; one block)
+// Blocks are concatenated at 8-aligned rank offsets; columns rw_b .. ld_out_b
+// of out_b are written as zeros; out2_b (optional) gets columns < ld_out2_b.
+struct RowProb {
+  const __nv_bfloat16* X;
+  int ldx, T, C;
+  int nblk;
+  const __nv_bfloat16* W[kMaxRankBlocks];
+  int ldw[kMaxRankBlocks];
+  int rw[kMaxRankBlocks];
+  __nv_bfloat16* out[kMaxRankBlocks];
+  int ld_out[kMaxRankBlocks];
+  __nv_bfloat16* out2[kMaxRankBlocks];
+  int ld_out2[kMaxRankBlocks];
+  float scale;
+  int rpad;        // concatenated rank, rounded up to 16
+  int cps;         // 64-column chunks per split
+  int tile_begin;  // first 64-token tile of this problem in the launch
 };
-ColProjPlan plan_colproj(int T, int C, int num_sms);
-cudaError_t launch_colproj(const __nv_bfloat16* X, int ldx, const __nv_bfloat16* S, int lds, int T, int C,
-                           int r, const ColProjPlan& plan, float* part, float* out, bool out_cr,
-                           cudaStream_t stream);
+struct RowBatch {
+  RowProb p[kMaxRankProblems];
+  int n, tiles, splits, w_rc;
+};
+
+// Column product problem: out_b[c, j] = sum_t X[t, c] * S_b[t, j] for every
+// block b sharing X [T, C]; S_b has row stride lds_b (a multiple of 8) and
+// zeros in columns rs_b .. pad8(rs_b).  out_cr: out_b[c * rs_b + j] (dB),
+// else out_b[j * C + c] (dA).
+struct ColProb {
+  const __nv_bfloat16* X;
+  int ldx, T, C;
+  int nblk;
+  const __nv_bfloat16* S[kMaxRankBlocks];
+  int lds[kMaxRankBlocks];
+  int rs[kMaxRankBlocks];
+  float* out[kMaxRankBlocks];
+  int out_cr;
+  int rpad;
+  int cps;         // 64-token chunks per split
+  int tile_begin;  // first 64-column tile of this problem in the launch
+};
+struct ColBatch {
+  ColProb p[kMaxRankProblems];
+  int n, tiles, splits;
+};
+
+int rank_tile();
+// Cluster size (1, 2, 4 or 8) splitting each reduction so that the launch fills the GPU.
+int rank_splits(int tiles, int max_chunks, int num_sms);
+cudaError_t launch_rowprod(const RowBatch& b, int rmax, cudaStream_t stream);
+cudaError_t launch_colprod(const ColBatch& b, int rmax, cudaStream_t stream);
 
 // dst[i, j] = j < r ? src[i * r + j] : 0  for j < ld_dst (zero-padded copy of an [rows, r] matrix).
 cudaError_t launch_pad_cols(const __nv_bfloat16* src, int rows, int r, __nv_bfloat16* dst, int ld_dst,

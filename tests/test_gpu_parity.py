@@ -207,16 +207,24 @@ def test_layer_stack(name):
 
 
 def test_stack_equals_single_calls():
-    """The grouped launch computes every tile exactly as a single call does."""
+    """The grouped launches compute y, su and dx tile by tile exactly as single
+    calls do; dA and dB may be summed in another order (the split of the token
+    reduction depends on how many tiles a launch has), so they agree to fp32
+    rounding; and a repeated stack call is bit-identical."""
     wl = workloads.llama_sweep(256, 16)
     ps = build_layer(wl, seed=3)
     G.run_stack(ps)
+    first = [(p.dA.clone(), p.dB.clone(), p.y.clone()) for p in ps]
+    G.run_stack(ps)
+    for p, (dA, dB, y) in zip(ps, first):
+        assert torch.equal(p.dA, dA) and torch.equal(p.dB, dB) and torch.equal(p.y.view(torch.int16), y.view(torch.int16))
     for i, pr in enumerate(wl.projs):
         q = G.DevProj(*(ps[i].bits[k] for k in ("x", "W", "A", "B", "dy")), wl.scale)
         G.run_single(q)
         for n in ("y", "su", "dx"):
             assert torch.equal(getattr(q, n).view(torch.int16), getattr(ps[i], n).view(torch.int16)), (pr.name, n)
-        assert torch.equal(q.dA, ps[i].dA) and torch.equal(q.dB, ps[i].dB), pr.name
+        assert G.rel_fro(G.host_f64(q.dA), G.host_f64(ps[i].dA)) < 1e-6, pr.name
+        assert G.rel_fro(G.host_f64(q.dB), G.host_f64(ps[i].dB)) < 1e-6, pr.name
 
 
 SWEEP = [(T, r) for T in workloads.SWEEP_TOKENS for r in workloads.SWEEP_RANKS]
