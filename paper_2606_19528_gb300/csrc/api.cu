@@ -318,15 +318,27 @@ int launch_cols(std::vector<ColProb>& probs, int num_sms, cudaStream_t st) {
 }
 
 // ------------------------------------------------------------------ forward
-int add_fwd_problem(GemmBatch& b, const lora_proj& p, const Operands& o) {
+// CTA pairs per cluster for a batch of fused contractions over tokens T_i:
+// two pairs (weight tile shared) unless stacking 512 rows would waste work.
+int choose_pairs(const std::vector<int64_t>& Ts) {
+  for (int64_t T : Ts) {
+    const int64_t rows1 = (T + 255) / 256 * 256, rows2 = (T + 511) / 512 * 512;
+    if (rows2 * 100 > rows1 * 107) return 1;
+  }
+  return 2;
+}
+
+int add_fwd_problem(GemmBatch& b, const lora_proj& p, const Operands& o, int pairs) {
   const lora_shape& s = p.shape;
   const int i = b.num_problems;
   const int64_t T = s.T, K = s.d_in, N = s.d_out, r = s.rank;
   int rc;
+  // activation boxes: one CTA's 128 rows x 64 contraction elements; weight
+  // boxes: 64 rows x 64 (two per CTA, shared between the pairs of a cluster)
   if ((rc = make_map(&b.tmA[i], p.x, K, T, K, 64, 128)) != LORA_OK) return rc;
   if ((rc = make_map(&b.tmA2[i], o.s_in, r, T, o.ld_s, 64, 128)) != LORA_OK) return rc;
-  if ((rc = make_map(&b.tmB[i], p.W, K, N, K, 64, 256)) != LORA_OK) return rc;
-  if ((rc = make_map(&b.tmB2[i], o.B, r, N, o.ld_b, 64, 256)) != LORA_OK) return rc;
+  if ((rc = make_map(&b.tmB[i], p.W, K, N, K, 64, 64)) != LORA_OK) return rc;
+  if ((rc = make_map(&b.tmB2[i], o.B, r, N, o.ld_b, 64, 64)) != LORA_OK) return rc;
   GemmProblem& g = b.prob[i];
   g.out = mb(p.y);
   g.ldo = (int)N;
@@ -335,7 +347,7 @@ int add_fwd_problem(GemmBatch& b, const lora_proj& p, const Operands& o) {
   g.Kmain = (int)K;
   g.r = (int)r;
   g.num_n_tiles = cdiv(N, gemm_tile_n());
-  g.num_m_tiles = cdiv(T, gemm_tile_m());
+  g.num_m_tiles = cdiv(T, (int64_t)gemm_tile_m() * pairs);
   g.m_fast = N >= T ? 1 : 0;  // weight operand [N, K] at least as large as x [T, K]
   g.kb_main = cdiv(K, gemm_tile_k());
   g.kb_total = g.kb_main + cdiv(r, gemm_tile_k());
@@ -346,7 +358,7 @@ int add_fwd_problem(GemmBatch& b, const lora_proj& p, const Operands& o) {
 }
 
 // ------------------------------------------------------------------ backward
-int add_bwd_problem(GemmBatch& b, const lora_proj& p, const Operands& o) {
+int add_bwd_problem(GemmBatch& b, const lora_proj& p, const Operands& o, int pairs) {
   const lora_shape& s = p.shape;
   const int i = b.num_problems;
   const int64_t T = s.T, K = s.d_in, N = s.d_out, r = s.rank;
@@ -364,7 +376,7 @@ int add_bwd_problem(GemmBatch& b, const lora_proj& p, const Operands& o) {
   g.Kmain = (int)N;
   g.r = (int)r;
   g.num_n_tiles = cdiv(K, gemm_tile_n());
-  g.num_m_tiles = cdiv(T, gemm_tile_m());
+  g.num_m_tiles = cdiv(T, (int64_t)gemm_tile_m() * pairs);
   g.m_fast = K >= T ? 1 : 0;  // weight operand [N, K] at least as large as dy [T, N]
   g.kb_main = cdiv(N, gemm_tile_k());
   g.kb_total = g.kb_main + cdiv(r, gemm_tile_k());
@@ -452,10 +464,13 @@ int run_step(const lora_proj* projs, int n, int mode, void* ws, const std::vecto
       GemmBatch b;
       init_batch(b, d);
       b.tile_counter = counters + next_counter++;
+      std::vector<int64_t> Ts;
+      for (int i = i0; i < n && i < i0 + kMaxProblems; ++i) Ts.push_back(projs[order[i]].shape.T);
+      const int pairs = choose_pairs(Ts);
       for (int i = i0; i < n && i < i0 + kMaxProblems; ++i)
-        if ((rc = add_fwd_problem(b, projs[order[i]], ops[order[i]])) != LORA_OK) return rc;
+        if ((rc = add_fwd_problem(b, projs[order[i]], ops[order[i]], pairs)) != LORA_OK) return rc;
       ProfScope ps(LORA_KERNEL_GEMM_FWD, st);
-      if (launch_fused_gemm(b, false, d->num_sms, st) != cudaSuccess) return LORA_ECUDA;
+      if (launch_fused_gemm(b, false, pairs, d->num_sms, st) != cudaSuccess) return LORA_ECUDA;
     }
   }
   if (mode & LORA_BWD) {
@@ -516,10 +531,13 @@ int run_step(const lora_proj* projs, int n, int mode, void* ws, const std::vecto
       GemmBatch b;
       init_batch(b, d);
       b.tile_counter = counters + next_counter++;
+      std::vector<int64_t> Ts;
+      for (size_t i = i0; i < order.size() && i < i0 + kMaxProblems; ++i) Ts.push_back(projs[order[i]].shape.T);
+      const int pairs = choose_pairs(Ts);
       for (size_t i = i0; i < order.size() && i < i0 + kMaxProblems; ++i)
-        if ((rc = add_bwd_problem(b, projs[order[i]], ops[order[i]])) != LORA_OK) return rc;
+        if ((rc = add_bwd_problem(b, projs[order[i]], ops[order[i]], pairs)) != LORA_OK) return rc;
       ProfScope ps(LORA_KERNEL_GEMM_BWD, st);
-      if (launch_fused_gemm(b, true, d->num_sms, st) != cudaSuccess) return LORA_ECUDA;
+      if (launch_fused_gemm(b, true, pairs, d->num_sms, st) != cudaSuccess) return LORA_ECUDA;
     }
   }
   return LORA_OK;

@@ -13,18 +13,28 @@
 // the second operand W [N, K] is contracted over its rows, i.e. it is read
 // MN-major straight from the frozen weight (no transposed copy of W).
 //
-// Structure: persistent CTAs (one per SM) take tiles from a tile list
-// spanning every problem of a batch (up to kMaxProblems projections, heavier
-// first) through a global atomic counter, so that tiles of unequal depth
-// balance across SMs; 128 x 256 output tiles, 64-deep contraction blocks.
-// Within a problem, consecutive tiles walk M when the weight operand is the
-// larger one, so each weight tile is read from DRAM once.
-//   warp 0      tile scheduler and TMA producer: 4-stage shared-memory ring,
-//               128-byte swizzle
-//   warp 1      tcgen05.mma issuer (one thread); owns the TMEM allocation
+// Structure: persistent clusters of P CTA pairs (P = 1 or 2; one CTA per SM)
+// take "super-tiles" of P vertically adjacent 256 x 256 output tiles from a
+// tile list spanning every problem of a batch (up to kMaxProblems
+// projections, heavier first) through a global atomic counter, so that tiles
+// of unequal depth balance across SMs.  Each 256 x 256 tile is one 2-CTA
+// tensor-core contraction (tcgen05 cta_group::2, M = 256, N = 256, K = 16
+// per instruction): each CTA of a pair stages its own 128 rows of the
+// activation operand and its own 128 columns of the weight operand, and
+// holds its 128 x 256 half of the fp32 accumulator in its own tensor memory.
+// With P = 2 the two pairs share the weight tile: each CTA loads half of its
+// weight half and multicasts it to its counterpart in the other pair, so
+// L2-to-SM traffic drops by a quarter (the operand feed, not the tensor
+// pipe, bounds a single pair).  Within a problem, consecutive super-tiles
+// walk M when the weight operand is the larger one, so each weight tile is
+// read from DRAM once.
+//   warp 0      tile scheduler (cluster rank 0) and TMA producer (every CTA):
+//               6-stage shared-memory ring of 32 KB, 128-byte swizzle
+//   warp 1      TMEM allocation (every CTA); tcgen05.mma issuer (even CTAs)
 //   warps 2..5  epilogue: TMEM -> registers -> bf16 -> global
-// Two 256-column fp32 accumulators in TMEM (512 columns) let the epilogue of
-// one tile overlap the main loop of the next.  Every wait is bounded.
+// Two 256-column fp32 accumulators per CTA (512 TMEM columns) let the
+// epilogue of one tile overlap the main loop of the next.  Every wait is
+// bounded.
 #include "common.cuh"
 #include "kernels.h"
 
@@ -32,26 +42,29 @@ namespace lora {
 
 namespace {
 
-constexpr int kBM = 128;
-constexpr int kBN = 256;
+constexpr int kBM = 256;                          // tile rows (128 per CTA of a pair)
+constexpr int kHalf = 128;
+constexpr int kBN = 256;                          // tile columns (128 weight rows/columns per CTA)
 constexpr int kBK = 64;
-constexpr int kStages = 4;
-constexpr uint32_t kAStage = kBM * kBK * 2;        // 16 KB
-constexpr uint32_t kBStage = kBN * kBK * 2;        // 32 KB
-constexpr uint32_t kStageBytes = kAStage + kBStage;
-constexpr uint32_t kMnChunk = 64 * kBK * 2;        // one 64-wide MN chunk of B, 8 KB
+constexpr int kStages = 6;
+constexpr uint32_t kAHalf = kHalf * kBK * 2;      // 16 KB
+constexpr uint32_t kBHalf = kHalf * kBK * 2;      // 16 KB
+constexpr uint32_t kStageBytes = kAHalf + kBHalf;
+constexpr uint32_t kBox = 64 * kBK * 2;           // one 64 x 64 box of the weight operand, 8 KB
 constexpr int kThreads = 192;
+constexpr int kEpiWarps = 4;
 constexpr uint32_t kTmemCols = 512;
-constexpr int kTileRing = 4;  // tile ids handed from the producer to the MMA and epilogue warps
+constexpr int kTileRing = 4;  // tile ids handed from the scheduler to the other roles
+constexpr long long kDrainNs = 1000000000ll;
 
 struct __align__(8) Ctl {
-  uint64_t full[kStages];
-  uint64_t empty[kStages];
-  uint64_t tfull[2];
-  uint64_t tempty[2];
-  uint64_t tile_full[kTileRing];
-  uint64_t tile_empty[kTileRing];
-  uint64_t drain;
+  uint64_t full[kStages];          // even CTAs: both CTAs' halves of a stage landed
+  uint64_t empty[kStages];         // every CTA: every pair's MMAs finished reading a stage
+  uint64_t tfull[2];               // every CTA: accumulator complete
+  uint64_t tempty[2];              // even CTAs: the pair's epilogues drained an accumulator
+  uint64_t tile_full[kTileRing];   // every CTA: tile id written
+  uint64_t tile_empty[kTileRing];  // cluster rank 0: every consumer of the cluster read the slot
+  uint64_t drain;                  // every CTA: every MMA of its pair completed
   int tile_id[kTileRing];
   uint32_t tmem_base;
   int abort;
@@ -59,32 +72,25 @@ struct __align__(8) Ctl {
 
 constexpr size_t kSmemBytes = 1024 + (size_t)kStages * kStageBytes + sizeof(Ctl);
 
+// Problem p, first row m0 of the super-tile (P tiles stacked along M) and column n0.
+template <int P>
 __device__ __forceinline__ void decode_tile(const GemmBatch& b, int t, int& p, int& m0, int& n0) {
   p = 0;
   while (p + 1 < b.num_problems && t >= b.prob[p + 1].tile_begin) ++p;
-  const GemmProblem& P = b.prob[p];
-  const int local = t - P.tile_begin;
-  if (P.m_fast) {
-    m0 = (local % P.num_m_tiles) * kBM;
-    n0 = (local / P.num_m_tiles) * kBN;
+  const GemmProblem& Q = b.prob[p];
+  const int local = t - Q.tile_begin;
+  if (Q.m_fast) {
+    m0 = (local % Q.num_m_tiles) * kBM * P;
+    n0 = (local / Q.num_m_tiles) * kBN;
   } else {
-    m0 = (local / P.num_n_tiles) * kBM;
-    n0 = (local % P.num_n_tiles) * kBN;
+    m0 = (local / Q.num_n_tiles) * kBM * P;
+    n0 = (local % Q.num_n_tiles) * kBN;
   }
 }
 
-// Consumer side of the tile ring: the id of this role's it-th tile (-1: no more).
-__device__ __forceinline__ bool next_tile(Ctl* ctl, int it, const WaitCtl& wc, volatile int* abort, int* t) {
-  const int slot = it % kTileRing;
-  const uint32_t par = (uint32_t)((it / kTileRing) & 1);
-  if (!mbar_wait(smem_u32(&ctl->tile_full[slot]), par, wc, abort)) return false;
-  *t = *reinterpret_cast<volatile int*>(&ctl->tile_id[slot]);
-  mbar_arrive(smem_u32(&ctl->tile_empty[slot]));
-  return true;
-}
-
-template <bool kBMn>
+template <bool kBMn, int P>
 __global__ void __launch_bounds__(kThreads, 1) fused_lora_gemm(const __grid_constant__ GemmBatch b) {
+  constexpr int C = 2 * P;  // CTAs per cluster
   extern __shared__ uint8_t smem_raw[];
   const uint32_t raw = smem_u32(smem_raw);
   const uint32_t base = (raw + 1023u) & ~1023u;
@@ -93,86 +99,113 @@ __global__ void __launch_bounds__(kThreads, 1) fused_lora_gemm(const __grid_cons
 
   const int warp = threadIdx.x >> 5;
   const int lane = threadIdx.x & 31;
+  const int rank = (int)cluster_ctarank();
+  const int pair = rank >> 1;       // which pair of the cluster
+  const int c = rank & 1;           // position within the pair
+  const uint32_t pair_leader = (uint32_t)(rank & ~1);
   const WaitCtl wc{b.status, b.limit_ns};
 
   if (threadIdx.x == 0) {
     for (int s = 0; s < kStages; ++s) {
       mbar_init(smem_u32(&ctl->full[s]), 1);
-      mbar_init(smem_u32(&ctl->empty[s]), 1);
+      mbar_init(smem_u32(&ctl->empty[s]), P);  // one commit from every pair
     }
     for (int a = 0; a < 2; ++a) {
       mbar_init(smem_u32(&ctl->tfull[a]), 1);
-      mbar_init(smem_u32(&ctl->tempty[a]), 128);
+      mbar_init(smem_u32(&ctl->tempty[a]), 2 * kEpiWarps);
     }
     for (int k = 0; k < kTileRing; ++k) {
       mbar_init(smem_u32(&ctl->tile_full[k]), 1);
-      mbar_init(smem_u32(&ctl->tile_empty[k]), 1 + 128);  // MMA thread + epilogue threads
+      // MMA threads of the pairs, epilogue warps of every CTA, producers of the other CTAs
+      mbar_init(smem_u32(&ctl->tile_empty[k]), P + C * kEpiWarps + (C - 1));
     }
     mbar_init(smem_u32(&ctl->drain), 1);
     ctl->abort = 0;
     fence_mbar_init();
   }
   if (warp == 0 && lane == 0) {
-    for (int p = 0; p < b.num_problems; ++p) {
-      tma_prefetch_desc(&b.tmA[p]);
-      tma_prefetch_desc(&b.tmA2[p]);
-      tma_prefetch_desc(&b.tmB[p]);
-      tma_prefetch_desc(&b.tmB2[p]);
+    for (int q = 0; q < b.num_problems; ++q) {
+      tma_prefetch_desc(&b.tmA[q]);
+      tma_prefetch_desc(&b.tmA2[q]);
+      tma_prefetch_desc(&b.tmB[q]);
+      tma_prefetch_desc(&b.tmB2[q]);
     }
   }
   if (warp == 1) {
-    tmem_alloc(smem_u32(&ctl->tmem_base), kTmemCols);
-    tmem_relinquish();
+    tmem_alloc_pair(smem_u32(&ctl->tmem_base), kTmemCols);
+    tmem_relinquish_pair();
   }
   tc_fence_before();
   __syncthreads();
   tc_fence_after();
+  cluster_sync_all();  // every CTA's barriers exist before any cross-CTA arrival
   const uint32_t tmem_base = ctl->tmem_base;
-  long long issued = 0;     // producer: TMA stage loads issued
-  bool issued_any = false;  // MMA issuer: any tcgen05.mma issued
+  const uint32_t tile_empty_root = mapa_shared(smem_u32(&ctl->tile_empty[0]), 0);
 
   if (warp == 0) {
-    // ------------------------------------------------------------ producer
+    // ------------------------------------------------------------ scheduler + producer
     if (lane == 0) {
+      const uint32_t full_pl = mapa_shared(smem_u32(&ctl->full[0]), pair_leader);
+      const uint16_t b_mask = (uint16_t)((1u << c) | (1u << (c + 2)));  // my position in both pairs
       int stage = 0;
       uint32_t phase = 0;
       for (int it = 0;; ++it) {
-        // fetch the next tile and hand its id to the other roles
         const int slot = it % kTileRing;
-        if (!mbar_wait(smem_u32(&ctl->tile_empty[slot]), (uint32_t)(((it / kTileRing) & 1) ^ 1), wc, abort_flag))
-          break;
-        int t = atomicAdd(b.tile_counter, 1);
-        if (t >= b.total_tiles) t = -1;
-        ctl->tile_id[slot] = t;
-        mbar_arrive(smem_u32(&ctl->tile_full[slot]));
+        const uint32_t par = (uint32_t)((it / kTileRing) & 1);
+        int t;
+        if (rank == 0) {
+          if (!mbar_wait_cluster(smem_u32(&ctl->tile_empty[slot]), par ^ 1u, wc, abort_flag)) break;
+          t = atomicAdd(b.tile_counter, 1);
+          if (t >= b.total_tiles) t = -1;
+          ctl->tile_id[slot] = t;
+          for (int r = 1; r < C; ++r) st_cluster_u32(mapa_shared(smem_u32(&ctl->tile_id[slot]), r), (uint32_t)t);
+          mbar_arrive(smem_u32(&ctl->tile_full[slot]));
+          for (int r = 1; r < C; ++r) mbar_arrive_cluster(mapa_shared(smem_u32(&ctl->tile_full[slot]), r));
+        } else {
+          if (!mbar_wait_cluster(smem_u32(&ctl->tile_full[slot]), par, wc, abort_flag)) break;
+          t = *reinterpret_cast<volatile int*>(&ctl->tile_id[slot]);
+          mbar_arrive_cluster(tile_empty_root + (uint32_t)slot * 8u);
+        }
         if (t < 0) break;
-        int p, m0, n0;
-        decode_tile(b, t, p, m0, n0);
-        const GemmProblem& P = b.prob[p];
-        // backward: 64-wide MN chunks of the weight tile that hold any column < N
-        const int chunks = kBMn ? min(4, (P.N - n0 + 63) / 64) : 0;
-        const uint32_t tx = kAStage + (kBMn ? (uint32_t)chunks * kMnChunk : kBStage);
+        int p, sm0, n0;
+        decode_tile<P>(b, t, p, sm0, n0);
+        const GemmProblem& Q = b.prob[p];
+        const int m0 = sm0 + pair * kBM;
+        const int my_m = m0 + c * kHalf;
+        const bool a_mine = my_m < Q.M;
+        // weight boxes of pair position c' hold columns n0 + 128 c' + 64 j, j = 0, 1
+        auto box_ok = [&](int cc, int j) { return n0 + cc * kHalf + j * 64 < Q.N; };
+        // bytes landing in this pair per stage (signalled on the pair's even CTA)
+        const uint32_t tx_pair = (m0 < Q.M ? kAHalf : 0u) + (m0 + kHalf < Q.M ? kAHalf : 0u) +
+                                 kBox * ((box_ok(0, 0) ? 1u : 0u) + (box_ok(0, 1) ? 1u : 0u) +
+                                         (box_ok(1, 0) ? 1u : 0u) + (box_ok(1, 1) ? 1u : 0u));
         bool ok = true;
-        for (int kb = 0; kb < P.kb_total; ++kb) {
-          if (!mbar_wait(smem_u32(&ctl->empty[stage]), phase ^ 1u, wc, abort_flag)) {
+        for (int kb = 0; kb < Q.kb_total; ++kb) {
+          if (!mbar_wait_cluster(smem_u32(&ctl->empty[stage]), phase ^ 1u, wc, abort_flag)) {
             ok = false;
             break;
           }
-          const uint32_t full = smem_u32(&ctl->full[stage]);
+          if (c == 0) mbar_arrive_expect_tx(smem_u32(&ctl->full[stage]), tx_pair);
+          const uint32_t bar = full_pl + (uint32_t)stage * 8u;
           const uint32_t a_dst = base + stage * kStageBytes;
-          const uint32_t b_dst = a_dst + kAStage;
-          mbar_arrive_expect_tx(full, tx);
-          const bool main = kb < P.kb_main;
-          const int kc = main ? kb * kBK : (kb - P.kb_main) * kBK;
+          const uint32_t b_dst = a_dst + kAHalf;
+          const bool main = kb < Q.kb_main;
+          const int kc = main ? kb * kBK : (kb - Q.kb_main) * kBK;
           const CUtensorMap* ta = main ? &b.tmA[p] : &b.tmA2[p];
           const CUtensorMap* tb = main ? &b.tmB[p] : &b.tmB2[p];
-          tma_load_2d(a_dst, ta, full, kc, m0);
-          if (!kBMn) {
-            tma_load_2d(b_dst, tb, full, kc, n0);
-          } else {
-            for (int c = 0; c < chunks; ++c) tma_load_2d(b_dst + c * kMnChunk, tb, full, n0 + 64 * c, kc);
+          if (a_mine) tma_load_2d_pair(a_dst, ta, bar, kc, my_m);
+#pragma unroll
+          for (int j = 0; j < 2; ++j) {
+            if (P == 2 && j != pair) continue;  // the other pair's CTA loads (and multicasts) box j
+            if (!box_ok(c, j)) continue;
+            const int col = n0 + c * kHalf + j * 64;
+            const int x = kBMn ? col : kc;
+            const int y = kBMn ? kc : col;
+            if (P == 1)
+              tma_load_2d_pair(b_dst + j * kBox, tb, bar, x, y);
+            else
+              tma_load_2d_pair_mc(b_dst + j * kBox, tb, bar, x, y, b_mask);
           }
-          ++issued;
           if (++stage == kStages) {
             stage = 0;
             phase ^= 1u;
@@ -182,82 +215,92 @@ __global__ void __launch_bounds__(kThreads, 1) fused_lora_gemm(const __grid_cons
       }
     }
   } else if (warp == 1) {
-    // ------------------------------------------------------------ MMA issuer
-    if (lane == 0) {
+    // ------------------------------------------------------------ MMA issuer (even CTAs)
+    if (c == 0 && lane == 0) {
       constexpr uint32_t idesc = idesc_bf16_f32(kBM, kBN, 0, kBMn ? 1 : 0);
+      constexpr uint16_t all_mask = (uint16_t)((1u << C) - 1u);
+      const uint16_t pair_mask = (uint16_t)(0x3u << (2 * pair));
       int stage = 0;
       uint32_t phase = 0;
       bool ok = true;
       for (int it = 0; ok; ++it) {
-        int t;
-        if (!next_tile(ctl, it, wc, abort_flag, &t) || t < 0) break;
-        int p, m0, n0;
-        decode_tile(b, t, p, m0, n0);
-        const GemmProblem& P = b.prob[p];
+        const int slot = it % kTileRing;
+        if (!mbar_wait_cluster(smem_u32(&ctl->tile_full[slot]), (uint32_t)((it / kTileRing) & 1), wc, abort_flag))
+          break;
+        const int t = *reinterpret_cast<volatile int*>(&ctl->tile_id[slot]);
+        mbar_arrive_cluster(tile_empty_root + (uint32_t)slot * 8u);
+        if (t < 0) break;
+        int p, sm0, n0;
+        decode_tile<P>(b, t, p, sm0, n0);
+        const GemmProblem& Q = b.prob[p];
         const int acc = it & 1;
         const uint32_t acc_par = (uint32_t)((it >> 1) & 1);
-        if (!mbar_wait(smem_u32(&ctl->tempty[acc]), acc_par ^ 1u, wc, abort_flag)) {
-          ok = false;
-          break;
-        }
+        if (!mbar_wait_cluster(smem_u32(&ctl->tempty[acc]), acc_par ^ 1u, wc, abort_flag)) break;
         tc_fence_after();
         const uint32_t d_tmem = tmem_base + (uint32_t)(acc * kBN);
-        for (int kb = 0; kb < P.kb_total; ++kb) {
+        for (int kb = 0; kb < Q.kb_total; ++kb) {
           if (!mbar_wait(smem_u32(&ctl->full[stage]), phase, wc, abort_flag)) {
             ok = false;
             break;
           }
           tc_fence_after();
           const uint32_t a_addr = base + stage * kStageBytes;
-          const uint32_t b_addr = a_addr + kAStage;
-          const int nk = kb < P.kb_main ? kBK / 16 : min(kBK / 16, (P.r - (kb - P.kb_main) * kBK + 15) / 16);
+          const uint32_t b_addr = a_addr + kAHalf;
+          const int nk = kb < Q.kb_main ? kBK / 16 : min(kBK / 16, (Q.r - (kb - Q.kb_main) * kBK + 15) / 16);
           for (int k = 0; k < nk; ++k) {
             const uint64_t adesc = sw128_desc(a_addr + k * 32, 16, 1024);
-            const uint64_t bdesc = kBMn ? sw128_desc(b_addr + k * 2048, kMnChunk, 1024)
+            const uint64_t bdesc = kBMn ? sw128_desc(b_addr + k * 2048, kBox, 1024)
                                         : sw128_desc(b_addr + k * 32, 16, 1024);
-            umma_bf16(d_tmem, adesc, bdesc, idesc, (kb | k) != 0 ? 1u : 0u);
+            umma_bf16_pair(d_tmem, adesc, bdesc, idesc, (kb | k) != 0 ? 1u : 0u);
           }
-          issued_any = true;
-          umma_commit(smem_u32(&ctl->empty[stage]));
+          // the stage is free in every CTA once every pair has consumed it
+          umma_commit_pair_mc(smem_u32(&ctl->empty[stage]), all_mask);
           if (++stage == kStages) {
             stage = 0;
             phase ^= 1u;
           }
         }
         if (!ok) break;
-        umma_commit(smem_u32(&ctl->tfull[acc]));
+        umma_commit_pair_mc(smem_u32(&ctl->tfull[acc]), pair_mask);
       }
+      // completes in both CTAs of the pair once every MMA issued above has finished
+      umma_commit_pair_mc(smem_u32(&ctl->drain), pair_mask);
     }
   } else {
-    // ------------------------------------------------------------ epilogue
+    // ------------------------------------------------------------ epilogue (every CTA)
     const int q = warp & 3;  // TMEM lane quadrant this warp may access
+    const uint32_t tempty_pl = mapa_shared(smem_u32(&ctl->tempty[0]), pair_leader);
     for (int it = 0;; ++it) {
-      int t;
-      bool got = next_tile(ctl, it, wc, abort_flag, &t);
+      const int slot = it % kTileRing;
+      bool got = mbar_wait_cluster(smem_u32(&ctl->tile_full[slot]), (uint32_t)((it / kTileRing) & 1), wc, abort_flag);
       got = __all_sync(0xffffffffu, got);
-      if (!got || t < 0) break;
-      int p, m0, n0;
-      decode_tile(b, t, p, m0, n0);
-      const GemmProblem& P = b.prob[p];
+      if (!got) break;
+      const int t = *reinterpret_cast<volatile int*>(&ctl->tile_id[slot]);
+      __syncwarp();
+      if (lane == 0) mbar_arrive_cluster(tile_empty_root + (uint32_t)slot * 8u);
+      if (t < 0) break;
+      int p, sm0, n0;
+      decode_tile<P>(b, t, p, sm0, n0);
+      const GemmProblem& Q = b.prob[p];
       const int acc = it & 1;
       const uint32_t acc_par = (uint32_t)((it >> 1) & 1);
-      bool ok = mbar_wait(smem_u32(&ctl->tfull[acc]), acc_par, wc, abort_flag);
+      bool ok = mbar_wait_cluster(smem_u32(&ctl->tfull[acc]), acc_par, wc, abort_flag);
       ok = __all_sync(0xffffffffu, ok);
       if (!ok) break;
       tc_fence_after();
-      const int row = m0 + q * 32 + lane;
+      const int row = sm0 + pair * kBM + c * kHalf + q * 32 + lane;
       const uint32_t taddr = tmem_base + ((uint32_t)(q * 32) << 16) + (uint32_t)(acc * kBN);
-      __nv_bfloat16* orow = P.out + (size_t)row * P.ldo;
-      for (int c = 0; c < kBN; c += 32) {
-        if (n0 + c >= P.N) break;  // uniform across the warp
+      __nv_bfloat16* orow = Q.out + (size_t)row * Q.ldo;
+      for (int cc = 0; cc < kBN; cc += 32) {
+        if (n0 + cc >= Q.N) break;  // uniform across the warp
         uint32_t v[32];
-        tmem_ld_32x32b_x32(taddr + (uint32_t)c, v);
+        tmem_ld_32x32b_x32(taddr + (uint32_t)cc, v);
         tmem_ld_wait();
-        if (row < P.M) {
+        if (row < Q.M) {
 #pragma unroll
           for (int g = 0; g < 4; ++g) {
-            const int col = n0 + c + g * 8;
-            if (col < P.N) {
+            const int col = n0 + cc + g * 8;
+            if (col < Q.N) {
               uint4 pk;
               pk.x = pack_bf16x2(__uint_as_float(v[g * 8 + 0]), __uint_as_float(v[g * 8 + 1]));
               pk.y = pack_bf16x2(__uint_as_float(v[g * 8 + 2]), __uint_as_float(v[g * 8 + 3]));
@@ -269,53 +312,70 @@ __global__ void __launch_bounds__(kThreads, 1) fused_lora_gemm(const __grid_cons
         }
       }
       tc_fence_before();
-      mbar_arrive(smem_u32(&ctl->tempty[acc]));
+      __syncwarp();
+      if (lane == 0) mbar_arrive_cluster(tempty_pl + (uint32_t)acc * 8u);
     }
   }
 
+  // ------------------------------------------------------------ teardown
   tc_fence_before();
   __syncthreads();
-  if (*abort_flag) {
-    // A wait gave up somewhere in the CTA.  Before shared and tensor memory
-    // are released, let every copy and MMA this CTA issued complete.
-    if (warp == 0 && lane == 0) {
-      const long long first = issued > kStages ? issued - kStages : 0;
-      for (long long j = first; j < issued; ++j)
-        mbar_wait_drain(smem_u32(&ctl->full[j % kStages]), (uint32_t)((j / kStages) & 1), 1000000000ll);
+  if (threadIdx.x == 0) {
+    // every MMA of the pair has finished before tensor memory is released
+    if (!mbar_wait_drain(smem_u32(&ctl->drain), 0, b.limit_ns > kDrainNs ? b.limit_ns : kDrainNs))
+      atomicCAS(b.status, 0, kStatusTimeout);
+    if (*abort_flag) {
+      // a wait gave up: give copies still in flight time to land (bounded)
+      const uint64_t t0 = global_timer_ns();
+      while (global_timer_ns() - t0 < 50000ull) {
+      }
     }
-    if (warp == 1 && lane == 0 && issued_any) {
-      umma_commit(smem_u32(&ctl->drain));
-      mbar_wait_drain(smem_u32(&ctl->drain), 0, 1000000000ll);
-    }
-    tc_fence_before();
-    __syncthreads();
   }
+  __syncthreads();
+  cluster_sync_all();  // no cross-CTA access is pending in any CTA of the cluster
   if (warp == 1) {
     tc_fence_after();
-    tmem_dealloc(tmem_base, kTmemCols);
+    tmem_dealloc_pair(tmem_base, kTmemCols);
   }
+}
+
+template <bool kBMn, int P>
+cudaError_t launch_variant(const GemmBatch& batch, int num_sms, cudaStream_t stream) {
+  static bool attr_done = false;
+  if (!attr_done) {
+    cudaError_t e = cudaFuncSetAttribute(fused_lora_gemm<kBMn, P>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                         (int)kSmemBytes);
+    if (e != cudaSuccess) return e;
+    attr_done = true;
+  }
+  const int max_clusters = num_sms / (2 * P);
+  const int clusters = batch.total_tiles < max_clusters ? batch.total_tiles : max_clusters;
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = dim3((unsigned)(2 * P * clusters), 1, 1);
+  cfg.blockDim = dim3(kThreads, 1, 1);
+  cfg.dynamicSmemBytes = kSmemBytes;
+  cfg.stream = stream;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeClusterDimension;
+  attr[0].val.clusterDim.x = 2 * P;
+  attr[0].val.clusterDim.y = 1;
+  attr[0].val.clusterDim.z = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  cudaError_t e = cudaLaunchKernelEx(&cfg, fused_lora_gemm<kBMn, P>, batch);
+  note_launch();
+  return e;
 }
 
 }  // namespace
 
 size_t fused_gemm_smem_bytes() { return kSmemBytes; }
 
-cudaError_t launch_fused_gemm(const GemmBatch& batch, bool b_mn_major, int num_sms, cudaStream_t stream) {
-  static bool attr_done[2] = {false, false};
-  const void* fn = b_mn_major ? (const void*)fused_lora_gemm<true> : (const void*)fused_lora_gemm<false>;
-  if (!attr_done[b_mn_major]) {
-    cudaError_t e = cudaFuncSetAttribute(fn, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)kSmemBytes);
-    if (e != cudaSuccess) return e;
-    attr_done[b_mn_major] = true;
-  }
+cudaError_t launch_fused_gemm(const GemmBatch& batch, bool b_mn_major, int pairs, int num_sms, cudaStream_t stream) {
   if (batch.total_tiles <= 0) return cudaSuccess;
-  const int grid = batch.total_tiles < num_sms ? batch.total_tiles : num_sms;
-  if (b_mn_major)
-    fused_lora_gemm<true><<<grid, kThreads, kSmemBytes, stream>>>(batch);
-  else
-    fused_lora_gemm<false><<<grid, kThreads, kSmemBytes, stream>>>(batch);
-  note_launch();
-  return cudaGetLastError();
+  if (pairs == 2) return b_mn_major ? launch_variant<true, 2>(batch, num_sms, stream)
+                                    : launch_variant<false, 2>(batch, num_sms, stream);
+  return b_mn_major ? launch_variant<true, 1>(batch, num_sms, stream) : launch_variant<false, 1>(batch, num_sms, stream);
 }
 
 int gemm_tile_m() { return kBM; }

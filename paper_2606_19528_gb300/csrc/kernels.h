@@ -27,7 +27,7 @@ struct GemmProblem {
   int kb_main;         // contraction blocks of the base part
   int kb_total;        // base + adapter blocks
   int m_fast;          // 1: consecutive tiles walk M (the weight tile stays put)
-  int num_m_tiles;
+  int num_m_tiles;     // super-tiles (pairs x 256 rows) along M
 };
 
 // One launch: up to kMaxProblems independent fused contractions.
@@ -47,7 +47,9 @@ struct GemmBatch {
   long long limit_ns;
 };
 
-cudaError_t launch_fused_gemm(const GemmBatch& batch, bool b_mn_major, int num_sms, cudaStream_t stream);
+// pairs: CTA pairs per cluster (1, or 2 to share the weight tile between two
+// vertically adjacent tiles); tiles of the batch must have been counted for it.
+cudaError_t launch_fused_gemm(const GemmBatch& batch, bool b_mn_major, int pairs, int num_sms, cudaStream_t stream);
 size_t fused_gemm_smem_bytes();
 int gemm_tile_m();
 int gemm_tile_n();
