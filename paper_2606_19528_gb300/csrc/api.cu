@@ -182,6 +182,20 @@ Ws plan_ws(const lora_shape& s, int mode) {
   return w;
 }
 
+// Workspace of a call: [GEMM tile counters | rank-r partials | per-projection regions].
+// The rank-r arenas are sized for the projections without input sharing,
+// an upper bound of what grouped problems need (a group's padded rank is at
+// most the sum of its members').
+enum { kPhFwdRows = 0, kPhBwdRows = 1, kPhBwdCols = 2, kPhases = 3 };
+
+struct Plan {
+  std::vector<Ws> ws;
+  std::vector<size_t> offs;
+  size_t part_off[kPhases] = {0, 0, 0}, n_partials[kPhases] = {0, 0, 0};
+  size_t zero_bytes = 0;  // [0, zero_bytes) is cleared at the start of a call
+  size_t total = 0;
+};
+
 template <typename T>
 T* at(void* ws, size_t off) {
   return reinterpret_cast<T*>(static_cast<uint8_t*>(ws) + off);
@@ -199,24 +213,47 @@ struct Operands {
   int ld_b;
 };
 
+// Host description of a rank-r problem before its tensor maps are encoded.
+struct RowSpec {
+  const bf* X;
+  int ldx, T, C, nblk;
+  float scale;
+  const bf* W[kMaxRankBlocks];
+  int ldw[kMaxRankBlocks], rw[kMaxRankBlocks];
+  bf* out[kMaxRankBlocks];
+  int ld_out[kMaxRankBlocks];
+  bf* out2[kMaxRankBlocks];
+  int ld_out2[kMaxRankBlocks];
+};
+struct ColSpec {
+  const bf* X;
+  int ldx, T, C, nblk, out_cr;
+  const bf* S[kMaxRankBlocks];
+  int lds[kMaxRankBlocks], rs[kMaxRankBlocks];
+  float* out[kMaxRankBlocks];
+};
+
+inline int used_rank(const int* r, int n) {
+  int u = 0;
+  for (int k = 0; k < n; ++k) u += rank_pad8(r[k]);
+  return u;
+}
+
 // Appends block (W, ldw, rw) -> (out, out2) to the row problem of activation X,
 // opening a new problem when X differs or the concatenated rank would pass 128.
-void add_row_block(std::vector<RowProb>& probs, const bf* X, int ldx, int T, int C, float scale, const bf* W,
+void add_row_block(std::vector<RowSpec>& probs, const bf* X, int ldx, int T, int C, float scale, const bf* W,
                    int ldw, int rw, bf* out, int ld_out, bf* out2, int ld_out2, bool fuse) {
-  RowProb* p = nullptr;
+  RowSpec* p = nullptr;
   if (fuse) {
-    for (RowProb& q : probs) {
-      int used = 0;
-      for (int b = 0; b < q.nblk; ++b) used += rank_pad8(q.rw[b]);
+    for (RowSpec& q : probs)
       if (q.X == X && q.T == T && q.C == C && q.ldx == ldx && q.scale == scale && q.nblk < kMaxRankBlocks &&
-          used + rank_pad8(rw) <= 128) {
+          used_rank(q.rw, q.nblk) + rank_pad8(rw) <= 128) {
         p = &q;
         break;
       }
-    }
   }
   if (!p) {
-    RowProb q;
+    RowSpec q;
     memset(&q, 0, sizeof(q));
     q.X = X;
     q.ldx = ldx;
@@ -236,22 +273,19 @@ void add_row_block(std::vector<RowProb>& probs, const bf* X, int ldx, int T, int
   p->ld_out2[b] = ld_out2;
 }
 
-void add_col_block(std::vector<ColProb>& probs, const bf* X, int ldx, int T, int C, const bf* S, int lds, int rs,
+void add_col_block(std::vector<ColSpec>& probs, const bf* X, int ldx, int T, int C, const bf* S, int lds, int rs,
                    float* out, int out_cr, bool fuse) {
-  ColProb* p = nullptr;
+  ColSpec* p = nullptr;
   if (fuse) {
-    for (ColProb& q : probs) {
-      int used = 0;
-      for (int b = 0; b < q.nblk; ++b) used += rank_pad8(q.rs[b]);
+    for (ColSpec& q : probs)
       if (q.X == X && q.T == T && q.C == C && q.ldx == ldx && q.out_cr == out_cr && q.nblk < kMaxRankBlocks &&
-          used + rank_pad8(rs) <= 128) {
+          used_rank(q.rs, q.nblk) + rank_pad8(rs) <= 128) {
         p = &q;
         break;
       }
-    }
   }
   if (!p) {
-    ColProb q;
+    ColSpec q;
     memset(&q, 0, sizeof(q));
     q.X = X;
     q.ldx = ldx;
@@ -268,73 +302,177 @@ void add_col_block(std::vector<ColProb>& probs, const bf* X, int ldx, int T, int
   p->out[b] = out;
 }
 
-int launch_rows(std::vector<RowProb>& probs, bool w_rc, int num_sms, cudaStream_t st) {
+// fp32 partials of one rank-r phase.
+struct Arena {
+  float* partials;
+  size_t n_partials;
+};
+
+constexpr int kMinUnitChunks = 8;  // smallest work unit (64-wide chunks); sizes the partial arenas
+
+// Chunks per unit for a launch.  The persistent grid (two CTAs per SM) takes
+// units round-robin, so the launch lasts about ceil(units / CTAs) units; the
+// cost of a size is that makespan in chunks, plus a fixed charge for the
+// partial-sum pass when any tile needs several units.  Ties go to the larger
+// unit (fewer partials).
+template <typename Spec, typename LenFn>
+int choose_unit_chunks(const std::vector<Spec>& specs, size_t i0, size_t i1, int num_sms, LenFn len) {
+  int best = kMinUnitChunks;
+  long long best_cost = -1;
+  for (int u : {64, 32, 16, 8}) {
+    long long units = 0;
+    bool partials = false;
+    for (size_t i = i0; i < i1; ++i) {
+      const auto tl = len(specs[i]);  // (tiles, reduction length)
+      const long long upt = cdiv(cdiv(tl.second, 64), u);
+      units += (long long)tl.first * upt;
+      partials = partials || upt > 1;
+    }
+    const long long ctas = std::min<long long>(units, 2LL * num_sms);
+    const long long cost = (units + ctas - 1) / ctas * u + (partials ? 4 : 0);
+    if (best_cost < 0 || cost < best_cost) {
+      best_cost = cost;
+      best = u;
+    }
+  }
+  return best;
+}
+
+// 2-D bf16 tensor map without swizzle (rank-side tiles).
+int make_map_plain(CUtensorMap* m, const void* ptr, uint64_t inner, uint64_t outer, uint64_t ld, uint32_t box_inner,
+                   uint32_t box_outer) {
+  cuuint64_t dims[2] = {inner, outer};
+  cuuint64_t strides[1] = {ld * 2};
+  cuuint32_t box[2] = {box_inner, box_outer};
+  cuuint32_t estr[2] = {1, 1};
+  CUresult r = g_encode(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void*>(ptr), dims, strides, box, estr,
+                        CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_NONE,
+                        CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+  return r == CUDA_SUCCESS ? LORA_OK : LORA_ECUDA;
+}
+
+int launch_rows(const std::vector<RowSpec>& specs, bool w_rc, const Arena& ar, const DeviceInfo* d,
+                cudaStream_t st) {
   const int tile = rank_tile();
-  for (size_t i0 = 0; i0 < probs.size(); i0 += kMaxRankProblems) {
+  size_t pf = 0;
+  int rc;
+  for (size_t i0 = 0; i0 < specs.size(); i0 += kMaxRankProblems) {
+    const size_t i1 = std::min(specs.size(), i0 + kMaxRankProblems);
     RowBatch b;
     memset(&b, 0, sizeof(b));
-    int rmax = 16, max_chunks = 1;
-    for (size_t i = i0; i < probs.size() && i < i0 + kMaxRankProblems; ++i) {
-      RowProb& p = probs[i];
-      int used = 0;
-      for (int k = 0; k < p.nblk; ++k) used += rank_pad8(p.rw[k]);
-      p.rpad = rank_pad16(used);
+    // (tiles, reduction length) of a row problem
+    b.unit_chunks = choose_unit_chunks(specs, i0, i1, d->num_sms, [&](const RowSpec& q) {
+      return std::make_pair(cdiv(q.T, tile), q.C);
+    });
+    int rmax = 16;
+    for (size_t i = i0; i < i1; ++i) {
+      const RowSpec& sp = specs[i];
+      RowProb& p = b.p[b.n++];
+      p.T = sp.T;
+      p.C = sp.C;
+      p.nblk = sp.nblk;
+      p.scale = sp.scale;
+      if ((rc = make_map(&p.tmX, sp.X, sp.C, sp.T, sp.ldx, 64, 64)) != LORA_OK) return rc;
+      int bytes = 64 * 64 * 2;
+      for (int k = 0; k < sp.nblk; ++k) {
+        p.rw[k] = sp.rw[k];
+        p.out[k] = sp.out[k];
+        p.ld_out[k] = sp.ld_out[k];
+        p.out2[k] = sp.out2[k];
+        p.ld_out2[k] = sp.ld_out2[k];
+        const int r8 = rank_pad8(sp.rw[k]);
+        if (w_rc)  // A_b [r_b, C]: 64 columns x r8 rows, rows past r_b zero-filled
+          rc = make_map(&p.tmW[k], sp.W[k], sp.C, sp.rw[k], sp.ldw[k], 64, r8);
+        else       // B [C, r] (row stride ldw, a multiple of 8): r8 entries x 64 rows
+          rc = make_map_plain(&p.tmW[k], sp.W[k], r8, sp.C, sp.ldw[k], r8, 64);
+        if (rc != LORA_OK) return rc;
+        bytes += 64 * r8 * 2;
+      }
+      p.tx_bytes = bytes;
+      p.rpad = rank_pad16(used_rank(sp.rw, sp.nblk));
       rmax = std::max(rmax, p.rpad);
-      max_chunks = std::max(max_chunks, cdiv(p.C, tile));
-      p.tile_begin = b.tiles;
-      b.tiles += cdiv(p.T, tile);
-      b.p[b.n++] = p;
+      const int tiles = cdiv(p.T, tile);
+      p.upt = cdiv(cdiv(p.C, tile), b.unit_chunks);
+      p.unit_begin = b.units;
+      b.units += tiles * p.upt;
+      p.part_off = (long long)pf;
+      p.red_begin = b.red_total;
+      if (p.upt > 1) {
+        pf += (size_t)tiles * p.upt * tile * p.rpad;
+        b.red_total += tiles * tile * p.rpad;
+      }
     }
-    b.splits = rank_splits(b.tiles, max_chunks, num_sms);
+    if (pf > ar.n_partials) return LORA_EWORKSPACE;  // planning bound violated
     b.w_rc = w_rc ? 1 : 0;
-    for (int i = 0; i < b.n; ++i) b.p[i].cps = cdiv(cdiv(b.p[i].C, tile), b.splits);
-    if (launch_rowprod(b, rmax, st) != cudaSuccess) return LORA_ECUDA;
+    b.partials = ar.partials;
+    b.status = d->status;
+    b.limit_ns = g_wait_limit_ns;
+    if (launch_rowprod(b, rmax, d->num_sms, st) != cudaSuccess) return LORA_ECUDA;
   }
   return LORA_OK;
 }
 
-int launch_cols(std::vector<ColProb>& probs, int num_sms, cudaStream_t st) {
+int launch_cols(const std::vector<ColSpec>& specs, const Arena& ar, const DeviceInfo* d, cudaStream_t st) {
   const int tile = rank_tile();
-  for (size_t i0 = 0; i0 < probs.size(); i0 += kMaxRankProblems) {
+  size_t pf = 0;
+  int rc;
+  for (size_t i0 = 0; i0 < specs.size(); i0 += kMaxRankProblems) {
+    const size_t i1 = std::min(specs.size(), i0 + kMaxRankProblems);
     ColBatch b;
     memset(&b, 0, sizeof(b));
-    int rmax = 16, max_chunks = 1;
-    for (size_t i = i0; i < probs.size() && i < i0 + kMaxRankProblems; ++i) {
-      ColProb& p = probs[i];
-      int used = 0;
-      for (int k = 0; k < p.nblk; ++k) used += rank_pad8(p.rs[k]);
-      p.rpad = rank_pad16(used);
+    b.unit_chunks = choose_unit_chunks(specs, i0, i1, d->num_sms, [&](const ColSpec& q) {
+      return std::make_pair(cdiv(q.C, tile), q.T);
+    });
+    int rmax = 16;
+    for (size_t i = i0; i < i1; ++i) {
+      const ColSpec& sp = specs[i];
+      ColProb& p = b.p[b.n++];
+      p.T = sp.T;
+      p.C = sp.C;
+      p.nblk = sp.nblk;
+      p.out_cr = sp.out_cr;
+      if ((rc = make_map(&p.tmX, sp.X, sp.C, sp.T, sp.ldx, 64, 64)) != LORA_OK) return rc;
+      int bytes = 64 * 64 * 2;
+      for (int k = 0; k < sp.nblk; ++k) {
+        p.rs[k] = sp.rs[k];
+        p.out[k] = sp.out[k];
+        const int r8 = rank_pad8(sp.rs[k]);
+        if ((rc = make_map_plain(&p.tmS[k], sp.S[k], r8, sp.T, sp.lds[k], r8, 64)) != LORA_OK) return rc;
+        bytes += 64 * r8 * 2;
+      }
+      p.tx_bytes = bytes;
+      p.rpad = rank_pad16(used_rank(sp.rs, sp.nblk));
       rmax = std::max(rmax, p.rpad);
-      max_chunks = std::max(max_chunks, cdiv(p.T, tile));
-      p.tile_begin = b.tiles;
-      b.tiles += cdiv(p.C, tile);
-      b.p[b.n++] = p;
+      const int tiles = cdiv(p.C, tile);
+      p.upt = cdiv(cdiv(p.T, tile), b.unit_chunks);
+      p.unit_begin = b.units;
+      b.units += tiles * p.upt;
+      p.part_off = (long long)pf;
+      p.red_begin = b.red_total;
+      if (p.upt > 1) {
+        pf += (size_t)tiles * p.upt * tile * p.rpad;
+        b.red_total += tiles * tile * p.rpad;
+      }
     }
-    b.splits = rank_splits(b.tiles, max_chunks, num_sms);
-    for (int i = 0; i < b.n; ++i) b.p[i].cps = cdiv(cdiv(b.p[i].T, tile), b.splits);
-    if (launch_colprod(b, rmax, st) != cudaSuccess) return LORA_ECUDA;
+    if (pf > ar.n_partials) return LORA_EWORKSPACE;
+    b.partials = ar.partials;
+    b.status = d->status;
+    b.limit_ns = g_wait_limit_ns;
+    if (launch_colprod(b, rmax, d->num_sms, st) != cudaSuccess) return LORA_ECUDA;
   }
   return LORA_OK;
 }
 
-// ------------------------------------------------------------------ forward
-// CTA pairs per cluster for a batch of fused contractions over tokens T_i:
-// two pairs (weight tile shared) unless stacking 512 rows would waste work.
-int choose_pairs(const std::vector<int64_t>& Ts) {
-  for (int64_t T : Ts) {
-    const int64_t rows1 = (T + 255) / 256 * 256, rows2 = (T + 511) / 512 * 512;
-    if (rows2 * 100 > rows1 * 107) return 1;
-  }
-  return 2;
-}
+Arena arena(void* ws, const Plan& pl, int phase) { return Arena{at<float>(ws, pl.part_off[phase]), pl.n_partials[phase]}; }
 
-int add_fwd_problem(GemmBatch& b, const lora_proj& p, const Operands& o, int pairs) {
+// ------------------------------------------------------------------ forward
+int add_fwd_problem(GemmBatch& b, const lora_proj& p, const Operands& o) {
   const lora_shape& s = p.shape;
   const int i = b.num_problems;
   const int64_t T = s.T, K = s.d_in, N = s.d_out, r = s.rank;
   int rc;
   // activation boxes: one CTA's 128 rows x 64 contraction elements; weight
-  // boxes: 64 rows x 64 (two per CTA, shared between the pairs of a cluster)
+  // boxes: 64 rows x 64 (two per CTA)
   if ((rc = make_map(&b.tmA[i], p.x, K, T, K, 64, 128)) != LORA_OK) return rc;
   if ((rc = make_map(&b.tmA2[i], o.s_in, r, T, o.ld_s, 64, 128)) != LORA_OK) return rc;
   if ((rc = make_map(&b.tmB[i], p.W, K, N, K, 64, 64)) != LORA_OK) return rc;
@@ -347,7 +485,7 @@ int add_fwd_problem(GemmBatch& b, const lora_proj& p, const Operands& o, int pai
   g.Kmain = (int)K;
   g.r = (int)r;
   g.num_n_tiles = cdiv(N, gemm_tile_n());
-  g.num_m_tiles = cdiv(T, (int64_t)gemm_tile_m() * pairs);
+  g.num_m_tiles = cdiv(T, gemm_tile_m());
   g.m_fast = N >= T ? 1 : 0;  // weight operand [N, K] at least as large as x [T, K]
   g.kb_main = cdiv(K, gemm_tile_k());
   g.kb_total = g.kb_main + cdiv(r, gemm_tile_k());
@@ -358,7 +496,7 @@ int add_fwd_problem(GemmBatch& b, const lora_proj& p, const Operands& o, int pai
 }
 
 // ------------------------------------------------------------------ backward
-int add_bwd_problem(GemmBatch& b, const lora_proj& p, const Operands& o, int pairs) {
+int add_bwd_problem(GemmBatch& b, const lora_proj& p, const Operands& o) {
   const lora_shape& s = p.shape;
   const int i = b.num_problems;
   const int64_t T = s.T, K = s.d_in, N = s.d_out, r = s.rank;
@@ -376,7 +514,7 @@ int add_bwd_problem(GemmBatch& b, const lora_proj& p, const Operands& o, int pai
   g.Kmain = (int)N;
   g.r = (int)r;
   g.num_n_tiles = cdiv(K, gemm_tile_n());
-  g.num_m_tiles = cdiv(T, (int64_t)gemm_tile_m() * pairs);
+  g.num_m_tiles = cdiv(T, gemm_tile_m());
   g.m_fast = K >= T ? 1 : 0;  // weight operand [N, K] at least as large as dy [T, N]
   g.kb_main = cdiv(N, gemm_tile_k());
   g.kb_total = g.kb_main + cdiv(r, gemm_tile_k());
@@ -416,17 +554,17 @@ int check_ws(void* ws, size_t ws_bytes, size_t need) {
 }
 
 // Runs the given projections in `mode`; every argument already validated.
-int run_step(const lora_proj* projs, int n, int mode, void* ws, const std::vector<Ws>& plans,
-             const std::vector<size_t>& offs, DeviceInfo* d, cudaStream_t st) {
+int run_step(const lora_proj* projs, int n, int mode, void* ws, const Plan& pl, DeviceInfo* d, cudaStream_t st) {
   int rc;
-  auto W_ = [&](int i) { return at<uint8_t>(ws, offs[i]); };
-  // tile counters of the fused-GEMM launches live in the workspace header
+  const std::vector<Ws>& plans = pl.ws;
+  auto W_ = [&](int i) { return at<uint8_t>(ws, pl.offs[i]); };
+  // tile counters of the fused-GEMM launches
   int* counters = at<int>(ws, 0);
   int next_counter = 0;
-  if (cudaMemsetAsync(counters, 0, kWsHeader, st) != cudaSuccess) return LORA_ECUDA;
+  if (cudaMemsetAsync(ws, 0, pl.zero_bytes, st) != cudaSuccess) return LORA_ECUDA;
   if (mode & LORA_FWD) {
     std::vector<Operands> ops(n);
-    std::vector<RowProb> rows;
+    std::vector<RowSpec> rows;
     {
       ProfScope ps(LORA_KERNEL_PAD, st);
       for (int i = 0; i < n; ++i) {
@@ -453,7 +591,7 @@ int run_step(const lora_proj* projs, int n, int mode, void* ws, const std::vecto
     }
     {
       ProfScope ps(LORA_KERNEL_ROWPROJ, st);
-      if ((rc = launch_rows(rows, true, d->num_sms, st)) != LORA_OK) return rc;
+      if ((rc = launch_rows(rows, true, arena(ws, pl, kPhFwdRows), d, st)) != LORA_OK) return rc;
     }
     // heavier problems first so that the static tile walk ends balanced
     std::vector<int> order(n);
@@ -464,19 +602,16 @@ int run_step(const lora_proj* projs, int n, int mode, void* ws, const std::vecto
       GemmBatch b;
       init_batch(b, d);
       b.tile_counter = counters + next_counter++;
-      std::vector<int64_t> Ts;
-      for (int i = i0; i < n && i < i0 + kMaxProblems; ++i) Ts.push_back(projs[order[i]].shape.T);
-      const int pairs = choose_pairs(Ts);
       for (int i = i0; i < n && i < i0 + kMaxProblems; ++i)
-        if ((rc = add_fwd_problem(b, projs[order[i]], ops[order[i]], pairs)) != LORA_OK) return rc;
+        if ((rc = add_fwd_problem(b, projs[order[i]], ops[order[i]])) != LORA_OK) return rc;
       ProfScope ps(LORA_KERNEL_GEMM_FWD, st);
-      if (launch_fused_gemm(b, false, pairs, d->num_sms, st) != cudaSuccess) return LORA_ECUDA;
+      if (launch_fused_gemm(b, false, d->num_sms, st) != cudaSuccess) return LORA_ECUDA;
     }
   }
   if (mode & LORA_BWD) {
     std::vector<Operands> ops(n);
-    std::vector<RowProb> rows;
-    std::vector<ColProb> cols;
+    std::vector<RowSpec> rows;
+    std::vector<ColSpec> cols;
     std::vector<const bf*> su_in(n);
     std::vector<int> ld_su(n);
     {
@@ -506,7 +641,7 @@ int run_step(const lora_proj* projs, int n, int mode, void* ws, const std::vecto
     }
     {
       ProfScope ps(LORA_KERNEL_ROWPROJ, st);
-      if ((rc = launch_rows(rows, false, d->num_sms, st)) != LORA_OK) return rc;
+      if ((rc = launch_rows(rows, false, arena(ws, pl, kPhBwdRows), d, st)) != LORA_OK) return rc;
     }
     for (int i = 0; i < n; ++i) {
       const lora_proj& p = projs[i];
@@ -520,7 +655,7 @@ int run_step(const lora_proj* projs, int n, int mode, void* ws, const std::vecto
     }
     {
       ProfScope ps(LORA_KERNEL_COLPROJ, st);
-      if ((rc = launch_cols(cols, d->num_sms, st)) != LORA_OK) return rc;
+      if ((rc = launch_cols(cols, arena(ws, pl, kPhBwdCols), d, st)) != LORA_OK) return rc;
     }
     std::vector<int> order;
     for (int i = 0; i < n; ++i)
@@ -531,31 +666,47 @@ int run_step(const lora_proj* projs, int n, int mode, void* ws, const std::vecto
       GemmBatch b;
       init_batch(b, d);
       b.tile_counter = counters + next_counter++;
-      std::vector<int64_t> Ts;
-      for (size_t i = i0; i < order.size() && i < i0 + kMaxProblems; ++i) Ts.push_back(projs[order[i]].shape.T);
-      const int pairs = choose_pairs(Ts);
       for (size_t i = i0; i < order.size() && i < i0 + kMaxProblems; ++i)
-        if ((rc = add_bwd_problem(b, projs[order[i]], ops[order[i]], pairs)) != LORA_OK) return rc;
+        if ((rc = add_bwd_problem(b, projs[order[i]], ops[order[i]])) != LORA_OK) return rc;
       ProfScope ps(LORA_KERNEL_GEMM_BWD, st);
-      if (launch_fused_gemm(b, true, pairs, d->num_sms, st) != cudaSuccess) return LORA_ECUDA;
+      if (launch_fused_gemm(b, true, d->num_sms, st) != cudaSuccess) return LORA_ECUDA;
     }
   }
   return LORA_OK;
 }
 
-int plan_all(const lora_proj* projs, int n, int mode, int num_sms, std::vector<Ws>* plans,
-             std::vector<size_t>* offs, size_t* total) {
-  size_t off = kWsHeader;
-  plans->resize(n);
-  offs->resize(n);
+int plan_all(const lora_proj* projs, int n, int mode, Plan* pl) {
+  const int tile = rank_tile();
+  // partials are bounded by the smallest unit size (most units per tile)
+  auto upt = [&](int64_t len) { return (size_t)cdiv(cdiv(len, tile), kMinUnitChunks); };
+  auto tiles = [&](int64_t len) { return (size_t)cdiv(len, tile); };
   for (int i = 0; i < n; ++i) {
     int rc = check_shape(&projs[i].shape);
     if (rc != LORA_OK) return rc;
-    (*plans)[i] = plan_ws(projs[i].shape, mode);
-    (*offs)[i] = off;
-    off += up256((*plans)[i].total);
+    const lora_shape& s = projs[i].shape;
+    const size_t r16 = (size_t)rank_pad16((int)s.rank);
+    if (mode & LORA_FWD) {
+      if (upt(s.d_in) > 1) pl->n_partials[kPhFwdRows] += tiles(s.T) * upt(s.d_in) * tile * r16;
+    }
+    if (mode & LORA_BWD) {
+      if (upt(s.d_out) > 1) pl->n_partials[kPhBwdRows] += tiles(s.T) * upt(s.d_out) * tile * r16;
+      if (upt(s.T) > 1) pl->n_partials[kPhBwdCols] += (tiles(s.d_out) + tiles(s.d_in)) * upt(s.T) * tile * r16;
+    }
   }
-  *total = off;
+  size_t off = kWsHeader;
+  pl->zero_bytes = kWsHeader;
+  for (int k = 0; k < kPhases; ++k) {
+    pl->part_off[k] = off;
+    off += up256(pl->n_partials[k] * sizeof(float));
+  }
+  pl->ws.resize(n);
+  pl->offs.resize(n);
+  for (int i = 0; i < n; ++i) {
+    pl->ws[i] = plan_ws(projs[i].shape, mode);
+    pl->offs[i] = off;
+    off += up256(pl->ws[i].total);
+  }
+  pl->total = off;
   return LORA_OK;
 }
 
@@ -603,12 +754,11 @@ int lora_workspace_size(const lora_shape* shape, int mode, size_t* bytes) {
 int lora_stack_workspace_size(const lora_proj* projs, int n_proj, int mode, size_t* bytes) {
   if (!projs || !bytes) return LORA_ENULL;
   if (n_proj < 1 || n_proj > 64 || mode < LORA_FWD || mode > LORA_FWD_BWD) return LORA_EINVAL;
-  DeviceInfo* d = nullptr;
-  int rc = device_info(&d);
+  Plan pl;
+  int rc = plan_all(projs, n_proj, mode, &pl);
   if (rc != LORA_OK) return rc;
-  std::vector<Ws> plans;
-  std::vector<size_t> offs;
-  return plan_all(projs, n_proj, mode, d->num_sms, &plans, &offs, bytes);
+  *bytes = pl.total;
+  return LORA_OK;
 }
 
 int lora_stack_step(const lora_proj* projs, int n_proj, int mode, void* workspace, size_t workspace_bytes,
@@ -618,17 +768,16 @@ int lora_stack_step(const lora_proj* projs, int n_proj, int mode, void* workspac
   DeviceInfo* d = nullptr;
   int rc = device_info(&d);
   if (rc != LORA_OK) return rc;
-  std::vector<Ws> plans;
-  std::vector<size_t> offs;
-  size_t need = 0;
-  if ((rc = plan_all(projs, n_proj, mode, d->num_sms, &plans, &offs, &need)) != LORA_OK) return rc;
+  Plan pl;
+  if ((rc = plan_all(projs, n_proj, mode, &pl)) != LORA_OK) return rc;
+  const size_t need = pl.total;
   for (int i = 0; i < n_proj; ++i) {
     if ((mode & LORA_FWD) && (rc = check_fwd_ptrs(projs[i])) != LORA_OK) return rc;
     if ((mode & LORA_BWD) && (rc = check_bwd_ptrs(projs[i])) != LORA_OK) return rc;
     if (mode == LORA_FWD_BWD && !projs[i].su) return LORA_ENULL;  // the backward needs the saved su
   }
   if ((rc = check_ws(workspace, workspace_bytes, need)) != LORA_OK) return rc;
-  return run_step(projs, n_proj, mode, workspace, plans, offs, d, static_cast<cudaStream_t>(stream));
+  return run_step(projs, n_proj, mode, workspace, pl, d, static_cast<cudaStream_t>(stream));
 }
 
 int lora_linear_fwd(const lora_shape* shape, const lora_bf16* x, const lora_bf16* W, const lora_bf16* A,

@@ -13,24 +13,19 @@
 // the second operand W [N, K] is contracted over its rows, i.e. it is read
 // MN-major straight from the frozen weight (no transposed copy of W).
 //
-// Structure: persistent clusters of P CTA pairs (P = 1 or 2; one CTA per SM)
-// take "super-tiles" of P vertically adjacent 256 x 256 output tiles from a
-// tile list spanning every problem of a batch (up to kMaxProblems
-// projections, heavier first) through a global atomic counter, so that tiles
-// of unequal depth balance across SMs.  Each 256 x 256 tile is one 2-CTA
-// tensor-core contraction (tcgen05 cta_group::2, M = 256, N = 256, K = 16
-// per instruction): each CTA of a pair stages its own 128 rows of the
-// activation operand and its own 128 columns of the weight operand, and
-// holds its 128 x 256 half of the fp32 accumulator in its own tensor memory.
-// With P = 2 the two pairs share the weight tile: each CTA loads half of its
-// weight half and multicasts it to its counterpart in the other pair, so
-// L2-to-SM traffic drops by a quarter (the operand feed, not the tensor
-// pipe, bounds a single pair).  Within a problem, consecutive super-tiles
-// walk M when the weight operand is the larger one, so each weight tile is
-// read from DRAM once.
-//   warp 0      tile scheduler (cluster rank 0) and TMA producer (every CTA):
+// Structure: persistent CTA pairs (thread-block clusters of 2, one CTA per
+// SM) take 256 x 256 output tiles from a tile list spanning every problem of
+// a batch (up to kMaxProblems projections, heavier first) through a global
+// atomic counter, so that tiles of unequal depth balance across SMs.  Each
+// tile is one 2-CTA tensor-core contraction (tcgen05 cta_group::2, M = 256,
+// N = 256, K = 16 per instruction): each CTA of the pair stages its own 128
+// rows of the activation operand and its own 128 columns of the weight
+// operand, and holds its 128 x 256 half of the fp32 accumulator in its own
+// tensor memory.  Within a problem, consecutive tiles walk M when the weight
+// operand is the larger one, so each weight tile is read from DRAM once.
+//   warp 0      tile scheduler (even CTA) and TMA producer (both CTAs):
 //               6-stage shared-memory ring of 32 KB, 128-byte swizzle
-//   warp 1      TMEM allocation (every CTA); tcgen05.mma issuer (even CTAs)
+//   warp 1      TMEM allocation (both CTAs); tcgen05.mma issuer (even CTA)
 //   warps 2..5  epilogue: TMEM -> registers -> bf16 -> global
 // Two 256-column fp32 accumulators per CTA (512 TMEM columns) let the
 // epilogue of one tile overlap the main loop of the next.  Every wait is
@@ -58,13 +53,13 @@ constexpr int kTileRing = 4;  // tile ids handed from the scheduler to the other
 constexpr long long kDrainNs = 1000000000ll;
 
 struct __align__(8) Ctl {
-  uint64_t full[kStages];          // even CTAs: both CTAs' halves of a stage landed
-  uint64_t empty[kStages];         // every CTA: every pair's MMAs finished reading a stage
-  uint64_t tfull[2];               // every CTA: accumulator complete
-  uint64_t tempty[2];              // even CTAs: the pair's epilogues drained an accumulator
-  uint64_t tile_full[kTileRing];   // every CTA: tile id written
-  uint64_t tile_empty[kTileRing];  // cluster rank 0: every consumer of the cluster read the slot
-  uint64_t drain;                  // every CTA: every MMA of its pair completed
+  uint64_t full[kStages];          // even CTA: both CTAs' halves of a stage landed
+  uint64_t empty[kStages];         // both CTAs: the pair's MMAs finished reading a stage
+  uint64_t tfull[2];               // both CTAs: accumulator complete
+  uint64_t tempty[2];              // even CTA: both CTAs' epilogues drained an accumulator
+  uint64_t tile_full[kTileRing];   // both CTAs: tile id written
+  uint64_t tile_empty[kTileRing];  // even CTA: every consumer of both CTAs read the slot
+  uint64_t drain;                  // both CTAs: every MMA of the pair completed
   int tile_id[kTileRing];
   uint32_t tmem_base;
   int abort;
@@ -72,25 +67,23 @@ struct __align__(8) Ctl {
 
 constexpr size_t kSmemBytes = 1024 + (size_t)kStages * kStageBytes + sizeof(Ctl);
 
-// Problem p, first row m0 of the super-tile (P tiles stacked along M) and column n0.
-template <int P>
+// Problem p, first row m0 and first column n0 of tile t.
 __device__ __forceinline__ void decode_tile(const GemmBatch& b, int t, int& p, int& m0, int& n0) {
   p = 0;
   while (p + 1 < b.num_problems && t >= b.prob[p + 1].tile_begin) ++p;
   const GemmProblem& Q = b.prob[p];
   const int local = t - Q.tile_begin;
   if (Q.m_fast) {
-    m0 = (local % Q.num_m_tiles) * kBM * P;
+    m0 = (local % Q.num_m_tiles) * kBM;
     n0 = (local / Q.num_m_tiles) * kBN;
   } else {
-    m0 = (local / Q.num_n_tiles) * kBM * P;
+    m0 = (local / Q.num_n_tiles) * kBM;
     n0 = (local % Q.num_n_tiles) * kBN;
   }
 }
 
-template <bool kBMn, int P>
+template <bool kBMn>
 __global__ void __launch_bounds__(kThreads, 1) fused_lora_gemm(const __grid_constant__ GemmBatch b) {
-  constexpr int C = 2 * P;  // CTAs per cluster
   extern __shared__ uint8_t smem_raw[];
   const uint32_t raw = smem_u32(smem_raw);
   const uint32_t base = (raw + 1023u) & ~1023u;
@@ -99,16 +92,13 @@ __global__ void __launch_bounds__(kThreads, 1) fused_lora_gemm(const __grid_cons
 
   const int warp = threadIdx.x >> 5;
   const int lane = threadIdx.x & 31;
-  const int rank = (int)cluster_ctarank();
-  const int pair = rank >> 1;       // which pair of the cluster
-  const int c = rank & 1;           // position within the pair
-  const uint32_t pair_leader = (uint32_t)(rank & ~1);
+  const int c = (int)cluster_ctarank();  // position within the pair (0: issues the MMAs)
   const WaitCtl wc{b.status, b.limit_ns};
 
   if (threadIdx.x == 0) {
     for (int s = 0; s < kStages; ++s) {
       mbar_init(smem_u32(&ctl->full[s]), 1);
-      mbar_init(smem_u32(&ctl->empty[s]), P);  // one commit from every pair
+      mbar_init(smem_u32(&ctl->empty[s]), 1);
     }
     for (int a = 0; a < 2; ++a) {
       mbar_init(smem_u32(&ctl->tfull[a]), 1);
@@ -116,8 +106,8 @@ __global__ void __launch_bounds__(kThreads, 1) fused_lora_gemm(const __grid_cons
     }
     for (int k = 0; k < kTileRing; ++k) {
       mbar_init(smem_u32(&ctl->tile_full[k]), 1);
-      // MMA threads of the pairs, epilogue warps of every CTA, producers of the other CTAs
-      mbar_init(smem_u32(&ctl->tile_empty[k]), P + C * kEpiWarps + (C - 1));
+      // MMA thread, epilogue warps of both CTAs, producer of the odd CTA
+      mbar_init(smem_u32(&ctl->tile_empty[k]), 2 + 2 * kEpiWarps);
     }
     mbar_init(smem_u32(&ctl->drain), 1);
     ctl->abort = 0;
@@ -138,39 +128,37 @@ __global__ void __launch_bounds__(kThreads, 1) fused_lora_gemm(const __grid_cons
   tc_fence_before();
   __syncthreads();
   tc_fence_after();
-  cluster_sync_all();  // every CTA's barriers exist before any cross-CTA arrival
+  cluster_sync_all();  // both CTAs' barriers exist before any cross-CTA arrival
   const uint32_t tmem_base = ctl->tmem_base;
   const uint32_t tile_empty_root = mapa_shared(smem_u32(&ctl->tile_empty[0]), 0);
 
   if (warp == 0) {
     // ------------------------------------------------------------ scheduler + producer
     if (lane == 0) {
-      const uint32_t full_pl = mapa_shared(smem_u32(&ctl->full[0]), pair_leader);
-      const uint16_t b_mask = (uint16_t)((1u << c) | (1u << (c + 2)));  // my position in both pairs
+      const uint32_t full_pl = mapa_shared(smem_u32(&ctl->full[0]), 0);
       int stage = 0;
       uint32_t phase = 0;
       for (int it = 0;; ++it) {
         const int slot = it % kTileRing;
         const uint32_t par = (uint32_t)((it / kTileRing) & 1);
         int t;
-        if (rank == 0) {
+        if (c == 0) {
           if (!mbar_wait_cluster(smem_u32(&ctl->tile_empty[slot]), par ^ 1u, wc, abort_flag)) break;
           t = atomicAdd(b.tile_counter, 1);
           if (t >= b.total_tiles) t = -1;
           ctl->tile_id[slot] = t;
-          for (int r = 1; r < C; ++r) st_cluster_u32(mapa_shared(smem_u32(&ctl->tile_id[slot]), r), (uint32_t)t);
+          st_cluster_u32(mapa_shared(smem_u32(&ctl->tile_id[slot]), 1), (uint32_t)t);
           mbar_arrive(smem_u32(&ctl->tile_full[slot]));
-          for (int r = 1; r < C; ++r) mbar_arrive_cluster(mapa_shared(smem_u32(&ctl->tile_full[slot]), r));
+          mbar_arrive_cluster(mapa_shared(smem_u32(&ctl->tile_full[slot]), 1));
         } else {
           if (!mbar_wait_cluster(smem_u32(&ctl->tile_full[slot]), par, wc, abort_flag)) break;
           t = *reinterpret_cast<volatile int*>(&ctl->tile_id[slot]);
           mbar_arrive_cluster(tile_empty_root + (uint32_t)slot * 8u);
         }
         if (t < 0) break;
-        int p, sm0, n0;
-        decode_tile<P>(b, t, p, sm0, n0);
+        int p, m0, n0;
+        decode_tile(b, t, p, m0, n0);
         const GemmProblem& Q = b.prob[p];
-        const int m0 = sm0 + pair * kBM;
         const int my_m = m0 + c * kHalf;
         const bool a_mine = my_m < Q.M;
         // weight boxes of pair position c' hold columns n0 + 128 c' + 64 j, j = 0, 1
@@ -196,15 +184,9 @@ __global__ void __launch_bounds__(kThreads, 1) fused_lora_gemm(const __grid_cons
           if (a_mine) tma_load_2d_pair(a_dst, ta, bar, kc, my_m);
 #pragma unroll
           for (int j = 0; j < 2; ++j) {
-            if (P == 2 && j != pair) continue;  // the other pair's CTA loads (and multicasts) box j
             if (!box_ok(c, j)) continue;
             const int col = n0 + c * kHalf + j * 64;
-            const int x = kBMn ? col : kc;
-            const int y = kBMn ? kc : col;
-            if (P == 1)
-              tma_load_2d_pair(b_dst + j * kBox, tb, bar, x, y);
-            else
-              tma_load_2d_pair_mc(b_dst + j * kBox, tb, bar, x, y, b_mask);
+            tma_load_2d_pair(b_dst + j * kBox, tb, bar, kBMn ? col : kc, kBMn ? kc : col);
           }
           if (++stage == kStages) {
             stage = 0;
@@ -218,8 +200,7 @@ __global__ void __launch_bounds__(kThreads, 1) fused_lora_gemm(const __grid_cons
     // ------------------------------------------------------------ MMA issuer (even CTAs)
     if (c == 0 && lane == 0) {
       constexpr uint32_t idesc = idesc_bf16_f32(kBM, kBN, 0, kBMn ? 1 : 0);
-      constexpr uint16_t all_mask = (uint16_t)((1u << C) - 1u);
-      const uint16_t pair_mask = (uint16_t)(0x3u << (2 * pair));
+      constexpr uint16_t pair_mask = 0x3;
       int stage = 0;
       uint32_t phase = 0;
       bool ok = true;
@@ -230,8 +211,8 @@ __global__ void __launch_bounds__(kThreads, 1) fused_lora_gemm(const __grid_cons
         const int t = *reinterpret_cast<volatile int*>(&ctl->tile_id[slot]);
         mbar_arrive_cluster(tile_empty_root + (uint32_t)slot * 8u);
         if (t < 0) break;
-        int p, sm0, n0;
-        decode_tile<P>(b, t, p, sm0, n0);
+        int p, m0, n0;
+        decode_tile(b, t, p, m0, n0);
         const GemmProblem& Q = b.prob[p];
         const int acc = it & 1;
         const uint32_t acc_par = (uint32_t)((it >> 1) & 1);
@@ -253,8 +234,7 @@ __global__ void __launch_bounds__(kThreads, 1) fused_lora_gemm(const __grid_cons
                                         : sw128_desc(b_addr + k * 32, 16, 1024);
             umma_bf16_pair(d_tmem, adesc, bdesc, idesc, (kb | k) != 0 ? 1u : 0u);
           }
-          // the stage is free in every CTA once every pair has consumed it
-          umma_commit_pair_mc(smem_u32(&ctl->empty[stage]), all_mask);
+          umma_commit_pair_mc(smem_u32(&ctl->empty[stage]), pair_mask);
           if (++stage == kStages) {
             stage = 0;
             phase ^= 1u;
@@ -269,7 +249,7 @@ __global__ void __launch_bounds__(kThreads, 1) fused_lora_gemm(const __grid_cons
   } else {
     // ------------------------------------------------------------ epilogue (every CTA)
     const int q = warp & 3;  // TMEM lane quadrant this warp may access
-    const uint32_t tempty_pl = mapa_shared(smem_u32(&ctl->tempty[0]), pair_leader);
+    const uint32_t tempty_pl = mapa_shared(smem_u32(&ctl->tempty[0]), 0);
     for (int it = 0;; ++it) {
       const int slot = it % kTileRing;
       bool got = mbar_wait_cluster(smem_u32(&ctl->tile_full[slot]), (uint32_t)((it / kTileRing) & 1), wc, abort_flag);
@@ -279,8 +259,8 @@ __global__ void __launch_bounds__(kThreads, 1) fused_lora_gemm(const __grid_cons
       __syncwarp();
       if (lane == 0) mbar_arrive_cluster(tile_empty_root + (uint32_t)slot * 8u);
       if (t < 0) break;
-      int p, sm0, n0;
-      decode_tile<P>(b, t, p, sm0, n0);
+      int p, m0, n0;
+      decode_tile(b, t, p, m0, n0);
       const GemmProblem& Q = b.prob[p];
       const int acc = it & 1;
       const uint32_t acc_par = (uint32_t)((it >> 1) & 1);
@@ -288,7 +268,7 @@ __global__ void __launch_bounds__(kThreads, 1) fused_lora_gemm(const __grid_cons
       ok = __all_sync(0xffffffffu, ok);
       if (!ok) break;
       tc_fence_after();
-      const int row = sm0 + pair * kBM + c * kHalf + q * 32 + lane;
+      const int row = m0 + c * kHalf + q * 32 + lane;
       const uint32_t taddr = tmem_base + ((uint32_t)(q * 32) << 16) + (uint32_t)(acc * kBN);
       __nv_bfloat16* orow = Q.out + (size_t)row * Q.ldo;
       for (int cc = 0; cc < kBN; cc += 32) {
@@ -332,50 +312,43 @@ __global__ void __launch_bounds__(kThreads, 1) fused_lora_gemm(const __grid_cons
     }
   }
   __syncthreads();
-  cluster_sync_all();  // no cross-CTA access is pending in any CTA of the cluster
+  cluster_sync_all();  // no cross-CTA access is pending in either CTA
   if (warp == 1) {
     tc_fence_after();
     tmem_dealloc_pair(tmem_base, kTmemCols);
   }
 }
 
-template <bool kBMn, int P>
-cudaError_t launch_variant(const GemmBatch& batch, int num_sms, cudaStream_t stream) {
-  static bool attr_done = false;
-  if (!attr_done) {
-    cudaError_t e = cudaFuncSetAttribute(fused_lora_gemm<kBMn, P>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                         (int)kSmemBytes);
+}  // namespace
+
+size_t fused_gemm_smem_bytes() { return kSmemBytes; }
+
+cudaError_t launch_fused_gemm(const GemmBatch& batch, bool b_mn_major, int num_sms, cudaStream_t stream) {
+  static bool attr_done[2] = {false, false};
+  const void* fn = b_mn_major ? (const void*)fused_lora_gemm<true> : (const void*)fused_lora_gemm<false>;
+  if (!attr_done[b_mn_major]) {
+    cudaError_t e = cudaFuncSetAttribute(fn, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)kSmemBytes);
     if (e != cudaSuccess) return e;
-    attr_done = true;
+    attr_done[b_mn_major] = true;
   }
-  const int max_clusters = num_sms / (2 * P);
-  const int clusters = batch.total_tiles < max_clusters ? batch.total_tiles : max_clusters;
+  if (batch.total_tiles <= 0) return cudaSuccess;
+  const int pairs = batch.total_tiles < num_sms / 2 ? batch.total_tiles : num_sms / 2;
   cudaLaunchConfig_t cfg = {};
-  cfg.gridDim = dim3((unsigned)(2 * P * clusters), 1, 1);
+  cfg.gridDim = dim3((unsigned)(2 * pairs), 1, 1);
   cfg.blockDim = dim3(kThreads, 1, 1);
   cfg.dynamicSmemBytes = kSmemBytes;
   cfg.stream = stream;
   cudaLaunchAttribute attr[1];
   attr[0].id = cudaLaunchAttributeClusterDimension;
-  attr[0].val.clusterDim.x = 2 * P;
+  attr[0].val.clusterDim.x = 2;
   attr[0].val.clusterDim.y = 1;
   attr[0].val.clusterDim.z = 1;
   cfg.attrs = attr;
   cfg.numAttrs = 1;
-  cudaError_t e = cudaLaunchKernelEx(&cfg, fused_lora_gemm<kBMn, P>, batch);
+  cudaError_t e = b_mn_major ? cudaLaunchKernelEx(&cfg, fused_lora_gemm<true>, batch)
+                             : cudaLaunchKernelEx(&cfg, fused_lora_gemm<false>, batch);
   note_launch();
   return e;
-}
-
-}  // namespace
-
-size_t fused_gemm_smem_bytes() { return kSmemBytes; }
-
-cudaError_t launch_fused_gemm(const GemmBatch& batch, bool b_mn_major, int pairs, int num_sms, cudaStream_t stream) {
-  if (batch.total_tiles <= 0) return cudaSuccess;
-  if (pairs == 2) return b_mn_major ? launch_variant<true, 2>(batch, num_sms, stream)
-                                    : launch_variant<false, 2>(batch, num_sms, stream);
-  return b_mn_major ? launch_variant<true, 1>(batch, num_sms, stream) : launch_variant<false, 1>(batch, num_sms, stream);
 }
 
 int gemm_tile_m() { return kBM; }
