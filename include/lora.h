@@ -63,7 +63,8 @@ enum {
   LORA_ECUDA = -4,       /* a CUDA runtime call or launch failed */
   LORA_ETIMEOUT = -5,    /* a device-side bounded wait expired */
   LORA_EWORKSPACE = -6,  /* workspace missing or smaller than required */
-  LORA_EDEVICE = -7      /* current device is not a compute capability 10.3 GPU */
+  LORA_EDEVICE = -7,     /* current device is not a compute capability 10.3 GPU */
+  LORA_ESCRATCH = -8     /* needs more scratch than lora_linear_fwd_noalloc's fixed array */
 };
 
 enum { LORA_FWD = 1, LORA_BWD = 2, LORA_FWD_BWD = 3 };
@@ -88,6 +89,25 @@ int lora_workspace_size(const lora_shape* shape, int mode, size_t* bytes);
 int lora_linear_fwd(const lora_shape* shape, const lora_bf16* x, const lora_bf16* W,
                     const lora_bf16* A, const lora_bf16* B, lora_bf16* y, lora_bf16* su,
                     void* workspace, size_t workspace_bytes, void* stream);
+
+/* Forward of one LoRA linear exactly as lora_linear_fwd computes it, but
+ * with no workspace argument, for callers that cannot allocate device memory
+ * when they call: an operator running inside another framework's execution
+ * callback, where allocating is not allowed, or a latency-bound path that
+ * cannot afford the device-wide synchronisation cudaMalloc and cudaFree
+ * cause.  Its scratch is one fixed array of 4 MiB in device memory that the
+ * library owns; every GPU that loads the library keeps it until the process
+ * exits.  Shapes whose forward needs more scratch than that are rejected
+ * with LORA_ESCRATCH before anything is enqueued (roughly when tokens x
+ * d_in x rank reaches 2^29; 4096 tokens x d_in 4096 at rank 16 fit).  The first call on a device looks up the
+ * array's device address; make that first call before any stream capture.
+ * All calls share the array and leave their scratch in it: calls that
+ * overlap on the GPU (for example on two streams at once) race and give
+ * wrong results.  Nothing is allocated.  The paper has no counterpart of
+ * this entry point.  Returns as lora_linear_fwd, or LORA_ESCRATCH. */
+int lora_linear_fwd_noalloc(const lora_shape* shape, const lora_bf16* x, const lora_bf16* W,
+                            const lora_bf16* A, const lora_bf16* B, lora_bf16* y, lora_bf16* su,
+                            void* stream);
 
 /* Backward of one LoRA linear with W frozen.
  * su is the forward's saved s x A^T.  dx may be NULL (no input gradient

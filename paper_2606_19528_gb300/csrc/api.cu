@@ -732,6 +732,7 @@ const char* lora_strerror(int code) {
     case LORA_ETIMEOUT: return "a device-side bounded wait expired";
     case LORA_EWORKSPACE: return "workspace missing or too small";
     case LORA_EDEVICE: return "current device is not a compute capability 10.3 (GB300) GPU";
+    case LORA_ESCRATCH: return "shape needs more scratch than the fixed 4 MiB array of lora_linear_fwd_noalloc";
     default: return "unknown error";
   }
 }
@@ -864,3 +865,61 @@ int lora_read_status(void* stream, int* status, int reset) {
 }
 
 }  // extern "C"
+
+// ---------------------------------------------------------------------------
+// Forward for callers that cannot allocate.
+//
+// A caller running inside another framework's execution callback may not be
+// allowed to allocate device memory, and a latency-bound caller may not
+// afford the synchronisation of cudaMalloc; lora_linear_fwd_noalloc takes its
+// scratch from the fixed array below instead of a caller workspace.  The
+// array is a host-side stand-in in host code: its device address is looked
+// up once per device with cudaGetSymbolAddress and passed to the kernels.
+namespace lora {
+
+constexpr size_t kNoAllocScratchBytes = (size_t)4 << 20;  // 4 MiB, held by every GPU that loads the library
+static __device__ __align__(256) unsigned char g_noalloc_scratch[kNoAllocScratchBytes];
+
+namespace {
+std::mutex g_noalloc_mu;
+void* g_noalloc_addr[kMaxDevices] = {};
+}  // namespace
+
+}  // namespace lora
+
+extern "C" int lora_linear_fwd_noalloc(const lora_shape* shape, const lora_bf16* x, const lora_bf16* W,
+                                       const lora_bf16* A, const lora_bf16* B, lora_bf16* y, lora_bf16* su,
+                                       void* stream) {
+  if (!shape) return LORA_ENULL;
+  DeviceInfo* d = nullptr;
+  int rc = device_info(&d);
+  if (rc != LORA_OK) return rc;
+  lora_proj p;
+  memset(&p, 0, sizeof(p));
+  p.shape = *shape;
+  p.x = x;
+  p.W = W;
+  p.A = A;
+  p.B = B;
+  p.y = y;
+  p.su = su;
+  Plan pl;
+  if ((rc = plan_all(&p, 1, LORA_FWD, &pl)) != LORA_OK) return rc;
+  if (pl.total > kNoAllocScratchBytes) return LORA_ESCRATCH;
+  if ((rc = check_fwd_ptrs(p)) != LORA_OK) return rc;
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= kMaxDevices) return LORA_ECUDA;
+  void* scratch = nullptr;
+  {
+    // first call on this device (with it current): find the array's device address
+    std::lock_guard<std::mutex> lk(g_noalloc_mu);
+    if (g_noalloc_addr[dev] == nullptr) {
+      void* a = nullptr;
+      if (cudaGetSymbolAddress(&a, g_noalloc_scratch) != cudaSuccess || a == nullptr) return LORA_ECUDA;
+      g_noalloc_addr[dev] = a;
+    }
+    scratch = g_noalloc_addr[dev];
+  }
+  // run_step clears the part of the scratch that must start at zero
+  return run_step(&p, 1, LORA_FWD, scratch, pl, d, static_cast<cudaStream_t>(stream));
+}

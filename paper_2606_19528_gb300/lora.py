@@ -24,13 +24,14 @@ LORA_ECUDA = -4
 LORA_ETIMEOUT = -5
 LORA_EWORKSPACE = -6
 LORA_EDEVICE = -7
+LORA_ESCRATCH = -8
 
 LORA_FWD = 1
 LORA_BWD = 2
 LORA_FWD_BWD = 3
 
 # every symbol that include/lora.h declares
-EXPORTS = ("lora_workspace_size", "lora_linear_fwd", "lora_linear_bwd", "lora_stack_workspace_size",
+EXPORTS = ("lora_workspace_size", "lora_linear_fwd", "lora_linear_fwd_noalloc", "lora_linear_bwd", "lora_stack_workspace_size",
            "lora_stack_step", "lora_read_status", "lora_set_wait_limit_ns", "lora_launch_count",
            "lora_profile_begin", "lora_profile_end", "lora_strerror", "lora_version")
 
@@ -73,6 +74,7 @@ def library(path: str = _LIB_PATH) -> ctypes.CDLL:
         P = ctypes.POINTER
         lib.lora_workspace_size.argtypes = [P(lora_shape), i32, P(sz)]
         lib.lora_linear_fwd.argtypes = [P(lora_shape), vp, vp, vp, vp, vp, vp, vp, sz, vp]
+        lib.lora_linear_fwd_noalloc.argtypes = [P(lora_shape), vp, vp, vp, vp, vp, vp, vp]
         lib.lora_linear_bwd.argtypes = [P(lora_shape), vp, vp, vp, vp, vp, vp, vp, vp, vp, vp, sz, vp]
         lib.lora_stack_workspace_size.argtypes = [P(lora_proj), i32, i32, P(sz)]
         lib.lora_stack_step.argtypes = [P(lora_proj), i32, i32, vp, sz, vp]
@@ -133,6 +135,14 @@ def lora_workspace_size(shape: lora_shape, mode: int) -> int:
 def lora_linear_fwd(shape, x, W, A, B, y, su, workspace, workspace_bytes, stream=None) -> None:
     _check(library().lora_linear_fwd(ctypes.byref(shape), _ptr(x), _ptr(W), _ptr(A), _ptr(B), _ptr(y), _ptr(su),
                                      _ptr(workspace), int(workspace_bytes), _stream(stream)), "lora_linear_fwd")
+
+
+def lora_linear_fwd_noalloc(shape, x, W, A, B, y, su, stream=None) -> None:
+    """Forward without a workspace argument (scratch in a fixed 4 MiB array
+    inside the library), for callers that cannot allocate device memory when
+    they call; see include/lora.h."""
+    _check(library().lora_linear_fwd_noalloc(ctypes.byref(shape), _ptr(x), _ptr(W), _ptr(A), _ptr(B), _ptr(y),
+                                             _ptr(su), _stream(stream)), "lora_linear_fwd_noalloc")
 
 
 def lora_linear_bwd(shape, dy, x, W, A, B, su, dx, dA, dB, workspace, workspace_bytes, stream=None) -> None:
