@@ -41,6 +41,33 @@ FALLBACK_PEAKS = {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "bf16_tflops_sustain
 L2_FLUSH_BYTES = 256 << 20
 
 
+GEMM_PROFILE = os.path.join(ROOT, "profiles", "fused_gemm_llama_layer_T2048_r16.md")
+GEMM_SOURCES = ("paper_2606_19528_gb300/csrc/fused_gemm.cu", "paper_2606_19528_gb300/csrc/common.cuh")
+
+
+def gemm_traffic(workload_name: str):
+    """DRAM bytes per step of the two fused-GEMM launches from the committed ncu
+    summary, or None when the workload differs or the kernel sources changed
+    since the counters were taken."""
+    import hashlib
+    import re
+    if workload_name != workloads.llama_layer_T2048().name:
+        return None
+    try:
+        text = open(GEMM_PROFILE).read()
+        h = hashlib.sha256()
+        for f in GEMM_SOURCES:
+            with open(os.path.join(ROOT, f), "rb") as fh:
+                h.update(fh.read())
+    except OSError:
+        return None
+    m = re.search(r"traffic_bytes_per_step:\s*(\d+)", text)
+    sha = re.search(r"source_sha256:\s*([0-9a-f]{64})", text)
+    if not m or not sha or sha.group(1) != h.hexdigest():
+        return None
+    return int(m.group(1))
+
+
 def load_peaks():
     try:
         with open(PEAKS_FILE) as f:
@@ -410,7 +437,8 @@ def run_gpu(args, wl):
                              "source": peaks_src},
         "roofline": {"kernel": "fused_lora_gemm (fwd and bwd launches)", "bound": "tensor",
                      "achieved": gemm_tflops, "peak": sustained, "unit": "TFLOP/s",
-                     "frac": gemm_tflops / sustained, "traffic": None,
+                     "frac": gemm_tflops / sustained, "traffic": gemm_traffic(wl.name),
+                     "traffic_unit": "bytes per step (forward + backward launch), ncu dram__bytes_read+write",
                      "peak_kind": f"bf16 sustained, of {peaks_src}",
                      "frac_of_burst": gemm_tflops / burst,
                      "flops_per_step": f_fwd + f_bwd, "ms_per_step": gemm_ms},
