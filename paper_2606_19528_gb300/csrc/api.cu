@@ -477,6 +477,7 @@ int add_fwd_problem(GemmBatch& b, const lora_proj& p, const Operands& o) {
   if ((rc = make_map(&b.tmA2[i], o.s_in, r, T, o.ld_s, 64, 128)) != LORA_OK) return rc;
   if ((rc = make_map(&b.tmB[i], p.W, K, N, K, 64, 64)) != LORA_OK) return rc;
   if ((rc = make_map(&b.tmB2[i], o.B, r, N, o.ld_b, 64, 64)) != LORA_OK) return rc;
+  if ((rc = make_map(&b.tmOut[i], p.y, N, T, N, 64, 32)) != LORA_OK) return rc;
   GemmProblem& g = b.prob[i];
   g.out = mb(p.y);
   g.ldo = (int)N;
@@ -506,6 +507,7 @@ int add_bwd_problem(GemmBatch& b, const lora_proj& p, const Operands& o) {
   // W [N, K] read MN-major: inner dimension K (the GEMM's output columns), rows = contraction
   if ((rc = make_map(&b.tmB[i], p.W, K, N, K, 64, 64)) != LORA_OK) return rc;
   if ((rc = make_map(&b.tmB2[i], p.A, K, r, K, 64, 64)) != LORA_OK) return rc;
+  if ((rc = make_map(&b.tmOut[i], p.dx, K, T, K, 64, 32)) != LORA_OK) return rc;
   GemmProblem& g = b.prob[i];
   g.out = mb(p.dx);
   g.ldo = (int)K;

@@ -14,22 +14,25 @@
 // MN-major straight from the frozen weight (no transposed copy of W).
 //
 // Structure: persistent CTA pairs (thread-block clusters of 2, one CTA per
-// SM) take 256 x 256 output tiles from a tile list spanning every problem of
+// SM) take 256 x 512 output tiles from a tile list spanning every problem of
 // a batch (up to kMaxProblems projections, heavier first) through a global
-// atomic counter, so that tiles of unequal depth balance across SMs.  Each
-// tile is one 2-CTA tensor-core contraction (tcgen05 cta_group::2, M = 256,
-// N = 256, K = 16 per instruction): each CTA of the pair stages its own 128
-// rows of the activation operand and its own 128 columns of the weight
-// operand, and holds its 128 x 256 half of the fp32 accumulator in its own
-// tensor memory.  Within a problem, consecutive tiles walk M when the weight
+// atomic counter, so that tiles of unequal depth balance across SMs.  A tile
+// is two 2-CTA tensor-core contractions per 16-deep step (tcgen05
+// cta_group::2, M = 256, N = 256 each, one per 256-column segment): each CTA
+// of the pair stages its own 128 rows of the activation operand and its own
+// 2 x 128 columns of the weight operand, and holds its 128 x 512 half of the
+// fp32 accumulator in all 512 columns of its tensor memory.  The wide tile
+// halves the shared-memory traffic per FLOP of a 256 x 256 tile, which keeps
+// the operand feed ahead of the tensor pipe.  The epilogue drains segment 0
+// first and releases it, so the next tile's first MMAs overlap the drain of
+// segment 1.  Within a problem, consecutive tiles walk M when the weight
 // operand is the larger one, so each weight tile is read from DRAM once.
 //   warp 0      tile scheduler (even CTA) and TMA producer (both CTAs):
-//               6-stage shared-memory ring of 32 KB, 128-byte swizzle
+//               4-stage shared-memory ring of 48 KB, 128-byte swizzle
 //   warp 1      TMEM allocation (both CTAs); tcgen05.mma issuer (even CTA)
-//   warps 2..5  epilogue: TMEM -> registers -> bf16 -> global
-// Two 256-column fp32 accumulators per CTA (512 TMEM columns) let the
-// epilogue of one tile overlap the main loop of the next.  Every wait is
-// bounded.
+//   warps 2..9  epilogue: TMEM -> registers -> bf16 -> swizzled shared-memory
+//               block (32 rows x 64 columns per warp) -> TMA tensor store
+// Every wait is bounded.
 #include "common.cuh"
 #include "kernels.h"
 
@@ -39,24 +42,26 @@ namespace {
 
 constexpr int kBM = 256;                          // tile rows (128 per CTA of a pair)
 constexpr int kHalf = 128;
-constexpr int kBN = 256;                          // tile columns (128 weight rows/columns per CTA)
+constexpr int kSeg = 256;                         // columns of one MMA / accumulator segment
+constexpr int kBN = 2 * kSeg;                     // tile columns
 constexpr int kBK = 64;
-constexpr int kStages = 6;
-constexpr uint32_t kAHalf = kHalf * kBK * 2;      // 16 KB
-constexpr uint32_t kBHalf = kHalf * kBK * 2;      // 16 KB
-constexpr uint32_t kStageBytes = kAHalf + kBHalf;
+constexpr int kStages = 4;
+constexpr uint32_t kAHalf = kHalf * kBK * 2;      // 16 KB: this CTA's activation rows
+constexpr uint32_t kBSeg = kHalf * kBK * 2;       // 16 KB: this CTA's weight rows of one segment
+constexpr uint32_t kStageBytes = kAHalf + 2 * kBSeg;
 constexpr uint32_t kBox = 64 * kBK * 2;           // one 64 x 64 box of the weight operand, 8 KB
-constexpr int kThreads = 192;
-constexpr int kEpiWarps = 4;
+constexpr int kEpiWarps = 8;                      // two per TMEM lane quadrant
+constexpr uint32_t kEpiStage = 32 * 128;          // per-warp output block: 32 rows x 64 bf16, 4 KB
+constexpr int kThreads = (2 + kEpiWarps) * 32;
 constexpr uint32_t kTmemCols = 512;
 constexpr int kTileRing = 4;  // tile ids handed from the scheduler to the other roles
 constexpr long long kDrainNs = 1000000000ll;
 
 struct __align__(8) Ctl {
-  uint64_t full[kStages];          // even CTA: both CTAs' halves of a stage landed
+  uint64_t full[kStages];          // even CTA: both CTAs' parts of a stage landed
   uint64_t empty[kStages];         // both CTAs: the pair's MMAs finished reading a stage
-  uint64_t tfull[2];               // both CTAs: accumulator complete
-  uint64_t tempty[2];              // even CTA: both CTAs' epilogues drained an accumulator
+  uint64_t tfull;                  // both CTAs: accumulator complete
+  uint64_t tempty[2];              // even CTA: both CTAs' epilogues drained a segment
   uint64_t tile_full[kTileRing];   // both CTAs: tile id written
   uint64_t tile_empty[kTileRing];  // even CTA: every consumer of both CTAs read the slot
   uint64_t drain;                  // both CTAs: every MMA of the pair completed
@@ -65,7 +70,7 @@ struct __align__(8) Ctl {
   int abort;
 };
 
-constexpr size_t kSmemBytes = 1024 + (size_t)kStages * kStageBytes + sizeof(Ctl);
+constexpr size_t kSmemBytes = 1024 + (size_t)kStages * kStageBytes + (size_t)kEpiWarps * kEpiStage + sizeof(Ctl);
 
 // Problem p, first row m0 and first column n0 of tile t.
 __device__ __forceinline__ void decode_tile(const GemmBatch& b, int t, int& p, int& m0, int& n0) {
@@ -87,7 +92,9 @@ __global__ void __launch_bounds__(kThreads, 1) fused_lora_gemm(const __grid_cons
   extern __shared__ uint8_t smem_raw[];
   const uint32_t raw = smem_u32(smem_raw);
   const uint32_t base = (raw + 1023u) & ~1023u;
-  Ctl* ctl = reinterpret_cast<Ctl*>(smem_raw + (base - raw) + (size_t)kStages * kStageBytes);
+  const uint32_t epi_base = base + kStages * kStageBytes;  // 1024-aligned output staging blocks
+  Ctl* ctl = reinterpret_cast<Ctl*>(smem_raw + (base - raw) + (size_t)kStages * kStageBytes +
+                                    (size_t)kEpiWarps * kEpiStage);
   volatile int* abort_flag = &ctl->abort;
 
   const int warp = threadIdx.x >> 5;
@@ -100,10 +107,8 @@ __global__ void __launch_bounds__(kThreads, 1) fused_lora_gemm(const __grid_cons
       mbar_init(smem_u32(&ctl->full[s]), 1);
       mbar_init(smem_u32(&ctl->empty[s]), 1);
     }
-    for (int a = 0; a < 2; ++a) {
-      mbar_init(smem_u32(&ctl->tfull[a]), 1);
-      mbar_init(smem_u32(&ctl->tempty[a]), 2 * kEpiWarps);
-    }
+    mbar_init(smem_u32(&ctl->tfull), 1);
+    for (int h = 0; h < 2; ++h) mbar_init(smem_u32(&ctl->tempty[h]), 2 * kEpiWarps);
     for (int k = 0; k < kTileRing; ++k) {
       mbar_init(smem_u32(&ctl->tile_full[k]), 1);
       // MMA thread, epilogue warps of both CTAs, producer of the odd CTA
@@ -119,6 +124,7 @@ __global__ void __launch_bounds__(kThreads, 1) fused_lora_gemm(const __grid_cons
       tma_prefetch_desc(&b.tmA2[q]);
       tma_prefetch_desc(&b.tmB[q]);
       tma_prefetch_desc(&b.tmB2[q]);
+      tma_prefetch_desc(&b.tmOut[q]);
     }
   }
   if (warp == 1) {
@@ -161,12 +167,14 @@ __global__ void __launch_bounds__(kThreads, 1) fused_lora_gemm(const __grid_cons
         const GemmProblem& Q = b.prob[p];
         const int my_m = m0 + c * kHalf;
         const bool a_mine = my_m < Q.M;
-        // weight boxes of pair position c' hold columns n0 + 128 c' + 64 j, j = 0, 1
-        auto box_ok = [&](int cc, int j) { return n0 + cc * kHalf + j * 64 < Q.N; };
-        // bytes landing in this pair per stage (signalled on the pair's even CTA)
-        const uint32_t tx_pair = (m0 < Q.M ? kAHalf : 0u) + (m0 + kHalf < Q.M ? kAHalf : 0u) +
-                                 kBox * ((box_ok(0, 0) ? 1u : 0u) + (box_ok(0, 1) ? 1u : 0u) +
-                                         (box_ok(1, 0) ? 1u : 0u) + (box_ok(1, 1) ? 1u : 0u));
+        // weight box (segment h, pair position cc, j): columns n0 + 256 h + 128 cc + 64 j
+        auto box_ok = [&](int h, int cc, int j) { return n0 + h * kSeg + cc * kHalf + j * 64 < Q.N; };
+        uint32_t boxes = 0;
+        for (int h = 0; h < 2; ++h)
+          for (int cc = 0; cc < 2; ++cc)
+            for (int j = 0; j < 2; ++j) boxes += box_ok(h, cc, j) ? 1u : 0u;
+        // bytes landing in this pair per stage (signalled on the even CTA)
+        const uint32_t tx_pair = (m0 < Q.M ? kAHalf : 0u) + (m0 + kHalf < Q.M ? kAHalf : 0u) + kBox * boxes;
         bool ok = true;
         for (int kb = 0; kb < Q.kb_total; ++kb) {
           if (!mbar_wait_cluster(smem_u32(&ctl->empty[stage]), phase ^ 1u, wc, abort_flag)) {
@@ -183,10 +191,13 @@ __global__ void __launch_bounds__(kThreads, 1) fused_lora_gemm(const __grid_cons
           const CUtensorMap* tb = main ? &b.tmB[p] : &b.tmB2[p];
           if (a_mine) tma_load_2d_pair(a_dst, ta, bar, kc, my_m);
 #pragma unroll
-          for (int j = 0; j < 2; ++j) {
-            if (!box_ok(c, j)) continue;
-            const int col = n0 + c * kHalf + j * 64;
-            tma_load_2d_pair(b_dst + j * kBox, tb, bar, kBMn ? col : kc, kBMn ? kc : col);
+          for (int h = 0; h < 2; ++h) {
+#pragma unroll
+            for (int j = 0; j < 2; ++j) {
+              if (!box_ok(h, c, j)) continue;
+              const int col = n0 + h * kSeg + c * kHalf + j * 64;
+              tma_load_2d_pair(b_dst + h * kBSeg + j * kBox, tb, bar, kBMn ? col : kc, kBMn ? kc : col);
+            }
           }
           if (++stage == kStages) {
             stage = 0;
@@ -197,9 +208,9 @@ __global__ void __launch_bounds__(kThreads, 1) fused_lora_gemm(const __grid_cons
       }
     }
   } else if (warp == 1) {
-    // ------------------------------------------------------------ MMA issuer (even CTAs)
+    // ------------------------------------------------------------ MMA issuer (even CTA)
     if (c == 0 && lane == 0) {
-      constexpr uint32_t idesc = idesc_bf16_f32(kBM, kBN, 0, kBMn ? 1 : 0);
+      constexpr uint32_t idesc = idesc_bf16_f32(kBM, kSeg, 0, kBMn ? 1 : 0);
       constexpr uint16_t pair_mask = 0x3;
       int stage = 0;
       uint32_t phase = 0;
@@ -214,11 +225,9 @@ __global__ void __launch_bounds__(kThreads, 1) fused_lora_gemm(const __grid_cons
         int p, m0, n0;
         decode_tile(b, t, p, m0, n0);
         const GemmProblem& Q = b.prob[p];
-        const int acc = it & 1;
-        const uint32_t acc_par = (uint32_t)((it >> 1) & 1);
-        if (!mbar_wait_cluster(smem_u32(&ctl->tempty[acc]), acc_par ^ 1u, wc, abort_flag)) break;
-        tc_fence_after();
-        const uint32_t d_tmem = tmem_base + (uint32_t)(acc * kBN);
+        const int nseg = Q.N - n0 > kSeg ? 2 : 1;  // segments holding any column < N
+        // segment h is free once both epilogues drained it for the previous tile
+        const uint32_t drained_par = (uint32_t)((it & 1) ^ 1);
         for (int kb = 0; kb < Q.kb_total; ++kb) {
           if (!mbar_wait(smem_u32(&ctl->full[stage]), phase, wc, abort_flag)) {
             ok = false;
@@ -228,12 +237,24 @@ __global__ void __launch_bounds__(kThreads, 1) fused_lora_gemm(const __grid_cons
           const uint32_t a_addr = base + stage * kStageBytes;
           const uint32_t b_addr = a_addr + kAHalf;
           const int nk = kb < Q.kb_main ? kBK / 16 : min(kBK / 16, (Q.r - (kb - Q.kb_main) * kBK + 15) / 16);
-          for (int k = 0; k < nk; ++k) {
-            const uint64_t adesc = sw128_desc(a_addr + k * 32, 16, 1024);
-            const uint64_t bdesc = kBMn ? sw128_desc(b_addr + k * 2048, kBox, 1024)
-                                        : sw128_desc(b_addr + k * 32, 16, 1024);
-            umma_bf16_pair(d_tmem, adesc, bdesc, idesc, (kb | k) != 0 ? 1u : 0u);
+          for (int h = 0; h < 2; ++h) {
+            if (kb == 0) {
+              if (!mbar_wait_cluster(smem_u32(&ctl->tempty[h]), drained_par, wc, abort_flag)) {
+                ok = false;
+                break;
+              }
+              tc_fence_after();
+            }
+            if (h >= nseg) continue;
+            const uint32_t d_tmem = tmem_base + (uint32_t)(h * kSeg);
+            const uint32_t bseg = b_addr + (uint32_t)h * kBSeg;
+            for (int k = 0; k < nk; ++k) {
+              const uint64_t adesc = sw128_desc(a_addr + k * 32, 16, 1024);
+              const uint64_t bdesc = kBMn ? sw128_desc(bseg + k * 2048, kBox, 1024) : sw128_desc(bseg + k * 32, 16, 1024);
+              umma_bf16_pair(d_tmem, adesc, bdesc, idesc, (kb | k) != 0 ? 1u : 0u);
+            }
           }
+          if (!ok) break;
           umma_commit_pair_mc(smem_u32(&ctl->empty[stage]), pair_mask);
           if (++stage == kStages) {
             stage = 0;
@@ -241,14 +262,15 @@ __global__ void __launch_bounds__(kThreads, 1) fused_lora_gemm(const __grid_cons
           }
         }
         if (!ok) break;
-        umma_commit_pair_mc(smem_u32(&ctl->tfull[acc]), pair_mask);
+        umma_commit_pair_mc(smem_u32(&ctl->tfull), pair_mask);
       }
       // completes in both CTAs of the pair once every MMA issued above has finished
       umma_commit_pair_mc(smem_u32(&ctl->drain), pair_mask);
     }
   } else {
-    // ------------------------------------------------------------ epilogue (every CTA)
-    const int q = warp & 3;  // TMEM lane quadrant this warp may access
+    // ------------------------------------------------------------ epilogue (both CTAs)
+    const int q = warp & 3;                 // TMEM lane quadrant this warp may access
+    const int part = (warp - 2) >> 2;       // which 128 columns of each segment
     const uint32_t tempty_pl = mapa_shared(smem_u32(&ctl->tempty[0]), 0);
     for (int it = 0;; ++it) {
       const int slot = it % kTileRing;
@@ -262,39 +284,51 @@ __global__ void __launch_bounds__(kThreads, 1) fused_lora_gemm(const __grid_cons
       int p, m0, n0;
       decode_tile(b, t, p, m0, n0);
       const GemmProblem& Q = b.prob[p];
-      const int acc = it & 1;
-      const uint32_t acc_par = (uint32_t)((it >> 1) & 1);
-      bool ok = mbar_wait_cluster(smem_u32(&ctl->tfull[acc]), acc_par, wc, abort_flag);
+      bool ok = mbar_wait_cluster(smem_u32(&ctl->tfull), (uint32_t)(it & 1), wc, abort_flag);
       ok = __all_sync(0xffffffffu, ok);
       if (!ok) break;
       tc_fence_after();
-      const int row = m0 + c * kHalf + q * 32 + lane;
-      const uint32_t taddr = tmem_base + ((uint32_t)(q * 32) << 16) + (uint32_t)(acc * kBN);
-      __nv_bfloat16* orow = Q.out + (size_t)row * Q.ldo;
-      for (int cc = 0; cc < kBN; cc += 32) {
-        if (n0 + cc >= Q.N) break;  // uniform across the warp
-        uint32_t v[32];
-        tmem_ld_32x32b_x32(taddr + (uint32_t)cc, v);
-        tmem_ld_wait();
-        if (row < Q.M) {
+      const int row0 = m0 + c * kHalf + q * 32;  // first of this warp's 32 rows
+      const uint32_t stg = epi_base + (uint32_t)(warp - 2) * kEpiStage;
+      for (int h = 0; h < 2; ++h) {
+        for (int cc = 0; cc < kHalf; cc += 64) {
+          const int col0 = h * kSeg + part * kHalf + cc;  // tile column of this 64-column block
+          if (n0 + col0 >= Q.N || row0 >= Q.M) break;     // uniform across the warp
+          const uint32_t taddr = tmem_base + ((uint32_t)(q * 32) << 16) + (uint32_t)col0;
+          uint32_t v[32], w[32];
+          tmem_ld_32x32b_x32(taddr, v);
+          tmem_ld_32x32b_x32(taddr + 32u, w);
+          tmem_ld_wait();
+          // the previous block's store must have read the staging buffer
+          if (lane == 0) bulk_wait_read0();
+          __syncwarp();
+          // row `lane` of the block: 8 chunks of 16 B, chunk k at k ^ (row mod 8) (128-byte swizzle)
+          const uint32_t rbase = stg + (uint32_t)lane * 128u;
 #pragma unroll
-          for (int g = 0; g < 4; ++g) {
-            const int col = n0 + cc + g * 8;
-            if (col < Q.N) {
-              uint4 pk;
-              pk.x = pack_bf16x2(__uint_as_float(v[g * 8 + 0]), __uint_as_float(v[g * 8 + 1]));
-              pk.y = pack_bf16x2(__uint_as_float(v[g * 8 + 2]), __uint_as_float(v[g * 8 + 3]));
-              pk.z = pack_bf16x2(__uint_as_float(v[g * 8 + 4]), __uint_as_float(v[g * 8 + 5]));
-              pk.w = pack_bf16x2(__uint_as_float(v[g * 8 + 6]), __uint_as_float(v[g * 8 + 7]));
-              *reinterpret_cast<uint4*>(orow + col) = pk;
-            }
+          for (int k = 0; k < 8; ++k) {
+            const uint32_t* src = k < 4 ? &v[k * 8] : &w[(k - 4) * 8];
+            const uint32_t a = pack_bf16x2(__uint_as_float(src[0]), __uint_as_float(src[1]));
+            const uint32_t b2 = pack_bf16x2(__uint_as_float(src[2]), __uint_as_float(src[3]));
+            const uint32_t c2 = pack_bf16x2(__uint_as_float(src[4]), __uint_as_float(src[5]));
+            const uint32_t d2 = pack_bf16x2(__uint_as_float(src[6]), __uint_as_float(src[7]));
+            const uint32_t dst = rbase + (uint32_t)(((k ^ (lane & 7)) & 7) << 4);
+            asm volatile("st.shared.v4.b32 [%0], {%1, %2, %3, %4};" ::"r"(dst), "r"(a), "r"(b2), "r"(c2), "r"(d2)
+                         : "memory");
+          }
+          fence_proxy_async_smem();
+          __syncwarp();
+          if (lane == 0) {
+            tma_store_2d(&b.tmOut[p], stg, n0 + col0, row0);
+            bulk_commit();
           }
         }
+        tc_fence_before();
+        __syncwarp();
+        if (lane == 0) mbar_arrive_cluster(tempty_pl + (uint32_t)h * 8u);
       }
-      tc_fence_before();
-      __syncwarp();
-      if (lane == 0) mbar_arrive_cluster(tempty_pl + (uint32_t)acc * 8u);
     }
+    // the output must be written before the CTA exits
+    if (lane == 0) bulk_wait0();
   }
 
   // ------------------------------------------------------------ teardown

@@ -39,6 +39,7 @@ struct GemmBatch {
   CUtensorMap tmA2[kMaxProblems];
   CUtensorMap tmB[kMaxProblems];
   CUtensorMap tmB2[kMaxProblems];
+  CUtensorMap tmOut[kMaxProblems];  // out [M, N]: 64 columns x 32 rows boxes, 128-byte swizzle
   GemmProblem prob[kMaxProblems];
   int num_problems;
   int total_tiles;
