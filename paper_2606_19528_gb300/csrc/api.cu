@@ -161,7 +161,7 @@ int check_shape(const lora_shape* s) {
 
 // Workspace regions of one projection.
 struct Ws {
-  size_t su_pad = 0, b_pad = 0, sv = 0;
+  size_t su_pad = 0, b_pad = 0, sv = 0, bt = 0, sut = 0, svt = 0;
   size_t total = 0;
 };
 
@@ -177,12 +177,19 @@ Ws plan_ws(const lora_shape& s, int mode) {
   };
   w.su_pad = take((size_t)T * r8 * 2);
   if (pad) w.b_pad = take((size_t)N * r8 * 2);
-  if (mode & LORA_BWD) w.sv = take((size_t)T * r8 * 2);
+  if (mode & LORA_BWD) {
+    w.sv = take((size_t)T * r8 * 2);
+    w.bt = take((size_t)N * r8 * 2);   // B^T, zero rows past r
+    w.sut = take((size_t)T * r8 * 2);  // su^T, zero rows past r
+    w.svt = take((size_t)T * r8 * 2);  // sv^T, zero rows past r
+  }
   w.total = off;
   return w;
 }
 
-// Workspace of a call: [GEMM tile counters | rank-r partials | per-projection regions].
+// Workspace of a call: [GEMM tile counters | rank-r partials |
+// per-projection regions]; the counters are cleared by one memset at the
+// start of a call.
 // The rank-r arenas are sized for the projections without input sharing,
 // an upper bound of what grouped problems need (a group's padded rank is at
 // most the sum of its members').
@@ -224,6 +231,7 @@ struct RowSpec {
   int ld_out[kMaxRankBlocks];
   bf* out2[kMaxRankBlocks];
   int ld_out2[kMaxRankBlocks];
+  bf* outT[kMaxRankBlocks];
 };
 struct ColSpec {
   const bf* X;
@@ -239,10 +247,11 @@ inline int used_rank(const int* r, int n) {
   return u;
 }
 
-// Appends block (W, ldw, rw) -> (out, out2) to the row problem of activation X,
-// opening a new problem when X differs or the concatenated rank would pass 128.
+// Appends block (W, ldw, rw) -> (out, out2, outT) to the row problem of
+// activation X, opening a new problem when X differs or the concatenated rank
+// would pass 128.
 void add_row_block(std::vector<RowSpec>& probs, const bf* X, int ldx, int T, int C, float scale, const bf* W,
-                   int ldw, int rw, bf* out, int ld_out, bf* out2, int ld_out2, bool fuse) {
+                   int ldw, int rw, bf* out, int ld_out, bf* out2, int ld_out2, bf* outT, bool fuse) {
   RowSpec* p = nullptr;
   if (fuse) {
     for (RowSpec& q : probs)
@@ -271,6 +280,7 @@ void add_row_block(std::vector<RowSpec>& probs, const bf* X, int ldx, int T, int
   p->ld_out[b] = ld_out;
   p->out2[b] = out2;
   p->ld_out2[b] = ld_out2;
+  p->outT[b] = outT;
 }
 
 void add_col_block(std::vector<ColSpec>& probs, const bf* X, int ldx, int T, int C, const bf* S, int lds, int rs,
@@ -310,13 +320,13 @@ struct Arena {
 
 constexpr int kMinUnitChunks = 8;  // smallest work unit (64-wide chunks); sizes the partial arenas
 
-// Chunks per unit for a launch.  The persistent grid (two CTAs per SM) takes
+// Chunks per unit for a launch.  The persistent grid (max_ctas CTAs) takes
 // units round-robin, so the launch lasts about ceil(units / CTAs) units; the
 // cost of a size is that makespan in chunks, plus a fixed charge for the
 // partial-sum pass when any tile needs several units.  Ties go to the larger
 // unit (fewer partials).
 template <typename Spec, typename LenFn>
-int choose_unit_chunks(const std::vector<Spec>& specs, size_t i0, size_t i1, int num_sms, LenFn len) {
+int choose_unit_chunks(const std::vector<Spec>& specs, size_t i0, size_t i1, int max_ctas, LenFn len) {
   int best = kMinUnitChunks;
   long long best_cost = -1;
   for (int u : {64, 32, 16, 8}) {
@@ -328,7 +338,7 @@ int choose_unit_chunks(const std::vector<Spec>& specs, size_t i0, size_t i1, int
       units += (long long)tl.first * upt;
       partials = partials || upt > 1;
     }
-    const long long ctas = std::min<long long>(units, 2LL * num_sms);
+    const long long ctas = std::min<long long>(units, (long long)max_ctas);
     const long long cost = (units + ctas - 1) / ctas * u + (partials ? 4 : 0);
     if (best_cost < 0 || cost < best_cost) {
       best_cost = cost;
@@ -338,29 +348,16 @@ int choose_unit_chunks(const std::vector<Spec>& specs, size_t i0, size_t i1, int
   return best;
 }
 
-// 2-D bf16 tensor map without swizzle (rank-side tiles).
-int make_map_plain(CUtensorMap* m, const void* ptr, uint64_t inner, uint64_t outer, uint64_t ld, uint32_t box_inner,
-                   uint32_t box_outer) {
-  cuuint64_t dims[2] = {inner, outer};
-  cuuint64_t strides[1] = {ld * 2};
-  cuuint32_t box[2] = {box_inner, box_outer};
-  cuuint32_t estr[2] = {1, 1};
-  CUresult r = g_encode(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void*>(ptr), dims, strides, box, estr,
-                        CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_NONE,
-                        CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
-  return r == CUDA_SUCCESS ? LORA_OK : LORA_ECUDA;
-}
-
-int launch_rows(const std::vector<RowSpec>& specs, bool w_rc, const Arena& ar, const DeviceInfo* d,
-                cudaStream_t st) {
-  const int tile = rank_tile();
+int launch_rows(const std::vector<RowSpec>& specs, const Arena& ar, const DeviceInfo* d, cudaStream_t st) {
+  const int tile = rank_mma_tile();
   size_t pf = 0;
   int rc;
   for (size_t i0 = 0; i0 < specs.size(); i0 += kMaxRankProblems) {
     const size_t i1 = std::min(specs.size(), i0 + kMaxRankProblems);
     RowBatch b;
     memset(&b, 0, sizeof(b));
-    // (tiles, reduction length) of a row problem
+    b.tile_rows = tile;
+    // one persistent CTA per SM; (tiles, reduction length) of a row problem
     b.unit_chunks = choose_unit_chunks(specs, i0, i1, d->num_sms, [&](const RowSpec& q) {
       return std::make_pair(cdiv(q.T, tile), q.C);
     });
@@ -372,27 +369,25 @@ int launch_rows(const std::vector<RowSpec>& specs, bool w_rc, const Arena& ar, c
       p.C = sp.C;
       p.nblk = sp.nblk;
       p.scale = sp.scale;
-      if ((rc = make_map(&p.tmX, sp.X, sp.C, sp.T, sp.ldx, 64, 64)) != LORA_OK) return rc;
-      int bytes = 64 * 64 * 2;
+      if ((rc = make_map(&p.tmX, sp.X, sp.C, sp.T, sp.ldx, 64, tile)) != LORA_OK) return rc;
+      int bytes = tile * 64 * 2;
       for (int k = 0; k < sp.nblk; ++k) {
         p.rw[k] = sp.rw[k];
         p.out[k] = sp.out[k];
         p.ld_out[k] = sp.ld_out[k];
         p.out2[k] = sp.out2[k];
         p.ld_out2[k] = sp.ld_out2[k];
+        p.outT[k] = sp.outT[k];
         const int r8 = rank_pad8(sp.rw[k]);
-        if (w_rc)  // A_b [r_b, C]: 64 columns x r8 rows, rows past r_b zero-filled
-          rc = make_map(&p.tmW[k], sp.W[k], sp.C, sp.rw[k], sp.ldw[k], 64, r8);
-        else       // B [C, r] (row stride ldw, a multiple of 8): r8 entries x 64 rows
-          rc = make_map_plain(&p.tmW[k], sp.W[k], r8, sp.C, sp.ldw[k], r8, 64);
-        if (rc != LORA_OK) return rc;
+        // W_b [r_b, C]: 64 columns x r8 rows, rows past r_b zero-filled
+        if ((rc = make_map(&p.tmW[k], sp.W[k], sp.C, sp.rw[k], sp.ldw[k], 64, r8)) != LORA_OK) return rc;
         bytes += 64 * r8 * 2;
       }
       p.tx_bytes = bytes;
       p.rpad = rank_pad16(used_rank(sp.rw, sp.nblk));
       rmax = std::max(rmax, p.rpad);
       const int tiles = cdiv(p.T, tile);
-      p.upt = cdiv(cdiv(p.C, tile), b.unit_chunks);
+      p.upt = cdiv(cdiv(p.C, 64), b.unit_chunks);
       p.unit_begin = b.units;
       b.units += tiles * p.upt;
       p.part_off = (long long)pf;
@@ -403,24 +398,26 @@ int launch_rows(const std::vector<RowSpec>& specs, bool w_rc, const Arena& ar, c
       }
     }
     if (pf > ar.n_partials) return LORA_EWORKSPACE;  // planning bound violated
-    b.w_rc = w_rc ? 1 : 0;
     b.partials = ar.partials;
     b.status = d->status;
     b.limit_ns = g_wait_limit_ns;
-    if (launch_rowprod(b, rmax, d->num_sms, st) != cudaSuccess) return LORA_ECUDA;
+    if (launch_rowmma(b, rmax, d->num_sms, st) != cudaSuccess) return LORA_ECUDA;
   }
   return LORA_OK;
 }
 
-int launch_cols(const std::vector<ColSpec>& specs, const Arena& ar, const DeviceInfo* d, cudaStream_t st) {
-  const int tile = rank_tile();
+// Column products of one phase on `ctas` persistent CTAs (one per SM).
+int launch_cols(const std::vector<ColSpec>& specs, const Arena& ar, const DeviceInfo* d, int ctas, cudaStream_t st) {
+  const int tile = rank_mma_tile();
   size_t pf = 0;
   int rc;
   for (size_t i0 = 0; i0 < specs.size(); i0 += kMaxRankProblems) {
     const size_t i1 = std::min(specs.size(), i0 + kMaxRankProblems);
     ColBatch b;
     memset(&b, 0, sizeof(b));
-    b.unit_chunks = choose_unit_chunks(specs, i0, i1, d->num_sms, [&](const ColSpec& q) {
+    b.tile_rows = tile;
+    // (tiles, reduction length) of a column problem
+    b.unit_chunks = choose_unit_chunks(specs, i0, i1, ctas, [&](const ColSpec& q) {
       return std::make_pair(cdiv(q.C, tile), q.T);
     });
     int rmax = 16;
@@ -431,20 +428,22 @@ int launch_cols(const std::vector<ColSpec>& specs, const Arena& ar, const Device
       p.C = sp.C;
       p.nblk = sp.nblk;
       p.out_cr = sp.out_cr;
+      // X^T tiles: two boxes of 64 columns x 64 tokens
       if ((rc = make_map(&p.tmX, sp.X, sp.C, sp.T, sp.ldx, 64, 64)) != LORA_OK) return rc;
-      int bytes = 64 * 64 * 2;
+      int bytes = tile * 64 * 2;
       for (int k = 0; k < sp.nblk; ++k) {
         p.rs[k] = sp.rs[k];
         p.out[k] = sp.out[k];
         const int r8 = rank_pad8(sp.rs[k]);
-        if ((rc = make_map_plain(&p.tmS[k], sp.S[k], r8, sp.T, sp.lds[k], r8, 64)) != LORA_OK) return rc;
+        // S_b^T [rs_b, T]: 64 tokens x r8 rows, rows past rs_b zero-filled
+        if ((rc = make_map(&p.tmS[k], sp.S[k], sp.T, sp.rs[k], sp.lds[k], 64, r8)) != LORA_OK) return rc;
         bytes += 64 * r8 * 2;
       }
       p.tx_bytes = bytes;
       p.rpad = rank_pad16(used_rank(sp.rs, sp.nblk));
       rmax = std::max(rmax, p.rpad);
       const int tiles = cdiv(p.C, tile);
-      p.upt = cdiv(cdiv(p.T, tile), b.unit_chunks);
+      p.upt = cdiv(cdiv(p.T, 64), b.unit_chunks);
       p.unit_begin = b.units;
       b.units += tiles * p.upt;
       p.part_off = (long long)pf;
@@ -454,16 +453,18 @@ int launch_cols(const std::vector<ColSpec>& specs, const Arena& ar, const Device
         b.red_total += tiles * tile * p.rpad;
       }
     }
-    if (pf > ar.n_partials) return LORA_EWORKSPACE;
+    if (pf > ar.n_partials) return LORA_EWORKSPACE;  // planning bound violated
     b.partials = ar.partials;
     b.status = d->status;
     b.limit_ns = g_wait_limit_ns;
-    if (launch_colprod(b, rmax, d->num_sms, st) != cudaSuccess) return LORA_ECUDA;
+    if (launch_colmma(b, rmax, ctas, st) != cudaSuccess) return LORA_ECUDA;
   }
   return LORA_OK;
 }
 
-Arena arena(void* ws, const Plan& pl, int phase) { return Arena{at<float>(ws, pl.part_off[phase]), pl.n_partials[phase]}; }
+Arena arena(void* ws, const Plan& pl, int phase) {
+  return Arena{at<float>(ws, pl.part_off[phase]), pl.n_partials[phase]};
+}
 
 // ------------------------------------------------------------------ forward
 int add_fwd_problem(GemmBatch& b, const lora_proj& p, const Operands& o) {
@@ -577,7 +578,8 @@ int run_step(const lora_proj* projs, int n, int mode, void* ws, const Plan& pl, 
         bf* su_gemm = (p.su && !pad) ? mb(p.su) : at<bf>(W_(i), plans[i].su_pad);
         const int ld_gemm = (p.su && !pad) ? r : r8;
         bf* su_user2 = (p.su && pad) ? mb(p.su) : nullptr;
-        add_row_block(rows, cb(p.x), K, T, K, p.shape.scale, cb(p.A), K, r, su_gemm, ld_gemm, su_user2, r, true);
+        add_row_block(rows, cb(p.x), K, T, K, p.shape.scale, cb(p.A), K, r, su_gemm, ld_gemm, su_user2, r, nullptr,
+                      true);
         ops[i].s_in = su_gemm;
         ops[i].ld_s = ld_gemm;
         if (pad) {
@@ -593,7 +595,7 @@ int run_step(const lora_proj* projs, int n, int mode, void* ws, const Plan& pl, 
     }
     {
       ProfScope ps(LORA_KERNEL_ROWPROJ, st);
-      if ((rc = launch_rows(rows, true, arena(ws, pl, kPhFwdRows), d, st)) != LORA_OK) return rc;
+      if ((rc = launch_rows(rows, arena(ws, pl, kPhFwdRows), d, st)) != LORA_OK) return rc;
     }
     // heavier problems first so that the static tile walk ends balanced
     std::vector<int> order(n);
@@ -614,50 +616,60 @@ int run_step(const lora_proj* projs, int n, int mode, void* ws, const Plan& pl, 
     std::vector<Operands> ops(n);
     std::vector<RowSpec> rows;
     std::vector<ColSpec> cols;
-    std::vector<const bf*> su_in(n);
-    std::vector<int> ld_su(n);
+    std::vector<bf*> sut(n), svt(n);
+    TransposeJobs tj;
+    memset(&tj, 0, sizeof(tj));
     {
       ProfScope ps(LORA_KERNEL_PAD, st);
+      // rank sides as K-major tensor-core operands: B^T for sv = s dy B and
+      // su^T for dB = dy^T su, zero rows past r
+      auto transpose = [&](const bf* src, int rows_, int r, bf* dst) -> int {
+        if (tj.count == kMaxTransposes) {
+          if (launch_transposes(tj, st) != cudaSuccess) return LORA_ECUDA;
+          memset(&tj, 0, sizeof(tj));
+        }
+        const int k = tj.count++;
+        tj.src[k] = src;
+        tj.dst[k] = dst;
+        tj.n[k] = rows_;
+        tj.r[k] = r;
+        tj.ld[k] = r;
+        tj.r8[k] = rank_pad8(r);
+        tj.max_elems = std::max(tj.max_elems, (long long)rows_ * tj.r8[k]);
+        return LORA_OK;
+      };
       for (int i = 0; i < n; ++i) {
         const lora_proj& p = projs[i];
         const int T = (int)p.shape.T, N = (int)p.shape.d_out, r = (int)p.shape.rank, r8 = rank_pad8(r);
-        const bool pad = (r % 8) != 0;
-        const bf* B_in = cb(p.B);
-        int ld_b = r;
-        su_in[i] = cb(p.su);
-        ld_su[i] = r;
-        if (pad) {
-          if (launch_pad_cols(cb(p.su), T, r, at<bf>(W_(i), plans[i].su_pad), r8, st) != cudaSuccess ||
-              launch_pad_cols(cb(p.B), N, r, at<bf>(W_(i), plans[i].b_pad), r8, st) != cudaSuccess)
-            return LORA_ECUDA;
-          su_in[i] = at<bf>(W_(i), plans[i].su_pad);
-          ld_su[i] = r8;
-          B_in = at<bf>(W_(i), plans[i].b_pad);
-          ld_b = r8;
-        }
+        bf* bt = at<bf>(W_(i), plans[i].bt);
+        sut[i] = at<bf>(W_(i), plans[i].sut);
+        svt[i] = at<bf>(W_(i), plans[i].svt);
+        if ((rc = transpose(cb(p.B), N, r, bt)) != LORA_OK) return rc;
+        if ((rc = transpose(cb(p.su), T, r, sut[i])) != LORA_OK) return rc;
         bf* sv = at<bf>(W_(i), plans[i].sv);
-        add_row_block(rows, cb(p.dy), N, T, N, p.shape.scale, B_in, ld_b, r, sv, r8, nullptr, 0, false);
+        add_row_block(rows, cb(p.dy), N, T, N, p.shape.scale, bt, N, r, sv, r8, nullptr, 0, svt[i], false);
         ops[i].s_in = sv;
         ops[i].ld_s = r8;
       }
+      if (launch_transposes(tj, st) != cudaSuccess) return LORA_ECUDA;
     }
     {
       ProfScope ps(LORA_KERNEL_ROWPROJ, st);
-      if ((rc = launch_rows(rows, false, arena(ws, pl, kPhBwdRows), d, st)) != LORA_OK) return rc;
+      if ((rc = launch_rows(rows, arena(ws, pl, kPhBwdRows), d, st)) != LORA_OK) return rc;
     }
     for (int i = 0; i < n; ++i) {
       const lora_proj& p = projs[i];
-      const int T = (int)p.shape.T, K = (int)p.shape.d_in, N = (int)p.shape.d_out, r = (int)p.shape.rank;
-      add_col_block(cols, cb(p.dy), N, T, N, su_in[i], ld_su[i], r, p.dB, 1, false);
+      const int T = (int)p.shape.T, N = (int)p.shape.d_out, r = (int)p.shape.rank;
+      add_col_block(cols, cb(p.dy), N, T, N, sut[i], T, r, p.dB, 1, false);
     }
     for (int i = 0; i < n; ++i) {
       const lora_proj& p = projs[i];
       const int T = (int)p.shape.T, K = (int)p.shape.d_in, r = (int)p.shape.rank;
-      add_col_block(cols, cb(p.x), K, T, K, ops[i].s_in, ops[i].ld_s, r, p.dA, 0, true);
+      add_col_block(cols, cb(p.x), K, T, K, svt[i], T, r, p.dA, 0, true);
     }
     {
       ProfScope ps(LORA_KERNEL_COLPROJ, st);
-      if ((rc = launch_cols(cols, arena(ws, pl, kPhBwdCols), d, st)) != LORA_OK) return rc;
+      if ((rc = launch_cols(cols, arena(ws, pl, kPhBwdCols), d, d->num_sms, st)) != LORA_OK) return rc;
     }
     std::vector<int> order;
     for (int i = 0; i < n; ++i)
@@ -678,25 +690,23 @@ int run_step(const lora_proj* projs, int n, int mode, void* ws, const Plan& pl, 
 }
 
 int plan_all(const lora_proj* projs, int n, int mode, Plan* pl) {
-  const int tile = rank_tile();
   // partials are bounded by the smallest unit size (most units per tile)
-  auto upt = [&](int64_t len) { return (size_t)cdiv(cdiv(len, tile), kMinUnitChunks); };
+  const int tile = rank_mma_tile();
+  auto upt = [&](int64_t len) { return (size_t)cdiv(cdiv(len, 64), kMinUnitChunks); };
   auto tiles = [&](int64_t len) { return (size_t)cdiv(len, tile); };
   for (int i = 0; i < n; ++i) {
     int rc = check_shape(&projs[i].shape);
     if (rc != LORA_OK) return rc;
     const lora_shape& s = projs[i].shape;
     const size_t r16 = (size_t)rank_pad16((int)s.rank);
-    if (mode & LORA_FWD) {
-      if (upt(s.d_in) > 1) pl->n_partials[kPhFwdRows] += tiles(s.T) * upt(s.d_in) * tile * r16;
-    }
+    if ((mode & LORA_FWD) && upt(s.d_in) > 1) pl->n_partials[kPhFwdRows] += tiles(s.T) * upt(s.d_in) * tile * r16;
     if (mode & LORA_BWD) {
       if (upt(s.d_out) > 1) pl->n_partials[kPhBwdRows] += tiles(s.T) * upt(s.d_out) * tile * r16;
       if (upt(s.T) > 1) pl->n_partials[kPhBwdCols] += (tiles(s.d_out) + tiles(s.d_in)) * upt(s.T) * tile * r16;
     }
   }
   size_t off = kWsHeader;
-  pl->zero_bytes = kWsHeader;
+  pl->zero_bytes = off;
   for (int k = 0; k < kPhases; ++k) {
     pl->part_off[k] = off;
     off += up256(pl->n_partials[k] * sizeof(float));

@@ -61,16 +61,15 @@ inline int rank_pad8(int r) { return (r + 7) / 8 * 8; }
 constexpr int kMaxRankBlocks = 4;     // projections fused into one problem
 constexpr int kMaxRankProblems = 12;  // problems per launch
 
-// Row product problem: out_b[t, j] = scale * sum_c X[t, c] * Wv_b(j, c) for
-// every block b (one projection each) sharing the activation X [T, C].
-//   w_rc launches: Wv_b(j, c) = W_b[j * ldw_b + c]   (A of the adapter, [r_b, C])
-//   otherwise:     Wv_0(j, c) = W_0[c * ldw_0 + j]   (B of the adapter, [C, r]; one block)
+// Row product problem: out_b[t, j] = scale * sum_c X[t, c] * W_b[j, c] for
+// every block b (one projection each) sharing the activation X [T, C]; W_b
+// is [r_b, C] row-major (A of the adapter, or B of the adapter transposed).
 // Blocks are concatenated at 8-aligned rank offsets; columns rw_b .. ld_out_b
-// of out_b are written as zeros; out2_b (optional) gets columns < ld_out2_b.
+// of out_b are written as zeros; out2_b (optional) gets columns < ld_out2_b
+// and outT_b (optional) the transpose [pad8(r_b), T], zero rows past r_b.
 struct RowProb {
-  CUtensorMap tmX;                   // X [T, C]: box 64 columns x 64 tokens, 128-byte swizzle
-  CUtensorMap tmW[kMaxRankBlocks];   // w_rc: A_b [r_b, C], box 64 x pad8(r_b), 128-byte swizzle;
-                                     // else: B [C, r] (one block), box pad8(r) x 64, no swizzle
+  CUtensorMap tmX;                   // X [T, C]: box 64 columns x 128 tokens, 128-byte swizzle
+  CUtensorMap tmW[kMaxRankBlocks];   // W_b [r_b, C]: box 64 columns x pad8(r_b) rows, 128-byte swizzle
   int T, C;
   int nblk;
   int rw[kMaxRankBlocks];
@@ -78,38 +77,40 @@ struct RowProb {
   int ld_out[kMaxRankBlocks];
   __nv_bfloat16* out2[kMaxRankBlocks];
   int ld_out2[kMaxRankBlocks];
+  __nv_bfloat16* outT[kMaxRankBlocks];
   float scale;
   int rpad;            // concatenated rank, rounded up to 16
   int tx_bytes;        // bytes one chunk stage receives (X box + rank-side boxes)
-  int upt;             // work units per 64-token tile (each unit_chunks x 64 columns)
+  int upt;             // work units per 128-token tile (each unit_chunks x 64 columns)
   int unit_begin;      // first unit of this problem in the launch
-  int red_begin;       // first element of this problem in the reduction pass (upt > 1)
+  int red_begin;       // first element of this problem in the partial-sum pass (upt > 1)
   long long part_off;  // first fp32 partial of this problem (used when upt > 1)
 };
 struct RowBatch {
   RowProb p[kMaxRankProblems];
-  int n, units, w_rc;
+  int n, units;
+  int tile_rows;    // tokens per tile
   int unit_chunks;  // 64-wide reduction chunks per unit
-  int red_total;    // elements of the reduction pass (0: none)
-  float* partials;  // [tile][unit][64][rpad] per problem
+  int red_total;    // elements of the partial-sum pass (0: none)
+  float* partials;  // [tile][unit][tile_rows][rpad] per problem
   int* status;
   long long limit_ns;
 };
 
 // Column product problem: out_b[c, j] = sum_t X[t, c] * S_b[t, j] for every
-// block b sharing X [T, C]; S_b is [T, pad8(rs_b)] with zeros beyond rs_b.
-// out_cr: out_b[c * rs_b + j] (dB), else out_b[j * C + c] (dA).
+// block b sharing X [T, C]; S_b is given transposed, S_b^T [rs_b, T]
+// row-major.  out_cr: out_b[c * rs_b + j] (dB), else out_b[j * C + c] (dA).
 struct ColProb {
   CUtensorMap tmX;                   // X [T, C]: box 64 columns x 64 tokens, 128-byte swizzle
-  CUtensorMap tmS[kMaxRankBlocks];   // S_b: box pad8(rs_b) x 64 tokens, no swizzle
+  CUtensorMap tmS[kMaxRankBlocks];   // S_b^T [rs_b, T]: box 64 tokens x pad8(rs_b) rows, 128-byte swizzle
   int T, C;
   int nblk;
   int rs[kMaxRankBlocks];
   float* out[kMaxRankBlocks];
   int out_cr;
   int rpad;
-  int tx_bytes;
-  int upt;             // work units per 64-column tile (each unit_chunks x 64 tokens)
+  int tx_bytes;        // bytes of a full chunk stage (both X boxes + rank-side boxes)
+  int upt;             // work units per 128-column tile (each unit_chunks x 64 tokens)
   int unit_begin;
   int red_begin;
   long long part_off;
@@ -117,6 +118,7 @@ struct ColProb {
 struct ColBatch {
   ColProb p[kMaxRankProblems];
   int n, units;
+  int tile_rows;    // columns per tile
   int unit_chunks;
   int red_total;
   float* partials;
@@ -124,9 +126,25 @@ struct ColBatch {
   long long limit_ns;
 };
 
-int rank_tile();
-cudaError_t launch_rowprod(const RowBatch& b, int rmax, int num_sms, cudaStream_t stream);
-cudaError_t launch_colprod(const ColBatch& b, int rmax, int num_sms, cudaStream_t stream);
+// Output rows (tokens of a row product, columns of a column product) per tile.
+int rank_mma_tile();
+// Rank-r products on the tensor cores, then their partial-sum pass when needed;
+// `ctas` persistent CTAs (one per SM).
+cudaError_t launch_rowmma(const RowBatch& b, int rmax, int ctas, cudaStream_t stream);
+cudaError_t launch_colmma(const ColBatch& b, int rmax, int ctas, cudaStream_t stream);
+cudaError_t launch_reduce_rows(const RowBatch& b, cudaStream_t stream);
+cudaError_t launch_reduce_cols(const ColBatch& b, cudaStream_t stream);
+// Batched transposes: dst_i[j, n] = src_i[n, j] for j < r_i, 0 for r_i <= j < r8_i
+// (src_i [n_i, r_i] with row stride ld_i), every job in one launch.
+constexpr int kMaxTransposes = 128;
+struct TransposeJobs {
+  const __nv_bfloat16* src[kMaxTransposes];
+  __nv_bfloat16* dst[kMaxTransposes];
+  int n[kMaxTransposes], r[kMaxTransposes], ld[kMaxTransposes], r8[kMaxTransposes];
+  int count;
+  long long max_elems;  // largest n_i * r8_i
+};
+cudaError_t launch_transposes(const TransposeJobs& jobs, cudaStream_t stream);
 
 // dst[i, j] = j < r ? src[i * r + j] : 0  for j < ld_dst (zero-padded copy of an [rows, r] matrix).
 cudaError_t launch_pad_cols(const __nv_bfloat16* src, int rows, int r, __nv_bfloat16* dst, int ld_dst,
