@@ -175,6 +175,10 @@ int64_t lora_launch_count(void);
  * and launches[LORA_KERNEL_KINDS] (either may be NULL), and stops recording.
  * Returns LORA_OK, LORA_EINVAL (end without begin) or LORA_ECUDA. */
 int lora_profile_begin(void);
+/* As lora_profile_begin, but only the launch groups of the kinds whose bit
+ * (1u << LORA_KERNEL_*) is set in kind_mask are bracketed; the others run
+ * with no event between their launches. */
+int lora_profile_begin_kinds(uint32_t kind_mask);
 int lora_profile_end(double* ms, int64_t* launches);
 
 /* Static message for a LORA_* code. */

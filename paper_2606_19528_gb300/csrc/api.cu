@@ -10,6 +10,7 @@
 
 #include <algorithm>
 #include <atomic>
+#include <cstdlib>
 #include <mutex>
 #include <vector>
 
@@ -48,6 +49,7 @@ struct ProfRec {
 
 struct Profiler {
   bool on = false;
+  uint32_t mask = 0;  // kinds bracketed with events
   std::vector<cudaEvent_t> pool;  // events are reused across sessions
   size_t next = 0;
   std::vector<ProfRec> recs;
@@ -69,7 +71,7 @@ class ProfScope {
  public:
   ProfScope(int kind, cudaStream_t st) : kind_(kind), st_(st) {
     std::lock_guard<std::mutex> lk(g_prof_mu);
-    if (!g_prof.on) return;
+    if (!g_prof.on || !((g_prof.mask >> kind) & 1u)) return;
     a_ = g_prof.take();
     b_ = g_prof.take();
     if (a_ && b_ && cudaEventRecord(a_, st_) == cudaSuccess) {
@@ -726,6 +728,14 @@ int plan_all(const lora_proj* projs, int n, int mode, Plan* pl) {
 
 void note_launch() { g_launches.fetch_add(1, std::memory_order_relaxed); }
 
+bool pdl_enabled() {
+  static const bool on = [] {
+    const char* e = getenv("LORA_PDL");
+    return !(e && e[0] == '0' && e[1] == 0);
+  }();
+  return on;
+}
+
 }  // namespace lora
 
 using namespace lora;
@@ -830,13 +840,16 @@ int lora_linear_bwd(const lora_shape* shape, const lora_bf16* dy, const lora_bf1
 
 int64_t lora_launch_count(void) { return (int64_t)g_launches.load(); }
 
-int lora_profile_begin(void) {
+int lora_profile_begin_kinds(uint32_t kind_mask) {
   std::lock_guard<std::mutex> lk(g_prof_mu);
   g_prof.recs.clear();
   g_prof.next = 0;
+  g_prof.mask = kind_mask;
   g_prof.on = true;
   return LORA_OK;
 }
+
+int lora_profile_begin(void) { return lora_profile_begin_kinds((1u << LORA_KERNEL_KINDS) - 1u); }
 
 int lora_profile_end(double* ms, int64_t* launches) {
   std::lock_guard<std::mutex> lk(g_prof_mu);

@@ -36,6 +36,14 @@ __device__ __forceinline__ void mbar_init(uint32_t bar, uint32_t count) {
   asm volatile("mbarrier.init.shared::cta.b64 [%0], %1;" ::"r"(bar), "r"(count) : "memory");
 }
 
+// Programmatic dependent launch.  griddep_wait blocks until every grid this
+// one depends on has completed and its writes are visible (a no-op for a grid
+// launched without the attribute); every kernel calls it before its first
+// global access.  griddep_launch_dependents lets the next grid of the stream
+// start launching (its CTAs run their prologue and then wait themselves).
+__device__ __forceinline__ void griddep_wait() { asm volatile("griddepcontrol.wait;" ::: "memory"); }
+__device__ __forceinline__ void griddep_launch_dependents() { asm volatile("griddepcontrol.launch_dependents;" ::: "memory"); }
+
 __device__ __forceinline__ void fence_mbar_init() {
   asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
 }

@@ -135,6 +135,7 @@ __global__ void __launch_bounds__(kThreads, 1) fused_lora_gemm(const __grid_cons
   __syncthreads();
   tc_fence_after();
   cluster_sync_all();  // both CTAs' barriers exist before any cross-CTA arrival
+  griddep_wait();      // the previous grid's outputs (su, sv, tile counter) are ready
   const uint32_t tmem_base = ctl->tmem_base;
   const uint32_t tile_empty_root = mapa_shared(smem_u32(&ctl->tile_empty[0]), 0);
 
@@ -161,7 +162,10 @@ __global__ void __launch_bounds__(kThreads, 1) fused_lora_gemm(const __grid_cons
           t = *reinterpret_cast<volatile int*>(&ctl->tile_id[slot]);
           mbar_arrive_cluster(tile_empty_root + (uint32_t)slot * 8u);
         }
-        if (t < 0) break;
+        if (t < 0) {
+          griddep_launch_dependents();  // no tile left for this pair
+          break;
+        }
         int p, m0, n0;
         decode_tile(b, t, p, m0, n0);
         const GemmProblem& Q = b.prob[p];
@@ -221,7 +225,10 @@ __global__ void __launch_bounds__(kThreads, 1) fused_lora_gemm(const __grid_cons
           break;
         const int t = *reinterpret_cast<volatile int*>(&ctl->tile_id[slot]);
         mbar_arrive_cluster(tile_empty_root + (uint32_t)slot * 8u);
-        if (t < 0) break;
+        if (t < 0) {
+          griddep_launch_dependents();  // no tile left for this pair
+          break;
+        }
         int p, m0, n0;
         decode_tile(b, t, p, m0, n0);
         const GemmProblem& Q = b.prob[p];
@@ -367,22 +374,9 @@ cudaError_t launch_fused_gemm(const GemmBatch& batch, bool b_mn_major, int num_s
   }
   if (batch.total_tiles <= 0) return cudaSuccess;
   const int pairs = batch.total_tiles < num_sms / 2 ? batch.total_tiles : num_sms / 2;
-  cudaLaunchConfig_t cfg = {};
-  cfg.gridDim = dim3((unsigned)(2 * pairs), 1, 1);
-  cfg.blockDim = dim3(kThreads, 1, 1);
-  cfg.dynamicSmemBytes = kSmemBytes;
-  cfg.stream = stream;
-  cudaLaunchAttribute attr[1];
-  attr[0].id = cudaLaunchAttributeClusterDimension;
-  attr[0].val.clusterDim.x = 2;
-  attr[0].val.clusterDim.y = 1;
-  attr[0].val.clusterDim.z = 1;
-  cfg.attrs = attr;
-  cfg.numAttrs = 1;
-  cudaError_t e = b_mn_major ? cudaLaunchKernelEx(&cfg, fused_lora_gemm<true>, batch)
-                             : cudaLaunchKernelEx(&cfg, fused_lora_gemm<false>, batch);
-  note_launch();
-  return e;
+  const dim3 grid((unsigned)(2 * pairs)), block(kThreads);
+  return b_mn_major ? launch_kernel(fused_lora_gemm<true>, grid, block, kSmemBytes, stream, 2, batch)
+                    : launch_kernel(fused_lora_gemm<false>, grid, block, kSmemBytes, stream, 2, batch);
 }
 
 int gemm_tile_m() { return kBM; }

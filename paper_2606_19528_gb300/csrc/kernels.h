@@ -12,6 +12,41 @@ namespace lora {
 // Counts one kernel launch (defined with the C ABI).
 void note_launch();
 
+// Whether kernels are launched with programmatic dependent launch (on unless
+// the environment sets LORA_PDL=0).
+bool pdl_enabled();
+
+// Launches `kernel` on `st` with programmatic stream serialization (when
+// enabled) and, for cluster_x > 1, clusters of cluster_x CTAs; counts it.
+template <typename... KArgs, typename... Args>
+cudaError_t launch_kernel(void (*kernel)(KArgs...), dim3 grid, dim3 block, size_t smem, cudaStream_t st,
+                          int cluster_x, Args&&... args) {
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = grid;
+  cfg.blockDim = block;
+  cfg.dynamicSmemBytes = smem;
+  cfg.stream = st;
+  cudaLaunchAttribute attr[2];
+  unsigned n = 0;
+  if (pdl_enabled()) {
+    attr[n].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    attr[n].val.programmaticStreamSerializationAllowed = 1;
+    ++n;
+  }
+  if (cluster_x > 1) {
+    attr[n].id = cudaLaunchAttributeClusterDimension;
+    attr[n].val.clusterDim.x = (unsigned)cluster_x;
+    attr[n].val.clusterDim.y = 1;
+    attr[n].val.clusterDim.z = 1;
+    ++n;
+  }
+  cfg.attrs = attr;
+  cfg.numAttrs = n;
+  const cudaError_t e = cudaLaunchKernelEx(&cfg, kernel, static_cast<Args&&>(args)...);
+  note_launch();
+  return e != cudaSuccess ? e : cudaGetLastError();
+}
+
 // ---------------------------------------------------------------- fused GEMM
 constexpr int kMaxProblems = 8;
 

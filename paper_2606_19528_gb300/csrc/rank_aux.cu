@@ -16,6 +16,8 @@ namespace {
 // row); the loads of all units are independent and issued together.
 template <typename Batch, bool kRow>
 __global__ void __launch_bounds__(256) reduce_partials_kernel(const __grid_constant__ Batch b, int total4) {
+  griddep_wait();
+  griddep_launch_dependents();
   const int i4 = blockIdx.x * blockDim.x + threadIdx.x;
   if (i4 >= total4) return;
   const int i = i4 * 4;
@@ -53,6 +55,8 @@ __global__ void __launch_bounds__(256) reduce_partials_kernel(const __grid_const
 // K-major operand of the tensor cores): job blockIdx.y, output element
 // (j, n) per thread, n fastest so that the writes coalesce.
 __global__ void transposes_kernel(const __grid_constant__ TransposeJobs jobs) {
+  griddep_wait();
+  griddep_launch_dependents();
   const int k = blockIdx.y;
   const int n = jobs.n[k];
   const long long total = (long long)n * jobs.r8[k];
@@ -66,6 +70,8 @@ __global__ void transposes_kernel(const __grid_constant__ TransposeJobs jobs) {
 
 __global__ void pad_cols_kernel(const __nv_bfloat16* __restrict__ src, int rows, int r,
                                 __nv_bfloat16* __restrict__ dst, int ld_dst) {
+  griddep_wait();
+  griddep_launch_dependents();
   const size_t n = (size_t)rows * ld_dst;
   for (size_t i = blockIdx.x * (size_t)blockDim.x + threadIdx.x; i < n; i += (size_t)gridDim.x * blockDim.x) {
     const size_t row = i / ld_dst;
@@ -86,33 +92,27 @@ int grid_for(size_t n, int threads) {
 cudaError_t launch_transposes(const TransposeJobs& jobs, cudaStream_t st) {
   if (jobs.count <= 0 || jobs.max_elems <= 0) return cudaSuccess;
   const int bx = std::min(grid_for((size_t)jobs.max_elems, 256), 64);
-  transposes_kernel<<<dim3(bx, jobs.count), 256, 0, st>>>(jobs);
-  note_launch();
-  return cudaGetLastError();
+  return launch_kernel(transposes_kernel, dim3(bx, jobs.count), dim3(256), 0, st, 1, jobs);
 }
 
 cudaError_t launch_reduce_rows(const RowBatch& b, cudaStream_t st) {
   if (b.red_total <= 0) return cudaSuccess;
   const int total4 = b.red_total / 4;
-  reduce_partials_kernel<RowBatch, true><<<(total4 + 255) / 256, 256, 0, st>>>(b, total4);
-  note_launch();
-  return cudaGetLastError();
+  return launch_kernel(reduce_partials_kernel<RowBatch, true>, dim3((total4 + 255) / 256), dim3(256), 0, st, 1, b,
+                       total4);
 }
 
 cudaError_t launch_reduce_cols(const ColBatch& b, cudaStream_t st) {
   if (b.red_total <= 0) return cudaSuccess;
   const int total4 = b.red_total / 4;
-  reduce_partials_kernel<ColBatch, false><<<(total4 + 255) / 256, 256, 0, st>>>(b, total4);
-  note_launch();
-  return cudaGetLastError();
+  return launch_kernel(reduce_partials_kernel<ColBatch, false>, dim3((total4 + 255) / 256), dim3(256), 0, st, 1, b,
+                       total4);
 }
 
 cudaError_t launch_pad_cols(const __nv_bfloat16* src, int rows, int r, __nv_bfloat16* dst, int ld_dst,
                             cudaStream_t st) {
   const size_t n = (size_t)rows * ld_dst;
-  pad_cols_kernel<<<grid_for(n, 256), 256, 0, st>>>(src, rows, r, dst, ld_dst);
-  note_launch();
-  return cudaGetLastError();
+  return launch_kernel(pad_cols_kernel, dim3(grid_for(n, 256)), dim3(256), 0, st, 1, src, rows, r, dst, ld_dst);
 }
 
 }  // namespace lora

@@ -122,6 +122,7 @@ __global__ void __launch_bounds__(kThreads, 1) rank_mma_kernel(const __grid_cons
   tc_fence_before();
   __syncthreads();
   tc_fence_after();
+  griddep_wait();  // X and the rank sides may come from the previous grid
   const uint32_t tmem_base = ctl->tmem_base;
   long long issued = 0;     // producer: stages issued
   bool issued_any = false;  // MMA issuer: any MMA issued
@@ -170,6 +171,7 @@ __global__ void __launch_bounds__(kThreads, 1) rank_mma_kernel(const __grid_cons
           }
         }
       }
+      griddep_launch_dependents();  // every load of this CTA is issued
     }
   } else if (warp == 1) {
     // ---------------------------------------------------------------- MMA issuer
@@ -293,9 +295,7 @@ cudaError_t launch_r(const typename Side<kCol>::Batch& b, int ctas, cudaStream_t
     attr_done = true;
   }
   const int grid = b.units < ctas ? b.units : ctas;
-  rank_mma_kernel<R, kCol><<<grid, kThreads, smem, st>>>(b);
-  note_launch();
-  return cudaGetLastError();
+  return launch_kernel(rank_mma_kernel<R, kCol>, dim3(grid), dim3(kThreads), smem, st, 1, b);
 }
 
 template <bool kCol>

@@ -33,7 +33,7 @@ LORA_FWD_BWD = 3
 # every symbol that include/lora.h declares
 EXPORTS = ("lora_workspace_size", "lora_linear_fwd", "lora_linear_fwd_noalloc", "lora_linear_bwd", "lora_stack_workspace_size",
            "lora_stack_step", "lora_read_status", "lora_set_wait_limit_ns", "lora_launch_count",
-           "lora_profile_begin", "lora_profile_end", "lora_strerror", "lora_version")
+           "lora_profile_begin", "lora_profile_begin_kinds", "lora_profile_end", "lora_strerror", "lora_version")
 
 LORA_KERNEL_GEMM_FWD = 0
 LORA_KERNEL_GEMM_BWD = 1
@@ -82,6 +82,7 @@ def library(path: str = _LIB_PATH) -> ctypes.CDLL:
         lib.lora_set_wait_limit_ns.argtypes = [i64]
         lib.lora_launch_count.argtypes = []
         lib.lora_profile_begin.argtypes = []
+        lib.lora_profile_begin_kinds.argtypes = [ctypes.c_uint32]
         lib.lora_profile_end.argtypes = [P(ctypes.c_double), P(i64)]
         lib.lora_strerror.argtypes = [i32]
         lib.lora_strerror.restype = ctypes.c_char_p
@@ -183,8 +184,16 @@ def lora_launch_count() -> int:
     return int(library().lora_launch_count())
 
 
-def lora_profile_begin() -> None:
-    _check(library().lora_profile_begin(), "lora_profile_begin")
+def lora_profile_begin(kinds=None) -> None:
+    """Starts a profiling session over every launch group, or only the groups
+    of the LORA_KERNEL_* kinds listed in `kinds`."""
+    if kinds is None:
+        _check(library().lora_profile_begin(), "lora_profile_begin")
+    else:
+        mask = 0
+        for k in kinds:
+            mask |= 1 << int(k)
+        _check(library().lora_profile_begin_kinds(mask), "lora_profile_begin_kinds")
 
 
 def lora_profile_end():
