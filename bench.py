@@ -89,9 +89,10 @@ def gen_layer_bits(wl: workloads.Workload, seed: int = 0, T: int | None = None):
             xs[p.group] = synth.gen_x(seed, wl.cfg, p.group, 0, T, p.d_in)
         out.append({
             "x": xs[p.group], "group": p.group,
-            "W": synth.gen_W(seed, wl.cfg, i, 0, p.d_out, p.d_in),
+            "W": None if wl.q4 else synth.gen_W(seed, wl.cfg, i, 0, p.d_out, p.d_in),
             "A": synth.gen_A(seed, wl.cfg, i, 0, wl.rank, p.d_in),
             "B": synth.gen_B(seed, wl.cfg, i, 0, p.d_out, wl.rank, zero=wl.zero_B),
+            "Wq": synth.gen_Wq(seed, wl.cfg, i, 0, p.d_out, p.d_in) if wl.q4 else None,
             "dy": synth.gen_dy(seed, wl.cfg, i, 0, T, p.d_out),
         })
     return out
@@ -166,19 +167,33 @@ class ClockSampler:
 # ----------------------------------------------------------------------------- CPU oracle timing
 
 def oracle_sample(wl: workloads.Workload, tokens: int, seed: int = 0):
-    """fp64 inputs of a `tokens`-token sample of the workload (outside timing)."""
+    """fp64 inputs of a `tokens`-token sample of the workload (outside timing);
+    4-bit weights stay as codes and (s, b) pairs."""
     bits = gen_layer_bits(wl, seed, T=tokens)
     f = synth.bf16_bits_to_f64
-    return [{k: f(v) for k, v in p.items() if k != "group"} for p in bits]
+    out = []
+    for p in bits:
+        e = {k: f(v) for k, v in p.items() if k not in ("group", "Wq", "W")}
+        if p["Wq"] is not None:
+            sb = f(p["Wq"][1])
+            e["Wq"] = (p["Wq"][0], sb[..., 0], sb[..., 1])
+        else:
+            e["W"] = f(p["W"])
+        out.append(e)
+    return out
 
 
 def time_oracle_step(sample, s: float):
+    """One oracle fwd+bwd over the sample; 4-bit weights are dequantized
+    (Algorithm 1) for the forward and again for the backward, inside the timing."""
     import oracle
     t0 = time.perf_counter()
     c0 = time.process_time()
     for p in sample:
-        oracle.lora_forward(p["x"], p["W"], p["A"], p["B"], s)
-        oracle.lora_backward(p["dy"], p["x"], p["W"], p["A"], p["B"], s)
+        W = oracle.dequant_q4(*p["Wq"]) if "Wq" in p else p["W"]
+        oracle.lora_forward(p["x"], W, p["A"], p["B"], s)
+        W = oracle.dequant_q4(*p["Wq"]) if "Wq" in p else p["W"]
+        oracle.lora_backward(p["dy"], p["x"], W, p["A"], p["B"], s)
     return time.perf_counter() - t0, time.process_time() - c0
 
 
@@ -293,7 +308,13 @@ class LayerOnDevice:
         for pb, pr in zip(bits, wl.projs):
             if pr.group not in xs:
                 xs[pr.group] = d(pb["x"])
-            e = {"x": xs[pr.group], "W": d(pb["W"]), "A": d(pb["A"]), "B": d(pb["B"]), "dy": d(pb["dy"]),
+            wq = None
+            if pb["Wq"] is not None:
+                codes = torch.from_numpy(pb["Wq"][0]).to(dev)
+                params = d(pb["Wq"][1])
+                wq = (codes, params, lora.make_q4(codes, params))
+            e = {"x": xs[pr.group], "W": None if wq else d(pb["W"]), "Wq": wq,
+                 "A": d(pb["A"]), "B": d(pb["B"]), "dy": d(pb["dy"]),
                  "y": torch.empty(T, pr.d_out, dtype=torch.bfloat16, device=dev),
                  "su": torch.empty(T, r, dtype=torch.bfloat16, device=dev),
                  "dx": torch.empty(T, pr.d_in, dtype=torch.bfloat16, device=dev),
@@ -303,7 +324,8 @@ class LayerOnDevice:
         self.xs = xs
         self.projs = [lora.make_proj(lora.make_shape(T, pr.d_in, pr.d_out, r, wl.scale), x=e["x"], W=e["W"],
                                      A=e["A"], B=e["B"], dy=e["dy"], y=e["y"], su=e["su"], dx=e["dx"], dA=e["dA"],
-                                     dB=e["dB"]) for e, pr in zip(self.p, wl.projs)]
+                                     dB=e["dB"], Wq=e["Wq"][2] if e["Wq"] else None)
+                      for e, pr in zip(self.p, wl.projs)]
         n = lora.lora_stack_workspace_size(self.projs, lora.LORA_FWD_BWD)
         self.ws = torch.empty(max(n, 256), dtype=torch.uint8, device=dev)
 
@@ -316,7 +338,8 @@ class LayerOnDevice:
         dys2 = [torch.empty_like(e["dy"]) for e in self.p]
         projs2 = [lora.make_proj(lora.make_shape(T, pr.d_in, pr.d_out, r, self.wl.scale), x=xs2[pr.group],
                                  W=e["W"], A=e["A"], B=e["B"], dy=dy, y=e["y"], su=e["su"], dx=e["dx"],
-                                 dA=e["dA"], dB=e["dB"]) for e, pr, dy in zip(self.p, self.wl.projs, dys2)]
+                                 dA=e["dA"], dB=e["dB"], Wq=e["Wq"][2] if e["Wq"] else None)
+                  for e, pr, dy in zip(self.p, self.wl.projs, dys2)]
         return xs2, dys2, projs2
 
     def step(self, lora, stream, projs=None):

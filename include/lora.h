@@ -117,9 +117,39 @@ int lora_linear_bwd(const lora_shape* shape, const lora_bf16* dy, const lora_bf1
                     const lora_bf16* su, lora_bf16* dx, float* dA, float* dB,
                     void* workspace, size_t workspace_bytes, void* stream);
 
+/* Frozen base weight in 4-bit form, dequantized on the fly inside the fused
+ * contractions (Algorithm 1, "On-the-fly Dequantization": W = s * W_q + b,
+ * rematerialized for the forward and again for the backward, never kept):
+ * the bf16 W is never written to memory.  One (s, b) pair per output row n
+ * and group of 64 consecutive input columns k = 64 g .. 64 g + 63; each
+ * dequantized element is bf16(s * q + b), rounded once.  The paper fixes
+ * neither the group size nor the code layout; these are the library's:
+ *   codes   [d_out][d_in / 2] bytes, codes q[n][k] in 0..15.  The
+ *           little-endian 32-bit word m of row n covers k = 8m .. 8m + 7:
+ *           q[n][8m + 2i] in bits 4i .. 4i + 3 and q[n][8m + 2i + 1] in bits
+ *           16 + 4i .. 16 + 4i + 3, for i = 0..3;
+ *   params  [d_out][d_in / 64][2] bf16: (s, b) of row n, group g.
+ * d_in must be a multiple of 256; both pointers 16-byte aligned. */
+typedef struct lora_q4_weight {
+  const uint8_t* codes;
+  const lora_bf16* params;
+} lora_q4_weight;
+
+/* As lora_linear_fwd / lora_linear_bwd with the base weight given as 4-bit
+ * codes (lora_q4_weight) instead of bf16 W.  Returns LORA_EINVAL when d_in is
+ * not a multiple of 256. */
+int lora_linear_fwd_q4(const lora_shape* shape, const lora_bf16* x, const lora_q4_weight* Wq,
+                       const lora_bf16* A, const lora_bf16* B, lora_bf16* y, lora_bf16* su,
+                       void* workspace, size_t workspace_bytes, void* stream);
+int lora_linear_bwd_q4(const lora_shape* shape, const lora_bf16* dy, const lora_bf16* x,
+                       const lora_q4_weight* Wq, const lora_bf16* A, const lora_bf16* B,
+                       const lora_bf16* su, lora_bf16* dx, float* dA, float* dB,
+                       void* workspace, size_t workspace_bytes, void* stream);
+
 /* One adapted projection of a decoder layer (q, k, v, o, gate, up, down).
  * Field meanings and rules as above; pointers a mode does not touch may be
- * NULL (forward: x W A B y [su]; backward: dy x W A B su dA dB [dx]). */
+ * NULL (forward: x W A B y [su]; backward: dy x W A B su dA dB [dx]).  The
+ * base weight is either W (bf16) or Wq (4-bit; then W must be NULL). */
 typedef struct lora_proj {
   lora_shape shape;
   const lora_bf16* x;
@@ -132,6 +162,7 @@ typedef struct lora_proj {
   lora_bf16* dx;
   float* dA;
   float* dB;
+  lora_q4_weight Wq;
 } lora_proj;
 
 /* Workspace bytes for lora_stack_step over `projs` in `mode`. */

@@ -4,4 +4,5 @@ Test infrastructure only: the tests, the smoke check and the benchmark's CPU
 baseline arm are its only users; the CUDA library never imports it.
 """
 from .lora_oracle import (lora_forward, lora_backward, lora_forward_rows,  # noqa: F401
-                          lora_backward_dx_rows, lora_adapter_grads, lora_step)
+                          lora_backward_dx_rows, lora_adapter_grads, lora_step,
+                          unpack_q4, dequant_q4)

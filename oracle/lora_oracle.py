@@ -20,6 +20,12 @@ y = x W^T and dx = dy W are Algorithm 1's y_base = W x and dx = W^T dy
 (column-vector form) transposed to this layout.  W is frozen, so dW is never
 formed (Section "Base Model Quantization": the base weights stay frozen).
 
+Algorithm 1 ("On-the-fly Dequantization") stores the frozen W as integer
+codes W_q with quantization parameters s, b and uses W = s W_q + b for both
+the forward and the backward; `dequant_q4` is that definition for the 4-bit
+layout of the CUDA library's interface (codes 0..15, one (s, b) pair per
+output row and group of 64 input columns; the paper fixes neither).
+
 Every function below is the plain definition: fp64 arithmetic on inputs that
 are exactly widened from bf16, with numpy's matrix product as the only
 library step; no blocking, fusion or reordering.  Pins that hold it to
@@ -88,3 +94,30 @@ def lora_step(proj_inputs, s: float):
         dx, dA, dB, _ = lora_backward(p["dy"], p["x"], p["W"], p["A"], p["B"], s)
         out.append({"y": y, "u": u, "dx": dx, "dA": dA, "dB": dB})
     return out
+
+
+def unpack_q4(codes) -> np.ndarray:
+    """Codes [N, K] (integers 0..15) from the packed bytes [N, K / 2].
+
+    Layout: the little-endian 32-bit word m of a row holds the codes of
+    columns 8m .. 8m + 7; column 8m + 2i sits in bits 4i .. 4i + 3 and column
+    8m + 2i + 1 in bits 16 + 4i .. 16 + 4i + 3 (i = 0..3)."""
+    c = np.ascontiguousarray(codes, dtype=np.uint8)
+    N, half = c.shape
+    words = c.view("<u4").astype(np.int64)  # [N, K / 8]
+    q = np.empty((N, words.shape[1], 8), dtype=np.int64)
+    for i in range(4):
+        q[:, :, 2 * i] = (words >> (4 * i)) & 15
+        q[:, :, 2 * i + 1] = (words >> (16 + 4 * i)) & 15
+    return q.reshape(N, 2 * half)
+
+
+def dequant_q4(codes, s, b) -> np.ndarray:
+    """Algorithm 1's dequantization W = s * W_q + b in fp64.
+
+    codes: packed bytes [N, K / 2] (see unpack_q4); s, b: [N, K / 64] per
+    output row and group of 64 consecutive input columns."""
+    q = unpack_q4(codes).astype(np.float64)
+    s, b = _f64(s), _f64(b)
+    g = np.arange(q.shape[1]) // 64
+    return s[:, g] * q + b[:, g]

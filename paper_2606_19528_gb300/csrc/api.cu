@@ -147,6 +147,20 @@ int make_map(CUtensorMap* m, const void* ptr, uint64_t inner, uint64_t outer, ui
   return r == CUDA_SUCCESS ? LORA_OK : LORA_ECUDA;
 }
 
+// 2-D tensor map of `dtype` elements over a row-major [outer, inner] matrix
+// with row stride `ld` elements, no swizzle (staging boxes read by threads).
+int make_map_plain(CUtensorMap* m, CUtensorMapDataType dtype, int esize, const void* ptr, uint64_t inner,
+                   uint64_t outer, uint64_t ld, uint32_t box_inner, uint32_t box_outer) {
+  cuuint64_t dims[2] = {inner, outer};
+  cuuint64_t strides[1] = {ld * (uint64_t)esize};
+  cuuint32_t box[2] = {box_inner, box_outer};
+  cuuint32_t estr[2] = {1, 1};
+  CUresult r = g_encode(m, dtype, 2, const_cast<void*>(ptr), dims, strides, box, estr, CU_TENSOR_MAP_INTERLEAVE_NONE,
+                        CU_TENSOR_MAP_SWIZZLE_NONE, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+                        CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+  return r == CUDA_SUCCESS ? LORA_OK : LORA_ECUDA;
+}
+
 inline size_t up256(size_t x) { return (x + 255) & ~(size_t)255; }
 inline bool aligned16(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
 inline int cdiv(int64_t a, int64_t b) { return (int)((a + b - 1) / b); }
@@ -213,6 +227,8 @@ T* at(void* ws, size_t off) {
 typedef __nv_bfloat16 bf;
 inline const bf* cb(const lora_bf16* p) { return reinterpret_cast<const bf*>(p); }
 inline bf* mb(lora_bf16* p) { return reinterpret_cast<bf*>(p); }
+
+inline bool is_q4(const lora_proj& p) { return p.Wq.codes != nullptr; }
 
 // Adapter operands of one projection's fused contraction.
 struct Operands {
@@ -478,7 +494,17 @@ int add_fwd_problem(GemmBatch& b, const lora_proj& p, const Operands& o) {
   // boxes: 64 rows x 64 (two per CTA)
   if ((rc = make_map(&b.tmA[i], p.x, K, T, K, 64, 128)) != LORA_OK) return rc;
   if ((rc = make_map(&b.tmA2[i], o.s_in, r, T, o.ld_s, 64, 128)) != LORA_OK) return rc;
-  if ((rc = make_map(&b.tmB[i], p.W, K, N, K, 64, 64)) != LORA_OK) return rc;
+  if (is_q4(p)) {
+    // 4-bit W: a box is 64 rows x 64 codes (32 bytes); (s, b) boxes are 128 rows x 4 groups
+    if ((rc = make_map_plain(&b.tmQ[i], CU_TENSOR_MAP_DATA_TYPE_UINT8, 1, p.Wq.codes, K / 2, N, K / 2, 32, 64)) !=
+        LORA_OK)
+      return rc;
+    if ((rc = make_map_plain(&b.tmP[i], CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, p.Wq.params, K / 32, N, K / 32, 8,
+                             128)) != LORA_OK)
+      return rc;
+  } else if ((rc = make_map(&b.tmB[i], p.W, K, N, K, 64, 64)) != LORA_OK) {
+    return rc;
+  }
   if ((rc = make_map(&b.tmB2[i], o.B, r, N, o.ld_b, 64, 64)) != LORA_OK) return rc;
   if ((rc = make_map(&b.tmOut[i], p.y, N, T, N, 64, 32)) != LORA_OK) return rc;
   GemmProblem& g = b.prob[i];
@@ -508,7 +534,17 @@ int add_bwd_problem(GemmBatch& b, const lora_proj& p, const Operands& o) {
   if ((rc = make_map(&b.tmA[i], p.dy, N, T, N, 64, 128)) != LORA_OK) return rc;
   if ((rc = make_map(&b.tmA2[i], o.s_in, r, T, o.ld_s, 64, 128)) != LORA_OK) return rc;
   // W [N, K] read MN-major: inner dimension K (the GEMM's output columns), rows = contraction
-  if ((rc = make_map(&b.tmB[i], p.W, K, N, K, 64, 64)) != LORA_OK) return rc;
+  if (is_q4(p)) {
+    // 4-bit W: a box is 64 rows x 128 codes (64 bytes); (s, b) boxes are 64 rows x 4 groups
+    if ((rc = make_map_plain(&b.tmQ[i], CU_TENSOR_MAP_DATA_TYPE_UINT8, 1, p.Wq.codes, K / 2, N, K / 2, 64, 64)) !=
+        LORA_OK)
+      return rc;
+    if ((rc = make_map_plain(&b.tmP[i], CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, p.Wq.params, K / 32, N, K / 32, 8,
+                             64)) != LORA_OK)
+      return rc;
+  } else if ((rc = make_map(&b.tmB[i], p.W, K, N, K, 64, 64)) != LORA_OK) {
+    return rc;
+  }
   if ((rc = make_map(&b.tmB2[i], p.A, K, r, K, 64, 64)) != LORA_OK) return rc;
   if ((rc = make_map(&b.tmOut[i], p.dx, K, T, K, 64, 32)) != LORA_OK) return rc;
   GemmProblem& g = b.prob[i];
@@ -536,20 +572,31 @@ void init_batch(GemmBatch& b, const DeviceInfo* d) {
 }
 
 // ------------------------------------------------------------------ checks
-int check_fwd_ptrs(const lora_proj& p) {
-  if (!p.x || !p.W || !p.A || !p.B || !p.y) return LORA_ENULL;
-  const void* ps[] = {p.x, p.W, p.A, p.B, p.y, p.su};
-  for (const void* q : ps)
-    if (q && !aligned16(q)) return LORA_EALIGN;
+// The base weight: bf16 W, or 4-bit codes with their (s, b) pairs (exactly one).
+int check_weight(const lora_proj& p) {
+  const bool q = p.Wq.codes != nullptr || p.Wq.params != nullptr;
+  if (q && p.W) return LORA_EINVAL;
+  if (!q) return p.W ? LORA_OK : LORA_ENULL;
+  if (!p.Wq.codes || !p.Wq.params) return LORA_ENULL;
+  if (p.shape.d_in % 256) return LORA_EINVAL;  // whole 64-wide groups, 16-byte (s, b) rows
+  if (!aligned16(p.Wq.codes) || !aligned16(p.Wq.params)) return LORA_EALIGN;
   return LORA_OK;
 }
 
+int check_fwd_ptrs(const lora_proj& p) {
+  if (!p.x || !p.A || !p.B || !p.y) return LORA_ENULL;
+  const void* ps[] = {p.x, p.W, p.A, p.B, p.y, p.su};
+  for (const void* q : ps)
+    if (q && !aligned16(q)) return LORA_EALIGN;
+  return check_weight(p);
+}
+
 int check_bwd_ptrs(const lora_proj& p) {
-  if (!p.dy || !p.x || !p.W || !p.A || !p.B || !p.su || !p.dA || !p.dB) return LORA_ENULL;
+  if (!p.dy || !p.x || !p.A || !p.B || !p.su || !p.dA || !p.dB) return LORA_ENULL;
   const void* ps[] = {p.dy, p.x, p.W, p.A, p.B, p.su, p.dx, p.dA, p.dB};
   for (const void* q : ps)
     if (q && !aligned16(q)) return LORA_EALIGN;
-  return LORA_OK;
+  return check_weight(p);
 }
 
 int check_ws(void* ws, size_t ws_bytes, size_t need) {
@@ -599,19 +646,23 @@ int run_step(const lora_proj* projs, int n, int mode, void* ws, const Plan& pl, 
       ProfScope ps(LORA_KERNEL_ROWPROJ, st);
       if ((rc = launch_rows(rows, arena(ws, pl, kPhFwdRows), d, st)) != LORA_OK) return rc;
     }
-    // heavier problems first so that the static tile walk ends balanced
-    std::vector<int> order(n);
-    for (int i = 0; i < n; ++i) order[i] = i;
-    std::stable_sort(order.begin(), order.end(),
-                     [&](int a, int b) { return projs[a].shape.d_in > projs[b].shape.d_in; });
-    for (int i0 = 0; i0 < n; i0 += kMaxProblems) {
-      GemmBatch b;
-      init_batch(b, d);
-      b.tile_counter = counters + next_counter++;
-      for (int i = i0; i < n && i < i0 + kMaxProblems; ++i)
-        if ((rc = add_fwd_problem(b, projs[order[i]], ops[order[i]])) != LORA_OK) return rc;
-      ProfScope ps(LORA_KERNEL_GEMM_FWD, st);
-      if (launch_fused_gemm(b, false, d->num_sms, st) != cudaSuccess) return LORA_ECUDA;
+    // one launch per batch of bf16-weight, then of 4-bit-weight problems;
+    // heavier problems first so that the tile walk ends balanced
+    for (int q4 = 0; q4 < 2; ++q4) {
+      std::vector<int> order;
+      for (int i = 0; i < n; ++i)
+        if (is_q4(projs[i]) == (q4 != 0)) order.push_back(i);
+      std::stable_sort(order.begin(), order.end(),
+                       [&](int a, int b) { return projs[a].shape.d_in > projs[b].shape.d_in; });
+      for (size_t i0 = 0; i0 < order.size(); i0 += kMaxProblems) {
+        GemmBatch b;
+        init_batch(b, d);
+        b.tile_counter = counters + next_counter++;
+        for (size_t i = i0; i < order.size() && i < i0 + kMaxProblems; ++i)
+          if ((rc = add_fwd_problem(b, projs[order[i]], ops[order[i]])) != LORA_OK) return rc;
+        ProfScope ps(LORA_KERNEL_GEMM_FWD, st);
+        if (launch_fused_gemm(b, false, q4 != 0, d->num_sms, st) != cudaSuccess) return LORA_ECUDA;
+      }
     }
   }
   if (mode & LORA_BWD) {
@@ -673,19 +724,21 @@ int run_step(const lora_proj* projs, int n, int mode, void* ws, const Plan& pl, 
       ProfScope ps(LORA_KERNEL_COLPROJ, st);
       if ((rc = launch_cols(cols, arena(ws, pl, kPhBwdCols), d, d->num_sms, st)) != LORA_OK) return rc;
     }
-    std::vector<int> order;
-    for (int i = 0; i < n; ++i)
-      if (projs[i].dx) order.push_back(i);
-    std::stable_sort(order.begin(), order.end(),
-                     [&](int a, int b) { return projs[a].shape.d_out > projs[b].shape.d_out; });
-    for (size_t i0 = 0; i0 < order.size(); i0 += kMaxProblems) {
-      GemmBatch b;
-      init_batch(b, d);
-      b.tile_counter = counters + next_counter++;
-      for (size_t i = i0; i < order.size() && i < i0 + kMaxProblems; ++i)
-        if ((rc = add_bwd_problem(b, projs[order[i]], ops[order[i]])) != LORA_OK) return rc;
-      ProfScope ps(LORA_KERNEL_GEMM_BWD, st);
-      if (launch_fused_gemm(b, true, d->num_sms, st) != cudaSuccess) return LORA_ECUDA;
+    for (int q4 = 0; q4 < 2; ++q4) {
+      std::vector<int> order;
+      for (int i = 0; i < n; ++i)
+        if (projs[i].dx && is_q4(projs[i]) == (q4 != 0)) order.push_back(i);
+      std::stable_sort(order.begin(), order.end(),
+                       [&](int a, int b) { return projs[a].shape.d_out > projs[b].shape.d_out; });
+      for (size_t i0 = 0; i0 < order.size(); i0 += kMaxProblems) {
+        GemmBatch b;
+        init_batch(b, d);
+        b.tile_counter = counters + next_counter++;
+        for (size_t i = i0; i < order.size() && i < i0 + kMaxProblems; ++i)
+          if ((rc = add_bwd_problem(b, projs[order[i]], ops[order[i]])) != LORA_OK) return rc;
+        ProfScope ps(LORA_KERNEL_GEMM_BWD, st);
+        if (launch_fused_gemm(b, true, q4 != 0, d->num_sms, st) != cudaSuccess) return LORA_ECUDA;
+      }
     }
   }
   return LORA_OK;
@@ -742,7 +795,7 @@ using namespace lora;
 
 extern "C" {
 
-int lora_version(void) { return 100; }
+int lora_version(void) { return 200; }
 
 const char* lora_strerror(int code) {
   switch (code) {
@@ -835,6 +888,43 @@ int lora_linear_bwd(const lora_shape* shape, const lora_bf16* dy, const lora_bf1
   p.dx = dx;
   p.dA = dA;
   p.dB = dB;
+  return lora_stack_step(&p, 1, LORA_BWD, workspace, workspace_bytes, stream);
+}
+
+int lora_linear_fwd_q4(const lora_shape* shape, const lora_bf16* x, const lora_q4_weight* Wq, const lora_bf16* A,
+                       const lora_bf16* B, lora_bf16* y, lora_bf16* su, void* workspace, size_t workspace_bytes,
+                       void* stream) {
+  if (!shape || !Wq) return LORA_ENULL;
+  lora_proj p;
+  memset(&p, 0, sizeof(p));
+  p.shape = *shape;
+  p.x = x;
+  p.Wq = *Wq;
+  p.A = A;
+  p.B = B;
+  p.y = y;
+  p.su = su;
+  if (!p.Wq.codes || !p.Wq.params) return LORA_ENULL;
+  return lora_stack_step(&p, 1, LORA_FWD, workspace, workspace_bytes, stream);
+}
+
+int lora_linear_bwd_q4(const lora_shape* shape, const lora_bf16* dy, const lora_bf16* x, const lora_q4_weight* Wq,
+                       const lora_bf16* A, const lora_bf16* B, const lora_bf16* su, lora_bf16* dx, float* dA,
+                       float* dB, void* workspace, size_t workspace_bytes, void* stream) {
+  if (!shape || !Wq) return LORA_ENULL;
+  lora_proj p;
+  memset(&p, 0, sizeof(p));
+  p.shape = *shape;
+  p.dy = dy;
+  p.x = x;
+  p.Wq = *Wq;
+  p.A = A;
+  p.B = B;
+  p.su = const_cast<lora_bf16*>(su);
+  p.dx = dx;
+  p.dA = dA;
+  p.dB = dB;
+  if (!p.Wq.codes || !p.Wq.params) return LORA_ENULL;
   return lora_stack_step(&p, 1, LORA_BWD, workspace, workspace_bytes, stream);
 }
 

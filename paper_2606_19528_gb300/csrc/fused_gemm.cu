@@ -32,7 +32,20 @@
 //   warp 1      TMEM allocation (both CTAs); tcgen05.mma issuer (even CTA)
 //   warps 2..9  epilogue: TMEM -> registers -> bf16 -> swizzled shared-memory
 //               block (32 rows x 64 columns per warp) -> TMA tensor store
+//               (warps 2..5 with 4-bit weights)
 // Every wait is bounded.
+//
+// 4-bit weights (Algorithm 1's on-the-fly dequantization, W = s * W_q + b with
+// one (s, b) per output row and 64-wide group along d_in): three decoupled
+// rings per CTA.  Warp 0 streams the activation boxes (4 deep); warp 10
+// streams this CTA's codes and (s, b) pairs by TMA (a quarter of the bf16
+// weight bytes, 4 deep); warps 6..9 dequantize a block with packed bf16
+// FMAs straight into the 128-byte-swizzled operand layout the tensor core
+// reads, in a ring of 3 bf16 weight tiles, releasing the code slot at once;
+// warp 11 relays "tile dequantized" to the MMA issuer (one cluster-scope
+// arrive per block and CTA, kept off the dequantizing warps' path); the MMA
+// waits for an activation stage and a weight tile.  Each ring has a
+// block of slack over its refill latency; the bf16 weight never exists in HBM.
 #include "common.cuh"
 #include "kernels.h"
 
@@ -45,21 +58,53 @@ constexpr int kHalf = 128;
 constexpr int kSeg = 256;                         // columns of one MMA / accumulator segment
 constexpr int kBN = 2 * kSeg;                     // tile columns
 constexpr int kBK = 64;
-constexpr int kStages = 4;
 constexpr uint32_t kAHalf = kHalf * kBK * 2;      // 16 KB: this CTA's activation rows
 constexpr uint32_t kBSeg = kHalf * kBK * 2;       // 16 KB: this CTA's weight rows of one segment
-constexpr uint32_t kStageBytes = kAHalf + 2 * kBSeg;
 constexpr uint32_t kBox = 64 * kBK * 2;           // one 64 x 64 box of the weight operand, 8 KB
-constexpr int kEpiWarps = 8;                      // two per TMEM lane quadrant
+constexpr int kEpiWarps = 8;                      // bf16 weights: two per TMEM lane quadrant
 constexpr uint32_t kEpiStage = 32 * 128;          // per-warp output block: 32 rows x 64 bf16, 4 KB
-constexpr int kThreads = (2 + kEpiWarps) * 32;
 constexpr uint32_t kTmemCols = 512;
+constexpr int kConvWarps = 4;                     // 4-bit weights: dequantizing warps per CTA
+
+constexpr int kMaxStages = 4;
+constexpr uint32_t kStageBytes = kAHalf + 2 * kBSeg;  // bf16 weights: activation + weight boxes
+constexpr uint32_t kQCodes = 8192;                    // 4-bit block: 256 weight rows x 64 codes
+constexpr uint32_t kQSlot = kQCodes + 4096;           // + (s, b) boxes
+constexpr int kQStages = 4;                           // 4-bit: code slots
+constexpr int kWStages = 3;                           // 4-bit: dequantized bf16 weight tiles
+constexpr uint32_t kWTile = 2 * kBSeg;
+
+// Shared-memory layout and warps of the bf16-weight (kQ false) and
+// 4-bit-weight (kQ true) kernels.  bf16: 4 stages of [activation | weight],
+// 8 epilogue warps; 4-bit: 4 activation boxes, 3 bf16 weight tiles, 4 code
+// slots, 4 epilogue warps (its tiles take longer, so one warp per TMEM lane
+// quadrant drains in time) and 4 dequantizing warps.
+template <bool kQ>
+struct Cfg {
+  static constexpr int kStages = 4;  // activation ring
+  static constexpr int kEpi = kQ ? 4 : kEpiWarps;
+  static constexpr int kParts = kEpi / 4;          // epilogue warps per TMEM lane quadrant
+  static constexpr int kPartCols = kSeg / kParts;  // columns of a segment per epilogue warp
+  static constexpr uint32_t kRing = kQ ? kStages * kAHalf + kWStages * kWTile + kQStages * kQSlot
+                                       : kStages * kStageBytes;
+  static constexpr int kThreads = (2 + kEpi + (kQ ? kConvWarps + 2 : 0)) * 32;
+  __device__ static uint32_t a_addr(uint32_t base, int s) { return base + (uint32_t)s * (kQ ? kAHalf : kStageBytes); }
+  __device__ static uint32_t w_tile(uint32_t base, int w) { return base + kStages * kAHalf + (uint32_t)w * kWTile; }
+  __device__ static uint32_t q_slot(uint32_t base, int s) {
+    return base + kStages * kAHalf + kWStages * kWTile + (uint32_t)s * kQSlot;
+  }
+};
 constexpr int kTileRing = 4;  // tile ids handed from the scheduler to the other roles
 constexpr long long kDrainNs = 1000000000ll;
 
 struct __align__(8) Ctl {
-  uint64_t full[kStages];          // even CTA: both CTAs' parts of a stage landed
-  uint64_t empty[kStages];         // both CTAs: the pair's MMAs finished reading a stage
+  uint64_t full[kMaxStages];       // even CTA: both CTAs' parts of a stage landed
+  uint64_t empty[kMaxStages];      // both CTAs: the pair's MMAs finished reading a stage
+  uint64_t qfull[kQStages];        // both CTAs, 4-bit: this CTA's codes and (s, b) of a block landed
+  uint64_t qempty[kQStages];       // both CTAs, 4-bit: this CTA's dequantizers read a code slot
+  uint64_t wfull[kWStages];        // even CTA, 4-bit: both CTAs' weight tile dequantized (or loaded)
+  uint64_t convd[kWStages];        // both CTAs, 4-bit: this CTA's dequantizing warps finished a weight tile
+  uint64_t wempty[kWStages];       // both CTAs, 4-bit: the pair's MMAs finished reading a weight tile
   uint64_t tfull;                  // both CTAs: accumulator complete
   uint64_t tempty[2];              // even CTA: both CTAs' epilogues drained a segment
   uint64_t tile_full[kTileRing];   // both CTAs: tile id written
@@ -70,7 +115,10 @@ struct __align__(8) Ctl {
   int abort;
 };
 
-constexpr size_t kSmemBytes = 1024 + (size_t)kStages * kStageBytes + (size_t)kEpiWarps * kEpiStage + sizeof(Ctl);
+template <bool kQ>
+constexpr size_t smem_bytes() {
+  return 1024 + (size_t)Cfg<kQ>::kRing + (size_t)Cfg<kQ>::kEpi * kEpiStage + sizeof(Ctl);
+}
 
 // Problem p, first row m0 and first column n0 of tile t.
 __device__ __forceinline__ void decode_tile(const GemmBatch& b, int t, int& p, int& m0, int& n0) {
@@ -87,14 +135,75 @@ __device__ __forceinline__ void decode_tile(const GemmBatch& b, int t, int& p, i
   }
 }
 
+// Two 4-bit codes -> bf16x2 (s * q + b): the codes sit at bits 0..3 and
+// 16..19 of `w`; OR-ing in the exponent of 128 gives exactly 128 + q per half,
+// the first FMA takes 128 off (exact), the second rounds s * q + b once.
+__device__ __forceinline__ uint32_t dq_pair(uint32_t w, uint32_t s2, uint32_t b2) {
+  const uint32_t v = (w & 0x000F000Fu) | 0x43004300u;
+  uint32_t q, r;
+  asm("fma.rn.bf16x2 %0, %1, %2, %3;" : "=r"(q) : "r"(v), "r"(0x3F803F80u), "r"(0xC300C300u));
+  asm("fma.rn.bf16x2 %0, %1, %2, %3;" : "=r"(r) : "r"(q), "r"(s2), "r"(b2));
+  return r;
+}
+
+// Dequantizes this CTA's weight operand of one contraction block from the
+// staged codes and (s, b) pairs into the 128-byte-swizzled bf16 boxes the MMA
+// reads.  Row rho of box (h, j) is weight column / row col0 = n0 + 256 h +
+// 128 c + 64 j of the tile: the forward's rows are W rows col0 + rho at
+// k-group kb; the backward's are W rows 64 kb + rho at k-group col0 / 64.
+// Staged boxes: forward, codes (h, j) 64 rows x 32 B at 2 KB (2 h + j), (s, b)
+// h 128 rows x 4 groups at 2 KB h; backward, codes h 64 rows x 64 B at 4 KB h,
+// (s, b) h 64 rows x 4 groups at 1 KB h.  A thread takes half rows (32 codes,
+// 16 bytes) ordered so that a warp reads 512 contiguous bytes of codes.
 template <bool kBMn>
-__global__ void __launch_bounds__(kThreads, 1) fused_lora_gemm(const __grid_constant__ GemmBatch b) {
+__device__ __forceinline__ void dequant_stage(uint32_t slot, uint32_t wdst, int ct, int c, int n0, int kb,
+                                              int ncols) {
+  constexpr int kThr = kConvWarps * 32;
+  const uint32_t codes = slot;
+  const uint32_t params = slot + kQCodes;
+#pragma unroll
+  for (int rep = 0; rep < 512 / kThr; ++rep) {
+    const int hu = ct + rep * kThr;  // half row
+    const int half = hu & 1, h = hu >> 8;
+    const int j = kBMn ? (hu >> 1) & 1 : (hu >> 7) & 1;
+    const int rho = kBMn ? (hu >> 2) & 63 : (hu >> 1) & 63;
+    const int colh = n0 + h * kSeg + c * kHalf;
+    if (colh + j * 64 >= ncols) continue;  // box not loaded: its MMA columns are never stored
+    uint32_t csrc, psrc;
+    if (kBMn) {
+      const int g = (colh >> 6) + j, gb = (colh >> 6) & ~3;
+      csrc = codes + (uint32_t)(h * 4096 + rho * 64 + j * 32 + half * 16);
+      psrc = params + (uint32_t)(h * 1024 + rho * 16 + (g - gb) * 4);
+    } else {
+      csrc = codes + (uint32_t)((h * 2 + j) * 2048 + rho * 32 + half * 16);
+      psrc = params + (uint32_t)(h * 2048 + (j * 64 + rho) * 16 + (kb & 3) * 4);
+    }
+    uint32_t w[4], sb;
+    asm volatile("ld.shared.v4.b32 {%0, %1, %2, %3}, [%4];"
+                 : "=r"(w[0]), "=r"(w[1]), "=r"(w[2]), "=r"(w[3]) : "r"(csrc) : "memory");
+    asm volatile("ld.shared.b32 %0, [%1];" : "=r"(sb) : "r"(psrc) : "memory");
+    const uint32_t s2 = (sb & 0xFFFFu) * 0x10001u, b2 = (sb >> 16) * 0x10001u;
+    const uint32_t row = wdst + (uint32_t)(h * kBSeg + j * kBox + rho * 128);
+#pragma unroll
+    for (int m = 0; m < 4; ++m) {
+      const uint32_t o0 = dq_pair(w[m], s2, b2), o1 = dq_pair(w[m] >> 4, s2, b2);
+      const uint32_t o2 = dq_pair(w[m] >> 8, s2, b2), o3 = dq_pair(w[m] >> 12, s2, b2);
+      const uint32_t dst = row + (uint32_t)((((half * 4 + m) ^ (rho & 7)) & 7) << 4);
+      asm volatile("st.shared.v4.b32 [%0], {%1, %2, %3, %4};" ::"r"(dst), "r"(o0), "r"(o1), "r"(o2), "r"(o3)
+                   : "memory");
+    }
+  }
+}
+
+template <bool kBMn, bool kQ>
+__global__ void __launch_bounds__(Cfg<kQ>::kThreads, 1) fused_lora_gemm(const __grid_constant__ GemmBatch b) {
+  constexpr int kStages = Cfg<kQ>::kStages;
   extern __shared__ uint8_t smem_raw[];
   const uint32_t raw = smem_u32(smem_raw);
   const uint32_t base = (raw + 1023u) & ~1023u;
-  const uint32_t epi_base = base + kStages * kStageBytes;  // 1024-aligned output staging blocks
-  Ctl* ctl = reinterpret_cast<Ctl*>(smem_raw + (base - raw) + (size_t)kStages * kStageBytes +
-                                    (size_t)kEpiWarps * kEpiStage);
+  const uint32_t epi_base = base + Cfg<kQ>::kRing;  // 1024-aligned output staging blocks
+  constexpr int kEpi = Cfg<kQ>::kEpi;
+  Ctl* ctl = reinterpret_cast<Ctl*>(smem_raw + (base - raw) + (size_t)Cfg<kQ>::kRing + (size_t)kEpi * kEpiStage);
   volatile int* abort_flag = &ctl->abort;
 
   const int warp = threadIdx.x >> 5;
@@ -104,15 +213,25 @@ __global__ void __launch_bounds__(kThreads, 1) fused_lora_gemm(const __grid_cons
 
   if (threadIdx.x == 0) {
     for (int s = 0; s < kStages; ++s) {
+      // producer (expect_tx), plus every dequantizing warp of both CTAs
       mbar_init(smem_u32(&ctl->full[s]), 1);
       mbar_init(smem_u32(&ctl->empty[s]), 1);
     }
+    for (int q = 0; q < kQStages; ++q) {
+      mbar_init(smem_u32(&ctl->qfull[q]), 1);
+      mbar_init(smem_u32(&ctl->qempty[q]), kConvWarps);
+    }
+    for (int w = 0; w < kWStages; ++w) {
+      mbar_init(smem_u32(&ctl->wfull[w]), 2);  // the relay of each CTA
+      mbar_init(smem_u32(&ctl->convd[w]), kConvWarps);
+      mbar_init(smem_u32(&ctl->wempty[w]), 1);
+    }
     mbar_init(smem_u32(&ctl->tfull), 1);
-    for (int h = 0; h < 2; ++h) mbar_init(smem_u32(&ctl->tempty[h]), 2 * kEpiWarps);
+    for (int h = 0; h < 2; ++h) mbar_init(smem_u32(&ctl->tempty[h]), 2 * kEpi);
     for (int k = 0; k < kTileRing; ++k) {
       mbar_init(smem_u32(&ctl->tile_full[k]), 1);
-      // MMA thread, epilogue warps of both CTAs, producer of the odd CTA
-      mbar_init(smem_u32(&ctl->tile_empty[k]), 2 + 2 * kEpiWarps);
+      // MMA thread, epilogue (and dequantizing, code producer, relay) warps of both CTAs, producer of the odd CTA
+      mbar_init(smem_u32(&ctl->tile_empty[k]), 2 + 2 * kEpi + (kQ ? 2 * kConvWarps + 4 : 0));
     }
     mbar_init(smem_u32(&ctl->drain), 1);
     ctl->abort = 0;
@@ -122,7 +241,12 @@ __global__ void __launch_bounds__(kThreads, 1) fused_lora_gemm(const __grid_cons
     for (int q = 0; q < b.num_problems; ++q) {
       tma_prefetch_desc(&b.tmA[q]);
       tma_prefetch_desc(&b.tmA2[q]);
-      tma_prefetch_desc(&b.tmB[q]);
+      if (kQ) {
+        tma_prefetch_desc(&b.tmQ[q]);
+        tma_prefetch_desc(&b.tmP[q]);
+      } else {
+        tma_prefetch_desc(&b.tmB[q]);
+      }
       tma_prefetch_desc(&b.tmB2[q]);
       tma_prefetch_desc(&b.tmOut[q]);
     }
@@ -178,29 +302,34 @@ __global__ void __launch_bounds__(kThreads, 1) fused_lora_gemm(const __grid_cons
           for (int cc = 0; cc < 2; ++cc)
             for (int j = 0; j < 2; ++j) boxes += box_ok(h, cc, j) ? 1u : 0u;
         // bytes landing in this pair per stage (signalled on the even CTA)
-        const uint32_t tx_pair = (m0 < Q.M ? kAHalf : 0u) + (m0 + kHalf < Q.M ? kAHalf : 0u) + kBox * boxes;
+        const uint32_t tx_a = (m0 < Q.M ? kAHalf : 0u) + (m0 + kHalf < Q.M ? kAHalf : 0u);
+        const uint32_t tx_pair = tx_a + kBox * boxes;
         bool ok = true;
         for (int kb = 0; kb < Q.kb_total; ++kb) {
           if (!mbar_wait_cluster(smem_u32(&ctl->empty[stage]), phase ^ 1u, wc, abort_flag)) {
             ok = false;
             break;
           }
-          if (c == 0) mbar_arrive_expect_tx(smem_u32(&ctl->full[stage]), tx_pair);
-          const uint32_t bar = full_pl + (uint32_t)stage * 8u;
-          const uint32_t a_dst = base + stage * kStageBytes;
-          const uint32_t b_dst = a_dst + kAHalf;
           const bool main = kb < Q.kb_main;
+          // with 4-bit weights the dequantizing warps fill the weight tiles
+          const bool w_tma = !kQ;
+          if (c == 0) mbar_arrive_expect_tx(smem_u32(&ctl->full[stage]), w_tma ? tx_pair : tx_a);
+          const uint32_t bar = full_pl + (uint32_t)stage * 8u;
+          const uint32_t a_dst = Cfg<kQ>::a_addr(base, stage);
+          const uint32_t b_dst = a_dst + kAHalf;
           const int kc = main ? kb * kBK : (kb - Q.kb_main) * kBK;
           const CUtensorMap* ta = main ? &b.tmA[p] : &b.tmA2[p];
           const CUtensorMap* tb = main ? &b.tmB[p] : &b.tmB2[p];
           if (a_mine) tma_load_2d_pair(a_dst, ta, bar, kc, my_m);
+          if (w_tma) {
 #pragma unroll
-          for (int h = 0; h < 2; ++h) {
+            for (int h = 0; h < 2; ++h) {
 #pragma unroll
-            for (int j = 0; j < 2; ++j) {
-              if (!box_ok(h, c, j)) continue;
-              const int col = n0 + h * kSeg + c * kHalf + j * 64;
-              tma_load_2d_pair(b_dst + h * kBSeg + j * kBox, tb, bar, kBMn ? col : kc, kBMn ? kc : col);
+              for (int j = 0; j < 2; ++j) {
+                if (!box_ok(h, c, j)) continue;
+                const int col = n0 + h * kSeg + c * kHalf + j * 64;
+                tma_load_2d_pair(b_dst + h * kBSeg + j * kBox, tb, bar, kBMn ? col : kc, kBMn ? kc : col);
+              }
             }
           }
           if (++stage == kStages) {
@@ -218,6 +347,7 @@ __global__ void __launch_bounds__(kThreads, 1) fused_lora_gemm(const __grid_cons
       constexpr uint16_t pair_mask = 0x3;
       int stage = 0;
       uint32_t phase = 0;
+      uint32_t wseq = 0;  // 4-bit: contraction blocks so far (weight tile wseq % 2)
       bool ok = true;
       for (int it = 0; ok; ++it) {
         const int slot = it % kTileRing;
@@ -240,9 +370,14 @@ __global__ void __launch_bounds__(kThreads, 1) fused_lora_gemm(const __grid_cons
             ok = false;
             break;
           }
+          const int wt = (int)(wseq % kWStages);
+          if (kQ && !mbar_wait_cluster(smem_u32(&ctl->wfull[wt]), (wseq / kWStages) & 1u, wc, abort_flag)) {
+            ok = false;
+            break;
+          }
           tc_fence_after();
-          const uint32_t a_addr = base + stage * kStageBytes;
-          const uint32_t b_addr = a_addr + kAHalf;
+          const uint32_t a_addr = Cfg<kQ>::a_addr(base, stage);
+          const uint32_t b_addr = kQ ? Cfg<kQ>::w_tile(base, wt) : a_addr + kAHalf;
           const int nk = kb < Q.kb_main ? kBK / 16 : min(kBK / 16, (Q.r - (kb - Q.kb_main) * kBK + 15) / 16);
           for (int h = 0; h < 2; ++h) {
             if (kb == 0) {
@@ -263,6 +398,8 @@ __global__ void __launch_bounds__(kThreads, 1) fused_lora_gemm(const __grid_cons
           }
           if (!ok) break;
           umma_commit_pair_mc(smem_u32(&ctl->empty[stage]), pair_mask);
+          if (kQ) umma_commit_pair_mc(smem_u32(&ctl->wempty[wt]), pair_mask);
+          ++wseq;
           if (++stage == kStages) {
             stage = 0;
             phase ^= 1u;
@@ -274,10 +411,10 @@ __global__ void __launch_bounds__(kThreads, 1) fused_lora_gemm(const __grid_cons
       // completes in both CTAs of the pair once every MMA issued above has finished
       umma_commit_pair_mc(smem_u32(&ctl->drain), pair_mask);
     }
-  } else {
+  } else if (warp < 2 + kEpi) {
     // ------------------------------------------------------------ epilogue (both CTAs)
     const int q = warp & 3;                 // TMEM lane quadrant this warp may access
-    const int part = (warp - 2) >> 2;       // which 128 columns of each segment
+    const int part = (warp - 2) >> 2;       // which kPartCols columns of each segment
     const uint32_t tempty_pl = mapa_shared(smem_u32(&ctl->tempty[0]), 0);
     for (int it = 0;; ++it) {
       const int slot = it % kTileRing;
@@ -298,8 +435,8 @@ __global__ void __launch_bounds__(kThreads, 1) fused_lora_gemm(const __grid_cons
       const int row0 = m0 + c * kHalf + q * 32;  // first of this warp's 32 rows
       const uint32_t stg = epi_base + (uint32_t)(warp - 2) * kEpiStage;
       for (int h = 0; h < 2; ++h) {
-        for (int cc = 0; cc < kHalf; cc += 64) {
-          const int col0 = h * kSeg + part * kHalf + cc;  // tile column of this 64-column block
+        for (int cc = 0; cc < Cfg<kQ>::kPartCols; cc += 64) {
+          const int col0 = h * kSeg + part * Cfg<kQ>::kPartCols + cc;  // tile column of this 64-column block
           if (n0 + col0 >= Q.N || row0 >= Q.M) break;     // uniform across the warp
           const uint32_t taddr = tmem_base + ((uint32_t)(q * 32) << 16) + (uint32_t)col0;
           uint32_t v[32], w[32];
@@ -336,6 +473,161 @@ __global__ void __launch_bounds__(kThreads, 1) fused_lora_gemm(const __grid_cons
     }
     // the output must be written before the CTA exits
     if (lane == 0) bulk_wait0();
+  } else if (kQ && warp < 2 + kEpi + kConvWarps) {
+    // ------------------------------------------------------------ weight dequantizers (both CTAs)
+    const int cw = warp - 2 - kEpi;
+    const int ct = cw * 32 + lane;
+    const uint32_t wfull_pl = mapa_shared(smem_u32(&ctl->wfull[0]), 0);  // adapter-block TMA completions
+    int qs = 0;          // code slot of the next main block
+    uint32_t qpar = 0;   // its qfull parity
+    uint32_t wseq = 0;   // contraction blocks so far: weight tile wseq % kWStages
+    for (int it = 0;; ++it) {
+      const int slot = it % kTileRing;
+      bool got = mbar_wait_cluster(smem_u32(&ctl->tile_full[slot]), (uint32_t)((it / kTileRing) & 1), wc, abort_flag);
+      got = __all_sync(0xffffffffu, got);
+      if (!got) break;
+      const int t = *reinterpret_cast<volatile int*>(&ctl->tile_id[slot]);
+      __syncwarp();
+      if (lane == 0) mbar_arrive_cluster(tile_empty_root + (uint32_t)slot * 8u);
+      if (t < 0) break;
+      int p, m0, n0;
+      decode_tile(b, t, p, m0, n0);
+      const GemmProblem& Q = b.prob[p];
+      auto box_ok = [&](int h, int cc, int j) { return n0 + h * kSeg + cc * kHalf + j * 64 < Q.N; };
+      bool ok = true;
+      for (int kb = 0; kb < Q.kb_total; ++kb) {
+        const bool main = kb < Q.kb_main;
+        const int wt = (int)(wseq % kWStages);
+        // the weight tile's previous contents are consumed by the MMAs
+        ok = mbar_wait_cluster(smem_u32(&ctl->wempty[wt]), ((wseq / kWStages) & 1u) ^ 1u, wc, abort_flag);
+        if (ok && main) ok = mbar_wait(smem_u32(&ctl->qfull[qs]), qpar, wc, abort_flag);
+        ok = __all_sync(0xffffffffu, ok);
+        if (!ok) break;
+        const uint32_t wdst = Cfg<kQ>::w_tile(base, wt);
+        if (main) {
+          dequant_stage<kBMn>(Cfg<kQ>::q_slot(base, qs), wdst, ct, c, n0, kb, Q.N);
+          fence_proxy_async_smem();  // the tensor core reads what these threads wrote
+          __syncwarp();
+          if (lane == 0) {
+            mbar_arrive(smem_u32(&ctl->qempty[qs]));  // the code slot may be refilled
+            mbar_arrive(smem_u32(&ctl->convd[wt]));
+          }
+          if (++qs == kQStages) {
+            qs = 0;
+            qpar ^= 1u;
+          }
+        } else {
+          // adapter block: the bf16 rank-side boxes go straight into the weight tile by TMA
+          if (cw == 0 && lane == 0) {
+            const int kc = (kb - Q.kb_main) * kBK;
+            const uint32_t bar = wfull_pl + (uint32_t)wt * 8u;
+            if (c == 0) {
+              // before this CTA's relay can arrive: the phase cannot complete without these bytes
+              uint32_t boxes = 0;
+              for (int h = 0; h < 2; ++h)
+                for (int cc = 0; cc < 2; ++cc)
+                  for (int j = 0; j < 2; ++j) boxes += box_ok(h, cc, j) ? 1u : 0u;
+              mbar_expect_tx(smem_u32(&ctl->wfull[wt]), kBox * boxes);
+            }
+            for (int h = 0; h < 2; ++h) {
+              for (int j = 0; j < 2; ++j) {
+                if (!box_ok(h, c, j)) continue;
+                const int col = n0 + h * kSeg + c * kHalf + j * 64;
+                tma_load_2d_pair(wdst + h * kBSeg + j * kBox, &b.tmB2[p], bar, kBMn ? col : kc, kBMn ? kc : col);
+              }
+            }
+          }
+          __syncwarp();
+          if (lane == 0) mbar_arrive(smem_u32(&ctl->convd[wt]));
+        }
+        ++wseq;
+      }
+      if (!ok) break;
+    }
+  } else if (kQ && warp == 2 + kEpi + kConvWarps + 1) {
+    // ------------------------------------------------------------ relay (both CTAs)
+    if (lane == 0) {
+      const uint32_t wfull_pl = mapa_shared(smem_u32(&ctl->wfull[0]), 0);
+      uint32_t wseq = 0;
+      for (int it = 0;; ++it) {
+        const int slot = it % kTileRing;
+        if (!mbar_wait_cluster(smem_u32(&ctl->tile_full[slot]), (uint32_t)((it / kTileRing) & 1), wc, abort_flag))
+          break;
+        const int t = *reinterpret_cast<volatile int*>(&ctl->tile_id[slot]);
+        mbar_arrive_cluster(tile_empty_root + (uint32_t)slot * 8u);
+        if (t < 0) break;
+        int p, m0, n0;
+        decode_tile(b, t, p, m0, n0);
+        bool ok = true;
+        for (int kb = 0; kb < b.prob[p].kb_total; ++kb, ++wseq) {
+          const int wt = (int)(wseq % kWStages);
+          if (!mbar_wait(smem_u32(&ctl->convd[wt]), (wseq / kWStages) & 1u, wc, abort_flag)) {
+            ok = false;
+            break;
+          }
+          // cumulative release: covers the dequantizing warps' writes this thread acquired
+          mbar_arrive_cluster(wfull_pl + (uint32_t)wt * 8u);
+        }
+        if (!ok) break;
+      }
+    }
+  } else if (kQ) {
+    // ------------------------------------------------------------ code producer (both CTAs)
+    if (lane == 0) {
+      int qs = 0;
+      uint32_t qpar = 0;
+      for (int it = 0;; ++it) {
+        const int slot = it % kTileRing;
+        if (!mbar_wait_cluster(smem_u32(&ctl->tile_full[slot]), (uint32_t)((it / kTileRing) & 1), wc, abort_flag))
+          break;
+        const int t = *reinterpret_cast<volatile int*>(&ctl->tile_id[slot]);
+        mbar_arrive_cluster(tile_empty_root + (uint32_t)slot * 8u);
+        if (t < 0) break;
+        int p, m0, n0;
+        decode_tile(b, t, p, m0, n0);
+        const GemmProblem& Q = b.prob[p];
+        auto box_ok = [&](int h, int j) { return n0 + h * kSeg + c * kHalf + j * 64 < Q.N; };
+        // bytes of this CTA's code and (s, b) boxes per block
+        uint32_t tx_q = 0;
+        for (int h = 0; h < 2; ++h) {
+          if (kBMn) {
+            tx_q += box_ok(h, 0) ? 4096u + 1024u : 0u;
+          } else {
+            tx_q += box_ok(h, 0) ? 2048u : 0u;
+            for (int j = 0; j < 2; ++j) tx_q += box_ok(h, j) ? 2048u : 0u;
+          }
+        }
+        bool ok = true;
+        for (int kb = 0; kb < Q.kb_main; ++kb) {
+          if (!mbar_wait(smem_u32(&ctl->qempty[qs]), qpar ^ 1u, wc, abort_flag)) {
+            ok = false;
+            break;
+          }
+          const uint32_t qbar = smem_u32(&ctl->qfull[qs]);
+          const uint32_t codes = Cfg<kQ>::q_slot(base, qs);
+          const uint32_t params = codes + kQCodes;
+          mbar_arrive_expect_tx(qbar, tx_q);
+          for (int h = 0; h < 2; ++h) {
+            const int colh = n0 + h * kSeg + c * kHalf;
+            if (!box_ok(h, 0)) continue;
+            if (kBMn) {
+              // W rows 64 kb ..; this CTA's 128 output columns = 64 code bytes, 2 groups
+              tma_load_2d(codes + h * 4096, &b.tmQ[p], qbar, colh / 2, kb * kBK);
+              tma_load_2d(params + h * 1024, &b.tmP[p], qbar, ((colh >> 6) & ~3) * 2, kb * kBK);
+            } else {
+              for (int j = 0; j < 2; ++j)
+                if (box_ok(h, j)) tma_load_2d(codes + (h * 2 + j) * 2048, &b.tmQ[p], qbar, kb * 32, colh + j * 64);
+              tma_load_2d(params + h * 2048, &b.tmP[p], qbar, (kb & ~3) * 2, colh);
+            }
+          }
+          if (++qs == kQStages) {
+            qs = 0;
+            qpar ^= 1u;
+          }
+        }
+        if (!ok) break;
+      }
+    }
   }
 
   // ------------------------------------------------------------ teardown
@@ -362,21 +654,27 @@ __global__ void __launch_bounds__(kThreads, 1) fused_lora_gemm(const __grid_cons
 
 }  // namespace
 
-size_t fused_gemm_smem_bytes() { return kSmemBytes; }
+size_t fused_gemm_smem_bytes() { return smem_bytes<false>(); }
 
-cudaError_t launch_fused_gemm(const GemmBatch& batch, bool b_mn_major, int num_sms, cudaStream_t stream) {
-  static bool attr_done[2] = {false, false};
-  const void* fn = b_mn_major ? (const void*)fused_lora_gemm<true> : (const void*)fused_lora_gemm<false>;
-  if (!attr_done[b_mn_major]) {
-    cudaError_t e = cudaFuncSetAttribute(fn, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)kSmemBytes);
+template <bool kBMn, bool kQ>
+cudaError_t launch_variant(const GemmBatch& batch, int pairs, cudaStream_t stream) {
+  constexpr size_t smem = smem_bytes<kQ>();
+  static bool attr_done = false;
+  if (!attr_done) {
+    cudaError_t e = cudaFuncSetAttribute(fused_lora_gemm<kBMn, kQ>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                         (int)smem);
     if (e != cudaSuccess) return e;
-    attr_done[b_mn_major] = true;
+    attr_done = true;
   }
+  return launch_kernel(fused_lora_gemm<kBMn, kQ>, dim3((unsigned)(2 * pairs)), dim3(Cfg<kQ>::kThreads), smem,
+                       stream, 2, batch);
+}
+
+cudaError_t launch_fused_gemm(const GemmBatch& batch, bool b_mn_major, bool q4, int num_sms, cudaStream_t stream) {
   if (batch.total_tiles <= 0) return cudaSuccess;
   const int pairs = batch.total_tiles < num_sms / 2 ? batch.total_tiles : num_sms / 2;
-  const dim3 grid((unsigned)(2 * pairs)), block(kThreads);
-  return b_mn_major ? launch_kernel(fused_lora_gemm<true>, grid, block, kSmemBytes, stream, 2, batch)
-                    : launch_kernel(fused_lora_gemm<false>, grid, block, kSmemBytes, stream, 2, batch);
+  if (q4) return b_mn_major ? launch_variant<true, true>(batch, pairs, stream) : launch_variant<false, true>(batch, pairs, stream);
+  return b_mn_major ? launch_variant<true, false>(batch, pairs, stream) : launch_variant<false, false>(batch, pairs, stream);
 }
 
 int gemm_tile_m() { return kBM; }

@@ -63,6 +63,7 @@ struct GemmProblem {
   int kb_total;        // base + adapter blocks
   int m_fast;          // 1: consecutive tiles walk M (the weight tile stays put)
   int num_m_tiles;
+
 };
 
 // One launch: up to kMaxProblems independent fused contractions.
@@ -75,6 +76,9 @@ struct GemmBatch {
   CUtensorMap tmB[kMaxProblems];
   CUtensorMap tmB2[kMaxProblems];
   CUtensorMap tmOut[kMaxProblems];  // out [M, N]: 64 columns x 32 rows boxes, 128-byte swizzle
+  // 4-bit weights only: codes [d_out, d_in / 2] bytes and (s, b) pairs [d_out, d_in / 64, 2] bf16
+  CUtensorMap tmQ[kMaxProblems];
+  CUtensorMap tmP[kMaxProblems];
   GemmProblem prob[kMaxProblems];
   int num_problems;
   int total_tiles;
@@ -83,7 +87,9 @@ struct GemmBatch {
   long long limit_ns;
 };
 
-cudaError_t launch_fused_gemm(const GemmBatch& batch, bool b_mn_major, int num_sms, cudaStream_t stream);
+// b_mn_major: the weight operand is contracted over its rows (backward);
+// q4: every problem's base weight is given as 4-bit codes (tmQ, tmP).
+cudaError_t launch_fused_gemm(const GemmBatch& batch, bool b_mn_major, bool q4, int num_sms, cudaStream_t stream);
 size_t fused_gemm_smem_bytes();
 int gemm_tile_m();
 int gemm_tile_n();

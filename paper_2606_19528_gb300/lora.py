@@ -31,7 +31,8 @@ LORA_BWD = 2
 LORA_FWD_BWD = 3
 
 # every symbol that include/lora.h declares
-EXPORTS = ("lora_workspace_size", "lora_linear_fwd", "lora_linear_fwd_noalloc", "lora_linear_bwd", "lora_stack_workspace_size",
+EXPORTS = ("lora_workspace_size", "lora_linear_fwd", "lora_linear_fwd_noalloc", "lora_linear_bwd",
+           "lora_linear_fwd_q4", "lora_linear_bwd_q4", "lora_stack_workspace_size",
            "lora_stack_step", "lora_read_status", "lora_set_wait_limit_ns", "lora_launch_count",
            "lora_profile_begin", "lora_profile_begin_kinds", "lora_profile_end", "lora_strerror", "lora_version")
 
@@ -56,11 +57,15 @@ class lora_shape(ctypes.Structure):
                 ("rank", ctypes.c_int64), ("scale", ctypes.c_float)]
 
 
+class lora_q4_weight(ctypes.Structure):
+    _fields_ = [("codes", ctypes.c_void_p), ("params", ctypes.c_void_p)]
+
+
 class lora_proj(ctypes.Structure):
     _fields_ = [("shape", lora_shape),
                 ("x", ctypes.c_void_p), ("W", ctypes.c_void_p), ("A", ctypes.c_void_p), ("B", ctypes.c_void_p),
                 ("dy", ctypes.c_void_p), ("y", ctypes.c_void_p), ("su", ctypes.c_void_p), ("dx", ctypes.c_void_p),
-                ("dA", ctypes.c_void_p), ("dB", ctypes.c_void_p)]
+                ("dA", ctypes.c_void_p), ("dB", ctypes.c_void_p), ("Wq", lora_q4_weight)]
 
 
 def library(path: str = _LIB_PATH) -> ctypes.CDLL:
@@ -76,6 +81,9 @@ def library(path: str = _LIB_PATH) -> ctypes.CDLL:
         lib.lora_linear_fwd.argtypes = [P(lora_shape), vp, vp, vp, vp, vp, vp, vp, sz, vp]
         lib.lora_linear_fwd_noalloc.argtypes = [P(lora_shape), vp, vp, vp, vp, vp, vp, vp]
         lib.lora_linear_bwd.argtypes = [P(lora_shape), vp, vp, vp, vp, vp, vp, vp, vp, vp, vp, sz, vp]
+        lib.lora_linear_fwd_q4.argtypes = [P(lora_shape), vp, P(lora_q4_weight), vp, vp, vp, vp, vp, sz, vp]
+        lib.lora_linear_bwd_q4.argtypes = [P(lora_shape), vp, vp, P(lora_q4_weight), vp, vp, vp, vp, vp, vp, vp, sz,
+                                           vp]
         lib.lora_stack_workspace_size.argtypes = [P(lora_proj), i32, i32, P(sz)]
         lib.lora_stack_step.argtypes = [P(lora_proj), i32, i32, vp, sz, vp]
         lib.lora_read_status.argtypes = [vp, P(i32), i32]
@@ -121,10 +129,16 @@ def make_shape(T, d_in, d_out, rank, scale) -> lora_shape:
     return lora_shape(int(T), int(d_in), int(d_out), int(rank), float(scale))
 
 
+def make_q4(codes, params) -> lora_q4_weight:
+    """4-bit base weight: codes [d_out, d_in / 2] bytes and (s, b) pairs
+    [d_out, d_in / 64, 2] bf16 (layout in include/lora.h)."""
+    return lora_q4_weight(_ptr(codes), _ptr(params))
+
+
 def make_proj(shape: lora_shape, x=None, W=None, A=None, B=None, dy=None, y=None, su=None, dx=None, dA=None,
-              dB=None) -> lora_proj:
+              dB=None, Wq=None) -> lora_proj:
     return lora_proj(shape, _ptr(x), _ptr(W), _ptr(A), _ptr(B), _ptr(dy), _ptr(y), _ptr(su), _ptr(dx), _ptr(dA),
-                     _ptr(dB))
+                     _ptr(dB), Wq if Wq is not None else lora_q4_weight(None, None))
 
 
 def lora_workspace_size(shape: lora_shape, mode: int) -> int:
@@ -150,6 +164,19 @@ def lora_linear_bwd(shape, dy, x, W, A, B, su, dx, dA, dB, workspace, workspace_
     _check(library().lora_linear_bwd(ctypes.byref(shape), _ptr(dy), _ptr(x), _ptr(W), _ptr(A), _ptr(B), _ptr(su),
                                      _ptr(dx), _ptr(dA), _ptr(dB), _ptr(workspace), int(workspace_bytes),
                                      _stream(stream)), "lora_linear_bwd")
+
+
+def lora_linear_fwd_q4(shape, x, Wq: lora_q4_weight, A, B, y, su, workspace, workspace_bytes, stream=None) -> None:
+    _check(library().lora_linear_fwd_q4(ctypes.byref(shape), _ptr(x), ctypes.byref(Wq), _ptr(A), _ptr(B), _ptr(y),
+                                        _ptr(su), _ptr(workspace), int(workspace_bytes), _stream(stream)),
+           "lora_linear_fwd_q4")
+
+
+def lora_linear_bwd_q4(shape, dy, x, Wq: lora_q4_weight, A, B, su, dx, dA, dB, workspace, workspace_bytes,
+                       stream=None) -> None:
+    _check(library().lora_linear_bwd_q4(ctypes.byref(shape), _ptr(dy), _ptr(x), ctypes.byref(Wq), _ptr(A), _ptr(B),
+                                        _ptr(su), _ptr(dx), _ptr(dA), _ptr(dB), _ptr(workspace),
+                                        int(workspace_bytes), _stream(stream)), "lora_linear_bwd_q4")
 
 
 def _proj_array(projs):

@@ -22,6 +22,14 @@ Generator (counter based, so any slice can be drawn independently):
 Distributions of the LoRA workloads: x, dy ~ N(0, 1); W ~ N(0, 1/d_in)
 (variance 1/d_in); A ~ U(-1/sqrt(d_in), 1/sqrt(d_in)); B ~ N(0, 0.02**2)
 (standard deviation 0.02), or B = 0 for the LoRA initialisation case.
+
+4-bit base weights (the paper quantizes trained weights with a quantizer it
+does not specify; here the codes and parameters are drawn directly): every
+code byte is floor(256 u), so both 4-bit codes of a byte are uniform on
+0..15 and independent; per (row, 64-column group) the scale is
+s = s0 (0.5 + u1) with s0 = 2 sqrt(3) / (15 sqrt(d_in)) and the offset
+b = -(7.5 + (2 u2 - 1)) s, so that s q + b has mean about 0 and variance
+about 1/d_in, like W above; s and b are rounded to bf16.
 """
 from __future__ import annotations
 
@@ -37,7 +45,7 @@ _M2 = np.uint64(0x94D049BB133111EB)
 _CHUNK = 1 << 22
 
 # tensor identifiers used as stream tags
-TID_X, TID_W, TID_A, TID_B, TID_DY = 1, 2, 3, 4, 5
+TID_X, TID_W, TID_A, TID_B, TID_DY, TID_WQ, TID_WP = 1, 2, 3, 4, 5, 6, 7
 
 
 def _mix(z: np.ndarray) -> np.ndarray:
@@ -170,3 +178,18 @@ def gen_B(seed: int, cfg: int, proj: int, layer: int, N: int, r: int, zero: bool
     if zero:
         return np.zeros((N, r), dtype=np.uint16)
     return normal_bf16(stream_key(seed, cfg, TID_B, proj, layer), (N, r), 0.02)
+
+
+def gen_Wq(seed: int, cfg: int, proj: int, layer: int, N: int, K: int):
+    """4-bit frozen weight of a [N, K] projection: (codes [N, K / 2] uint8,
+    params [N, K / 64, 2] bf16 bits holding (s, b) per row and 64-column group)."""
+    u = uniform01(stream_key(seed, cfg, TID_WQ, proj, layer), N * (K // 2))
+    codes = np.minimum(np.floor(u * 256.0), 255.0).astype(np.uint8).reshape(N, K // 2)
+    G_ = K // 64
+    v = uniform01(stream_key(seed, cfg, TID_WP, proj, layer), 2 * N * G_).reshape(N, G_, 2)
+    s0 = 2.0 * math.sqrt(3.0) / (15.0 * math.sqrt(K))
+    sc = s0 * (0.5 + v[:, :, 0])
+    sc_b = bf16_bits_to_f64(to_bf16_bits(sc))
+    off = -(7.5 + (2.0 * v[:, :, 1] - 1.0)) * sc_b
+    params = np.stack([to_bf16_bits(sc), to_bf16_bits(off)], axis=-1)
+    return codes, params

@@ -35,6 +35,7 @@ class Workload:
     projs: List[Proj] = field(default_factory=list)
     layers: int = 1
     zero_B: bool = False
+    q4: bool = False      # base weights as 4-bit codes (Algorithm 1's on-the-fly dequantization)
 
     @property
     def scale(self) -> float:
@@ -97,6 +98,16 @@ def llama_stack28() -> Workload:
     return Workload("llama3b_stack28_T1024_r16", 5, 1024, 16, 32.0, llama_layer(), layers=28)
 
 
+def llama_layer_T2048_q4() -> Workload:
+    """The Llama layer at T = 2048, r = 16 with every base weight in 4-bit form."""
+    return Workload("llama3b_layer_T2048_r16_q4", 6, 2048, 16, 32.0, llama_layer(), q4=True)
+
+
+def llama_layer_T256(q4: bool = False) -> Workload:
+    """The Llama layer at T = 256, r = 16: few tokens, so the weight bytes bound the contractions."""
+    return Workload("llama3b_layer_T256_r16" + ("_q4" if q4 else ""), 7, 256, 16, 32.0, llama_layer(), q4=q4)
+
+
 BY_NAME = {
     "single": single_small,
     "single_B0": lambda: single_small(True),
@@ -104,4 +115,7 @@ BY_NAME = {
     "llama_layer": llama_layer_T2048,
     "qwen_layer": qwen_layer_T4096,
     "llama_stack28": llama_stack28,
+    "llama_layer_q4": llama_layer_T2048_q4,
+    "llama_layer_T256": llama_layer_T256,
+    "llama_layer_T256_q4": lambda: llama_layer_T256(True),
 }

@@ -174,3 +174,68 @@ def run_pin(pin, fwd, bwd, seed=0):
     if pin is pin_handworked:
         return pin(fwd, bwd)
     return pin(fwd, bwd, rng)
+
+
+# ---------------------------------------------------------------- 4-bit dequantization (Algorithm 1)
+
+def _q4_bytes_loop(codes_row_bytes, k):
+    """Code of column k read bit by bit from the packed row (the interface's
+    layout written out per element, independently of any vectorised unpack)."""
+    m, rem = divmod(k, 8)
+    i, hi = divmod(rem, 2)
+    bit = 4 * i + 16 * hi
+    byte = codes_row_bytes[4 * m + bit // 8]
+    return (byte >> (bit % 8)) & 15
+
+
+def pin_q4_handworked(unpack, dequant):
+    with open(os.path.join(GOLDEN, "q4_dequant_handworked_N2_K128.json")) as f:
+        g = json.load(f)
+    codes = np.array(g["codes"], dtype=np.uint8)
+    W = dequant(codes, np.array(g["s"]), np.array(g["b"]))
+    assert np.array_equal(W, np.array(g["W"], dtype=np.float64)), W
+    y = np.array(g["x"]) @ W.T
+    assert np.array_equal(y, np.array(g["y"], dtype=np.float64)), y
+
+
+def pin_q4_bitwise_layout(unpack, dequant, rng):
+    """Every code of a random packed matrix equals the per-element bit read."""
+    N, K = 3, 64
+    codes = rng.integers(0, 256, size=(N, K // 2), dtype=np.uint8)
+    q = unpack(codes)
+    for n in range(N):
+        row = [int(v) for v in codes[n]]
+        for k in range(K):
+            assert q[n, k] == _q4_bytes_loop(row, k), (n, k)
+
+
+def pin_q4_affine_groups(unpack, dequant, rng):
+    """s = 1, b = 0 gives the codes themselves; each group's (s, b) applies to
+    exactly its 64 columns (checked one group at a time against scalar loops)."""
+    N, K = 2, 192
+    codes = rng.integers(0, 256, size=(N, K // 2), dtype=np.uint8)
+    ones, zeros = np.ones((N, K // 64)), np.zeros((N, K // 64))
+    W = dequant(codes, ones, zeros)
+    for n in range(N):
+        row = [int(v) for v in codes[n]]
+        for k in range(K):
+            assert W[n, k] == _q4_bytes_loop(row, k)
+    s = rng.uniform(0.1, 2.0, (N, K // 64))
+    b = rng.uniform(-1.0, 1.0, (N, K // 64))
+    W = dequant(codes, s, b)
+    for n in range(N):
+        row = [int(v) for v in codes[n]]
+        for k in range(K):
+            g = k // 64
+            assert abs(W[n, k] - (s[n, g] * _q4_bytes_loop(row, k) + b[n, g])) <= 1e-15 * (1 + abs(W[n, k]))
+
+
+Q4_PINS = (pin_q4_handworked, pin_q4_bitwise_layout, pin_q4_affine_groups)
+
+
+def run_q4_pin(pin, unpack, dequant, seed=0):
+    rng = np.random.default_rng(seed)
+    if pin is pin_q4_handworked:
+        pin(unpack, dequant)
+    else:
+        pin(unpack, dequant, rng)

@@ -4,6 +4,7 @@ import numpy as np
 import pytest
 
 import oracle
+from oracle import lora_oracle as O
 from tests import oracle_pins as P
 
 
@@ -89,4 +90,62 @@ def test_pins_catch_planted_mistake(name, fwd, bwd):
             P.run_pin(pin, fwd, bwd)
         except (AssertionError, ValueError):
             failed.append(pin.__name__)
+    assert failed, f"no pin caught the planted mistake {name}"
+
+
+# ---- 4-bit dequantization -----------------------------------------------------
+
+@pytest.mark.parametrize("pin", P.Q4_PINS, ids=lambda p: p.__name__)
+def test_q4_pin(pin):
+    P.run_q4_pin(pin, O.unpack_q4, O.dequant_q4)
+
+
+def _unpack_swapped_halves(codes):
+    q = O.unpack_q4(codes)
+    out = q.copy()
+    out[:, 0::2], out[:, 1::2] = q[:, 1::2], q[:, 0::2]
+    return out
+
+
+def _unpack_nibble_order(codes):
+    c = np.ascontiguousarray(codes, dtype=np.uint8)
+    lo, hi = c & 15, c >> 4
+    return np.stack([lo, hi], axis=-1).reshape(c.shape[0], -1).astype(np.int64)
+
+
+def _dequant_from(unpack):
+    def dq(codes, s, b):
+        q = unpack(codes).astype(np.float64)
+        g = np.arange(q.shape[1]) // 64
+        return np.asarray(s, dtype=np.float64)[:, g] * q + np.asarray(b, dtype=np.float64)[:, g]
+    return dq
+
+
+def _dequant_group_32(codes, s, b):
+    q = O.unpack_q4(codes).astype(np.float64)
+    g = np.minimum(np.arange(q.shape[1]) // 32, np.asarray(s).shape[1] - 1)
+    return np.asarray(s, dtype=np.float64)[:, g] * q + np.asarray(b, dtype=np.float64)[:, g]
+
+
+def _dequant_no_offset(codes, s, b):
+    return O.dequant_q4(codes, s, np.zeros_like(np.asarray(b, dtype=np.float64)))
+
+
+Q4_MISTAKES = {
+    "swapped_pair_halves": (_unpack_swapped_halves, _dequant_from(_unpack_swapped_halves)),
+    "plain_nibble_order": (_unpack_nibble_order, _dequant_from(_unpack_nibble_order)),
+    "group_of_32": (O.unpack_q4, _dequant_group_32),
+    "dropped_offset": (O.unpack_q4, _dequant_no_offset),
+}
+
+
+@pytest.mark.parametrize("name", sorted(Q4_MISTAKES))
+def test_q4_pins_catch_planted_mistake(name):
+    unpack, dequant = Q4_MISTAKES[name]
+    failed = False
+    for pin in P.Q4_PINS:
+        try:
+            P.run_q4_pin(pin, unpack, dequant)
+        except AssertionError:
+            failed = True
     assert failed, f"no pin caught the planted mistake {name}"
