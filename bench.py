@@ -99,10 +99,11 @@ def gen_layer_bits(wl: workloads.Workload, seed: int = 0, T: int | None = None):
 
 
 def gemm_flops(wl: workloads.Workload):
-    """Algorithmic FLOPs of the two fused contractions of one step."""
+    """FLOPs the forward and backward fused-contraction launches of one step
+    execute (every layer; the checkpointed schedule runs each forward twice)."""
     T, r = wl.T, wl.rank
-    fwd = sum(2 * T * (p.d_in + r) * p.d_out for p in wl.projs)
-    bwd = sum(2 * T * (p.d_out + r) * p.d_in for p in wl.projs)
+    fwd = sum(2 * T * (p.d_in + r) * p.d_out for p in wl.projs) * wl.layers * (2 if wl.ckpt else 1)
+    bwd = sum(2 * T * (p.d_out + r) * p.d_in for p in wl.projs) * wl.layers
     return float(fwd), float(bwd)
 
 
@@ -347,6 +348,59 @@ class LayerOnDevice:
                              stream)
 
 
+class StackOnDevice:
+    """`wl.layers` layers of the workload's projections, each with its own
+    buffers (filled with the first layer's synthetic values), run forward of
+    every layer then backward of every layer in reverse, or with the
+    checkpointed schedule (Algorithm 2) when `wl.ckpt`."""
+
+    def __init__(self, wl, bits, torch, lora):
+        self.wl = wl
+        first = LayerOnDevice(wl, bits, torch, lora)
+        self.layers = [first]
+        for _ in range(wl.layers - 1):
+            L = LayerOnDevice.__new__(LayerOnDevice)
+            L.wl, L.torch = wl, torch
+            L.xs = {g: t.clone() for g, t in first.xs.items()}
+            L.p = []
+            for e, pr in zip(first.p, wl.projs):
+                c = {k: (v.clone() if hasattr(v, "clone") else v) for k, v in e.items() if k != "x"}
+                c["x"] = L.xs[pr.group]
+                L.p.append(c)
+            L.projs = [lora.make_proj(lora.make_shape(wl.T, pr.d_in, pr.d_out, wl.rank, wl.scale), x=e["x"],
+                                      W=e["W"], A=e["A"], B=e["B"], dy=e["dy"], y=e["y"], su=e["su"], dx=e["dx"],
+                                      dA=e["dA"], dB=e["dB"], Wq=None) for e, pr in zip(L.p, wl.projs)]
+            self.layers.append(L)
+        self.p = [e for L in self.layers for e in L.p]
+        self.lora = lora
+        layer_projs = [L.projs for L in self.layers]
+        if wl.ckpt:
+            n = lora.lora_stack_ckpt_workspace_size(layer_projs)
+        else:
+            n = max(max(lora.lora_stack_workspace_size(L.projs, m) for m in (lora.LORA_FWD, lora.LORA_BWD))
+                    for L in self.layers)
+        self.ws = torch.empty(max(n, 256), dtype=torch.uint8, device="cuda")
+
+    def step(self, lora, stream, projs=None):
+        if self.wl.ckpt:
+            lora.lora_stack_ckpt([L.projs for L in self.layers], self.ws, self.ws.numel(), stream)
+            return
+        for L in self.layers:
+            lora.lora_stack_step(L.projs, lora.LORA_FWD, self.ws, self.ws.numel(), stream)
+        for L in reversed(self.layers):
+            lora.lora_stack_step(L.projs, lora.LORA_BWD, self.ws, self.ws.numel(), stream)
+
+
+def step_desc(wl) -> str:
+    n = len(wl.projs)
+    if wl.layers == 1:
+        return f"lora_stack_step(LORA_FWD_BWD): {n} forwards then {n} backwards"
+    if wl.ckpt:
+        return (f"lora_stack_ckpt over {wl.layers} layers of {n} projections: every forward saving nothing, "
+                "then per layer from the last a re-forward and the backward (Algorithm 2)")
+    return f"{wl.layers} layers of {n} projections: every forward (saving su), then every backward in reverse"
+
+
 def run_gpu(args, wl):
     import torch
 
@@ -360,7 +414,13 @@ def run_gpu(args, wl):
     peaks, peaks_src = load_peaks()
 
     bits = gen_layer_bits(wl, seed=rank)
-    L = LayerOnDevice(wl, bits, torch, lora)
+    if wl.layers > 1:
+        if wl.q4:
+            raise SystemExit("stack workloads use bf16 weights")
+        L = StackOnDevice(wl, bits, torch, lora)
+        args.no_e2e = True  # the end-to-end copies are defined for the single-layer workloads
+    else:
+        L = LayerOnDevice(wl, bits, torch, lora)
     stream = torch.cuda.current_stream()
     flush = torch.empty(L2_FLUSH_BYTES, dtype=torch.uint8, device=device)
 
@@ -518,9 +578,10 @@ def run_gpu(args, wl):
         "metric": METRIC, "value": world * wl.T / (step_ms / 1e3), "unit": UNIT, "n_gpus": world,
         "steps": K, "warmup": W, "ms_per_step": step_ms, "higher_is_better": True, "scaling": "weak",
         "vs_baseline": None, "dtype": "bf16", "data": "synthetic",
-        "config": {"workload": wl.name, "T": wl.T, "rank": wl.rank, "alpha": wl.alpha,
+        "config": {"workload": wl.name, "T": wl.T, "rank": wl.rank, "alpha": wl.alpha, "layers": wl.layers,
+                   "weights": "4-bit codes + (s, b) per 64-group" if wl.q4 else "bf16",
                    "projections": [f"{p.name} {p.d_in}->{p.d_out}" for p in wl.projs],
-                   "step": "lora_stack_step(LORA_FWD_BWD): 7 forwards then 7 backwards",
+                   "step": step_desc(wl),
                    "flops_per_step": flops,
                    "l2": "256 MiB buffer written between timed steps (outside the step events); "
                          "inputs of one step (W 201 MB + x 71 MB + dy 113 MB) also exceed the 129 MB L2",

@@ -175,6 +175,22 @@ int lora_stack_workspace_size(const lora_proj* projs, int n_proj, int mode, size
 int lora_stack_step(const lora_proj* projs, int n_proj, int mode, void* workspace,
                     size_t workspace_bytes, void* stream);
 
+/* Memory-efficient checkpointed schedule over a stack of layers
+ * (Algorithm 2, "forward twice, backward once"): Stage I runs the forward of
+ * every layer without saving anything (as with su = NULL); Stage III walks
+ * the layers from the last to the first and for each re-runs its forward,
+ * keeping su only in the workspace, then its backward.  Only the layers'
+ * inputs (x, and dy for the backward) need to stay resident between the
+ * stages; no su of any layer outlives its backward.  `projs` holds
+ * n_layers x n_per_layer projections, layer-major, each with x, W (or Wq),
+ * A, B, dy, y, dA, dB (dx optional); their su fields are ignored.  y is
+ * written by both stages (with the same values).  Results equal those of
+ * lora_stack_step(LORA_FWD_BWD) layer by layer.  n_per_layer 1..64.
+ * Returns as lora_stack_step. */
+int lora_stack_ckpt_workspace_size(const lora_proj* projs, int n_layers, int n_per_layer, size_t* bytes);
+int lora_stack_ckpt(const lora_proj* projs, int n_layers, int n_per_layer, void* workspace,
+                    size_t workspace_bytes, void* stream);
+
 /* Waits for `stream`, then reads the device status word that bounded waits
  * set when they expire: *status = LORA_OK or LORA_ETIMEOUT.  reset != 0
  * clears it.  Returns LORA_OK or LORA_ECUDA. */

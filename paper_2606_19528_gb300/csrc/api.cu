@@ -777,6 +777,42 @@ int plan_all(const lora_proj* projs, int n, int mode, Plan* pl) {
   return LORA_OK;
 }
 
+
+// Checkpointed stack (Algorithm 2): scratch for one layer's saved su (the
+// largest layer) and for one stack step.
+int ckpt_layout(const lora_proj* projs, int n_layers, int n_per, size_t* su_bytes, size_t* step_bytes) {
+  if (!projs) return LORA_ENULL;
+  if (n_layers < 1 || n_per < 1 || n_per > 64) return LORA_EINVAL;
+  size_t sb = 0, wb = 0;
+  for (int l = 0; l < n_layers; ++l) {
+    const lora_proj* L = projs + (size_t)l * n_per;
+    size_t su = 0;
+    for (int i = 0; i < n_per; ++i) {
+      int rc = check_shape(&L[i].shape);
+      if (rc != LORA_OK) return rc;
+      su += up256((size_t)L[i].shape.T * (size_t)L[i].shape.rank * 2);
+    }
+    Plan pl;
+    int rc = plan_all(L, n_per, LORA_FWD_BWD, &pl);  // bounds the su-less forward's needs too
+    if (rc != LORA_OK) return rc;
+    sb = std::max(sb, su);
+    wb = std::max(wb, pl.total);
+  }
+  *su_bytes = up256(sb);
+  *step_bytes = wb;
+  return LORA_OK;
+}
+
+// One layer's projections with su placed in the scratch (or NULL).
+void layer_copy(const lora_proj* L, int n_per, uint8_t* su_scratch, std::vector<lora_proj>* out) {
+  out->assign(L, L + n_per);
+  size_t off = 0;
+  for (int i = 0; i < n_per; ++i) {
+    (*out)[i].su = su_scratch ? reinterpret_cast<lora_bf16*>(su_scratch + off) : nullptr;
+    off += up256((size_t)L[i].shape.T * (size_t)L[i].shape.rank * 2);
+  }
+}
+
 }  // namespace
 
 void note_launch() { g_launches.fetch_add(1, std::memory_order_relaxed); }
@@ -964,6 +1000,47 @@ int lora_profile_end(double* ms, int64_t* launches) {
   g_prof.next = 0;
   g_prof.on = false;
   return rc;
+}
+
+int lora_stack_ckpt_workspace_size(const lora_proj* projs, int n_layers, int n_per_layer, size_t* bytes) {
+  if (!bytes) return LORA_ENULL;
+  size_t sb = 0, wb = 0;
+  const int rc = ckpt_layout(projs, n_layers, n_per_layer, &sb, &wb);
+  if (rc != LORA_OK) return rc;
+  *bytes = sb + wb;
+  return LORA_OK;
+}
+
+int lora_stack_ckpt(const lora_proj* projs, int n_layers, int n_per_layer, void* workspace, size_t workspace_bytes,
+                    void* stream) {
+  size_t sb = 0, wb = 0;
+  int rc = ckpt_layout(projs, n_layers, n_per_layer, &sb, &wb);
+  if (rc != LORA_OK) return rc;
+  if ((rc = check_ws(workspace, workspace_bytes, sb + wb)) != LORA_OK) return rc;
+  DeviceInfo* d = nullptr;
+  if ((rc = device_info(&d)) != LORA_OK) return rc;
+  uint8_t* su_scratch = static_cast<uint8_t*>(workspace);
+  void* step_ws = su_scratch + sb;
+  std::vector<lora_proj> layer;
+  // every argument is checked before anything is enqueued
+  for (int l = 0; l < n_layers; ++l) {
+    layer_copy(projs + (size_t)l * n_per_layer, n_per_layer, su_scratch, &layer);
+    for (const lora_proj& p : layer) {
+      if ((rc = check_fwd_ptrs(p)) != LORA_OK) return rc;
+      if ((rc = check_bwd_ptrs(p)) != LORA_OK) return rc;
+    }
+  }
+  // Stage I: every layer's forward, saving nothing
+  for (int l = 0; l < n_layers; ++l) {
+    layer_copy(projs + (size_t)l * n_per_layer, n_per_layer, nullptr, &layer);
+    if ((rc = lora_stack_step(layer.data(), n_per_layer, LORA_FWD, step_ws, wb, stream)) != LORA_OK) return rc;
+  }
+  // Stage III: from the last layer back, re-run its forward saving su, then its backward
+  for (int l = n_layers - 1; l >= 0; --l) {
+    layer_copy(projs + (size_t)l * n_per_layer, n_per_layer, su_scratch, &layer);
+    if ((rc = lora_stack_step(layer.data(), n_per_layer, LORA_FWD_BWD, step_ws, wb, stream)) != LORA_OK) return rc;
+  }
+  return LORA_OK;
 }
 
 int lora_read_status(void* stream, int* status, int reset) {

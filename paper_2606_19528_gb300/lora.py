@@ -33,7 +33,7 @@ LORA_FWD_BWD = 3
 # every symbol that include/lora.h declares
 EXPORTS = ("lora_workspace_size", "lora_linear_fwd", "lora_linear_fwd_noalloc", "lora_linear_bwd",
            "lora_linear_fwd_q4", "lora_linear_bwd_q4", "lora_stack_workspace_size",
-           "lora_stack_step", "lora_read_status", "lora_set_wait_limit_ns", "lora_launch_count",
+           "lora_stack_step", "lora_stack_ckpt_workspace_size", "lora_stack_ckpt", "lora_read_status", "lora_set_wait_limit_ns", "lora_launch_count",
            "lora_profile_begin", "lora_profile_begin_kinds", "lora_profile_end", "lora_strerror", "lora_version")
 
 LORA_KERNEL_GEMM_FWD = 0
@@ -86,6 +86,8 @@ def library(path: str = _LIB_PATH) -> ctypes.CDLL:
                                            vp]
         lib.lora_stack_workspace_size.argtypes = [P(lora_proj), i32, i32, P(sz)]
         lib.lora_stack_step.argtypes = [P(lora_proj), i32, i32, vp, sz, vp]
+        lib.lora_stack_ckpt_workspace_size.argtypes = [P(lora_proj), i32, i32, P(sz)]
+        lib.lora_stack_ckpt.argtypes = [P(lora_proj), i32, i32, vp, sz, vp]
         lib.lora_read_status.argtypes = [vp, P(i32), i32]
         lib.lora_set_wait_limit_ns.argtypes = [i64]
         lib.lora_launch_count.argtypes = []
@@ -195,6 +197,26 @@ def lora_stack_step(projs, mode: int, workspace, workspace_bytes, stream=None) -
     arr = _proj_array(projs)
     _check(library().lora_stack_step(arr, len(projs), mode, _ptr(workspace), int(workspace_bytes),
                                      _stream(stream)), "lora_stack_step")
+
+
+def lora_stack_ckpt_workspace_size(layers) -> int:
+    """`layers`: a list of layers, each a list of projections (same count)."""
+    n_per = len(layers[0])
+    arr = _proj_array([p for L in layers for p in L])
+    n = ctypes.c_size_t(0)
+    _check(library().lora_stack_ckpt_workspace_size(arr, len(layers), n_per, ctypes.byref(n)),
+           "lora_stack_ckpt_workspace_size")
+    return n.value
+
+
+def lora_stack_ckpt(layers, workspace, workspace_bytes, stream=None) -> None:
+    """Checkpointed forward and backward of a stack of layers (see include/lora.h)."""
+    n_per = len(layers[0])
+    if any(len(L) != n_per for L in layers):
+        raise ValueError("every layer needs the same number of projections")
+    arr = _proj_array([p for L in layers for p in L])
+    _check(library().lora_stack_ckpt(arr, len(layers), n_per, _ptr(workspace), int(workspace_bytes),
+                                     _stream(stream)), "lora_stack_ckpt")
 
 
 def lora_read_status(stream=None, reset: bool = True) -> int:

@@ -36,6 +36,7 @@ class Workload:
     layers: int = 1
     zero_B: bool = False
     q4: bool = False      # base weights as 4-bit codes (Algorithm 1's on-the-fly dequantization)
+    ckpt: bool = False    # checkpointed stack schedule (Algorithm 2): forward twice, backward once
 
     @property
     def scale(self) -> float:
@@ -98,6 +99,13 @@ def llama_stack28() -> Workload:
     return Workload("llama3b_stack28_T1024_r16", 5, 1024, 16, 32.0, llama_layer(), layers=28)
 
 
+def llama_stack28_ckpt() -> Workload:
+    """The 28-layer stack under the checkpointed schedule (Algorithm 2): every
+    layer's forward saving nothing, then per layer from the last a re-forward
+    and the backward."""
+    return Workload("llama3b_stack28_T1024_r16_ckpt", 5, 1024, 16, 32.0, llama_layer(), layers=28, ckpt=True)
+
+
 def llama_layer_T2048_q4() -> Workload:
     """The Llama layer at T = 2048, r = 16 with every base weight in 4-bit form."""
     return Workload("llama3b_layer_T2048_r16_q4", 6, 2048, 16, 32.0, llama_layer(), q4=True)
@@ -115,6 +123,7 @@ BY_NAME = {
     "llama_layer": llama_layer_T2048,
     "qwen_layer": qwen_layer_T4096,
     "llama_stack28": llama_stack28,
+    "llama_stack28_ckpt": llama_stack28_ckpt,
     "llama_layer_q4": llama_layer_T2048_q4,
     "llama_layer_T256": llama_layer_T256,
     "llama_layer_T256_q4": lambda: llama_layer_T256(True),
