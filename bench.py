@@ -401,6 +401,193 @@ def step_desc(wl) -> str:
     return f"{wl.layers} layers of {n} projections: every forward (saving su), then every backward in reverse"
 
 
+# ----------------------------------------------------------------------------- LM-head cross entropy
+
+_CE_STATIC = {}
+
+
+def ce_inputs(wl, seed: int = 0, T: int | None = None):
+    """Seeded inputs of the LM-head workload (targets, mask and top-k table
+    with the locality described in synth); E and the table are drawn once."""
+    T = wl.T if T is None else T
+    key = (wl.name, seed)
+    if key not in _CE_STATIC:
+        E = synth.gen_E(seed, wl.cfg, wl.vocab, wl.hidden)
+        tab = synth.gen_topk_table(seed, wl.cfg, wl.vocab, wl.topk, wl.cluster) if wl.topk else None
+        _CE_STATIC[key] = (E, tab)
+    E, tab = _CE_STATIC[key]
+    h = synth.gen_h(seed, wl.cfg, T, wl.hidden)
+    y = synth.gen_targets(seed, wl.cfg, T, wl.vocab, wl.cluster)
+    m = synth.gen_mask(T, wl.trainable)
+    return h, E, y, m, tab
+
+
+def run_gpu_ce(args, wl):
+    """The LM-head node: reduced-vocabulary cross entropy with logits masking."""
+    import torch
+
+    from paper_2606_19528_gb300 import lora
+
+    dist, rank, world = dist_setup()
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    torch.cuda.set_device(local)
+    device = torch.device("cuda", local)
+    lora.library()
+    peaks, peaks_src = load_peaks()
+    h, E, y, m, tab = ce_inputs(wl, seed=rank)
+    dev = lambda b: torch.from_numpy(np.ascontiguousarray(b).view(np.int16)).to(device).view(torch.bfloat16)
+    d_h, d_E = dev(h), dev(E)
+    d_y, d_m = torch.from_numpy(y).to(device), torch.from_numpy(m).to(device)
+    d_tab = torch.from_numpy(tab).to(device) if tab is not None else None
+    loss = torch.empty(1, device=device)
+    token_loss = torch.empty(wl.T, device=device)
+    dh = torch.empty(wl.T, wl.hidden, dtype=torch.bfloat16, device=device)
+    args_ce = lora.make_ce_args(wl.T, wl.hidden, wl.vocab, d_h, d_E, d_y, loss, mask=d_m, topk=d_tab,
+                                ld_topk=wl.topk, k=wl.topk, token_loss=token_loss, dh=dh)
+    ws = torch.empty(lora.lora_ce_workspace_size(args_ce), dtype=torch.uint8, device=device)
+    stream = torch.cuda.current_stream()
+    flush = torch.empty(L2_FLUSH_BYTES, dtype=torch.uint8, device=device)
+
+    def step():
+        return lora.lora_ce_fwd_bwd(args_ce, ws, ws.numel(), stream)
+
+    W, K = max(3, args.warmup), args.steps
+    for _ in range(W):
+        nT, nJ = step()
+    torch.cuda.synchronize()
+    props = torch.cuda.get_device_properties(device)
+    gpu_id = str(getattr(props, "uuid", local))
+    if gpu_id and not gpu_id.startswith("GPU-") and len(gpu_id) == 36:
+        gpu_id = "GPU-" + gpu_id
+    ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in range(K)]
+    clocks = ClockSampler(gpu_id) if rank == 0 else None
+    barrier(dist, device)
+    torch.cuda.synchronize()
+    if clocks:
+        clocks.start()
+        time.sleep(0.3)
+    launches0 = lora.lora_launch_count()
+    lora.lora_profile_begin((lora.LORA_KERNEL_GEMM_FWD, lora.LORA_KERNEL_GEMM_BWD))
+    for i in range(K):
+        flush.zero_()
+        ev[i][0].record(stream)
+        step()
+        ev[i][1].record(stream)
+    torch.cuda.synchronize()
+    kern_ms, _ = lora.lora_profile_end()
+    launches = lora.lora_launch_count() - launches0
+    barrier(dist, device)
+    clk = clocks.stop() if clocks else None
+    step_ms = max_over_ranks(dist, sum(a.elapsed_time(b) for a, b in ev) / K, device)
+
+    # end to end: h, targets and mask from pinned host memory, loss back, every step
+    h_h = torch.from_numpy(np.ascontiguousarray(h).view(np.int16)).pin_memory()
+    h_y, h_m = torch.from_numpy(y).pin_memory(), torch.from_numpy(m).pin_memory()
+    h_loss = torch.empty(1).pin_memory()
+    Ke = max(10, min(K, 100))
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    torch.cuda.synchronize()
+    e0.record(stream)
+    for _ in range(Ke):
+        d_h.view(torch.int16).copy_(h_h, non_blocking=True)
+        d_y.copy_(h_y, non_blocking=True)
+        d_m.copy_(h_m, non_blocking=True)
+        step()
+        h_loss.copy_(loss, non_blocking=True)
+    e1.record(stream)
+    torch.cuda.synchronize()
+    e2e_ms = max_over_ranks(dist, e0.elapsed_time(e1) / Ke, device)
+    if rank != 0:
+        if dist is not None:
+            dist.destroy_process_group()
+        return 0
+    gemm_ms = (kern_ms["gemm_fwd"] + kern_ms["gemm_bwd"]) / K
+    flops = 4.0 * nT * nJ * wl.hidden  # logits and dh contractions
+    sustained = peaks.get("bf16_tflops_sustained", FALLBACK_PEAKS["bf16_tflops_sustained"])
+    burst = peaks.get("bf16_tflops", FALLBACK_PEAKS["bf16_tflops"])
+    gemm_tf = flops / (gemm_ms / 1e3) / 1e12 if gemm_ms > 0 else None
+    line = {
+        "metric": METRIC, "value": world * wl.T / (step_ms / 1e3), "unit": UNIT, "n_gpus": world,
+        "steps": K, "warmup": W, "ms_per_step": step_ms, "higher_is_better": True, "scaling": "weak",
+        "vs_baseline": None, "dtype": "bf16", "data": "synthetic",
+        "config": {"workload": wl.name, "T": wl.T, "vocab": wl.vocab, "hidden": wl.hidden, "topk": wl.topk,
+                   "trainable_fraction": wl.trainable, "trainable_positions": nT, "reduced_vocab": nJ,
+                   "step": "lora_ce_fwd_bwd: index pass, logits of trainable positions over J, softmax CE, dh",
+                   "l2": "256 MiB buffer written between timed steps (outside the step events)",
+                   "parallelism": f"{world} independent replica(s), no collective"},
+        "tflops": flops / (step_ms / 1e3) / 1e12,
+        "roofline": {"kernel": "fused_lora_gemm (logits and dh contractions)", "bound": "tensor",
+                     "achieved": gemm_tf, "peak": sustained, "unit": "TFLOP/s",
+                     "frac": gemm_tf / sustained if gemm_tf else None, "traffic": None,
+                     "peak_kind": f"bf16 sustained, of {peaks_src}", "frac_of_burst": gemm_tf / burst if gemm_tf else None,
+                     "flops_per_step": flops, "ms_per_step": gemm_ms},
+        "gpu_launches": launches,
+        "clocks": clk,
+        "status": lora.lora_strerror(lora.lora_read_status()),
+        "e2e": {"value": world * wl.T / (e2e_ms / 1e3), "unit": UNIT, "ms_per_step": e2e_ms, "steps": Ke,
+                "h2d_bytes_per_step": h_h.numel() * 2 + h_y.numel() * 4 + h_m.numel(),
+                "d2h_bytes_per_step": 4},
+    }
+    if world == 1 and not args.no_cpu_baseline:
+        line["cpu_baseline"] = cpu_baseline_ce(wl, budget_s=args.cpu_budget)
+    print(json.dumps(line), flush=True)
+    if dist is not None:
+        dist.destroy_process_group()
+    return 0
+
+
+def time_oracle_ce(wl, T: int):
+    import oracle
+    h, E, y, m, tab = ce_inputs(wl, T=T)
+    hf, Ef = synth.bf16_bits_to_f64(h), synth.bf16_bits_to_f64(E)
+    mb = m.astype(bool)
+    t0, c0 = time.perf_counter(), time.process_time()
+    J = np.arange(wl.vocab) if tab is None else oracle.reduced_vocab(y, mb, tab, wl.topk)
+    oracle.ce_forward_backward(hf, Ef, y, mb, J)
+    return time.perf_counter() - t0, time.process_time() - c0
+
+
+def cpu_baseline_ce(wl, budget_s: float = 15.0):
+    """The oracle on the host cores over the first positions of the sequence."""
+    T = 64
+    w, _ = time_oracle_ce(wl, T)
+    T = int(min(wl.T, max(64, T * budget_s / max(w, 1e-3) / 2)))
+    w, c = time_oracle_ce(wl, T)
+    return {"value": T / w, "unit": UNIT, "cores": max(1, round(c / w)), "kind": "oracle",
+            "host_cpus": os.cpu_count(),
+            "sample": f"fp64 oracle on the first {T} of {wl.T} positions (same trainable fraction), one run, "
+                      f"{w:.2f} s"}
+
+
+def run_reference_ce(args, wl):
+    """--impl reference for the LM-head workload: the oracle on a bounded sample of positions."""
+    if int(os.environ.get("RANK", "0")) != 0:
+        return 0
+    W, K = args.warmup, args.steps
+    w64, _ = time_oracle_ce(wl, 64)
+    T = int(min(wl.T, max(64, 64 * (90.0 / max(1, W + K)) / max(w64, 1e-3))))
+    for _ in range(W):
+        time_oracle_ce(wl, T)
+    walls, cpus = [], []
+    for _ in range(K):
+        w, c = time_oracle_ce(wl, T)
+        walls.append(w)
+        cpus.append(c)
+    total = sum(walls)
+    value = T * K / total
+    line = {"impl": "reference", "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": args.gpus, "steps": K,
+            "warmup": W, "ms_per_step": 1e3 * total / K, "higher_is_better": True, "scaling": "weak",
+            "vs_baseline": None, "dtype": "f64", "data": "synthetic",
+            "config": {"workload": wl.name, "T": wl.T, "vocab": wl.vocab, "hidden": wl.hidden, "topk": wl.topk,
+                       "sample_positions_per_step": T},
+            "cpu_baseline": {"value": value, "unit": UNIT, "cores": max(1, round(sum(cpus) / total)),
+                             "kind": "oracle", "host_cpus": os.cpu_count(),
+                             "sample": f"first {T} of {wl.T} positions per step"},
+            "e2e": {"value": value, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
+    print(json.dumps(line), flush=True)
+    return 0
+
+
 def run_gpu(args, wl):
     import torch
 
@@ -623,6 +810,8 @@ def main(argv=None):
     ap.add_argument("--cpu-budget", type=float, default=15.0)
     args = ap.parse_args(argv)
     wl = workloads.BY_NAME[args.workload]()
+    if wl.kind == "ce":
+        return run_reference_ce(args, wl) if args.impl == "reference" else run_gpu_ce(args, wl)
     if args.impl == "reference":
         return run_reference(args, wl)
     return run_gpu(args, wl)

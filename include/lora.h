@@ -191,6 +191,43 @@ int lora_stack_ckpt_workspace_size(const lora_proj* projs, int n_layers, int n_p
 int lora_stack_ckpt(const lora_proj* projs, int n_layers, int n_per_layer, void* workspace,
                     size_t workspace_bytes, void* stream);
 
+/* Reduced-vocabulary LM-head cross entropy with logits masking (Sections
+ * "Softmax Approximation" and "Logits Masking").  Hidden states h [T, d]
+ * enter the frozen LM head E [V, d] (one row per vocabulary token).  With
+ * trainable positions T_set (mask) and targets y, the reduced vocabulary is
+ *     J = union over t in T_set of topk[y_t, 0..k-1]     (every token when topk is NULL)
+ * logits are formed only for t in T_set and only over J:
+ *     z_t[j] = h_t . E_j,   loss = sum_{t in T_set} (log sum_{j in J} exp z_t[j] - z_t[y_t])
+ * and the only gradient (E frozen) is
+ *     dh_t = sum_{j in J} (softmax_J(z_t)[j] - [j == y_t]) E_j for t in T_set, 0 elsewhere.
+ * Row i of the top-k table lists tokens by descending similarity to token i
+ * and starts with i (so every trainable target is in J); it is the table
+ * lora_topk_table builds.  The call synchronizes `stream` once, after the
+ * index pass, to size the two contractions by |T_set| and |J| (so it cannot
+ * be captured into a CUDA graph).  Logits are accumulated in fp32 and kept in
+ * fp32; softmax - onehot enters the dh contraction in bf16; dh is bf16.
+ * Requirements: d a multiple of 8, T >= 1, V >= 1, 1 <= k <= ld_topk; targets
+ * of trainable positions in [0, V) and table entries in [0, V) (else
+ * LORA_EINVAL after the index pass, outputs untouched). */
+typedef struct lora_ce_args {
+  int64_t T, d, V;
+  const lora_bf16* h;       /* [T, d] */
+  const lora_bf16* E;       /* [V, d] */
+  const int32_t* targets;   /* [T] */
+  const uint8_t* mask;      /* [T], nonzero = trainable; NULL = every position */
+  const int32_t* topk;      /* [V, ld_topk], or NULL for the full vocabulary */
+  int64_t ld_topk, k;
+  float* loss;              /* [1]: the sum over trainable positions */
+  float* token_loss;        /* [T] or NULL: per-position losses, 0 off T_set */
+  lora_bf16* dh;            /* [T, d] or NULL (no backward) */
+  int32_t* vocab;           /* [V] or NULL: receives J in ascending order */
+  int64_t* counts;          /* host [2] or NULL: receives |T_set| and |J| */
+} lora_ce_args;
+
+/* Workspace bytes for the worst case |T_set| = T, |J| = V. */
+int lora_ce_workspace_size(const lora_ce_args* args, size_t* bytes);
+int lora_ce_fwd_bwd(const lora_ce_args* args, void* workspace, size_t workspace_bytes, void* stream);
+
 /* Waits for `stream`, then reads the device status word that bounded waits
  * set when they expire: *status = LORA_OK or LORA_ETIMEOUT.  reset != 0
  * clears it.  Returns LORA_OK or LORA_ECUDA. */

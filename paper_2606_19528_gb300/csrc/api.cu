@@ -133,17 +133,18 @@ int device_info(DeviceInfo** out) {
   return LORA_OK;
 }
 
-// 2-D bf16 tensor map over a row-major [outer, inner] matrix with row stride
-// `ld` elements, 128-byte swizzle, zero fill outside the matrix.
+// 2-D bf16 (or fp32) tensor map over a row-major [outer, inner] matrix with
+// row stride `ld` elements, 128-byte swizzle, zero fill outside the matrix.
 int make_map(CUtensorMap* m, const void* ptr, uint64_t inner, uint64_t outer, uint64_t ld, uint32_t box_inner,
-             uint32_t box_outer) {
+             uint32_t box_outer, bool f32 = false) {
   cuuint64_t dims[2] = {inner, outer};
-  cuuint64_t strides[1] = {ld * 2};
+  cuuint64_t strides[1] = {ld * (f32 ? 4 : 2)};
   cuuint32_t box[2] = {box_inner, box_outer};
   cuuint32_t estr[2] = {1, 1};
-  CUresult r = g_encode(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void*>(ptr), dims, strides, box, estr,
-                        CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
-                        CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+  CUresult r = g_encode(m, f32 ? CU_TENSOR_MAP_DATA_TYPE_FLOAT32 : CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2,
+                        const_cast<void*>(ptr), dims, strides, box, estr, CU_TENSOR_MAP_INTERLEAVE_NONE,
+                        CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+                        CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
   return r == CUDA_SUCCESS ? LORA_OK : LORA_ECUDA;
 }
 
@@ -813,6 +814,84 @@ void layer_copy(const lora_proj* L, int n_per, uint8_t* su_scratch, std::vector<
   }
 }
 
+
+// ------------------------------------------------------------------ reduced-vocabulary cross entropy
+inline int64_t rup(int64_t x, int64_t m) { return (x + m - 1) / m * m; }
+
+struct CePlan {
+  size_t flags, counts, J, pos, tl, tpos, ycol, rowloss, ht, ej, z, g, dht, tiles, total;
+};
+
+int ce_check(const lora_ce_args* a, CePlan* pl) {
+  if (!a) return LORA_ENULL;
+  if (a->T < 1 || a->V < 1 || a->d < 8 || (a->d % 8) || a->T > (1ll << 24) || a->V > (1ll << 24) ||
+      a->d > (1ll << 20))
+    return LORA_EINVAL;
+  if (a->topk && (a->k < 1 || a->ld_topk < a->k)) return LORA_EINVAL;
+  if (!a->h || !a->E || !a->targets || !a->loss) return LORA_ENULL;
+  const void* ps[] = {a->h, a->E, a->dh};
+  for (const void* q : ps)
+    if (q && !aligned16(q)) return LORA_EALIGN;
+  const int64_t T = a->T, V = a->V, d = a->d;
+  size_t off = 0;
+  auto take = [&](size_t bytes) {
+    const size_t o = off;
+    off += up256(bytes);
+    return o;
+  };
+  pl->tiles = take(16);
+  pl->counts = take(16);
+  pl->flags = take((size_t)V);
+  pl->J = take((size_t)V * 4);
+  pl->pos = take((size_t)V * 4);
+  pl->tl = take((size_t)T * 4);
+  pl->tpos = take((size_t)T * 4);
+  pl->ycol = take((size_t)T * 4);
+  pl->rowloss = take((size_t)T * 4);
+  pl->ht = take((size_t)T * d * 2);
+  pl->ej = take((size_t)V * d * 2);
+  pl->z = take((size_t)T * rup(V, 4) * 4);
+  pl->g = take((size_t)T * rup(V, 8) * 2);
+  pl->dht = take((size_t)T * d * 2);
+  pl->total = off;
+  return LORA_OK;
+}
+
+// One-problem batch of the fused contraction with no adapter slab: out [M, N] = A [M, K] . B, B given
+// as [N, K] (K-major, b_mn false) or [K, N] (MN-major, b_mn true).
+int ce_gemm(const DeviceInfo* d, int* counter, const void* A, int64_t lda, const void* B, int64_t ldb, void* out,
+            int64_t ldo, int64_t M, int64_t N, int64_t K, bool b_mn, bool f32_out, cudaStream_t st) {
+  GemmBatch b;
+  init_batch(b, d);
+  b.tile_counter = counter;
+  int rc;
+  if ((rc = make_map(&b.tmA[0], A, K, M, lda, 64, 128)) != LORA_OK) return rc;
+  b.tmA2[0] = b.tmA[0];
+  if (b_mn) {
+    if ((rc = make_map(&b.tmB[0], B, N, K, ldb, 64, 64)) != LORA_OK) return rc;
+  } else if ((rc = make_map(&b.tmB[0], B, K, N, ldb, 64, 64)) != LORA_OK) {
+    return rc;
+  }
+  b.tmB2[0] = b.tmB[0];
+  if ((rc = make_map(&b.tmOut[0], out, N, M, ldo, f32_out ? 32 : 64, 32, f32_out)) != LORA_OK) return rc;
+  GemmProblem& g = b.prob[0];
+  g.out = static_cast<bf*>(out);
+  g.ldo = (int)ldo;
+  g.M = (int)M;
+  g.N = (int)N;
+  g.Kmain = (int)K;
+  g.r = 0;
+  g.num_n_tiles = cdiv(N, gemm_tile_n());
+  g.num_m_tiles = cdiv(M, gemm_tile_m());
+  g.m_fast = N >= M ? 1 : 0;
+  g.kb_main = cdiv(K, gemm_tile_k());
+  g.kb_total = g.kb_main;
+  g.tile_begin = 0;
+  b.total_tiles = g.num_m_tiles * g.num_n_tiles;
+  b.num_problems = 1;
+  return launch_fused_gemm(b, b_mn, false, d->num_sms, st, f32_out) == cudaSuccess ? LORA_OK : LORA_ECUDA;
+}
+
 }  // namespace
 
 void note_launch() { g_launches.fetch_add(1, std::memory_order_relaxed); }
@@ -1040,6 +1119,85 @@ int lora_stack_ckpt(const lora_proj* projs, int n_layers, int n_per_layer, void*
     layer_copy(projs + (size_t)l * n_per_layer, n_per_layer, su_scratch, &layer);
     if ((rc = lora_stack_step(layer.data(), n_per_layer, LORA_FWD_BWD, step_ws, wb, stream)) != LORA_OK) return rc;
   }
+  return LORA_OK;
+}
+
+int lora_ce_workspace_size(const lora_ce_args* args, size_t* bytes) {
+  if (!bytes) return LORA_ENULL;
+  CePlan pl;
+  const int rc = ce_check(args, &pl);
+  if (rc != LORA_OK) return rc;
+  *bytes = pl.total;
+  return LORA_OK;
+}
+
+int lora_ce_fwd_bwd(const lora_ce_args* a, void* workspace, size_t workspace_bytes, void* stream) {
+  CePlan pl;
+  int rc = ce_check(a, &pl);
+  if (rc != LORA_OK) return rc;
+  if ((rc = check_ws(workspace, workspace_bytes, pl.total)) != LORA_OK) return rc;
+  DeviceInfo* d = nullptr;
+  if ((rc = device_info(&d)) != LORA_OK) return rc;
+  cudaStream_t st = static_cast<cudaStream_t>(stream);
+  const int T = (int)a->T, V = (int)a->V, D = (int)a->d;
+  uint8_t* ws = static_cast<uint8_t*>(workspace);
+  // tile counters, counts and vocabulary flags start at zero
+  if (cudaMemsetAsync(ws, 0, pl.flags + (size_t)V, st) != cudaSuccess) return LORA_ECUDA;
+  CeIndex ix;
+  ix.targets = a->targets;
+  ix.mask = a->mask;
+  ix.T = T;
+  ix.V = V;
+  ix.topk = a->topk;
+  ix.ld_topk = a->ld_topk;
+  ix.k = (int)a->k;
+  ix.flags = ws + pl.flags;
+  ix.J = at<int32_t>(ws, pl.J);
+  ix.pos = at<int32_t>(ws, pl.pos);
+  ix.tl = at<int32_t>(ws, pl.tl);
+  ix.tpos = at<int32_t>(ws, pl.tpos);
+  ix.ycol = at<int32_t>(ws, pl.ycol);
+  ix.counts = at<int32_t>(ws, pl.counts);
+  if (launch_ce_index(ix, st) != cudaSuccess) return LORA_ECUDA;
+  // |T_set| and |J| size the contractions
+  int32_t counts[3] = {0, 0, 0};
+  if (cudaMemcpyAsync(counts, ix.counts, sizeof(counts), cudaMemcpyDeviceToHost, st) != cudaSuccess ||
+      cudaStreamSynchronize(st) != cudaSuccess)
+    return LORA_ECUDA;
+  if (counts[2]) return LORA_EINVAL;
+  const int nT = counts[0], nJ = counts[1];
+  if (a->counts) {
+    a->counts[0] = nT;
+    a->counts[1] = nJ;
+  }
+  float* rowloss = at<float>(ws, pl.rowloss);
+  if (nT > 0) {
+    bf* ht = at<bf>(ws, pl.ht);
+    bf* ej = at<bf>(ws, pl.ej);
+    float* z = at<float>(ws, pl.z);
+    bf* g = at<bf>(ws, pl.g);
+    const int ldz = (int)rup(nJ, 4), ldg = (int)rup(nJ, 8);
+    int* tiles = at<int>(ws, pl.tiles);
+    if (launch_gather_rows(cb(a->h), D, ix.tl, nT, D, ht, st) != cudaSuccess ||
+        launch_gather_rows(cb(a->E), D, ix.J, nJ, D, ej, st) != cudaSuccess)
+      return LORA_ECUDA;
+    {
+      ProfScope ps(LORA_KERNEL_GEMM_FWD, st);
+      if ((rc = ce_gemm(d, tiles, ht, D, ej, D, z, ldz, nT, nJ, D, false, true, st)) != LORA_OK) return rc;
+    }
+    if (launch_ce_rows(z, ldz, nJ, ix.ycol, nT, g, ldg, rowloss, st) != cudaSuccess) return LORA_ECUDA;
+    if (a->dh) {
+      bf* dht = at<bf>(ws, pl.dht);
+      ProfScope ps(LORA_KERNEL_GEMM_BWD, st);
+      if ((rc = ce_gemm(d, tiles + 1, g, ldg, ej, D, dht, D, nT, D, nJ, true, false, st)) != LORA_OK) return rc;
+    }
+  }
+  if (launch_ce_finish(rowloss, nT, ix.tpos, T, a->token_loss, a->loss, st) != cudaSuccess) return LORA_ECUDA;
+  if (a->dh && launch_scatter_rows(at<bf>(ws, pl.dht), ix.tpos, T, D, mb(a->dh), st) != cudaSuccess)
+    return LORA_ECUDA;
+  if (a->vocab && nJ > 0 &&
+      cudaMemcpyAsync(a->vocab, ix.J, (size_t)nJ * 4, cudaMemcpyDeviceToDevice, st) != cudaSuccess)
+    return LORA_ECUDA;
   return LORA_OK;
 }
 

@@ -195,7 +195,7 @@ __device__ __forceinline__ void dequant_stage(uint32_t slot, uint32_t wdst, int 
   }
 }
 
-template <bool kBMn, bool kQ>
+template <bool kBMn, bool kQ, bool kF32 = false>
 __global__ void __launch_bounds__(Cfg<kQ>::kThreads, 1) fused_lora_gemm(const __grid_constant__ GemmBatch b) {
   constexpr int kStages = Cfg<kQ>::kStages;
   extern __shared__ uint8_t smem_raw[];
@@ -435,13 +435,15 @@ __global__ void __launch_bounds__(Cfg<kQ>::kThreads, 1) fused_lora_gemm(const __
       const int row0 = m0 + c * kHalf + q * 32;  // first of this warp's 32 rows
       const uint32_t stg = epi_base + (uint32_t)(warp - 2) * kEpiStage;
       for (int h = 0; h < 2; ++h) {
-        for (int cc = 0; cc < Cfg<kQ>::kPartCols; cc += 64) {
-          const int col0 = h * kSeg + part * Cfg<kQ>::kPartCols + cc;  // tile column of this 64-column block
+        // a staged block is 32 rows x 128 bytes: 64 bf16 columns, or 32 fp32 columns
+        constexpr int kBlockCols = kF32 ? 32 : 64;
+        for (int cc = 0; cc < Cfg<kQ>::kPartCols; cc += kBlockCols) {
+          const int col0 = h * kSeg + part * Cfg<kQ>::kPartCols + cc;  // tile column of this block
           if (n0 + col0 >= Q.N || row0 >= Q.M) break;     // uniform across the warp
           const uint32_t taddr = tmem_base + ((uint32_t)(q * 32) << 16) + (uint32_t)col0;
           uint32_t v[32], w[32];
           tmem_ld_32x32b_x32(taddr, v);
-          tmem_ld_32x32b_x32(taddr + 32u, w);
+          if (!kF32) tmem_ld_32x32b_x32(taddr + 32u, w);
           tmem_ld_wait();
           // the previous block's store must have read the staging buffer
           if (lane == 0) bulk_wait_read0();
@@ -450,11 +452,19 @@ __global__ void __launch_bounds__(Cfg<kQ>::kThreads, 1) fused_lora_gemm(const __
           const uint32_t rbase = stg + (uint32_t)lane * 128u;
 #pragma unroll
           for (int k = 0; k < 8; ++k) {
-            const uint32_t* src = k < 4 ? &v[k * 8] : &w[(k - 4) * 8];
-            const uint32_t a = pack_bf16x2(__uint_as_float(src[0]), __uint_as_float(src[1]));
-            const uint32_t b2 = pack_bf16x2(__uint_as_float(src[2]), __uint_as_float(src[3]));
-            const uint32_t c2 = pack_bf16x2(__uint_as_float(src[4]), __uint_as_float(src[5]));
-            const uint32_t d2 = pack_bf16x2(__uint_as_float(src[6]), __uint_as_float(src[7]));
+            uint32_t a, b2, c2, d2;
+            if (kF32) {
+              a = v[4 * k];
+              b2 = v[4 * k + 1];
+              c2 = v[4 * k + 2];
+              d2 = v[4 * k + 3];
+            } else {
+              const uint32_t* src = k < 4 ? &v[k * 8] : &w[(k - 4) * 8];
+              a = pack_bf16x2(__uint_as_float(src[0]), __uint_as_float(src[1]));
+              b2 = pack_bf16x2(__uint_as_float(src[2]), __uint_as_float(src[3]));
+              c2 = pack_bf16x2(__uint_as_float(src[4]), __uint_as_float(src[5]));
+              d2 = pack_bf16x2(__uint_as_float(src[6]), __uint_as_float(src[7]));
+            }
             const uint32_t dst = rbase + (uint32_t)(((k ^ (lane & 7)) & 7) << 4);
             asm volatile("st.shared.v4.b32 [%0], {%1, %2, %3, %4};" ::"r"(dst), "r"(a), "r"(b2), "r"(c2), "r"(d2)
                          : "memory");
@@ -656,25 +666,33 @@ __global__ void __launch_bounds__(Cfg<kQ>::kThreads, 1) fused_lora_gemm(const __
 
 size_t fused_gemm_smem_bytes() { return smem_bytes<false>(); }
 
-template <bool kBMn, bool kQ>
+template <bool kBMn, bool kQ, bool kF32>
 cudaError_t launch_variant(const GemmBatch& batch, int pairs, cudaStream_t stream) {
   constexpr size_t smem = smem_bytes<kQ>();
   static bool attr_done = false;
   if (!attr_done) {
-    cudaError_t e = cudaFuncSetAttribute(fused_lora_gemm<kBMn, kQ>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+    cudaError_t e = cudaFuncSetAttribute(fused_lora_gemm<kBMn, kQ, kF32>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                          (int)smem);
     if (e != cudaSuccess) return e;
     attr_done = true;
   }
-  return launch_kernel(fused_lora_gemm<kBMn, kQ>, dim3((unsigned)(2 * pairs)), dim3(Cfg<kQ>::kThreads), smem,
+  return launch_kernel(fused_lora_gemm<kBMn, kQ, kF32>, dim3((unsigned)(2 * pairs)), dim3(Cfg<kQ>::kThreads), smem,
                        stream, 2, batch);
 }
 
-cudaError_t launch_fused_gemm(const GemmBatch& batch, bool b_mn_major, bool q4, int num_sms, cudaStream_t stream) {
+cudaError_t launch_fused_gemm(const GemmBatch& batch, bool b_mn_major, bool q4, int num_sms, cudaStream_t stream,
+                              bool f32_out) {
   if (batch.total_tiles <= 0) return cudaSuccess;
   const int pairs = batch.total_tiles < num_sms / 2 ? batch.total_tiles : num_sms / 2;
-  if (q4) return b_mn_major ? launch_variant<true, true>(batch, pairs, stream) : launch_variant<false, true>(batch, pairs, stream);
-  return b_mn_major ? launch_variant<true, false>(batch, pairs, stream) : launch_variant<false, false>(batch, pairs, stream);
+  if (f32_out) {
+    if (b_mn_major || q4) return cudaErrorInvalidValue;  // only the plain forward form writes fp32
+    return launch_variant<false, false, true>(batch, pairs, stream);
+  }
+  if (q4)
+    return b_mn_major ? launch_variant<true, true, false>(batch, pairs, stream)
+                      : launch_variant<false, true, false>(batch, pairs, stream);
+  return b_mn_major ? launch_variant<true, false, false>(batch, pairs, stream)
+                    : launch_variant<false, false, false>(batch, pairs, stream);
 }
 
 int gemm_tile_m() { return kBM; }

@@ -75,7 +75,7 @@ struct GemmBatch {
   CUtensorMap tmA2[kMaxProblems];
   CUtensorMap tmB[kMaxProblems];
   CUtensorMap tmB2[kMaxProblems];
-  CUtensorMap tmOut[kMaxProblems];  // out [M, N]: 64 columns x 32 rows boxes, 128-byte swizzle
+  CUtensorMap tmOut[kMaxProblems];  // out [M, N]: 128-byte rows of 32 rows (64 bf16 or 32 fp32), 128-byte swizzle
   // 4-bit weights only: codes [d_out, d_in / 2] bytes and (s, b) pairs [d_out, d_in / 64, 2] bf16
   CUtensorMap tmQ[kMaxProblems];
   CUtensorMap tmP[kMaxProblems];
@@ -89,7 +89,10 @@ struct GemmBatch {
 
 // b_mn_major: the weight operand is contracted over its rows (backward);
 // q4: every problem's base weight is given as 4-bit codes (tmQ, tmP).
-cudaError_t launch_fused_gemm(const GemmBatch& batch, bool b_mn_major, bool q4, int num_sms, cudaStream_t stream);
+// f32_out (forward form, bf16 weights only): the output is fp32 (tmOut an fp32
+// map with 32 x 32 boxes) instead of bf16.
+cudaError_t launch_fused_gemm(const GemmBatch& batch, bool b_mn_major, bool q4, int num_sms, cudaStream_t stream,
+                              bool f32_out = false);
 size_t fused_gemm_smem_bytes();
 int gemm_tile_m();
 int gemm_tile_n();
@@ -186,6 +189,37 @@ struct TransposeJobs {
   long long max_elems;  // largest n_i * r8_i
 };
 cudaError_t launch_transposes(const TransposeJobs& jobs, cudaStream_t stream);
+
+// ---------------------------------------------------------------- reduced-vocabulary cross entropy
+// Index pass: J (ascending) = union of the trainable targets' first k top-k
+// entries (every token when topk is null), pos[v] = column of v in J or -1,
+// tl = trainable positions (ascending), tpos[t] = row of t in tl or -1,
+// ycol[i] = column in J of the target of tl[i]; counts = {|tl|, |J|, bad
+// input flag}.  flags (V bytes) and counts must be zero at launch.
+struct CeIndex {
+  const int32_t* targets;
+  const uint8_t* mask;  // null: every position trainable
+  int T, V;
+  const int32_t* topk;  // [V, ld_topk], null: full vocabulary
+  long long ld_topk;
+  int k;
+  uint8_t* flags;
+  int32_t *J, *pos, *tl, *tpos, *ycol, *counts;
+};
+cudaError_t launch_ce_index(const CeIndex& a, cudaStream_t stream);
+// dst[i, :] = src[idx[i], :] for i < n (rows of d bf16, d a multiple of 8).
+cudaError_t launch_gather_rows(const __nv_bfloat16* src, long long ld, const int32_t* idx, int n, int d,
+                               __nv_bfloat16* dst, cudaStream_t stream);
+// Per row i < nT of the fp32 logits Z [nT, ldz]: rowloss[i] = lse - z[ycol[i]] and
+// G[i, :] = bf16(softmax - onehot), zero in columns [nJ, ldg).
+cudaError_t launch_ce_rows(const float* Z, int ldz, int nJ, const int32_t* ycol, int nT, __nv_bfloat16* G, int ldg,
+                           float* rowloss, cudaStream_t stream);
+// token_loss[t] (optional) and *loss = sum of rowloss in a fixed order.
+cudaError_t launch_ce_finish(const float* rowloss, int nT, const int32_t* tpos, int T, float* token_loss,
+                             float* loss, cudaStream_t stream);
+// dst[t, :] = src[tpos[t], :] or zeros when tpos[t] < 0.
+cudaError_t launch_scatter_rows(const __nv_bfloat16* src, const int32_t* tpos, int T, int d, __nv_bfloat16* dst,
+                                cudaStream_t stream);
 
 // dst[i, j] = j < r ? src[i * r + j] : 0  for j < ld_dst (zero-padded copy of an [rows, r] matrix).
 cudaError_t launch_pad_cols(const __nv_bfloat16* src, int rows, int r, __nv_bfloat16* dst, int ld_dst,

@@ -1,0 +1,267 @@
+// Reduced-vocabulary LM-head cross entropy with logits masking (Sections
+// "Softmax Approximation" and "Logits Masking"): the index and element-wise
+// passes around the two tensor-core contractions (fused_gemm.cu), which
+// compute the logits of the trainable positions over the reduced vocabulary
+// J and the hidden-state gradient.
+//   vocab_mark      J = union of the trainable targets' first k top-k entries
+//   compact         J and the trainable positions as ascending lists, their
+//                   inverse maps, each trainable target's column in J
+//   gather_rows     rows of h (trainable positions) and of E (J) made dense
+//   ce_rows         per trainable position: log-sum-exp over J, its loss, and
+//                   G = softmax_J - onehot(target) in bf16 for the dh contraction
+//   ce_finish       per-position losses and their sum, in a fixed order
+//   scatter_rows    dh rows of trainable positions, zeros elsewhere
+#include <math.h>
+
+#include "common.cuh"
+#include "kernels.h"
+
+namespace lora {
+
+namespace {
+
+constexpr int kScanThreads = 1024;
+
+__global__ void vocab_mark_kernel(const int32_t* __restrict__ targets, const uint8_t* __restrict__ mask, int T,
+                                  const int32_t* __restrict__ topk, long long ld, int k, int V,
+                                  uint8_t* __restrict__ flags, int32_t* __restrict__ counts) {
+  griddep_wait();
+  griddep_launch_dependents();
+  const long long n = (long long)T * k;
+  for (long long e = blockIdx.x * (long long)blockDim.x + threadIdx.x; e < n; e += (long long)gridDim.x * blockDim.x) {
+    const int t = (int)(e / k), j = (int)(e % k);
+    if (mask && !mask[t]) continue;
+    const int y = targets[t];
+    if (y < 0 || y >= V) {
+      counts[2] = 1;  // invalid target
+      continue;
+    }
+    const int v = topk[(long long)y * ld + j];
+    if (v < 0 || v >= V) {
+      counts[2] = 1;  // invalid table entry
+      continue;
+    }
+    flags[v] = 1;
+  }
+}
+
+// Exclusive scan of one value per thread over the block; returns the total.
+__device__ __forceinline__ int block_scan(int v, int* excl) {
+  __shared__ int warp_tot[kScanThreads / 32];
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+  int x = v;
+#pragma unroll
+  for (int o = 1; o < 32; o <<= 1) {
+    const int y = __shfl_up_sync(0xffffffffu, x, o);
+    if (lane >= o) x += y;
+  }
+  if (lane == 31) warp_tot[warp] = x;
+  __syncthreads();
+  if (warp == 0) {
+    int w = lane < kScanThreads / 32 ? warp_tot[lane] : 0;
+#pragma unroll
+    for (int o = 1; o < 32; o <<= 1) {
+      const int y = __shfl_up_sync(0xffffffffu, w, o);
+      if (lane >= o) w += y;
+    }
+    if (lane < kScanThreads / 32) warp_tot[lane] = w;  // inclusive
+  }
+  __syncthreads();
+  const int before = (warp > 0 ? warp_tot[warp - 1] : 0) + x - v;
+  const int total = warp_tot[kScanThreads / 32 - 1];
+  __syncthreads();
+  *excl = before;
+  return total;
+}
+
+// Ascending compaction of the set entries of [0, n) (flag(i) != 0) into
+// list, with inv[i] = position in list or -1.  One block.
+template <typename Flag>
+__device__ int compact(int n, Flag flag, int32_t* list, int32_t* inv) {
+  const int per = (n + kScanThreads - 1) / kScanThreads;
+  const int b0 = min(n, (int)threadIdx.x * per), b1 = min(n, b0 + per);
+  int cnt = 0;
+  for (int i = b0; i < b1; ++i) cnt += flag(i) ? 1 : 0;
+  int off;
+  const int total = block_scan(cnt, &off);
+  for (int i = b0; i < b1; ++i) {
+    if (flag(i)) {
+      list[off] = i;
+      if (inv) inv[i] = off;
+      ++off;
+    } else if (inv) {
+      inv[i] = -1;
+    }
+  }
+  return total;
+}
+
+__global__ void __launch_bounds__(kScanThreads) compact_kernel(const uint8_t* __restrict__ flags, int V, int full,
+                                                               const uint8_t* __restrict__ mask,
+                                                               const int32_t* __restrict__ targets, int T,
+                                                               int32_t* J, int32_t* pos, int32_t* tl, int32_t* tpos,
+                                                               int32_t* ycol, int32_t* counts) {
+  griddep_wait();
+  griddep_launch_dependents();
+  const int nJ = compact(V, [&](int i) { return full || flags[i] != 0; }, J, pos);
+  const int nT = compact(T, [&](int t) { return !mask || mask[t] != 0; }, tl, tpos);
+  __syncthreads();  // pos and tl complete
+  for (int i = threadIdx.x; i < nT; i += kScanThreads) {
+    const int y = targets[tl[i]];
+    const int c = (y >= 0 && y < V) ? pos[y] : -1;
+    if (c < 0) counts[2] = 1;  // a trainable target outside J (or out of range)
+    ycol[i] = c < 0 ? 0 : c;
+  }
+  if (threadIdx.x == 0) {
+    counts[0] = nT;
+    counts[1] = nJ;
+  }
+}
+
+__global__ void gather_rows_kernel(const __nv_bfloat16* __restrict__ src, long long ld,
+                                   const int32_t* __restrict__ idx, int n, int d, __nv_bfloat16* __restrict__ dst) {
+  griddep_wait();
+  griddep_launch_dependents();
+  const int vpr = d / 8;  // 16-byte vectors per row
+  const long long total = (long long)n * vpr;
+  for (long long e = blockIdx.x * (long long)blockDim.x + threadIdx.x; e < total;
+       e += (long long)gridDim.x * blockDim.x) {
+    const int i = (int)(e / vpr), v = (int)(e % vpr);
+    const uint4* s = reinterpret_cast<const uint4*>(src + (long long)idx[i] * ld) + v;
+    reinterpret_cast<uint4*>(dst + (long long)i * d)[v] = __ldg(s);
+  }
+}
+
+// Combine two (max, sum of exp(x - max)) pairs.
+__device__ __forceinline__ void lse_merge(float& m, float& s, float m2, float s2) {
+  if (m2 > m) {
+    s = s * expf(m - m2) + s2;
+    m = m2;
+  } else if (m2 > -INFINITY) {
+    s += s2 * expf(m2 - m);
+  }
+}
+
+// One block per trainable position i: lse over its nJ logits, its loss, and
+// G[i, :] = bf16(exp(z - lse) - [j == ycol]) with zeros in [nJ, ldg).
+__global__ void __launch_bounds__(256) ce_rows_kernel(const float* __restrict__ Z, int ldz, int nJ,
+                                                      const int32_t* __restrict__ ycol, __nv_bfloat16* __restrict__ G,
+                                                      int ldg, float* __restrict__ rowloss) {
+  griddep_wait();
+  griddep_launch_dependents();
+  __shared__ float sm[8], ss[8];
+  __shared__ float s_lse;
+  const int i = blockIdx.x;
+  const float* z = Z + (long long)i * ldz;
+  float m = -INFINITY, s = 0.f;
+  for (int j = threadIdx.x; j < nJ; j += blockDim.x) lse_merge(m, s, z[j], 1.f);
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) {
+    const float m2 = __shfl_xor_sync(0xffffffffu, m, o), s2 = __shfl_xor_sync(0xffffffffu, s, o);
+    lse_merge(m, s, m2, s2);
+  }
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  if (lane == 0) {
+    sm[warp] = m;
+    ss[warp] = s;
+  }
+  __syncthreads();
+  if (threadIdx.x == 0) {
+    float M = sm[0], S = ss[0];
+    for (int w = 1; w < (int)(blockDim.x >> 5); ++w) lse_merge(M, S, sm[w], ss[w]);
+    const float lse = M + logf(S);
+    s_lse = lse;
+    rowloss[i] = lse - z[ycol[i]];
+  }
+  __syncthreads();
+  const float lse = s_lse;
+  const int yc = ycol[i];
+  __nv_bfloat16* g = G + (long long)i * ldg;
+  for (int j = threadIdx.x; j < ldg; j += blockDim.x) {
+    float v = 0.f;
+    if (j < nJ) v = expf(z[j] - lse) - (j == yc ? 1.f : 0.f);
+    g[j] = __float2bfloat16_rn(v);
+  }
+}
+
+// Per-position losses (zeros off the trainable set) and their sum in a fixed order.
+__global__ void __launch_bounds__(256) ce_finish_kernel(const float* __restrict__ rowloss, int nT,
+                                                        const int32_t* __restrict__ tpos, int T,
+                                                        float* __restrict__ token_loss, float* __restrict__ loss) {
+  griddep_wait();
+  griddep_launch_dependents();
+  __shared__ double part[256];
+  if (token_loss)
+    for (int t = threadIdx.x; t < T; t += blockDim.x) token_loss[t] = tpos[t] >= 0 ? rowloss[tpos[t]] : 0.f;
+  double acc = 0.0;
+  for (int i = threadIdx.x; i < nT; i += blockDim.x) acc += (double)rowloss[i];
+  part[threadIdx.x] = acc;
+  __syncthreads();
+  for (int w = blockDim.x / 2; w > 0; w >>= 1) {
+    if ((int)threadIdx.x < w) part[threadIdx.x] += part[threadIdx.x + w];
+    __syncthreads();
+  }
+  if (threadIdx.x == 0) *loss = (float)part[0];
+}
+
+__global__ void scatter_rows_kernel(const __nv_bfloat16* __restrict__ src, const int32_t* __restrict__ tpos, int T,
+                                    int d, __nv_bfloat16* __restrict__ dst) {
+  griddep_wait();
+  griddep_launch_dependents();
+  const int vpr = d / 8;
+  const long long total = (long long)T * vpr;
+  for (long long e = blockIdx.x * (long long)blockDim.x + threadIdx.x; e < total;
+       e += (long long)gridDim.x * blockDim.x) {
+    const int t = (int)(e / vpr), v = (int)(e % vpr);
+    const int i = tpos[t];
+    const uint4 x = i >= 0 ? reinterpret_cast<const uint4*>(src + (long long)i * d)[v] : make_uint4(0u, 0u, 0u, 0u);
+    reinterpret_cast<uint4*>(dst + (long long)t * d)[v] = x;
+  }
+}
+
+int grid_for(long long n, int threads, int cap) {
+  long long b = (n + threads - 1) / threads;
+  if (b < 1) b = 1;
+  if (b > cap) b = cap;
+  return (int)b;
+}
+
+}  // namespace
+
+cudaError_t launch_ce_index(const CeIndex& a, cudaStream_t st) {
+  cudaError_t e;
+  if (a.topk) {
+    const long long n = (long long)a.T * a.k;
+    e = launch_kernel(vocab_mark_kernel, dim3(grid_for(n, 256, 4096)), dim3(256), 0, st, 1, a.targets, a.mask, a.T,
+                      a.topk, a.ld_topk, a.k, a.V, a.flags, a.counts);
+    if (e != cudaSuccess) return e;
+  }
+  return launch_kernel(compact_kernel, dim3(1), dim3(kScanThreads), 0, st, 1, (const uint8_t*)a.flags, a.V,
+                       a.topk ? 0 : 1, a.mask, a.targets, a.T, a.J, a.pos, a.tl, a.tpos, a.ycol, a.counts);
+}
+
+cudaError_t launch_gather_rows(const __nv_bfloat16* src, long long ld, const int32_t* idx, int n, int d,
+                               __nv_bfloat16* dst, cudaStream_t st) {
+  if (n <= 0) return cudaSuccess;
+  return launch_kernel(gather_rows_kernel, dim3(grid_for((long long)n * (d / 8), 256, 8192)), dim3(256), 0, st, 1,
+                       src, ld, idx, n, d, dst);
+}
+
+cudaError_t launch_ce_rows(const float* Z, int ldz, int nJ, const int32_t* ycol, int nT, __nv_bfloat16* G, int ldg,
+                           float* rowloss, cudaStream_t st) {
+  if (nT <= 0) return cudaSuccess;
+  return launch_kernel(ce_rows_kernel, dim3(nT), dim3(256), 0, st, 1, Z, ldz, nJ, ycol, G, ldg, rowloss);
+}
+
+cudaError_t launch_ce_finish(const float* rowloss, int nT, const int32_t* tpos, int T, float* token_loss,
+                             float* loss, cudaStream_t st) {
+  return launch_kernel(ce_finish_kernel, dim3(1), dim3(256), 0, st, 1, rowloss, nT, tpos, T, token_loss, loss);
+}
+
+cudaError_t launch_scatter_rows(const __nv_bfloat16* src, const int32_t* tpos, int T, int d, __nv_bfloat16* dst,
+                                cudaStream_t st) {
+  return launch_kernel(scatter_rows_kernel, dim3(grid_for((long long)T * (d / 8), 256, 8192)), dim3(256), 0, st, 1,
+                       src, tpos, T, d, dst);
+}
+
+}  // namespace lora

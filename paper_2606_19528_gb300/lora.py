@@ -33,7 +33,8 @@ LORA_FWD_BWD = 3
 # every symbol that include/lora.h declares
 EXPORTS = ("lora_workspace_size", "lora_linear_fwd", "lora_linear_fwd_noalloc", "lora_linear_bwd",
            "lora_linear_fwd_q4", "lora_linear_bwd_q4", "lora_stack_workspace_size",
-           "lora_stack_step", "lora_stack_ckpt_workspace_size", "lora_stack_ckpt", "lora_read_status", "lora_set_wait_limit_ns", "lora_launch_count",
+           "lora_stack_step", "lora_stack_ckpt_workspace_size", "lora_stack_ckpt", "lora_ce_workspace_size",
+           "lora_ce_fwd_bwd", "lora_read_status", "lora_set_wait_limit_ns", "lora_launch_count",
            "lora_profile_begin", "lora_profile_begin_kinds", "lora_profile_end", "lora_strerror", "lora_version")
 
 LORA_KERNEL_GEMM_FWD = 0
@@ -68,6 +69,14 @@ class lora_proj(ctypes.Structure):
                 ("dA", ctypes.c_void_p), ("dB", ctypes.c_void_p), ("Wq", lora_q4_weight)]
 
 
+class lora_ce_args(ctypes.Structure):
+    _fields_ = [("T", ctypes.c_int64), ("d", ctypes.c_int64), ("V", ctypes.c_int64),
+                ("h", ctypes.c_void_p), ("E", ctypes.c_void_p), ("targets", ctypes.c_void_p),
+                ("mask", ctypes.c_void_p), ("topk", ctypes.c_void_p), ("ld_topk", ctypes.c_int64),
+                ("k", ctypes.c_int64), ("loss", ctypes.c_void_p), ("token_loss", ctypes.c_void_p),
+                ("dh", ctypes.c_void_p), ("vocab", ctypes.c_void_p), ("counts", ctypes.c_void_p)]
+
+
 def library(path: str = _LIB_PATH) -> ctypes.CDLL:
     """Load the CUDA library (once).  Raises OSError if it has not been built."""
     global _lib
@@ -88,6 +97,8 @@ def library(path: str = _LIB_PATH) -> ctypes.CDLL:
         lib.lora_stack_step.argtypes = [P(lora_proj), i32, i32, vp, sz, vp]
         lib.lora_stack_ckpt_workspace_size.argtypes = [P(lora_proj), i32, i32, P(sz)]
         lib.lora_stack_ckpt.argtypes = [P(lora_proj), i32, i32, vp, sz, vp]
+        lib.lora_ce_workspace_size.argtypes = [P(lora_ce_args), P(sz)]
+        lib.lora_ce_fwd_bwd.argtypes = [P(lora_ce_args), vp, sz, vp]
         lib.lora_read_status.argtypes = [vp, P(i32), i32]
         lib.lora_set_wait_limit_ns.argtypes = [i64]
         lib.lora_launch_count.argtypes = []
@@ -217,6 +228,31 @@ def lora_stack_ckpt(layers, workspace, workspace_bytes, stream=None) -> None:
     arr = _proj_array([p for L in layers for p in L])
     _check(library().lora_stack_ckpt(arr, len(layers), n_per, _ptr(workspace), int(workspace_bytes),
                                      _stream(stream)), "lora_stack_ckpt")
+
+
+def make_ce_args(T, d, V, h, E, targets, loss, mask=None, topk=None, ld_topk=0, k=0, token_loss=None, dh=None,
+                 vocab=None) -> lora_ce_args:
+    return lora_ce_args(int(T), int(d), int(V), _ptr(h), _ptr(E), _ptr(targets), _ptr(mask), _ptr(topk),
+                        int(ld_topk), int(k), _ptr(loss), _ptr(token_loss), _ptr(dh), _ptr(vocab), None)
+
+
+def lora_ce_workspace_size(args: lora_ce_args) -> int:
+    n = ctypes.c_size_t(0)
+    _check(library().lora_ce_workspace_size(ctypes.byref(args), ctypes.byref(n)), "lora_ce_workspace_size")
+    return n.value
+
+
+def lora_ce_fwd_bwd(args: lora_ce_args, workspace, workspace_bytes, stream=None):
+    """Reduced-vocabulary cross entropy with logits masking (see include/lora.h);
+    returns (|T_set|, |J|)."""
+    counts = (ctypes.c_int64 * 2)()
+    args.counts = ctypes.cast(counts, ctypes.c_void_p)
+    try:
+        _check(library().lora_ce_fwd_bwd(ctypes.byref(args), _ptr(workspace), int(workspace_bytes), _stream(stream)),
+               "lora_ce_fwd_bwd")
+    finally:
+        args.counts = None
+    return int(counts[0]), int(counts[1])
 
 
 def lora_read_status(stream=None, reset: bool = True) -> int:

@@ -30,6 +30,18 @@ code byte is floor(256 u), so both 4-bit codes of a byte are uniform on
 s = s0 (0.5 + u1) with s0 = 2 sqrt(3) / (15 sqrt(d_in)) and the offset
 b = -(7.5 + (2 u2 - 1)) s, so that s q + b has mean about 0 and variance
 about 1/d_in, like W above; s and b are rounded to bf16.
+
+LM-head inputs (the paper's XSum sequences and trained embeddings are not
+available): hidden states h ~ N(0, 1) and embedding rows E ~ N(0, 1/d);
+instruction-tuning masks, a prompt of non-trainable positions followed by a
+trainable response; targets drawn cluster-first: the vocabulary is split
+into clusters of consecutive ids, a target's cluster is Zipf-distributed
+(rank r with weight r^-2.5, which puts |J| for 30 % of 2048 positions and
+k = 500 near 9 k, inside the 2.7-14.4 k the paper reports for its top-k
+runs) and its member uniform; the top-k table lists, for
+token i, i itself, then the rest of its cluster in a seeded random order,
+then tokens of the following clusters -- the locality that makes the union
+of a sequence's top-k rows far smaller than the vocabulary.
 """
 from __future__ import annotations
 
@@ -46,6 +58,7 @@ _CHUNK = 1 << 22
 
 # tensor identifiers used as stream tags
 TID_X, TID_W, TID_A, TID_B, TID_DY, TID_WQ, TID_WP = 1, 2, 3, 4, 5, 6, 7
+TID_H, TID_E, TID_Y, TID_TOPK = 8, 9, 10, 11
 
 
 def _mix(z: np.ndarray) -> np.ndarray:
@@ -193,3 +206,51 @@ def gen_Wq(seed: int, cfg: int, proj: int, layer: int, N: int, K: int):
     off = -(7.5 + (2.0 * v[:, :, 1] - 1.0)) * sc_b
     params = np.stack([to_bf16_bits(sc), to_bf16_bits(off)], axis=-1)
     return codes, params
+
+
+def gen_h(seed: int, cfg: int, T: int, d: int) -> np.ndarray:
+    """Hidden states h [T, d] ~ N(0, 1) entering the LM head."""
+    return normal_bf16(stream_key(seed, cfg, TID_H), (T, d), 1.0)
+
+
+def gen_E(seed: int, cfg: int, V: int, d: int) -> np.ndarray:
+    """Frozen LM-head embedding E [V, d] ~ N(0, 1/d)."""
+    return normal_bf16(stream_key(seed, cfg, TID_E), (V, d), 1.0 / math.sqrt(d))
+
+
+def gen_mask(T: int, trainable_frac: float) -> np.ndarray:
+    """Prompt then response: the last round(frac T) positions are trainable."""
+    n = int(round(T * trainable_frac))
+    m = np.zeros(T, dtype=np.uint8)
+    if n > 0:
+        m[T - n:] = 1
+    return m
+
+
+def gen_targets(seed: int, cfg: int, T: int, V: int, cluster: int, zipf: float = 2.5) -> np.ndarray:
+    """Targets [T] int32: Zipf-distributed cluster, uniform member."""
+    n_cl = (V + cluster - 1) // cluster
+    u = uniform01(stream_key(seed, cfg, TID_Y), 2 * T).reshape(T, 2)
+    w = np.arange(1, n_cl + 1, dtype=np.float64) ** -zipf
+    cdf = np.cumsum(w) / w.sum()
+    cl = np.minimum(np.searchsorted(cdf, u[:, 0]), n_cl - 1)
+    size = np.minimum(cluster, V - cl * cluster)
+    return (cl * cluster + np.minimum(np.floor(u[:, 1] * size), size - 1)).astype(np.int32)
+
+
+def gen_topk_table(seed: int, cfg: int, V: int, k: int, cluster: int) -> np.ndarray:
+    """Top-k table [V, k] int32 with cluster locality (see the module notes)."""
+    out = np.empty((V, k), dtype=np.int32)
+    key = stream_key(seed, cfg, TID_TOPK)
+    n_cl = (V + cluster - 1) // cluster
+    for c in range(n_cl):
+        lo, hi = c * cluster, min(V, (c + 1) * cluster)
+        members = np.arange(lo, hi)
+        nxt = np.concatenate([np.arange(hi, V), np.arange(0, lo)])[: max(0, k - 1)]
+        u = uniform01(key, (hi - lo) * (hi - lo), offset=lo * cluster).reshape(hi - lo, hi - lo)
+        for r, i in enumerate(members):
+            others = members[members != i]
+            order = others[np.argsort(u[r, : len(others)], kind="stable")]
+            row = np.concatenate([[i], order, nxt])[:k]
+            out[i, : len(row)] = row
+    return out

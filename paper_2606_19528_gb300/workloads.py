@@ -37,6 +37,12 @@ class Workload:
     zero_B: bool = False
     q4: bool = False      # base weights as 4-bit codes (Algorithm 1's on-the-fly dequantization)
     ckpt: bool = False    # checkpointed stack schedule (Algorithm 2): forward twice, backward once
+    kind: str = "lora"    # "lora": adapted projections; "ce": reduced-vocabulary LM-head cross entropy
+    vocab: int = 0        # ce: vocabulary size V
+    hidden: int = 0       # ce: hidden size d
+    topk: int = 0         # ce: k of the top-k table (0: full vocabulary)
+    trainable: float = 1.0  # ce: fraction of trainable positions (prompt first, then response)
+    cluster: int = 512    # ce: locality of the synthetic top-k table and targets
 
     @property
     def scale(self) -> float:
@@ -116,6 +122,20 @@ def llama_layer_T256(q4: bool = False) -> Workload:
     return Workload("llama3b_layer_T256_r16" + ("_q4" if q4 else ""), 7, 256, 16, 32.0, llama_layer(), q4=q4)
 
 
+def llama_lm_head_ce() -> Workload:
+    """Llama-3.2-3B LM head (V = 128256, d = 3072), T = 2048 positions of which
+    the last 30 % are trainable, top-500 reduced vocabulary: the LM-head node of
+    the paper's combined setting (top-k softmax approximation + logits masking)."""
+    return Workload("llama3b_lmhead_ce_T2048_top500_mask30", 12, 2048, 1, 1.0, [], kind="ce", vocab=128256,
+                    hidden=3072, topk=500, trainable=0.3)
+
+
+def llama_lm_head_ce_full() -> Workload:
+    """The same LM head with the full vocabulary (no top-k), logits masking only."""
+    return Workload("llama3b_lmhead_ce_T2048_full_mask30", 12, 2048, 1, 1.0, [], kind="ce", vocab=128256,
+                    hidden=3072, topk=0, trainable=0.3)
+
+
 BY_NAME = {
     "single": single_small,
     "single_B0": lambda: single_small(True),
@@ -124,6 +144,8 @@ BY_NAME = {
     "qwen_layer": qwen_layer_T4096,
     "llama_stack28": llama_stack28,
     "llama_stack28_ckpt": llama_stack28_ckpt,
+    "lm_head_ce": llama_lm_head_ce,
+    "lm_head_ce_full": llama_lm_head_ce_full,
     "llama_layer_q4": llama_layer_T2048_q4,
     "llama_layer_T256": llama_layer_T256,
     "llama_layer_T256_q4": lambda: llama_layer_T256(True),
