@@ -7,3 +7,4 @@ from .lora_oracle import (lora_forward, lora_backward, lora_forward_rows,  # noq
                           lora_backward_dx_rows, lora_adapter_grads, lora_step,
                           unpack_q4, dequant_q4)
 from .lm_head_oracle import reduced_vocab, ce_forward_backward  # noqa: F401,E402
+from .topk_oracle import normalize_rows, similarities, topk_table  # noqa: F401,E402
