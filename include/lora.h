@@ -228,9 +228,28 @@ typedef struct lora_ce_args {
 int lora_ce_workspace_size(const lora_ce_args* args, size_t* bytes);
 int lora_ce_fwd_bwd(const lora_ce_args* args, void* workspace, size_t workspace_bytes, void* stream);
 
+/* Top-k similarity table of a frozen embedding (Section "Softmax
+ * Approximation", "Choosing the Reduced Vocabulary Set"): with E~ the
+ * embedding's rows normalised (each row's sum of squares accumulated in fp32
+ * in index order, correctly rounded square root and division, rounded to
+ * bf16; a zero row stays zero), C = E~ E~^T holds the cosine similarities and
+ * row i of `table` [V, k] int32 lists the k tokens with the largest C[i, :],
+ * in descending order, the lower index first on equal similarities (row i
+ * starts with i unless another token has the same direction).  The V x V
+ * matrix is never formed: similarities are computed 512 rows at a time in
+ * fp32 on the tensor cores and each row's top k is selected from them.
+ * E [V, d] bf16 (16-byte aligned), d a multiple of 8, 1 <= k <= min(V, 1024).
+ * A row whose k-th similarity is shared by more candidates than the selection
+ * holds (thousands of exact ties) is left unwritten and lora_read_status
+ * reports LORA_EINVAL. */
+int lora_topk_workspace_size(int64_t V, int64_t d, int64_t k, size_t* bytes);
+int lora_topk_table(const lora_bf16* E, int64_t V, int64_t d, int64_t k, int32_t* table, void* workspace,
+                    size_t workspace_bytes, void* stream);
+
 /* Waits for `stream`, then reads the device status word that bounded waits
- * set when they expire: *status = LORA_OK or LORA_ETIMEOUT.  reset != 0
- * clears it.  Returns LORA_OK or LORA_ECUDA. */
+ * set when they expire (and lora_topk_table sets on an unresolved row):
+ * *status = LORA_OK, LORA_ETIMEOUT or LORA_EINVAL.  reset != 0 clears it.
+ * Returns LORA_OK or LORA_ECUDA. */
 int lora_read_status(void* stream, int* status, int reset);
 
 /* Limit, in nanoseconds of device time, of every bounded wait in the

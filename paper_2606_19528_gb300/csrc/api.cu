@@ -892,6 +892,36 @@ int ce_gemm(const DeviceInfo* d, int* counter, const void* A, int64_t lda, const
   return launch_fused_gemm(b, b_mn, false, d->num_sms, st, f32_out) == cudaSuccess ? LORA_OK : LORA_ECUDA;
 }
 
+
+// ------------------------------------------------------------------ top-k similarity table
+constexpr int kTopkChunk = 512;  // rows of similarities per contraction
+
+struct TopkPlan {
+  size_t counters, status, en, s, total;
+  int chunks;
+  long long lds;
+};
+
+int topk_check(const lora_bf16* E, int64_t V, int64_t d, int64_t k, TopkPlan* pl) {
+  if (V < 1 || d < 8 || (d % 8) || k < 1 || k > V || k > topk_max_k() || V > (1ll << 24) || d > (1ll << 20))
+    return LORA_EINVAL;
+  if (E && !aligned16(E)) return LORA_EALIGN;
+  pl->chunks = (int)cdiv(V, kTopkChunk);
+  pl->lds = rup(V, 4);
+  size_t off = 0;
+  auto take = [&](size_t bytes) {
+    const size_t o = off;
+    off += up256(bytes);
+    return o;
+  };
+  pl->counters = take((size_t)pl->chunks * 4);
+  pl->status = take(4);
+  pl->en = take((size_t)V * d * 2);
+  pl->s = take((size_t)std::min<int64_t>(V, kTopkChunk) * pl->lds * 4);
+  pl->total = off;
+  return LORA_OK;
+}
+
 }  // namespace
 
 void note_launch() { g_launches.fetch_add(1, std::memory_order_relaxed); }
@@ -1201,6 +1231,44 @@ int lora_ce_fwd_bwd(const lora_ce_args* a, void* workspace, size_t workspace_byt
   return LORA_OK;
 }
 
+int lora_topk_workspace_size(int64_t V, int64_t d, int64_t k, size_t* bytes) {
+  if (!bytes) return LORA_ENULL;
+  TopkPlan pl;
+  const int rc = topk_check(nullptr, V, d, k, &pl);
+  if (rc != LORA_OK) return rc;
+  *bytes = pl.total;
+  return LORA_OK;
+}
+
+int lora_topk_table(const lora_bf16* E, int64_t V, int64_t d, int64_t k, int32_t* table, void* workspace,
+                    size_t workspace_bytes, void* stream) {
+  if (!E || !table) return LORA_ENULL;
+  TopkPlan pl;
+  int rc = topk_check(E, V, d, k, &pl);
+  if (rc != LORA_OK) return rc;
+  if ((rc = check_ws(workspace, workspace_bytes, pl.total)) != LORA_OK) return rc;
+  DeviceInfo* dv = nullptr;
+  if ((rc = device_info(&dv)) != LORA_OK) return rc;
+  cudaStream_t st = static_cast<cudaStream_t>(stream);
+  uint8_t* ws = static_cast<uint8_t*>(workspace);
+  if (cudaMemsetAsync(ws, 0, pl.en, st) != cudaSuccess) return LORA_ECUDA;  // tile counters and status
+  bf* en = at<bf>(ws, pl.en);
+  float* S = at<float>(ws, pl.s);
+  if (launch_normalize_rows(cb(E), (int)V, (int)d, en, st) != cudaSuccess) return LORA_ECUDA;
+  for (int c = 0; c < pl.chunks; ++c) {
+    const int64_t r0 = (int64_t)c * kTopkChunk, rows = std::min<int64_t>(kTopkChunk, V - r0);
+    {
+      ProfScope ps(LORA_KERNEL_GEMM_FWD, st);
+      if ((rc = ce_gemm(dv, at<int>(ws, pl.counters) + c, en + r0 * d, d, en, d, S, pl.lds, rows, V, d, false,
+                        true, st)) != LORA_OK)
+        return rc;
+    }
+    if (launch_topk_select(S, pl.lds, (int)V, (int)k, (int)r0, (int)rows, table, dv->status, st) != cudaSuccess)
+      return LORA_ECUDA;
+  }
+  return LORA_OK;
+}
+
 int lora_read_status(void* stream, int* status, int reset) {
   if (!status) return LORA_ENULL;
   if (cudaStreamSynchronize(static_cast<cudaStream_t>(stream)) != cudaSuccess) return LORA_ECUDA;
@@ -1210,7 +1278,7 @@ int lora_read_status(void* stream, int* status, int reset) {
     const int z = 0;
     if (cudaMemcpyToSymbol(g_status, &z, sizeof(int)) != cudaSuccess) return LORA_ECUDA;
   }
-  *status = v ? LORA_ETIMEOUT : LORA_OK;
+  *status = v == 0 ? LORA_OK : v == kStatusTopkTies ? LORA_EINVAL : LORA_ETIMEOUT;
   return LORA_OK;
 }
 

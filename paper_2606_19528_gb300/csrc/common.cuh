@@ -16,6 +16,7 @@ namespace lora {
 
 // Error codes written to the device status word (first error wins).
 constexpr int kStatusTimeout = 1;
+constexpr int kStatusTopkTies = 2;  // a top-k row had more candidates tied at its k-th value than fit
 
 struct WaitCtl {
   int* status;         // device status word

@@ -221,6 +221,16 @@ cudaError_t launch_ce_finish(const float* rowloss, int nT, const int32_t* tpos, 
 cudaError_t launch_scatter_rows(const __nv_bfloat16* src, const int32_t* tpos, int T, int d, __nv_bfloat16* dst,
                                 cudaStream_t stream);
 
+// ---------------------------------------------------------------- top-k similarity table
+// En[i] = bf16(E[i] / ||E[i]||), the norm's sum of squares in fp32 in index order.
+cudaError_t launch_normalize_rows(const __nv_bfloat16* E, int V, int d, __nv_bfloat16* En, cudaStream_t stream);
+// Rows row0 .. row0 + nrows - 1 of the table from their similarities S [nrows, lds] fp32:
+// the k largest per row, descending, lower index first on ties; *status =
+// kStatusTopkTies when a row has too many candidates tied at its k-th value.
+cudaError_t launch_topk_select(const float* S, long long lds, int V, int k, int row0, int nrows, int32_t* table,
+                               int* status, cudaStream_t stream);
+int topk_max_k();
+
 // dst[i, j] = j < r ? src[i * r + j] : 0  for j < ld_dst (zero-padded copy of an [rows, r] matrix).
 cudaError_t launch_pad_cols(const __nv_bfloat16* src, int rows, int r, __nv_bfloat16* dst, int ld_dst,
                             cudaStream_t stream);

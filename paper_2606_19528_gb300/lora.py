@@ -34,7 +34,7 @@ LORA_FWD_BWD = 3
 EXPORTS = ("lora_workspace_size", "lora_linear_fwd", "lora_linear_fwd_noalloc", "lora_linear_bwd",
            "lora_linear_fwd_q4", "lora_linear_bwd_q4", "lora_stack_workspace_size",
            "lora_stack_step", "lora_stack_ckpt_workspace_size", "lora_stack_ckpt", "lora_ce_workspace_size",
-           "lora_ce_fwd_bwd", "lora_read_status", "lora_set_wait_limit_ns", "lora_launch_count",
+           "lora_ce_fwd_bwd", "lora_topk_workspace_size", "lora_topk_table", "lora_read_status", "lora_set_wait_limit_ns", "lora_launch_count",
            "lora_profile_begin", "lora_profile_begin_kinds", "lora_profile_end", "lora_strerror", "lora_version")
 
 LORA_KERNEL_GEMM_FWD = 0
@@ -99,6 +99,8 @@ def library(path: str = _LIB_PATH) -> ctypes.CDLL:
         lib.lora_stack_ckpt.argtypes = [P(lora_proj), i32, i32, vp, sz, vp]
         lib.lora_ce_workspace_size.argtypes = [P(lora_ce_args), P(sz)]
         lib.lora_ce_fwd_bwd.argtypes = [P(lora_ce_args), vp, sz, vp]
+        lib.lora_topk_workspace_size.argtypes = [i64, i64, i64, P(sz)]
+        lib.lora_topk_table.argtypes = [vp, i64, i64, i64, vp, vp, sz, vp]
         lib.lora_read_status.argtypes = [vp, P(i32), i32]
         lib.lora_set_wait_limit_ns.argtypes = [i64]
         lib.lora_launch_count.argtypes = []
@@ -253,6 +255,18 @@ def lora_ce_fwd_bwd(args: lora_ce_args, workspace, workspace_bytes, stream=None)
     finally:
         args.counts = None
     return int(counts[0]), int(counts[1])
+
+
+def lora_topk_workspace_size(V: int, d: int, k: int) -> int:
+    n = ctypes.c_size_t(0)
+    _check(library().lora_topk_workspace_size(int(V), int(d), int(k), ctypes.byref(n)), "lora_topk_workspace_size")
+    return n.value
+
+
+def lora_topk_table(E, V: int, d: int, k: int, table, workspace, workspace_bytes, stream=None) -> None:
+    """Top-k cosine-similarity table of the embedding E [V, d] into table [V, k] int32."""
+    _check(library().lora_topk_table(_ptr(E), int(V), int(d), int(k), _ptr(table), _ptr(workspace),
+                                     int(workspace_bytes), _stream(stream)), "lora_topk_table")
 
 
 def lora_read_status(stream=None, reset: bool = True) -> int:

@@ -37,7 +37,7 @@ class Workload:
     zero_B: bool = False
     q4: bool = False      # base weights as 4-bit codes (Algorithm 1's on-the-fly dequantization)
     ckpt: bool = False    # checkpointed stack schedule (Algorithm 2): forward twice, backward once
-    kind: str = "lora"    # "lora": adapted projections; "ce": reduced-vocabulary LM-head cross entropy
+    kind: str = "lora"    # "lora": adapted projections; "ce": LM-head cross entropy; "topk": similarity table
     vocab: int = 0        # ce: vocabulary size V
     hidden: int = 0       # ce: hidden size d
     topk: int = 0         # ce: k of the top-k table (0: full vocabulary)
@@ -136,6 +136,13 @@ def llama_lm_head_ce_full() -> Workload:
                     hidden=3072, topk=0, trainable=0.3)
 
 
+def llama_topk_table() -> Workload:
+    """The top-k similarity table of a Llama-3.2-3B-sized embedding (V = 128256,
+    d = 3072, k = 500, the paper's chosen k): a one-time precomputation."""
+    return Workload("llama3b_topk_table_V128256_k500", 13, 0, 1, 1.0, [], kind="topk", vocab=128256, hidden=3072,
+                    topk=500)
+
+
 BY_NAME = {
     "single": single_small,
     "single_B0": lambda: single_small(True),
@@ -146,6 +153,7 @@ BY_NAME = {
     "llama_stack28_ckpt": llama_stack28_ckpt,
     "lm_head_ce": llama_lm_head_ce,
     "lm_head_ce_full": llama_lm_head_ce_full,
+    "topk_table": llama_topk_table,
     "llama_layer_q4": llama_layer_T2048_q4,
     "llama_layer_T256": llama_layer_T256,
     "llama_layer_T256_q4": lambda: llama_layer_T256(True),
