@@ -819,7 +819,7 @@ void layer_copy(const lora_proj* L, int n_per, uint8_t* su_scratch, std::vector<
 inline int64_t rup(int64_t x, int64_t m) { return (x + m - 1) / m * m; }
 
 struct CePlan {
-  size_t flags, counts, J, pos, tl, tpos, ycol, rowloss, ht, ej, z, g, dht, tiles, total;
+  size_t flags, counts, segs, J, pos, tl, tpos, ycol, rowloss, ht, ej, z, g, dht, tiles, total;
 };
 
 int ce_check(const lora_ce_args* a, CePlan* pl) {
@@ -841,6 +841,7 @@ int ce_check(const lora_ce_args* a, CePlan* pl) {
   };
   pl->tiles = take(16);
   pl->counts = take(16);
+  pl->segs = take(128 * 4);
   pl->flags = take((size_t)V);
   pl->J = take((size_t)V * 4);
   pl->pos = take((size_t)V * 4);
@@ -1188,6 +1189,7 @@ int lora_ce_fwd_bwd(const lora_ce_args* a, void* workspace, size_t workspace_byt
   ix.tpos = at<int32_t>(ws, pl.tpos);
   ix.ycol = at<int32_t>(ws, pl.ycol);
   ix.counts = at<int32_t>(ws, pl.counts);
+  ix.seg_counts = at<int32_t>(ws, pl.segs);
   if (launch_ce_index(ix, st) != cudaSuccess) return LORA_ECUDA;
   // |T_set| and |J| size the contractions
   int32_t counts[3] = {0, 0, 0};

@@ -205,6 +205,7 @@ struct CeIndex {
   int k;
   uint8_t* flags;
   int32_t *J, *pos, *tl, *tpos, *ycol, *counts;
+  int32_t* seg_counts;  // 128 per-segment counts of the vocabulary compaction
 };
 cudaError_t launch_ce_index(const CeIndex& a, cudaStream_t stream);
 // dst[i, :] = src[idx[i], :] for i < n (rows of d bf16, d a multiple of 8).

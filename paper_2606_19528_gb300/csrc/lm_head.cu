@@ -4,8 +4,10 @@
 // compute the logits of the trainable positions over the reduced vocabulary
 // J and the hidden-state gradient.
 //   vocab_mark      J = union of the trainable targets' first k top-k entries
-//   compact         J and the trainable positions as ascending lists, their
-//                   inverse maps, each trainable target's column in J
+//   vocab_count,    J and the trainable positions as ascending lists and
+//   compact, ycol   their inverse maps (128 vocabulary segments counted,
+//                   then compacted in parallel), each trainable target's
+//                   column in J
 //   gather_rows     rows of h (trainable positions) and of E (J) made dense
 //   ce_rows         per trainable position: log-sum-exp over J, its loss, and
 //                   G = softmax_J - onehot(target) in bf16 for the dh contraction
@@ -96,25 +98,82 @@ __device__ int compact(int n, Flag flag, int32_t* list, int32_t* inv) {
   return total;
 }
 
-__global__ void __launch_bounds__(kScanThreads) compact_kernel(const uint8_t* __restrict__ flags, int V, int full,
-                                                               const uint8_t* __restrict__ mask,
-                                                               const int32_t* __restrict__ targets, int T,
-                                                               int32_t* J, int32_t* pos, int32_t* tl, int32_t* tpos,
-                                                               int32_t* ycol, int32_t* counts) {
+constexpr int kSegs = 128;  // vocabulary segments of the multi-block compaction
+
+// Set flags per vocabulary segment (every token in full-vocabulary mode).
+__global__ void __launch_bounds__(256) vocab_count_kernel(const uint8_t* __restrict__ flags, int V, int full,
+                                                          int32_t* __restrict__ seg_counts) {
   griddep_wait();
   griddep_launch_dependents();
-  const int nJ = compact(V, [&](int i) { return full || flags[i] != 0; }, J, pos);
+  const int seg = (V + kSegs - 1) / kSegs;
+  const int b0 = min(V, (int)blockIdx.x * seg), b1 = min(V, b0 + seg);
+  int c = 0;
+  for (int i = b0 + threadIdx.x; i < b1; i += blockDim.x) c += (full || flags[i]) ? 1 : 0;
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) c += __shfl_xor_sync(0xffffffffu, c, o);
+  __shared__ int wsum[8];
+  if ((threadIdx.x & 31) == 0) wsum[threadIdx.x >> 5] = c;
+  __syncthreads();
+  if (threadIdx.x == 0) {
+    int t = 0;
+    for (int w = 0; w < 8; ++w) t += wsum[w];
+    seg_counts[blockIdx.x] = t;
+  }
+}
+
+// Blocks 0 .. kSegs-1: their segment of J (ascending) and pos; block kSegs:
+// the trainable positions, their inverse map and the counts.
+__global__ void __launch_bounds__(kScanThreads) compact_kernel(const uint8_t* __restrict__ flags, int V, int full,
+                                                               const int32_t* __restrict__ seg_counts,
+                                                               const uint8_t* __restrict__ mask, int T,
+                                                               int32_t* J, int32_t* pos, int32_t* tl, int32_t* tpos,
+                                                               int32_t* counts) {
+  griddep_wait();
+  griddep_launch_dependents();
+  __shared__ int s_base;
+  if (blockIdx.x < kSegs) {
+    const int seg = (V + kSegs - 1) / kSegs;
+    const int b0 = min(V, (int)blockIdx.x * seg), b1 = min(V, b0 + seg);
+    if (threadIdx.x == 0) {
+      int base = 0;
+      for (int b = 0; b < (int)blockIdx.x; ++b) base += seg_counts[b];
+      s_base = base;
+    }
+    __syncthreads();
+    const int base = s_base;
+    compact(b1 - b0, [&](int i) { return full || flags[b0 + i] != 0; }, J + base, nullptr);
+    __syncthreads();
+    // pos over the segment: J[base .. base + cnt) are ascending tokens of [b0, b1)
+    for (int i = b0 + threadIdx.x; i < b1; i += kScanThreads) pos[i] = -1;
+    __syncthreads();
+    const int cnt = seg_counts[blockIdx.x];
+    for (int q = threadIdx.x; q < cnt; q += kScanThreads) {
+      J[base + q] += b0;  // compact wrote segment-relative indices
+      pos[J[base + q]] = base + q;
+    }
+    return;
+  }
   const int nT = compact(T, [&](int t) { return !mask || mask[t] != 0; }, tl, tpos);
-  __syncthreads();  // pos and tl complete
-  for (int i = threadIdx.x; i < nT; i += kScanThreads) {
+  if (threadIdx.x == 0) {
+    int nJ = 0;
+    for (int b = 0; b < kSegs; ++b) nJ += seg_counts[b];
+    counts[0] = nT;
+    counts[1] = nJ;
+  }
+}
+
+// Column in J of each trainable position's target (after the compaction).
+__global__ void ycol_kernel(const int32_t* __restrict__ targets, const int32_t* __restrict__ tl,
+                            const int32_t* __restrict__ pos, int V, int32_t* __restrict__ ycol,
+                            int32_t* __restrict__ counts) {
+  griddep_wait();
+  griddep_launch_dependents();
+  const int nT = counts[0];
+  for (int i = blockIdx.x * blockDim.x + threadIdx.x; i < nT; i += gridDim.x * blockDim.x) {
     const int y = targets[tl[i]];
     const int c = (y >= 0 && y < V) ? pos[y] : -1;
     if (c < 0) counts[2] = 1;  // a trainable target outside J (or out of range)
     ycol[i] = c < 0 ? 0 : c;
-  }
-  if (threadIdx.x == 0) {
-    counts[0] = nT;
-    counts[1] = nJ;
   }
 }
 
@@ -236,8 +295,15 @@ cudaError_t launch_ce_index(const CeIndex& a, cudaStream_t st) {
                       a.topk, a.ld_topk, a.k, a.V, a.flags, a.counts);
     if (e != cudaSuccess) return e;
   }
-  return launch_kernel(compact_kernel, dim3(1), dim3(kScanThreads), 0, st, 1, (const uint8_t*)a.flags, a.V,
-                       a.topk ? 0 : 1, a.mask, a.targets, a.T, a.J, a.pos, a.tl, a.tpos, a.ycol, a.counts);
+  const int full = a.topk ? 0 : 1;
+  e = launch_kernel(vocab_count_kernel, dim3(kSegs), dim3(256), 0, st, 1, (const uint8_t*)a.flags, a.V, full,
+                    a.seg_counts);
+  if (e != cudaSuccess) return e;
+  e = launch_kernel(compact_kernel, dim3(kSegs + 1), dim3(kScanThreads), 0, st, 1, (const uint8_t*)a.flags, a.V,
+                    full, (const int32_t*)a.seg_counts, a.mask, a.T, a.J, a.pos, a.tl, a.tpos, a.counts);
+  if (e != cudaSuccess) return e;
+  return launch_kernel(ycol_kernel, dim3(grid_for(a.T, 256, 64)), dim3(256), 0, st, 1, a.targets,
+                       (const int32_t*)a.tl, (const int32_t*)a.pos, a.V, a.ycol, a.counts);
 }
 
 cudaError_t launch_gather_rows(const __nv_bfloat16* src, long long ld, const int32_t* idx, int n, int d,

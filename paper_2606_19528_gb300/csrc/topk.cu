@@ -132,7 +132,7 @@ __global__ void __launch_bounds__(kSelThreads) topk_select_kernel(const float* _
   extern __shared__ uint8_t smem_raw[];
   SelShared& sh = *reinterpret_cast<SelShared*>(smem_raw);
   const int r = blockIdx.x;
-  const float* s = S + (long long)r * lds;
+  const float* s = S + (long long)r * lds;  // lds is a multiple of 4: 16-byte aligned rows
   // levels: (shift of the level's digit, digit bits); the prefix so far selects candidates
   const int shifts[3] = {21, 10, 0}, bits[3] = {11, 11, 10};
   uint32_t prefix = 0;  // chosen digits so far, as key >> shift of the current level
@@ -142,10 +142,18 @@ __global__ void __launch_bounds__(kSelThreads) topk_select_kernel(const float* _
     for (int b = threadIdx.x; b < nb; b += kSelThreads) sh.hist[b] = 0;
     __syncthreads();
     const int hi_shift = sh_ + bits[lvl];  // bits above this level's digit
-    for (int j = threadIdx.x; j < V; j += kSelThreads) {
-      const uint32_t key = ord_key(s[j]);
+    auto count = [&](float f) {
+      const uint32_t key = ord_key(f);
       if (lvl == 0 || (key >> hi_shift) == prefix) atomicAdd(&sh.hist[(key >> sh_) & (nb - 1)], 1);
+    };
+    for (int j4 = threadIdx.x; j4 < V / 4; j4 += kSelThreads) {
+      const float4 q = __ldg(reinterpret_cast<const float4*>(s) + j4);
+      count(q.x);
+      count(q.y);
+      count(q.z);
+      count(q.w);
     }
+    for (int j = (V & ~3) + (int)threadIdx.x; j < V; j += kSelThreads) count(s[j]);
     __syncthreads();
     find_bin(sh, nb, k_rem);
     prefix = (lvl == 0 ? 0u : prefix << bits[lvl]) | (uint32_t)sh.bin;
@@ -166,14 +174,22 @@ __global__ void __launch_bounds__(kSelThreads) topk_select_kernel(const float* _
   const int sh_ = shifts[lvl_found];
   if (threadIdx.x == 0) sh.ncand = 0;
   __syncthreads();
-  for (int j = threadIdx.x; j < V; j += kSelThreads) {
-    const uint32_t key = ord_key(s[j]);
+  auto take = [&](float f, int j) {
+    const uint32_t key = ord_key(f);
     if ((key >> sh_) >= prefix) {
       const int slot = atomicAdd(&sh.ncand, 1);
       sh.ckey[slot] = key;
       sh.cidx[slot] = j;
     }
+  };
+  for (int j4 = threadIdx.x; j4 < V / 4; j4 += kSelThreads) {
+    const float4 q = __ldcs(reinterpret_cast<const float4*>(s) + j4);  // last read of the row
+    take(q.x, 4 * j4);
+    take(q.y, 4 * j4 + 1);
+    take(q.z, 4 * j4 + 2);
+    take(q.w, 4 * j4 + 3);
   }
+  for (int j = (V & ~3) + (int)threadIdx.x; j < V; j += kSelThreads) take(s[j], j);
   __syncthreads();
   const int n = sh.ncand;
   int p2 = 1;
