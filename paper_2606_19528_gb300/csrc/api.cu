@@ -216,6 +216,10 @@ struct Plan {
   std::vector<Ws> ws;
   std::vector<size_t> offs;
   size_t part_off[kPhases] = {0, 0, 0}, n_partials[kPhases] = {0, 0, 0};
+  // split contractions: per projection, the split counts of its forward and
+  // backward contraction and its fp32 partial buffer (planned from the shapes)
+  std::vector<int> split_f, split_b;
+  std::vector<size_t> split_off;
   size_t zero_bytes = 0;  // [0, zero_bytes) is cleared at the start of a call
   size_t total = 0;
 };
@@ -230,6 +234,87 @@ inline const bf* cb(const lora_bf16* p) { return reinterpret_cast<const bf*>(p);
 inline bf* mb(lora_bf16* p) { return reinterpret_cast<bf*>(p); }
 
 inline bool is_q4(const lora_proj& p) { return p.Wq.codes != nullptr; }
+inline int64_t rup(int64_t x, int64_t m) { return (x + m - 1) / m * m; }
+
+// ------------------------------------------------------------------ fused-contraction problems
+// Output [M, N] over a contraction of Kc base columns plus an r-wide adapter
+// slab; one contraction pass, output written directly (no split).
+void gemm_shape(GemmProblem& g, int64_t M, int64_t N, int64_t Kc, int64_t r) {
+  g.ldo = (int)N;
+  g.out_f32 = 0;
+  g.M = (int)M;
+  g.N = (int)N;
+  g.Kmain = (int)Kc;
+  g.r = (int)r;
+  g.num_n_tiles = cdiv(N, gemm_tile_n());
+  g.num_m_tiles = cdiv(M, gemm_tile_m());
+  g.m_fast = N >= M ? 1 : 0;  // the weight operand at least as large as the activation operand
+  g.kb_main = cdiv(Kc, gemm_tile_k());
+  g.kb_total = g.kb_main + cdiv(r, gemm_tile_k());
+  g.splits = 1;
+  g.kb_split = g.kb_total;
+  g.m_pad = g.num_m_tiles * gemm_tile_m();
+  g.part = nullptr;
+  g.ldp = 0;
+}
+
+// Appends the problem just filled in at b.prob[b.num_problems].
+void add_problem(GemmBatch& b) {
+  GemmProblem& g = b.prob[b.num_problems];
+  g.tile_begin = b.total_tiles;
+  b.total_tiles += g.num_m_tiles * g.num_n_tiles * g.splits;
+  b.num_problems++;
+}
+
+constexpr int kPlanPairs = 76;  // CTA pairs the split rule plans for (one per two SMs of a GB300)
+
+// Split contraction for batches with fewer output tiles than CTA pairs: a
+// problem of kb blocks is cut into ceil(kb / L) splits (at most 8) with L the
+// batch's block-units per pair (at least 8 blocks), so the (tile, split) units
+// fill the pairs about once.  Writes each problem's split count (1: none).
+void choose_splits(const GemmBatch& b, int* splits) {
+  long long tiles = 0, work = 0;
+  for (int p = 0; p < b.num_problems; ++p) {
+    const GemmProblem& g = b.prob[p];
+    tiles += (long long)g.num_m_tiles * g.num_n_tiles;
+    work += (long long)g.num_m_tiles * g.num_n_tiles * g.kb_total;
+    splits[p] = 1;
+  }
+  if (tiles == 0 || tiles >= kPlanPairs) return;
+  const long long L = std::max<long long>(8, (work + kPlanPairs - 1) / kPlanPairs);
+  for (int p = 0; p < b.num_problems; ++p) {
+    const GemmProblem& g = b.prob[p];
+    int sp = (int)std::min<long long>(8, std::max<long long>(1, (g.kb_total + L - 1) / L));
+    if (sp > 1) sp = (g.kb_total + (g.kb_total + sp - 1) / sp - 1) / ((g.kb_total + sp - 1) / sp);  // no empty split
+    splits[p] = sp;
+  }
+}
+
+// fp32 partial elements of a problem cut into `sp` splits.
+size_t split_floats(const GemmProblem& g, int sp) {
+  return sp > 1 ? up256((size_t)sp * g.m_pad * (size_t)rup(g.N, 4) * 4) / 4 : 0;
+}
+
+// Applies split counts (partials of problem p at parts[p]): tile list, and
+// fp32 output maps over the partial buffers.
+int apply_splits(GemmBatch& b, const int* splits, float* const* parts) {
+  b.total_tiles = 0;
+  for (int p = 0; p < b.num_problems; ++p) {
+    GemmProblem& g = b.prob[p];
+    if (splits[p] > 1) {
+      g.splits = splits[p];
+      g.kb_split = (g.kb_total + g.splits - 1) / g.splits;
+      g.ldp = (int)rup(g.N, 4);
+      g.part = parts[p];
+      const int rc = make_map(&b.tmOut[p], g.part, g.N, (uint64_t)g.splits * g.m_pad, g.ldp, 32, 32, true);
+      if (rc != LORA_OK) return rc;
+    }
+    g.tile_begin = b.total_tiles;
+    b.total_tiles += g.num_m_tiles * g.num_n_tiles * g.splits;
+  }
+  return LORA_OK;
+}
+
 
 // Adapter operands of one projection's fused contraction.
 struct Operands {
@@ -509,20 +594,9 @@ int add_fwd_problem(GemmBatch& b, const lora_proj& p, const Operands& o) {
   if ((rc = make_map(&b.tmB2[i], o.B, r, N, o.ld_b, 64, 64)) != LORA_OK) return rc;
   if ((rc = make_map(&b.tmOut[i], p.y, N, T, N, 64, 32)) != LORA_OK) return rc;
   GemmProblem& g = b.prob[i];
+  gemm_shape(g, T, N, K, r);
   g.out = mb(p.y);
-  g.ldo = (int)N;
-  g.M = (int)T;
-  g.N = (int)N;
-  g.Kmain = (int)K;
-  g.r = (int)r;
-  g.num_n_tiles = cdiv(N, gemm_tile_n());
-  g.num_m_tiles = cdiv(T, gemm_tile_m());
-  g.m_fast = N >= T ? 1 : 0;  // weight operand [N, K] at least as large as x [T, K]
-  g.kb_main = cdiv(K, gemm_tile_k());
-  g.kb_total = g.kb_main + cdiv(r, gemm_tile_k());
-  g.tile_begin = b.total_tiles;
-  b.total_tiles += g.num_m_tiles * g.num_n_tiles;
-  b.num_problems++;
+  add_problem(b);
   return LORA_OK;
 }
 
@@ -549,20 +623,9 @@ int add_bwd_problem(GemmBatch& b, const lora_proj& p, const Operands& o) {
   if ((rc = make_map(&b.tmB2[i], p.A, K, r, K, 64, 64)) != LORA_OK) return rc;
   if ((rc = make_map(&b.tmOut[i], p.dx, K, T, K, 64, 32)) != LORA_OK) return rc;
   GemmProblem& g = b.prob[i];
+  gemm_shape(g, T, K, N, r);
   g.out = mb(p.dx);
-  g.ldo = (int)K;
-  g.M = (int)T;
-  g.N = (int)K;
-  g.Kmain = (int)N;
-  g.r = (int)r;
-  g.num_n_tiles = cdiv(K, gemm_tile_n());
-  g.num_m_tiles = cdiv(T, gemm_tile_m());
-  g.m_fast = K >= T ? 1 : 0;  // weight operand [N, K] at least as large as dy [T, N]
-  g.kb_main = cdiv(N, gemm_tile_k());
-  g.kb_total = g.kb_main + cdiv(r, gemm_tile_k());
-  g.tile_begin = b.total_tiles;
-  b.total_tiles += g.num_m_tiles * g.num_n_tiles;
-  b.num_problems++;
+  add_problem(b);
   return LORA_OK;
 }
 
@@ -659,10 +722,17 @@ int run_step(const lora_proj* projs, int n, int mode, void* ws, const Plan& pl, 
         GemmBatch b;
         init_batch(b, d);
         b.tile_counter = counters + next_counter++;
-        for (size_t i = i0; i < order.size() && i < i0 + kMaxProblems; ++i)
+        int sp[kMaxProblems];
+        float* parts[kMaxProblems];
+        for (size_t i = i0; i < order.size() && i < i0 + kMaxProblems; ++i) {
           if ((rc = add_fwd_problem(b, projs[order[i]], ops[order[i]])) != LORA_OK) return rc;
+          sp[i - i0] = pl.split_f[order[i]];
+          parts[i - i0] = at<float>(ws, pl.split_off[order[i]]);
+        }
+        if ((rc = apply_splits(b, sp, parts)) != LORA_OK) return rc;
         ProfScope ps(LORA_KERNEL_GEMM_FWD, st);
         if (launch_fused_gemm(b, false, q4 != 0, d->num_sms, st) != cudaSuccess) return LORA_ECUDA;
+        if (launch_split_reduce(b, st) != cudaSuccess) return LORA_ECUDA;
       }
     }
   }
@@ -735,17 +805,25 @@ int run_step(const lora_proj* projs, int n, int mode, void* ws, const Plan& pl, 
         GemmBatch b;
         init_batch(b, d);
         b.tile_counter = counters + next_counter++;
-        for (size_t i = i0; i < order.size() && i < i0 + kMaxProblems; ++i)
+        int sp[kMaxProblems];
+        float* parts[kMaxProblems];
+        for (size_t i = i0; i < order.size() && i < i0 + kMaxProblems; ++i) {
           if ((rc = add_bwd_problem(b, projs[order[i]], ops[order[i]])) != LORA_OK) return rc;
+          sp[i - i0] = pl.split_b[order[i]];
+          parts[i - i0] = at<float>(ws, pl.split_off[order[i]]);
+        }
+        if ((rc = apply_splits(b, sp, parts)) != LORA_OK) return rc;
         ProfScope ps(LORA_KERNEL_GEMM_BWD, st);
         if (launch_fused_gemm(b, true, q4 != 0, d->num_sms, st) != cudaSuccess) return LORA_ECUDA;
+        if (launch_split_reduce(b, st) != cudaSuccess) return LORA_ECUDA;
       }
     }
   }
   return LORA_OK;
 }
 
-int plan_all(const lora_proj* projs, int n, int mode, Plan* pl) {
+// allow_split false: every contraction in one pass (the fixed-scratch forward keeps its footprint).
+int plan_all(const lora_proj* projs, int n, int mode, Plan* pl, bool allow_split = true) {
   // partials are bounded by the smallest unit size (most units per tile)
   const int tile = rank_mma_tile();
   auto upt = [&](int64_t len) { return (size_t)cdiv(cdiv(len, 64), kMinUnitChunks); };
@@ -761,11 +839,52 @@ int plan_all(const lora_proj* projs, int n, int mode, Plan* pl) {
       if (upt(s.T) > 1) pl->n_partials[kPhBwdCols] += (tiles(s.d_out) + tiles(s.d_in)) * upt(s.T) * tile * r16;
     }
   }
+  // split contractions: batches as run_step forms them (every projection counted for the backward)
+  pl->split_f.assign(n, 1);
+  pl->split_b.assign(n, 1);
+  std::vector<size_t> split_need(n, 0);
+  for (int dir = 0; dir < 2; ++dir) {
+    if (!(mode & (dir == 0 ? LORA_FWD : LORA_BWD))) continue;
+    for (int q4 = 0; q4 < 2; ++q4) {
+      std::vector<int> order;
+      for (int i = 0; i < n; ++i)
+        if (is_q4(projs[i]) == (q4 != 0)) order.push_back(i);
+      std::stable_sort(order.begin(), order.end(), [&](int a, int b) {
+        return dir == 0 ? projs[a].shape.d_in > projs[b].shape.d_in : projs[a].shape.d_out > projs[b].shape.d_out;
+      });
+      for (size_t i0 = 0; i0 < order.size(); i0 += kMaxProblems) {
+        GemmBatch b;
+        memset(&b, 0, sizeof(b));
+        for (size_t i = i0; i < order.size() && i < i0 + kMaxProblems; ++i) {
+          const lora_shape& sh = projs[order[i]].shape;
+          if (dir == 0)
+            gemm_shape(b.prob[b.num_problems], sh.T, sh.d_out, sh.d_in, sh.rank);
+          else
+            gemm_shape(b.prob[b.num_problems], sh.T, sh.d_in, sh.d_out, sh.rank);
+          add_problem(b);
+        }
+        int sp[kMaxProblems];
+        choose_splits(b, sp);
+        if (!allow_split)
+          for (int q = 0; q < b.num_problems; ++q) sp[q] = 1;
+        for (int q = 0; q < b.num_problems; ++q) {
+          const int pi = order[i0 + q];
+          (dir == 0 ? pl->split_f : pl->split_b)[pi] = sp[q];
+          split_need[pi] = std::max(split_need[pi], split_floats(b.prob[q], sp[q]));
+        }
+      }
+    }
+  }
   size_t off = kWsHeader;
   pl->zero_bytes = off;
   for (int k = 0; k < kPhases; ++k) {
     pl->part_off[k] = off;
     off += up256(pl->n_partials[k] * sizeof(float));
+  }
+  pl->split_off.assign(n, 0);
+  for (int i = 0; i < n; ++i) {
+    pl->split_off[i] = off;
+    off += split_need[i] * sizeof(float);
   }
   pl->ws.resize(n);
   pl->offs.resize(n);
@@ -816,10 +935,13 @@ void layer_copy(const lora_proj* L, int n_per, uint8_t* su_scratch, std::vector<
 
 
 // ------------------------------------------------------------------ reduced-vocabulary cross entropy
-inline int64_t rup(int64_t x, int64_t m) { return (x + m - 1) / m * m; }
+
+// Split partials of one contraction: splits happen only below kPlanPairs output
+// tiles (M x N < kPlanPairs 256 x 512 padded), at most 8 of them.
+constexpr size_t kCeSplitFloats = (size_t)8 * kPlanPairs * 256 * 512 + 64 * 1024;
 
 struct CePlan {
-  size_t flags, counts, segs, J, pos, tl, tpos, ycol, rowloss, ht, ej, z, g, dht, tiles, total;
+  size_t flags, counts, segs, J, pos, tl, tpos, ycol, rowloss, ht, ej, z, g, dht, part, tiles, total;
 };
 
 int ce_check(const lora_ce_args* a, CePlan* pl) {
@@ -854,14 +976,16 @@ int ce_check(const lora_ce_args* a, CePlan* pl) {
   pl->z = take((size_t)T * rup(V, 4) * 4);
   pl->g = take((size_t)T * rup(V, 8) * 2);
   pl->dht = take((size_t)T * d * 2);
+  pl->part = take(kCeSplitFloats * 4);
   pl->total = off;
   return LORA_OK;
 }
 
 // One-problem batch of the fused contraction with no adapter slab: out [M, N] = A [M, K] . B, B given
-// as [N, K] (K-major, b_mn false) or [K, N] (MN-major, b_mn true).
+// as [N, K] (K-major, b_mn false) or [K, N] (MN-major, b_mn true); split when it has few tiles, with
+// its partials in `part` (kCeSplitFloats elements).
 int ce_gemm(const DeviceInfo* d, int* counter, const void* A, int64_t lda, const void* B, int64_t ldb, void* out,
-            int64_t ldo, int64_t M, int64_t N, int64_t K, bool b_mn, bool f32_out, cudaStream_t st) {
+            int64_t ldo, int64_t M, int64_t N, int64_t K, bool b_mn, bool f32_out, float* part, cudaStream_t st) {
   GemmBatch b;
   init_batch(b, d);
   b.tile_counter = counter;
@@ -876,21 +1000,17 @@ int ce_gemm(const DeviceInfo* d, int* counter, const void* A, int64_t lda, const
   b.tmB2[0] = b.tmB[0];
   if ((rc = make_map(&b.tmOut[0], out, N, M, ldo, f32_out ? 32 : 64, 32, f32_out)) != LORA_OK) return rc;
   GemmProblem& g = b.prob[0];
-  g.out = static_cast<bf*>(out);
+  gemm_shape(g, M, N, K, 0);
+  g.out = out;
   g.ldo = (int)ldo;
-  g.M = (int)M;
-  g.N = (int)N;
-  g.Kmain = (int)K;
-  g.r = 0;
-  g.num_n_tiles = cdiv(N, gemm_tile_n());
-  g.num_m_tiles = cdiv(M, gemm_tile_m());
-  g.m_fast = N >= M ? 1 : 0;
-  g.kb_main = cdiv(K, gemm_tile_k());
-  g.kb_total = g.kb_main;
-  g.tile_begin = 0;
-  b.total_tiles = g.num_m_tiles * g.num_n_tiles;
-  b.num_problems = 1;
-  return launch_fused_gemm(b, b_mn, false, d->num_sms, st, f32_out) == cudaSuccess ? LORA_OK : LORA_ECUDA;
+  g.out_f32 = f32_out ? 1 : 0;
+  add_problem(b);
+  int sp[1];
+  choose_splits(b, sp);
+  float* parts[1] = {part};
+  if ((rc = apply_splits(b, sp, parts)) != LORA_OK) return rc;
+  if (launch_fused_gemm(b, b_mn, false, d->num_sms, st, f32_out) != cudaSuccess) return LORA_ECUDA;
+  return launch_split_reduce(b, st) == cudaSuccess ? LORA_OK : LORA_ECUDA;
 }
 
 
@@ -898,7 +1018,7 @@ int ce_gemm(const DeviceInfo* d, int* counter, const void* A, int64_t lda, const
 constexpr int kTopkChunk = 512;  // rows of similarities per contraction
 
 struct TopkPlan {
-  size_t counters, status, en, s, total;
+  size_t counters, status, en, s, part, total;
   int chunks;
   long long lds;
 };
@@ -919,6 +1039,7 @@ int topk_check(const lora_bf16* E, int64_t V, int64_t d, int64_t k, TopkPlan* pl
   pl->status = take(4);
   pl->en = take((size_t)V * d * 2);
   pl->s = take((size_t)std::min<int64_t>(V, kTopkChunk) * pl->lds * 4);
+  pl->part = take(kCeSplitFloats * 4);  // small vocabularies: few tiles per chunk
   pl->total = off;
   return LORA_OK;
 }
@@ -1215,13 +1336,17 @@ int lora_ce_fwd_bwd(const lora_ce_args* a, void* workspace, size_t workspace_byt
       return LORA_ECUDA;
     {
       ProfScope ps(LORA_KERNEL_GEMM_FWD, st);
-      if ((rc = ce_gemm(d, tiles, ht, D, ej, D, z, ldz, nT, nJ, D, false, true, st)) != LORA_OK) return rc;
+      if ((rc = ce_gemm(d, tiles, ht, D, ej, D, z, ldz, nT, nJ, D, false, true, at<float>(ws, pl.part), st)) !=
+          LORA_OK)
+        return rc;
     }
     if (launch_ce_rows(z, ldz, nJ, ix.ycol, nT, g, ldg, rowloss, st) != cudaSuccess) return LORA_ECUDA;
     if (a->dh) {
       bf* dht = at<bf>(ws, pl.dht);
       ProfScope ps(LORA_KERNEL_GEMM_BWD, st);
-      if ((rc = ce_gemm(d, tiles + 1, g, ldg, ej, D, dht, D, nT, D, nJ, true, false, st)) != LORA_OK) return rc;
+      if ((rc = ce_gemm(d, tiles + 1, g, ldg, ej, D, dht, D, nT, D, nJ, true, false, at<float>(ws, pl.part), st)) !=
+          LORA_OK)
+        return rc;
     }
   }
   if (launch_ce_finish(rowloss, nT, ix.tpos, T, a->token_loss, a->loss, st) != cudaSuccess) return LORA_ECUDA;
@@ -1262,7 +1387,7 @@ int lora_topk_table(const lora_bf16* E, int64_t V, int64_t d, int64_t k, int32_t
     {
       ProfScope ps(LORA_KERNEL_GEMM_FWD, st);
       if ((rc = ce_gemm(dv, at<int>(ws, pl.counters) + c, en + r0 * d, d, en, d, S, pl.lds, rows, V, d, false,
-                        true, st)) != LORA_OK)
+                        true, at<float>(ws, pl.part), st)) != LORA_OK)
         return rc;
     }
     if (launch_topk_select(S, pl.lds, (int)V, (int)k, (int)r0, (int)rows, table, dv->status, st) != cudaSuccess)
@@ -1324,7 +1449,7 @@ extern "C" int lora_linear_fwd_noalloc(const lora_shape* shape, const lora_bf16*
   p.y = y;
   p.su = su;
   Plan pl;
-  if ((rc = plan_all(&p, 1, LORA_FWD, &pl)) != LORA_OK) return rc;
+  if ((rc = plan_all(&p, 1, LORA_FWD, &pl, false)) != LORA_OK) return rc;
   if (pl.total > kNoAllocScratchBytes) return LORA_ESCRATCH;
   if ((rc = check_fwd_ptrs(p)) != LORA_OK) return rc;
   int dev = 0;

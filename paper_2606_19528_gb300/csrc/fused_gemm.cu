@@ -120,12 +120,19 @@ constexpr size_t smem_bytes() {
   return 1024 + (size_t)Cfg<kQ>::kRing + (size_t)Cfg<kQ>::kEpi * kEpiStage + sizeof(Ctl);
 }
 
-// Problem p, first row m0 and first column n0 of tile t.
-__device__ __forceinline__ void decode_tile(const GemmBatch& b, int t, int& p, int& m0, int& n0) {
+// Problem p, first row m0 and first column n0 of tile t, its split ks and
+// that split's contraction blocks [kb0, kb1).
+__device__ __forceinline__ void decode_tile(const GemmBatch& b, int t, int& p, int& m0, int& n0, int& ks, int& kb0,
+                                            int& kb1) {
   p = 0;
   while (p + 1 < b.num_problems && t >= b.prob[p + 1].tile_begin) ++p;
   const GemmProblem& Q = b.prob[p];
-  const int local = t - Q.tile_begin;
+  int local = t - Q.tile_begin;
+  const int per = Q.num_m_tiles * Q.num_n_tiles;
+  ks = local / per;
+  local -= ks * per;
+  kb0 = ks * Q.kb_split;
+  kb1 = min(Q.kb_total, kb0 + Q.kb_split);
   if (Q.m_fast) {
     m0 = (local % Q.num_m_tiles) * kBM;
     n0 = (local / Q.num_m_tiles) * kBN;
@@ -290,8 +297,8 @@ __global__ void __launch_bounds__(Cfg<kQ>::kThreads, 1) fused_lora_gemm(const __
           griddep_launch_dependents();  // no tile left for this pair
           break;
         }
-        int p, m0, n0;
-        decode_tile(b, t, p, m0, n0);
+        int p, m0, n0, ks, kb0, kb1;
+        decode_tile(b, t, p, m0, n0, ks, kb0, kb1);
         const GemmProblem& Q = b.prob[p];
         const int my_m = m0 + c * kHalf;
         const bool a_mine = my_m < Q.M;
@@ -305,7 +312,7 @@ __global__ void __launch_bounds__(Cfg<kQ>::kThreads, 1) fused_lora_gemm(const __
         const uint32_t tx_a = (m0 < Q.M ? kAHalf : 0u) + (m0 + kHalf < Q.M ? kAHalf : 0u);
         const uint32_t tx_pair = tx_a + kBox * boxes;
         bool ok = true;
-        for (int kb = 0; kb < Q.kb_total; ++kb) {
+        for (int kb = kb0; kb < kb1; ++kb) {
           if (!mbar_wait_cluster(smem_u32(&ctl->empty[stage]), phase ^ 1u, wc, abort_flag)) {
             ok = false;
             break;
@@ -359,13 +366,13 @@ __global__ void __launch_bounds__(Cfg<kQ>::kThreads, 1) fused_lora_gemm(const __
           griddep_launch_dependents();  // no tile left for this pair
           break;
         }
-        int p, m0, n0;
-        decode_tile(b, t, p, m0, n0);
+        int p, m0, n0, ks, kb0, kb1;
+        decode_tile(b, t, p, m0, n0, ks, kb0, kb1);
         const GemmProblem& Q = b.prob[p];
         const int nseg = Q.N - n0 > kSeg ? 2 : 1;  // segments holding any column < N
         // segment h is free once both epilogues drained it for the previous tile
         const uint32_t drained_par = (uint32_t)((it & 1) ^ 1);
-        for (int kb = 0; kb < Q.kb_total; ++kb) {
+        for (int kb = kb0; kb < kb1; ++kb) {
           if (!mbar_wait(smem_u32(&ctl->full[stage]), phase, wc, abort_flag)) {
             ok = false;
             break;
@@ -380,7 +387,7 @@ __global__ void __launch_bounds__(Cfg<kQ>::kThreads, 1) fused_lora_gemm(const __
           const uint32_t b_addr = kQ ? Cfg<kQ>::w_tile(base, wt) : a_addr + kAHalf;
           const int nk = kb < Q.kb_main ? kBK / 16 : min(kBK / 16, (Q.r - (kb - Q.kb_main) * kBK + 15) / 16);
           for (int h = 0; h < 2; ++h) {
-            if (kb == 0) {
+            if (kb == kb0) {
               if (!mbar_wait_cluster(smem_u32(&ctl->tempty[h]), drained_par, wc, abort_flag)) {
                 ok = false;
                 break;
@@ -393,7 +400,7 @@ __global__ void __launch_bounds__(Cfg<kQ>::kThreads, 1) fused_lora_gemm(const __
             for (int k = 0; k < nk; ++k) {
               const uint64_t adesc = sw128_desc(a_addr + k * 32, 16, 1024);
               const uint64_t bdesc = kBMn ? sw128_desc(bseg + k * 2048, kBox, 1024) : sw128_desc(bseg + k * 32, 16, 1024);
-              umma_bf16_pair(d_tmem, adesc, bdesc, idesc, (kb | k) != 0 ? 1u : 0u);
+              umma_bf16_pair(d_tmem, adesc, bdesc, idesc, (kb != kb0 || k != 0) ? 1u : 0u);
             }
           }
           if (!ok) break;
@@ -425,8 +432,8 @@ __global__ void __launch_bounds__(Cfg<kQ>::kThreads, 1) fused_lora_gemm(const __
       __syncwarp();
       if (lane == 0) mbar_arrive_cluster(tile_empty_root + (uint32_t)slot * 8u);
       if (t < 0) break;
-      int p, m0, n0;
-      decode_tile(b, t, p, m0, n0);
+      int p, m0, n0, ks, kb0, kb1;
+      decode_tile(b, t, p, m0, n0, ks, kb0, kb1);
       const GemmProblem& Q = b.prob[p];
       bool ok = mbar_wait_cluster(smem_u32(&ctl->tfull), (uint32_t)(it & 1), wc, abort_flag);
       ok = __all_sync(0xffffffffu, ok);
@@ -436,14 +443,17 @@ __global__ void __launch_bounds__(Cfg<kQ>::kThreads, 1) fused_lora_gemm(const __
       const uint32_t stg = epi_base + (uint32_t)(warp - 2) * kEpiStage;
       for (int h = 0; h < 2; ++h) {
         // a staged block is 32 rows x 128 bytes: 64 bf16 columns, or 32 fp32 columns
-        constexpr int kBlockCols = kF32 ? 32 : 64;
-        for (int cc = 0; cc < Cfg<kQ>::kPartCols; cc += kBlockCols) {
+        // (fp32 output, or the partial of one split of the contraction)
+        const bool f32 = kF32 || Q.splits > 1;
+        const int block_cols = f32 ? 32 : 64;
+        const int row_st = (Q.splits > 1 ? ks * Q.m_pad : 0) + row0;  // stored row of this warp's first row
+        for (int cc = 0; cc < Cfg<kQ>::kPartCols; cc += block_cols) {
           const int col0 = h * kSeg + part * Cfg<kQ>::kPartCols + cc;  // tile column of this block
           if (n0 + col0 >= Q.N || row0 >= Q.M) break;     // uniform across the warp
           const uint32_t taddr = tmem_base + ((uint32_t)(q * 32) << 16) + (uint32_t)col0;
           uint32_t v[32], w[32];
           tmem_ld_32x32b_x32(taddr, v);
-          if (!kF32) tmem_ld_32x32b_x32(taddr + 32u, w);
+          if (!f32) tmem_ld_32x32b_x32(taddr + 32u, w);
           tmem_ld_wait();
           // the previous block's store must have read the staging buffer
           if (lane == 0) bulk_wait_read0();
@@ -453,7 +463,7 @@ __global__ void __launch_bounds__(Cfg<kQ>::kThreads, 1) fused_lora_gemm(const __
 #pragma unroll
           for (int k = 0; k < 8; ++k) {
             uint32_t a, b2, c2, d2;
-            if (kF32) {
+            if (f32) {
               a = v[4 * k];
               b2 = v[4 * k + 1];
               c2 = v[4 * k + 2];
@@ -472,7 +482,7 @@ __global__ void __launch_bounds__(Cfg<kQ>::kThreads, 1) fused_lora_gemm(const __
           fence_proxy_async_smem();
           __syncwarp();
           if (lane == 0) {
-            tma_store_2d(&b.tmOut[p], stg, n0 + col0, row0);
+            tma_store_2d(&b.tmOut[p], stg, n0 + col0, row_st);
             bulk_commit();
           }
         }
@@ -500,12 +510,12 @@ __global__ void __launch_bounds__(Cfg<kQ>::kThreads, 1) fused_lora_gemm(const __
       __syncwarp();
       if (lane == 0) mbar_arrive_cluster(tile_empty_root + (uint32_t)slot * 8u);
       if (t < 0) break;
-      int p, m0, n0;
-      decode_tile(b, t, p, m0, n0);
+      int p, m0, n0, ks, kb0, kb1;
+      decode_tile(b, t, p, m0, n0, ks, kb0, kb1);
       const GemmProblem& Q = b.prob[p];
       auto box_ok = [&](int h, int cc, int j) { return n0 + h * kSeg + cc * kHalf + j * 64 < Q.N; };
       bool ok = true;
-      for (int kb = 0; kb < Q.kb_total; ++kb) {
+      for (int kb = kb0; kb < kb1; ++kb) {
         const bool main = kb < Q.kb_main;
         const int wt = (int)(wseq % kWStages);
         // the weight tile's previous contents are consumed by the MMAs
@@ -566,10 +576,10 @@ __global__ void __launch_bounds__(Cfg<kQ>::kThreads, 1) fused_lora_gemm(const __
         const int t = *reinterpret_cast<volatile int*>(&ctl->tile_id[slot]);
         mbar_arrive_cluster(tile_empty_root + (uint32_t)slot * 8u);
         if (t < 0) break;
-        int p, m0, n0;
-        decode_tile(b, t, p, m0, n0);
+        int p, m0, n0, ks, kb0, kb1;
+        decode_tile(b, t, p, m0, n0, ks, kb0, kb1);
         bool ok = true;
-        for (int kb = 0; kb < b.prob[p].kb_total; ++kb, ++wseq) {
+        for (int kb = kb0; kb < kb1; ++kb, ++wseq) {
           const int wt = (int)(wseq % kWStages);
           if (!mbar_wait(smem_u32(&ctl->convd[wt]), (wseq / kWStages) & 1u, wc, abort_flag)) {
             ok = false;
@@ -593,8 +603,8 @@ __global__ void __launch_bounds__(Cfg<kQ>::kThreads, 1) fused_lora_gemm(const __
         const int t = *reinterpret_cast<volatile int*>(&ctl->tile_id[slot]);
         mbar_arrive_cluster(tile_empty_root + (uint32_t)slot * 8u);
         if (t < 0) break;
-        int p, m0, n0;
-        decode_tile(b, t, p, m0, n0);
+        int p, m0, n0, ks, kb0, kb1;
+        decode_tile(b, t, p, m0, n0, ks, kb0, kb1);
         const GemmProblem& Q = b.prob[p];
         auto box_ok = [&](int h, int j) { return n0 + h * kSeg + c * kHalf + j * 64 < Q.N; };
         // bytes of this CTA's code and (s, b) boxes per block
@@ -608,7 +618,7 @@ __global__ void __launch_bounds__(Cfg<kQ>::kThreads, 1) fused_lora_gemm(const __
           }
         }
         bool ok = true;
-        for (int kb = 0; kb < Q.kb_main; ++kb) {
+        for (int kb = kb0; kb < min(kb1, Q.kb_main); ++kb) {
           if (!mbar_wait(smem_u32(&ctl->qempty[qs]), qpar ^ 1u, wc, abort_flag)) {
             ok = false;
             break;
@@ -662,7 +672,57 @@ __global__ void __launch_bounds__(Cfg<kQ>::kThreads, 1) fused_lora_gemm(const __
   }
 }
 
+// out[m, n] = sum over s of part[s * m_pad + m, n], s in order; one thread per
+// 4 consecutive columns of a row of every split problem.
+__global__ void __launch_bounds__(256) split_reduce_kernel(const __grid_constant__ GemmBatch b, int total4) {
+  griddep_wait();
+  griddep_launch_dependents();
+  int e = blockIdx.x * blockDim.x + threadIdx.x;
+  if (e >= total4) return;
+  int p = 0;
+  for (; p < b.num_problems; ++p) {
+    const GemmProblem& Q = b.prob[p];
+    if (Q.splits <= 1) continue;
+    const int per = Q.M * ((Q.N + 3) / 4);
+    if (e < per) break;
+    e -= per;
+  }
+  const GemmProblem& Q = b.prob[p];
+  const int n4 = (Q.N + 3) / 4;
+  const int m = e / n4, n = (e % n4) * 4;
+  float acc[4] = {0.f, 0.f, 0.f, 0.f};
+  for (int s = 0; s < Q.splits; ++s) {
+    const float* src = Q.part + ((size_t)s * Q.m_pad + m) * Q.ldp + n;
+    if (n + 3 < Q.N) {
+      const float4 v = __ldcs(reinterpret_cast<const float4*>(src));
+      acc[0] += v.x;
+      acc[1] += v.y;
+      acc[2] += v.z;
+      acc[3] += v.w;
+    } else {
+      for (int q = 0; q < 4 && n + q < Q.N; ++q) acc[q] += src[q];
+    }
+  }
+  for (int q = 0; q < 4 && n + q < Q.N; ++q) {
+    if (Q.out_f32)
+      static_cast<float*>(Q.out)[(size_t)m * Q.ldo + n + q] = acc[q];
+    else
+      static_cast<__nv_bfloat16*>(Q.out)[(size_t)m * Q.ldo + n + q] = __float2bfloat16_rn(acc[q]);
+  }
+}
+
 }  // namespace
+
+cudaError_t launch_split_reduce(const GemmBatch& batch, cudaStream_t stream) {
+  long long total4 = 0;
+  for (int p = 0; p < batch.num_problems; ++p) {
+    const GemmProblem& Q = batch.prob[p];
+    if (Q.splits > 1) total4 += (long long)Q.M * ((Q.N + 3) / 4);
+  }
+  if (total4 == 0) return cudaSuccess;
+  return launch_kernel(split_reduce_kernel, dim3((unsigned)((total4 + 255) / 256)), dim3(256), 0, stream, 1, batch,
+                       (int)total4);
+}
 
 size_t fused_gemm_smem_bytes() { return smem_bytes<false>(); }
 

@@ -51,8 +51,9 @@ cudaError_t launch_kernel(void (*kernel)(KArgs...), dim3 grid, dim3 block, size_
 constexpr int kMaxProblems = 8;
 
 struct GemmProblem {
-  __nv_bfloat16* out;  // [M, N] bf16, leading dimension ldo
+  void* out;           // [M, N] bf16 (fp32 when out_f32), leading dimension ldo
   int ldo;
+  int out_f32;
   int M;               // tokens
   int N;               // output columns
   int Kmain;           // base contraction length
@@ -63,7 +64,14 @@ struct GemmProblem {
   int kb_total;        // base + adapter blocks
   int m_fast;          // 1: consecutive tiles walk M (the weight tile stays put)
   int num_m_tiles;
-
+  // split contraction: splits > 1 cuts [0, kb_total) into ranges of kb_split
+  // blocks; each (tile, split) writes an fp32 partial through tmOut, split s at
+  // rows s * m_pad.., and split_reduce sums the splits in order into out
+  int splits;
+  int kb_split;
+  int m_pad;           // num_m_tiles * tile rows
+  float* part;         // partials [splits * m_pad, ldp]
+  int ldp;
 };
 
 // One launch: up to kMaxProblems independent fused contractions.
@@ -94,6 +102,9 @@ struct GemmBatch {
 cudaError_t launch_fused_gemm(const GemmBatch& batch, bool b_mn_major, bool q4, int num_sms, cudaStream_t stream,
                               bool f32_out = false);
 size_t fused_gemm_smem_bytes();
+// out = sum over s of the split partials, in split order, for every problem
+// of the batch with splits > 1 (bf16 or fp32 per out_f32).
+cudaError_t launch_split_reduce(const GemmBatch& batch, cudaStream_t stream);
 int gemm_tile_m();
 int gemm_tile_n();
 int gemm_tile_k();

@@ -207,10 +207,11 @@ def test_layer_stack(name):
 
 
 def test_stack_equals_single_calls():
-    """The grouped launches compute y, su and dx tile by tile exactly as single
-    calls do; dA and dB may be summed in another order (the split of the token
-    reduction depends on how many tiles a launch has), so they agree to fp32
-    rounding; and a repeated stack call is bit-identical."""
+    """The grouped launches compute su exactly as single calls do; y and dx
+    agree up to the bf16 rounding of differently ordered fp32 sums (with few
+    output tiles the contractions are split, and how depends on the launch's
+    problems), dA and dB (whose token reduction is split by launch) to fp32
+    rounding; a repeated stack call is bit-identical."""
     wl = workloads.llama_sweep(256, 16)
     ps = build_layer(wl, seed=3)
     G.run_stack(ps)
@@ -221,8 +222,9 @@ def test_stack_equals_single_calls():
     for i, pr in enumerate(wl.projs):
         q = G.DevProj(*(ps[i].bits[k] for k in ("x", "W", "A", "B", "dy")), wl.scale)
         G.run_single(q)
-        for n in ("y", "su", "dx"):
-            assert torch.equal(getattr(q, n).view(torch.int16), getattr(ps[i], n).view(torch.int16)), (pr.name, n)
+        assert torch.equal(q.su.view(torch.int16), ps[i].su.view(torch.int16)), (pr.name, "su")
+        for n in ("y", "dx"):
+            assert G.rel_fro(G.host_f64(getattr(q, n)), G.host_f64(getattr(ps[i], n))) < 2e-3, (pr.name, n)
         assert G.rel_fro(G.host_f64(q.dA), G.host_f64(ps[i].dA)) < 1e-6, pr.name
         assert G.rel_fro(G.host_f64(q.dB), G.host_f64(ps[i].dB)) < 1e-6, pr.name
 
