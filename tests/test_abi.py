@@ -49,3 +49,57 @@ def test_null_arguments_are_rejected(lib):
     st = lora.make_shape(128, 256, 256, 8, 2.0)
     assert lib.lora_stack_step(ctypes.byref(lora.make_proj(st)), 0, 1, None, 0, None) == lora.LORA_EINVAL
     assert lib.lora_stack_step(ctypes.byref(lora.make_proj(st)), 1, 7, None, 0, None) == lora.LORA_EINVAL
+
+
+def test_workspace_sizes_plan_without_a_gpu(lib):
+    """Workspace planning is host arithmetic: sizes grow with the problem and
+    the split contraction adds partials only where its rule splits (few tiles)."""
+    small = lora.lora_workspace_size(lora.make_shape(256, 3072, 3072, 16, 2.0), lora.LORA_FWD_BWD)
+    big = lora.lora_workspace_size(lora.make_shape(4096, 3072, 3072, 16, 2.0), lora.LORA_FWD_BWD)
+    # T = 256: 1 x 6 output tiles (< 76 pairs), so each contraction splits (at least in two) and
+    # needs fp32 partials of 2 x 256 x 3072 x 4 bytes or more; T = 4096: 16 x 6 = 96 tiles, no
+    # partials, only the rank-r scratch (T x pad8(r) bf16 per buffer, a few MB)
+    assert small >= 2 * 256 * 3072 * 4
+    assert 0 < big < 16 * 2 ** 20
+
+
+def test_stack_ckpt_workspace_covers_the_largest_layer(lib):
+    st = lora.make_shape(1024, 3072, 3072, 16, 2.0)
+    layer = [lora.make_proj(st) for _ in range(3)]
+    one = lora.lora_stack_workspace_size(layer, lora.LORA_FWD_BWD)
+    n = lora.lora_stack_ckpt_workspace_size([layer, layer, layer])
+    assert n >= one + 3 * 1024 * 16 * 2  # a step's workspace plus one layer's su scratch
+    n_bad = ctypes.c_size_t(0)
+    arr = (lora.lora_proj * 3)(*layer)
+    assert lib.lora_stack_ckpt_workspace_size(arr, 0, 3, ctypes.byref(n_bad)) == lora.LORA_EINVAL
+    assert lib.lora_stack_ckpt_workspace_size(arr, 1, 65, ctypes.byref(n_bad)) == lora.LORA_EINVAL
+
+
+def test_q4_weights_validated_on_the_host(lib):
+    st = lora.make_shape(128, 128, 256, 8, 2.0)  # d_in not a multiple of 256
+    ws = ctypes.c_void_p(256)
+    wq = lora.make_q4(256, 256)
+    rc = lib.lora_linear_fwd_q4(ctypes.byref(st), 256, ctypes.byref(wq), 256, 256, 256, None, ws, 1 << 30, None)
+    assert rc in (lora.LORA_EINVAL, lora.LORA_EDEVICE, lora.LORA_ECUDA)
+    half = lora.make_q4(256, None)
+    st = lora.make_shape(128, 256, 256, 8, 2.0)
+    rc = lib.lora_linear_fwd_q4(ctypes.byref(st), 256, ctypes.byref(half), 256, 256, 256, None, ws, 1 << 30, None)
+    assert rc == lora.LORA_ENULL
+
+
+def test_ce_and_topk_sizes_and_arguments(lib):
+    a = lora.make_ce_args(2048, 3072, 128256, 256, 256, 256, 256, topk=256, ld_topk=500, k=500)
+    n = lora.lora_ce_workspace_size(a)
+    # worst case |T_set| = T, |J| = V: the fp32 logits alone take T x V x 4 bytes
+    assert n >= 2048 * 128256 * 4
+    n_bad = ctypes.c_size_t(0)
+    bad = lora.make_ce_args(2048, 3070, 128256, 256, 256, 256, 256)  # d not a multiple of 8
+    assert lib.lora_ce_workspace_size(ctypes.byref(bad), ctypes.byref(n_bad)) == lora.LORA_EINVAL
+    bad = lora.make_ce_args(2048, 3072, 128256, 256, 256, 256, 256, topk=256, ld_topk=10, k=11)  # k > ld_topk
+    assert lib.lora_ce_workspace_size(ctypes.byref(bad), ctypes.byref(n_bad)) == lora.LORA_EINVAL
+    bad = lora.make_ce_args(2048, 3072, 128256, None, 256, 256, 256)  # h missing
+    assert lib.lora_ce_workspace_size(ctypes.byref(bad), ctypes.byref(n_bad)) == lora.LORA_ENULL
+    t = lora.lora_topk_workspace_size(128256, 3072, 500)
+    assert t >= 128256 * 3072 * 2 + 512 * 128256 * 4  # normalised rows plus one chunk of similarities
+    for V, d, k in ((100, 12, 5), (100, 16, 101), (5000, 16, 1025), (0, 16, 1)):
+        assert lib.lora_topk_workspace_size(V, d, k, ctypes.byref(n_bad)) == lora.LORA_EINVAL
