@@ -252,6 +252,15 @@ int lora_topk_table(const lora_bf16* E, int64_t V, int64_t d, int64_t k, int32_t
  * Returns LORA_OK or LORA_ECUDA. */
 int lora_read_status(void* stream, int* status, int reset);
 
+/* Failure-detection self-check (the paper has no counterpart): enqueues one
+ * kernel that waits, with the same bounded wait every kernel of the library
+ * uses, on a barrier nothing arrives on.  After limit_ns (1 us .. 1 s) of
+ * device time the wait gives up, records LORA_ETIMEOUT in the status word and
+ * the kernel returns, leaving the context usable; lora_read_status then
+ * reports LORA_ETIMEOUT.  Returns LORA_OK once enqueued, LORA_EINVAL for a
+ * limit out of range. */
+int lora_wait_selftest(int64_t limit_ns, void* stream);
+
 /* Limit, in nanoseconds of device time, of every bounded wait in the
  * library's kernels (0 restores the default of 4 s).  For tests of the
  * timeout path; affects launches made after the call.  Returns LORA_OK. */

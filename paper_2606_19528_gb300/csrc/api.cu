@@ -1396,6 +1396,15 @@ int lora_topk_table(const lora_bf16* E, int64_t V, int64_t d, int64_t k, int32_t
   return LORA_OK;
 }
 
+int lora_wait_selftest(int64_t limit_ns, void* stream) {
+  if (limit_ns < 1000 || limit_ns > 1000000000ll) return LORA_EINVAL;
+  DeviceInfo* d = nullptr;
+  int rc = device_info(&d);
+  if (rc != LORA_OK) return rc;
+  return launch_wait_probe(d->status, limit_ns, static_cast<cudaStream_t>(stream)) == cudaSuccess ? LORA_OK
+                                                                                                    : LORA_ECUDA;
+}
+
 int lora_read_status(void* stream, int* status, int reset) {
   if (!status) return LORA_ENULL;
   if (cudaStreamSynchronize(static_cast<cudaStream_t>(stream)) != cudaSuccess) return LORA_ECUDA;

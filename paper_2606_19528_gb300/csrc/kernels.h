@@ -243,6 +243,9 @@ cudaError_t launch_topk_select(const float* S, long long lds, int V, int k, int 
                                int* status, cudaStream_t stream);
 int topk_max_k();
 
+// One bounded wait on a barrier nothing arrives on (failure-detection self-check).
+cudaError_t launch_wait_probe(int* status, long long limit_ns, cudaStream_t stream);
+
 // dst[i, j] = j < r ? src[i * r + j] : 0  for j < ld_dst (zero-padded copy of an [rows, r] matrix).
 cudaError_t launch_pad_cols(const __nv_bfloat16* src, int rows, int r, __nv_bfloat16* dst, int ld_dst,
                             cudaStream_t stream);

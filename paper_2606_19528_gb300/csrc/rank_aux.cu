@@ -80,6 +80,23 @@ __global__ void pad_cols_kernel(const __nv_bfloat16* __restrict__ src, int rows,
   }
 }
 
+// Failure-detection self-check: one thread waits, with the library's bounded
+// wait, on a barrier that nothing arrives on; the wait gives up after
+// limit_ns, records the timeout in the status word and the kernel returns.
+__global__ void wait_probe_kernel(int* status, long long limit_ns) {
+  griddep_wait();
+  griddep_launch_dependents();
+  __shared__ __align__(8) uint64_t bar;
+  __shared__ int abort_flag;
+  if (threadIdx.x == 0) {
+    mbar_init(smem_u32(&bar), 1);
+    abort_flag = 0;
+    fence_mbar_init();
+    const WaitCtl wc{status, limit_ns};
+    mbar_wait(smem_u32(&bar), 0, wc, &abort_flag);
+  }
+}
+
 int grid_for(size_t n, int threads) {
   size_t b = (n + threads - 1) / threads;
   if (b < 1) b = 1;
@@ -100,6 +117,10 @@ cudaError_t launch_reduce_rows(const RowBatch& b, cudaStream_t st) {
   const int total4 = b.red_total / 4;
   return launch_kernel(reduce_partials_kernel<RowBatch, true>, dim3((total4 + 255) / 256), dim3(256), 0, st, 1, b,
                        total4);
+}
+
+cudaError_t launch_wait_probe(int* status, long long limit_ns, cudaStream_t st) {
+  return launch_kernel(wait_probe_kernel, dim3(1), dim3(32), 0, st, 1, status, limit_ns);
 }
 
 cudaError_t launch_reduce_cols(const ColBatch& b, cudaStream_t st) {

@@ -34,7 +34,8 @@ LORA_FWD_BWD = 3
 EXPORTS = ("lora_workspace_size", "lora_linear_fwd", "lora_linear_fwd_noalloc", "lora_linear_bwd",
            "lora_linear_fwd_q4", "lora_linear_bwd_q4", "lora_stack_workspace_size",
            "lora_stack_step", "lora_stack_ckpt_workspace_size", "lora_stack_ckpt", "lora_ce_workspace_size",
-           "lora_ce_fwd_bwd", "lora_topk_workspace_size", "lora_topk_table", "lora_read_status", "lora_set_wait_limit_ns", "lora_launch_count",
+           "lora_ce_fwd_bwd", "lora_topk_workspace_size", "lora_topk_table", "lora_wait_selftest",
+           "lora_read_status", "lora_set_wait_limit_ns", "lora_launch_count",
            "lora_profile_begin", "lora_profile_begin_kinds", "lora_profile_end", "lora_strerror", "lora_version")
 
 LORA_KERNEL_GEMM_FWD = 0
@@ -101,6 +102,7 @@ def library(path: str = _LIB_PATH) -> ctypes.CDLL:
         lib.lora_ce_fwd_bwd.argtypes = [P(lora_ce_args), vp, sz, vp]
         lib.lora_topk_workspace_size.argtypes = [i64, i64, i64, P(sz)]
         lib.lora_topk_table.argtypes = [vp, i64, i64, i64, vp, vp, sz, vp]
+        lib.lora_wait_selftest.argtypes = [i64, vp]
         lib.lora_read_status.argtypes = [vp, P(i32), i32]
         lib.lora_set_wait_limit_ns.argtypes = [i64]
         lib.lora_launch_count.argtypes = []
@@ -267,6 +269,11 @@ def lora_topk_table(E, V: int, d: int, k: int, table, workspace, workspace_bytes
     """Top-k cosine-similarity table of the embedding E [V, d] into table [V, k] int32."""
     _check(library().lora_topk_table(_ptr(E), int(V), int(d), int(k), _ptr(table), _ptr(workspace),
                                      int(workspace_bytes), _stream(stream)), "lora_topk_table")
+
+
+def lora_wait_selftest(limit_ns: int, stream=None) -> None:
+    """Enqueue the bounded-wait self-check (see include/lora.h)."""
+    _check(library().lora_wait_selftest(int(limit_ns), _stream(stream)), "lora_wait_selftest")
 
 
 def lora_read_status(stream=None, reset: bool = True) -> int:

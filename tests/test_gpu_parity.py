@@ -292,3 +292,19 @@ def test_argument_errors():
     assert e.value.code == lora.LORA_ENULL
     torch.cuda.synchronize()
     assert torch.isnan(p.y).all(), "a rejected call must enqueue nothing"
+
+
+# --------------------------------------------------------------- failure detection
+
+def test_bounded_wait_expires_and_context_survives():
+    """A wait on a barrier nothing arrives on gives up after its limit, the
+    status word says LORA_ETIMEOUT, and the next call runs normally."""
+    torch.cuda.synchronize()
+    assert lora.lora_read_status() == lora.LORA_OK
+    lora.lora_wait_selftest(2_000_000)  # 2 ms
+    assert lora.lora_read_status(reset=True) == lora.LORA_ETIMEOUT
+    assert lora.lora_read_status() == lora.LORA_OK
+    s = 2.0
+    p = G.DevProj(*gen_proj(0, 7, 0, 128, 256, 256, 8, s), s)
+    G.run_single(p)
+    check_full(p)
