@@ -25,6 +25,7 @@ __device__ int g_status;  // first device-side error (kStatusTimeout), 0 if none
 
 constexpr int kMaxDevices = 64;
 constexpr size_t kWsHeader = 256;  // 64 tile counters, one per fused-GEMM launch of a call
+constexpr int kSideSms = 12;        // SMs the backward's rank-r work gets beside the contractions
 constexpr long long kDefaultWaitNs = 4000000000ll;
 
 struct DeviceInfo {
@@ -452,7 +453,8 @@ int choose_unit_chunks(const std::vector<Spec>& specs, size_t i0, size_t i1, int
   return best;
 }
 
-int launch_rows(const std::vector<RowSpec>& specs, const Arena& ar, const DeviceInfo* d, cudaStream_t st) {
+// Row products of one phase on `ctas` persistent CTAs (one per SM).
+int launch_rows(const std::vector<RowSpec>& specs, const Arena& ar, const DeviceInfo* d, int ctas, cudaStream_t st) {
   const int tile = rank_mma_tile();
   size_t pf = 0;
   int rc;
@@ -462,7 +464,7 @@ int launch_rows(const std::vector<RowSpec>& specs, const Arena& ar, const Device
     memset(&b, 0, sizeof(b));
     b.tile_rows = tile;
     // one persistent CTA per SM; (tiles, reduction length) of a row problem
-    b.unit_chunks = choose_unit_chunks(specs, i0, i1, d->num_sms, [&](const RowSpec& q) {
+    b.unit_chunks = choose_unit_chunks(specs, i0, i1, ctas, [&](const RowSpec& q) {
       return std::make_pair(cdiv(q.T, tile), q.C);
     });
     int rmax = 16;
@@ -505,7 +507,7 @@ int launch_rows(const std::vector<RowSpec>& specs, const Arena& ar, const Device
     b.partials = ar.partials;
     b.status = d->status;
     b.limit_ns = g_wait_limit_ns;
-    if (launch_rowmma(b, rmax, d->num_sms, st) != cudaSuccess) return LORA_ECUDA;
+    if (launch_rowmma(b, rmax, ctas, st) != cudaSuccess) return LORA_ECUDA;
   }
   return LORA_OK;
 }
@@ -669,6 +671,84 @@ int check_ws(void* ws, size_t ws_bytes, size_t need) {
   return LORA_OK;
 }
 
+// Side-stream schedule of a forward-and-backward call: fork after the
+// forward's row products; the dx contraction waits for sv, the end of the call
+// for dA and dB.  Each host thread has its own side stream and events per
+// device, so a stream capture on one thread never takes in another thread's
+// work; they are created on a thread's first such call and kept.
+bool overlap_enabled() {
+  static const bool on = [] {
+    const char* e = getenv("LORA_OVERLAP");
+    return !(e && e[0] == '0' && e[1] == 0);
+  }();
+  return on;
+}
+
+int side_sms_setting(int num_sms) {
+  static const int v = [] {
+    const char* e = getenv("LORA_SIDE_SMS");
+    return e ? atoi(e) : kSideSms;
+  }();
+  return std::max(2, std::min(num_sms / 4, v));
+}
+
+struct SideCtx {
+  cudaStream_t side = nullptr;
+  cudaEvent_t ev[3] = {nullptr, nullptr, nullptr};  // fork, sv ready, side done
+};
+
+struct ThreadSide {
+  SideCtx dev[kMaxDevices];
+  ~ThreadSide() {
+    for (SideCtx& c : dev) {
+      for (cudaEvent_t e : c.ev)
+        if (e) cudaEventDestroy(e);
+      if (c.side) cudaStreamDestroy(c.side);
+    }
+  }
+};
+
+thread_local ThreadSide t_side;
+
+struct Overlap {
+  bool on = false, forked = false, joined = false;
+  int side_ctas = 0;
+  cudaStream_t main = nullptr, side = nullptr;
+  cudaEvent_t ev_fork = nullptr, ev_sv = nullptr, ev_done = nullptr;
+  int init(const DeviceInfo* d, cudaStream_t st) {
+    if (!overlap_enabled()) return LORA_OK;
+    SideCtx& c = t_side.dev[d - g_dev];
+    if (!c.side && cudaStreamCreateWithFlags(&c.side, cudaStreamNonBlocking) != cudaSuccess) return LORA_ECUDA;
+    for (cudaEvent_t& e : c.ev)
+      if (!e && cudaEventCreateWithFlags(&e, cudaEventDisableTiming) != cudaSuccess) return LORA_ECUDA;
+    main = st;
+    side = c.side;
+    ev_fork = c.ev[0];
+    ev_sv = c.ev[1];
+    ev_done = c.ev[2];
+    side_ctas = side_sms_setting(d->num_sms);
+    on = true;
+    return LORA_OK;
+  }
+  int fork() {
+    forked = true;
+    return cudaEventRecord(ev_fork, main) == cudaSuccess && cudaStreamWaitEvent(side, ev_fork, 0) == cudaSuccess
+               ? LORA_OK
+               : LORA_ECUDA;
+  }
+  int wait_sv() { return cudaStreamWaitEvent(main, ev_sv, 0) == cudaSuccess ? LORA_OK : LORA_ECUDA; }
+  // the call ends when everything it put on the side stream is done
+  int join() {
+    joined = true;
+    return cudaEventRecord(ev_done, side) == cudaSuccess && cudaStreamWaitEvent(main, ev_done, 0) == cudaSuccess
+               ? LORA_OK
+               : LORA_ECUDA;
+  }
+  ~Overlap() {
+    if (forked && !joined) join();  // an error after the fork: still end after the side work
+  }
+};
+
 // Runs the given projections in `mode`; every argument already validated.
 int run_step(const lora_proj* projs, int n, int mode, void* ws, const Plan& pl, DeviceInfo* d, cudaStream_t st) {
   int rc;
@@ -678,6 +758,77 @@ int run_step(const lora_proj* projs, int n, int mode, void* ws, const Plan& pl, 
   int* counters = at<int>(ws, 0);
   int next_counter = 0;
   if (cudaMemsetAsync(ws, 0, pl.zero_bytes, st) != cudaSuccess) return LORA_ECUDA;
+  // forward and backward in one call: the backward's rank-r work runs on a side
+  // stream with a few SMs while the contractions use the rest
+  Overlap ov;
+  if (mode == LORA_FWD_BWD && (rc = ov.init(d, st)) != LORA_OK) return rc;
+  const int gemm_sms = ov.on ? d->num_sms - ov.side_ctas : d->num_sms;
+  // backward rank-r work: B^T, su^T, sv (and sv^T), then dB and dA; on `rs`
+  // with `ctas` persistent CTAs; the operands of the dx contraction go to bops
+  std::vector<Operands> bops(n);
+  auto bwd_rank = [&](cudaStream_t rs, int ctas) -> int {
+    int rc;
+    std::vector<RowSpec> rows;
+    std::vector<ColSpec> cols;
+    std::vector<bf*> sut(n), svt(n);
+    std::vector<Operands>& ops = bops;
+    TransposeJobs tj;
+    memset(&tj, 0, sizeof(tj));
+    {
+      ProfScope ps(LORA_KERNEL_PAD, rs);
+      // rank sides as K-major tensor-core operands: B^T for sv = s dy B and
+      // su^T for dB = dy^T su, zero rows past r
+      auto transpose = [&](const bf* src, int rows_, int r, bf* dst) -> int {
+        if (tj.count == kMaxTransposes) {
+          if (launch_transposes(tj, rs) != cudaSuccess) return LORA_ECUDA;
+          memset(&tj, 0, sizeof(tj));
+        }
+        const int k = tj.count++;
+        tj.src[k] = src;
+        tj.dst[k] = dst;
+        tj.n[k] = rows_;
+        tj.r[k] = r;
+        tj.ld[k] = r;
+        tj.r8[k] = rank_pad8(r);
+        tj.max_elems = std::max(tj.max_elems, (long long)rows_ * tj.r8[k]);
+        return LORA_OK;
+      };
+      for (int i = 0; i < n; ++i) {
+        const lora_proj& p = projs[i];
+        const int T = (int)p.shape.T, N = (int)p.shape.d_out, r = (int)p.shape.rank, r8 = rank_pad8(r);
+        bf* bt = at<bf>(W_(i), plans[i].bt);
+        sut[i] = at<bf>(W_(i), plans[i].sut);
+        svt[i] = at<bf>(W_(i), plans[i].svt);
+        if ((rc = transpose(cb(p.B), N, r, bt)) != LORA_OK) return rc;
+        if ((rc = transpose(cb(p.su), T, r, sut[i])) != LORA_OK) return rc;
+        bf* sv = at<bf>(W_(i), plans[i].sv);
+        add_row_block(rows, cb(p.dy), N, T, N, p.shape.scale, bt, N, r, sv, r8, nullptr, 0, svt[i], false);
+        ops[i].s_in = sv;
+        ops[i].ld_s = r8;
+      }
+      if (launch_transposes(tj, rs) != cudaSuccess) return LORA_ECUDA;
+    }
+    {
+      ProfScope ps(LORA_KERNEL_ROWPROJ, rs);
+      if ((rc = launch_rows(rows, arena(ws, pl, kPhBwdRows), d, ctas, rs)) != LORA_OK) return rc;
+    }
+    if (ov.on && cudaEventRecord(ov.ev_sv, rs) != cudaSuccess) return LORA_ECUDA;
+    for (int i = 0; i < n; ++i) {
+      const lora_proj& p = projs[i];
+      const int T = (int)p.shape.T, N = (int)p.shape.d_out, r = (int)p.shape.rank;
+      add_col_block(cols, cb(p.dy), N, T, N, sut[i], T, r, p.dB, 1, false);
+    }
+    for (int i = 0; i < n; ++i) {
+      const lora_proj& p = projs[i];
+      const int T = (int)p.shape.T, K = (int)p.shape.d_in, r = (int)p.shape.rank;
+      add_col_block(cols, cb(p.x), K, T, K, svt[i], T, r, p.dA, 0, true);
+    }
+    {
+      ProfScope ps(LORA_KERNEL_COLPROJ, rs);
+      if ((rc = launch_cols(cols, arena(ws, pl, kPhBwdCols), d, ctas, rs)) != LORA_OK) return rc;
+    }
+    return LORA_OK;
+  };
   if (mode & LORA_FWD) {
     std::vector<Operands> ops(n);
     std::vector<RowSpec> rows;
@@ -708,8 +859,11 @@ int run_step(const lora_proj* projs, int n, int mode, void* ws, const Plan& pl, 
     }
     {
       ProfScope ps(LORA_KERNEL_ROWPROJ, st);
-      if ((rc = launch_rows(rows, arena(ws, pl, kPhFwdRows), d, st)) != LORA_OK) return rc;
+      if ((rc = launch_rows(rows, arena(ws, pl, kPhFwdRows), d, d->num_sms, st)) != LORA_OK) return rc;
     }
+    // the backward's rank-r work needs su only: it may start now, beside the forward contractions
+    if (ov.on && (rc = ov.fork()) != LORA_OK) return rc;
+    if (ov.on && (rc = bwd_rank(ov.side, ov.side_ctas)) != LORA_OK) return rc;
     // one launch per batch of bf16-weight, then of 4-bit-weight problems;
     // heavier problems first so that the tile walk ends balanced
     for (int q4 = 0; q4 < 2; ++q4) {
@@ -731,70 +885,16 @@ int run_step(const lora_proj* projs, int n, int mode, void* ws, const Plan& pl, 
         }
         if ((rc = apply_splits(b, sp, parts)) != LORA_OK) return rc;
         ProfScope ps(LORA_KERNEL_GEMM_FWD, st);
-        if (launch_fused_gemm(b, false, q4 != 0, d->num_sms, st) != cudaSuccess) return LORA_ECUDA;
+        if (launch_fused_gemm(b, false, q4 != 0, gemm_sms, st) != cudaSuccess) return LORA_ECUDA;
         if (launch_split_reduce(b, st) != cudaSuccess) return LORA_ECUDA;
       }
     }
   }
   if (mode & LORA_BWD) {
-    std::vector<Operands> ops(n);
-    std::vector<RowSpec> rows;
-    std::vector<ColSpec> cols;
-    std::vector<bf*> sut(n), svt(n);
-    TransposeJobs tj;
-    memset(&tj, 0, sizeof(tj));
-    {
-      ProfScope ps(LORA_KERNEL_PAD, st);
-      // rank sides as K-major tensor-core operands: B^T for sv = s dy B and
-      // su^T for dB = dy^T su, zero rows past r
-      auto transpose = [&](const bf* src, int rows_, int r, bf* dst) -> int {
-        if (tj.count == kMaxTransposes) {
-          if (launch_transposes(tj, st) != cudaSuccess) return LORA_ECUDA;
-          memset(&tj, 0, sizeof(tj));
-        }
-        const int k = tj.count++;
-        tj.src[k] = src;
-        tj.dst[k] = dst;
-        tj.n[k] = rows_;
-        tj.r[k] = r;
-        tj.ld[k] = r;
-        tj.r8[k] = rank_pad8(r);
-        tj.max_elems = std::max(tj.max_elems, (long long)rows_ * tj.r8[k]);
-        return LORA_OK;
-      };
-      for (int i = 0; i < n; ++i) {
-        const lora_proj& p = projs[i];
-        const int T = (int)p.shape.T, N = (int)p.shape.d_out, r = (int)p.shape.rank, r8 = rank_pad8(r);
-        bf* bt = at<bf>(W_(i), plans[i].bt);
-        sut[i] = at<bf>(W_(i), plans[i].sut);
-        svt[i] = at<bf>(W_(i), plans[i].svt);
-        if ((rc = transpose(cb(p.B), N, r, bt)) != LORA_OK) return rc;
-        if ((rc = transpose(cb(p.su), T, r, sut[i])) != LORA_OK) return rc;
-        bf* sv = at<bf>(W_(i), plans[i].sv);
-        add_row_block(rows, cb(p.dy), N, T, N, p.shape.scale, bt, N, r, sv, r8, nullptr, 0, svt[i], false);
-        ops[i].s_in = sv;
-        ops[i].ld_s = r8;
-      }
-      if (launch_transposes(tj, st) != cudaSuccess) return LORA_ECUDA;
-    }
-    {
-      ProfScope ps(LORA_KERNEL_ROWPROJ, st);
-      if ((rc = launch_rows(rows, arena(ws, pl, kPhBwdRows), d, st)) != LORA_OK) return rc;
-    }
-    for (int i = 0; i < n; ++i) {
-      const lora_proj& p = projs[i];
-      const int T = (int)p.shape.T, N = (int)p.shape.d_out, r = (int)p.shape.rank;
-      add_col_block(cols, cb(p.dy), N, T, N, sut[i], T, r, p.dB, 1, false);
-    }
-    for (int i = 0; i < n; ++i) {
-      const lora_proj& p = projs[i];
-      const int T = (int)p.shape.T, K = (int)p.shape.d_in, r = (int)p.shape.rank;
-      add_col_block(cols, cb(p.x), K, T, K, svt[i], T, r, p.dA, 0, true);
-    }
-    {
-      ProfScope ps(LORA_KERNEL_COLPROJ, st);
-      if ((rc = launch_cols(cols, arena(ws, pl, kPhBwdCols), d, d->num_sms, st)) != LORA_OK) return rc;
-    }
+    if (!ov.on && (rc = bwd_rank(st, d->num_sms)) != LORA_OK) return rc;
+    // the dx contraction reads sv: with the side stream, wait for it
+    if (ov.on && (rc = ov.wait_sv()) != LORA_OK) return rc;
+    std::vector<Operands>& ops = bops;
     for (int q4 = 0; q4 < 2; ++q4) {
       std::vector<int> order;
       for (int i = 0; i < n; ++i)
@@ -814,11 +914,13 @@ int run_step(const lora_proj* projs, int n, int mode, void* ws, const Plan& pl, 
         }
         if ((rc = apply_splits(b, sp, parts)) != LORA_OK) return rc;
         ProfScope ps(LORA_KERNEL_GEMM_BWD, st);
-        if (launch_fused_gemm(b, true, q4 != 0, d->num_sms, st) != cudaSuccess) return LORA_ECUDA;
+        if (launch_fused_gemm(b, true, q4 != 0, gemm_sms, st) != cudaSuccess) return LORA_ECUDA;
         if (launch_split_reduce(b, st) != cudaSuccess) return LORA_ECUDA;
       }
     }
   }
+  // the call ends when the side stream's dA and dB are done
+  if (ov.on && (rc = ov.join()) != LORA_OK) return rc;
   return LORA_OK;
 }
 
