@@ -11,6 +11,8 @@
 #include <algorithm>
 #include <atomic>
 #include <cstdlib>
+#include <functional>
+#include <map>
 #include <mutex>
 #include <vector>
 
@@ -267,28 +269,93 @@ void add_problem(GemmBatch& b) {
   b.num_problems++;
 }
 
-constexpr int kPlanPairs = 76;  // CTA pairs the split rule plans for (one per two SMs of a GB300)
+constexpr int kPlanSms = 152;              // SMs the split rule plans for (a GB300)
+constexpr int kPlanPairs = kPlanSms / 2;  // CTA pairs of a launch on all of them
 
-// Split contraction for batches with fewer output tiles than CTA pairs: a
-// problem of kb blocks is cut into ceil(kb / L) splits (at most 8) with L the
-// batch's block-units per pair (at least 8 blocks), so the (tile, split) units
-// fill the pairs about once.  Writes each problem's split count (1: none).
-void choose_splits(const GemmBatch& b, int* splits) {
-  long long tiles = 0, work = 0;
+// Split contraction for batches with fewer output tiles than CTA pairs.  The
+// persistent kernel hands out (tile, split) units in order to whichever pair
+// is free, so for each candidate split length L (problem p cut into
+// ceil(kb_p / L) splits, at most 8) the walk is simulated on `pairs` pairs in
+// units of one k-block of a 256 x 512 tile (~0.77 us at the measured rate),
+// with a fixed cost per unit (pipeline fill, epilogue), one more for an fp32
+// partial epilogue, and the reduce launch plus its traffic; the cheapest
+// candidate wins (fewer splits on ties).  Choices are cached per shape set.
+constexpr double kUnitFixBlocks = 3.0;    // per unit: pipeline fill and epilogue
+constexpr double kPartEpiBlocks = 1.0;    // per split unit: fp32 partial tile instead of bf16
+constexpr double kReduceFixBlocks = 6.0;  // the reduce launch
+constexpr double kBytesPerBlock = 5.0e6;  // HBM bytes moved in one block time
+
+double simulate_splits(const GemmBatch& b, const int* sp, int pairs) {
+  std::vector<double> fin(pairs, 0.0);  // min-heap of pair finish times
+  std::make_heap(fin.begin(), fin.end(), std::greater<double>());
+  double reduce = 0.0;
+  bool any = false;
+  for (int p = 0; p < b.num_problems; ++p) {
+    const GemmProblem& g = b.prob[p];
+    const int per = g.num_m_tiles * g.num_n_tiles;
+    const int kbs = (g.kb_total + sp[p] - 1) / sp[p];
+    for (int ks = 0; ks < sp[p]; ++ks) {
+      const int len = std::min(g.kb_total, (ks + 1) * kbs) - ks * kbs;
+      const double d = len + kUnitFixBlocks + (sp[p] > 1 ? kPartEpiBlocks : 0.0);
+      for (int t = 0; t < per; ++t) {
+        std::pop_heap(fin.begin(), fin.end(), std::greater<double>());
+        fin.back() += d;
+        std::push_heap(fin.begin(), fin.end(), std::greater<double>());
+      }
+    }
+    if (sp[p] > 1) {
+      any = true;
+      reduce += (double)g.m_pad * g.N * (4.0 * sp[p] + 2.0) / kBytesPerBlock;
+    }
+  }
+  return *std::max_element(fin.begin(), fin.end()) + reduce + (any ? kReduceFixBlocks : 0.0);
+}
+
+void choose_splits(const GemmBatch& b, int* splits, int pairs = kPlanPairs) {
+  long long tiles = 0;
+  std::vector<long long> key;
+  key.push_back(pairs);
   for (int p = 0; p < b.num_problems; ++p) {
     const GemmProblem& g = b.prob[p];
     tiles += (long long)g.num_m_tiles * g.num_n_tiles;
-    work += (long long)g.num_m_tiles * g.num_n_tiles * g.kb_total;
+    key.insert(key.end(), {g.num_m_tiles, g.num_n_tiles, g.kb_total, g.m_pad, g.N});
     splits[p] = 1;
   }
-  if (tiles == 0 || tiles >= kPlanPairs) return;
-  const long long L = std::max<long long>(8, (work + kPlanPairs - 1) / kPlanPairs);
-  for (int p = 0; p < b.num_problems; ++p) {
-    const GemmProblem& g = b.prob[p];
-    int sp = (int)std::min<long long>(8, std::max<long long>(1, (g.kb_total + L - 1) / L));
-    if (sp > 1) sp = (g.kb_total + (g.kb_total + sp - 1) / sp - 1) / ((g.kb_total + sp - 1) / sp);  // no empty split
-    splits[p] = sp;
+  if (tiles == 0 || tiles >= pairs) return;
+  static std::mutex mu;
+  static std::map<std::vector<long long>, std::vector<int>> cache;
+  {
+    std::lock_guard<std::mutex> lk(mu);
+    auto it = cache.find(key);
+    if (it != cache.end()) {
+      std::copy(it->second.begin(), it->second.end(), splits);
+      return;
+    }
   }
+  std::vector<int> cand;
+  for (int p = 0; p < b.num_problems; ++p)
+    for (int s = 1; s <= 8; ++s) cand.push_back((b.prob[p].kb_total + s - 1) / s);
+  std::sort(cand.begin(), cand.end(), std::greater<int>());  // longest splits (fewest) first
+  cand.erase(std::unique(cand.begin(), cand.end()), cand.end());
+  std::vector<int> sp(b.num_problems), best(b.num_problems, 1);
+  double best_cost = simulate_splits(b, best.data(), pairs);
+  for (int L : cand) {
+    for (int p = 0; p < b.num_problems; ++p) {
+      const int kb = b.prob[p].kb_total;
+      int s = std::min(8, std::max(1, (kb + L - 1) / L));
+      if (s > 1) s = (kb + (kb + s - 1) / s - 1) / ((kb + s - 1) / s);  // no empty split
+      sp[p] = s;
+    }
+    const double c = simulate_splits(b, sp.data(), pairs);
+    if (c < best_cost - 1e-9) {
+      best_cost = c;
+      best = sp;
+    }
+  }
+  std::copy(best.begin(), best.end(), splits);
+  std::lock_guard<std::mutex> lk(mu);
+  if (cache.size() > 4096) cache.clear();
+  cache.emplace(key, best);
 }
 
 // fp32 partial elements of a problem cut into `sp` splits.
@@ -944,6 +1011,8 @@ int plan_all(const lora_proj* projs, int n, int mode, Plan* pl, bool allow_split
   // split contractions: batches as run_step forms them (every projection counted for the backward)
   pl->split_f.assign(n, 1);
   pl->split_b.assign(n, 1);
+  // a forward-and-backward call leaves the side stream's SMs out of the contractions
+  const int pairs = mode == LORA_FWD_BWD && overlap_enabled() ? (kPlanSms - side_sms_setting(kPlanSms)) / 2 : kPlanPairs;
   std::vector<size_t> split_need(n, 0);
   for (int dir = 0; dir < 2; ++dir) {
     if (!(mode & (dir == 0 ? LORA_FWD : LORA_BWD))) continue;
@@ -966,7 +1035,7 @@ int plan_all(const lora_proj* projs, int n, int mode, Plan* pl, bool allow_split
           add_problem(b);
         }
         int sp[kMaxProblems];
-        choose_splits(b, sp);
+        choose_splits(b, sp, pairs);
         if (!allow_split)
           for (int q = 0; q < b.num_problems; ++q) sp[q] = 1;
         for (int q = 0; q < b.num_problems; ++q) {
