@@ -259,6 +259,8 @@ void gemm_shape(GemmProblem& g, int64_t M, int64_t N, int64_t Kc, int64_t r) {
   g.m_pad = g.num_m_tiles * gemm_tile_m();
   g.part = nullptr;
   g.ldp = 0;
+  g.lse = nullptr;
+  g.ld_lse = 0;
 }
 
 // Appends the problem just filled in at b.prob[b.num_problems].
@@ -1112,7 +1114,8 @@ void layer_copy(const lora_proj* L, int n_per, uint8_t* su_scratch, std::vector<
 constexpr size_t kCeSplitFloats = (size_t)8 * kPlanPairs * 256 * 512 + 64 * 1024;
 
 struct CePlan {
-  size_t flags, counts, segs, J, pos, tl, tpos, ycol, rowloss, ht, ej, z, g, dht, part, tiles, total;
+  size_t flags, counts, segs, J, pos, tl, tpos, ycol, rowloss, lse, ht, ej, z, lse_part, g, dht, part, tiles, total;
+  int ld_lse;
 };
 
 int ce_check(const lora_ce_args* a, CePlan* pl) {
@@ -1142,9 +1145,13 @@ int ce_check(const lora_ce_args* a, CePlan* pl) {
   pl->tpos = take((size_t)T * 4);
   pl->ycol = take((size_t)T * 4);
   pl->rowloss = take((size_t)T * 4);
+  pl->lse = take((size_t)T * 4);
   pl->ht = take((size_t)T * d * 2);
-  pl->ej = take((size_t)V * d * 2);
+  // J is the whole vocabulary without a top-k table: E is read in place
+  pl->ej = take(a->topk ? (size_t)V * d * 2 : 0);
   pl->z = take((size_t)T * rup(V, 4) * 4);
+  pl->ld_lse = (int)cdiv(V, gemm_lse_group());
+  pl->lse_part = take((size_t)T * pl->ld_lse * 8);
   pl->g = take((size_t)T * rup(V, 8) * 2);
   pl->dht = take((size_t)T * d * 2);
   pl->part = take(kCeSplitFloats * 4);
@@ -1155,8 +1162,11 @@ int ce_check(const lora_ce_args* a, CePlan* pl) {
 // One-problem batch of the fused contraction with no adapter slab: out [M, N] = A [M, K] . B, B given
 // as [N, K] (K-major, b_mn false) or [K, N] (MN-major, b_mn true); split when it has few tiles, with
 // its partials in `part` (kCeSplitFloats elements).
+// lse (fp32 output only): per-row log-sum-exp partials [M, ld_lse], written by
+// the epilogue, or by the split reduce when the contraction is split.
 int ce_gemm(const DeviceInfo* d, int* counter, const void* A, int64_t lda, const void* B, int64_t ldb, void* out,
-            int64_t ldo, int64_t M, int64_t N, int64_t K, bool b_mn, bool f32_out, float* part, cudaStream_t st) {
+            int64_t ldo, int64_t M, int64_t N, int64_t K, bool b_mn, bool f32_out, float* part, cudaStream_t st,
+            float2* lse = nullptr, int ld_lse = 0) {
   GemmBatch b;
   init_batch(b, d);
   b.tile_counter = counter;
@@ -1175,6 +1185,8 @@ int ce_gemm(const DeviceInfo* d, int* counter, const void* A, int64_t lda, const
   g.out = out;
   g.ldo = (int)ldo;
   g.out_f32 = f32_out ? 1 : 0;
+  g.lse = lse;
+  g.ld_lse = ld_lse;
   add_problem(b);
   int sp[1];
   choose_splits(b, sp);
@@ -1497,21 +1509,28 @@ int lora_ce_fwd_bwd(const lora_ce_args* a, void* workspace, size_t workspace_byt
   float* rowloss = at<float>(ws, pl.rowloss);
   if (nT > 0) {
     bf* ht = at<bf>(ws, pl.ht);
-    bf* ej = at<bf>(ws, pl.ej);
     float* z = at<float>(ws, pl.z);
     bf* g = at<bf>(ws, pl.g);
+    float2* lse_part = at<float2>(ws, pl.lse_part);
     const int ldz = (int)rup(nJ, 4), ldg = (int)rup(nJ, 8);
     int* tiles = at<int>(ws, pl.tiles);
-    if (launch_gather_rows(cb(a->h), D, ix.tl, nT, D, ht, st) != cudaSuccess ||
-        launch_gather_rows(cb(a->E), D, ix.J, nJ, D, ej, st) != cudaSuccess)
-      return LORA_ECUDA;
+    if (launch_gather_rows(cb(a->h), D, ix.tl, nT, D, ht, st) != cudaSuccess) return LORA_ECUDA;
+    // J sorted ascending with |J| = V is every token in order: E serves as E_J
+    const bf* ej = cb(a->E);
+    if (nJ < V) {
+      bf* ejw = at<bf>(ws, pl.ej);
+      if (launch_gather_rows(cb(a->E), D, ix.J, nJ, D, ejw, st) != cudaSuccess) return LORA_ECUDA;
+      ej = ejw;
+    }
     {
       ProfScope ps(LORA_KERNEL_GEMM_FWD, st);
-      if ((rc = ce_gemm(d, tiles, ht, D, ej, D, z, ldz, nT, nJ, D, false, true, at<float>(ws, pl.part), st)) !=
-          LORA_OK)
+      if ((rc = ce_gemm(d, tiles, ht, D, ej, D, z, ldz, nT, nJ, D, false, true, at<float>(ws, pl.part), st, lse_part,
+                        pl.ld_lse)) != LORA_OK)
         return rc;
     }
-    if (launch_ce_rows(z, ldz, nJ, ix.ycol, nT, g, ldg, rowloss, st) != cudaSuccess) return LORA_ECUDA;
+    if (launch_ce_rows(lse_part, pl.ld_lse, z, ldz, nJ, ix.ycol, nT, at<float>(ws, pl.lse), rowloss, g, ldg,
+                       d->num_sms, st) != cudaSuccess)
+      return LORA_ECUDA;
     if (a->dh) {
       bf* dht = at<bf>(ws, pl.dht);
       ProfScope ps(LORA_KERNEL_GEMM_BWD, st);

@@ -447,6 +447,9 @@ __global__ void __launch_bounds__(Cfg<kQ>::kThreads, 1) fused_lora_gemm(const __
         const bool f32 = kF32 || Q.splits > 1;
         const int block_cols = f32 ? 32 : 64;
         const int row_st = (Q.splits > 1 ? ks * Q.m_pad : 0) + row0;  // stored row of this warp's first row
+        // log-sum-exp partial of this thread's row over the warp's column group
+        const bool lse_on = kF32 && Q.lse != nullptr && Q.splits == 1;  // split partials: the reduce does it
+        float lm = -INFINITY, ls = 0.f;
         for (int cc = 0; cc < Cfg<kQ>::kPartCols; cc += block_cols) {
           const int col0 = h * kSeg + part * Cfg<kQ>::kPartCols + cc;  // tile column of this block
           if (n0 + col0 >= Q.N || row0 >= Q.M) break;     // uniform across the warp
@@ -455,6 +458,20 @@ __global__ void __launch_bounds__(Cfg<kQ>::kThreads, 1) fused_lora_gemm(const __
           tmem_ld_32x32b_x32(taddr, v);
           if (!f32) tmem_ld_32x32b_x32(taddr + 32u, w);
           tmem_ld_wait();
+          if (lse_on) {
+            const int nv = min(32, Q.N - (n0 + col0));  // valid columns of the block, >= 1
+            float bm = __uint_as_float(v[0]);
+#pragma unroll
+            for (int j = 1; j < 32; ++j)
+              if (j < nv) bm = fmaxf(bm, __uint_as_float(v[j]));
+            const float mn = fmaxf(lm, bm);
+            float acc = ls * __expf(lm - mn);
+#pragma unroll
+            for (int j = 0; j < 32; ++j)
+              if (j < nv) acc += __expf(__uint_as_float(v[j]) - mn);
+            lm = mn;
+            ls = acc;
+          }
           // the previous block's store must have read the staging buffer
           if (lane == 0) bulk_wait_read0();
           __syncwarp();
@@ -485,6 +502,11 @@ __global__ void __launch_bounds__(Cfg<kQ>::kThreads, 1) fused_lora_gemm(const __
             tma_store_2d(&b.tmOut[p], stg, n0 + col0, row_st);
             bulk_commit();
           }
+        }
+        if (lse_on) {
+          const int gc = n0 + h * kSeg + part * Cfg<kQ>::kPartCols;  // first column of the group
+          if (gc < Q.N && row0 + lane < Q.M)
+            Q.lse[(long long)(row0 + lane) * Q.ld_lse + gc / Cfg<kQ>::kPartCols] = make_float2(lm, ls);
         }
         tc_fence_before();
         __syncwarp();
@@ -672,56 +694,97 @@ __global__ void __launch_bounds__(Cfg<kQ>::kThreads, 1) fused_lora_gemm(const __
   }
 }
 
-// out[m, n] = sum over s of part[s * m_pad + m, n], s in order; one thread per
-// 4 consecutive columns of a row of every split problem.
-__global__ void __launch_bounds__(256) split_reduce_kernel(const __grid_constant__ GemmBatch b, int total4) {
+constexpr int kLseGroup = 128;  // columns of one log-sum-exp partial
+static_assert(kLseGroup == Cfg<false>::kPartCols, "the epilogue's column group");
+
+// Threads the split reduce runs for a problem, a multiple of 32: one per 4
+// consecutive columns of a row; with log-sum-exp partials one warp per
+// (row, 128-column group).
+__host__ __device__ inline long long reduce_items(const GemmProblem& Q) {
+  if (Q.splits <= 1) return 0;
+  const long long n = Q.lse ? (long long)Q.M * ((Q.N + kLseGroup - 1) / kLseGroup) * 32
+                            : (long long)Q.M * ((Q.N + 3) / 4);
+  return (n + 31) / 32 * 32;
+}
+
+__device__ __forceinline__ void lse_merge2(float& m, float& s, float m2, float s2) {
+  if (m2 > m) {
+    s = s * __expf(m - m2) + s2;
+    m = m2;
+  } else if (m2 > -INFINITY) {
+    s += s2 * __expf(m2 - m);
+  }
+}
+
+// out[m, n] = sum over s of part[s * m_pad + m, n], s in order, 4 columns per
+// thread; for a problem with lse partials also each (row, column group)'s
+// (max, sum of exp) over the summed values, one warp per group.
+__global__ void __launch_bounds__(256) split_reduce_kernel(const __grid_constant__ GemmBatch b, long long total) {
   griddep_wait();
   griddep_launch_dependents();
-  int e = blockIdx.x * blockDim.x + threadIdx.x;
-  if (e >= total4) return;
+  long long e = blockIdx.x * (long long)blockDim.x + threadIdx.x;
+  if (e >= total) return;  // total is a multiple of 32: whole warps leave
   int p = 0;
   for (; p < b.num_problems; ++p) {
-    const GemmProblem& Q = b.prob[p];
-    if (Q.splits <= 1) continue;
-    const int per = Q.M * ((Q.N + 3) / 4);
+    const long long per = reduce_items(b.prob[p]);
     if (e < per) break;
     e -= per;
   }
   const GemmProblem& Q = b.prob[p];
-  const int n4 = (Q.N + 3) / 4;
-  const int m = e / n4, n = (e % n4) * 4;
+  int m, n;
+  if (Q.lse) {
+    const int ng = (Q.N + kLseGroup - 1) / kLseGroup;
+    const long long w = e >> 5;
+    m = (int)(w / ng);
+    n = (int)(w % ng) * kLseGroup + (int)(e & 31) * 4;
+  } else {
+    const int n4 = (Q.N + 3) / 4;
+    m = (int)(e / n4);
+    n = (int)(e % n4) * 4;
+  }
+  const bool row_ok = m < Q.M;
   float acc[4] = {0.f, 0.f, 0.f, 0.f};
-  for (int s = 0; s < Q.splits; ++s) {
-    const float* src = Q.part + ((size_t)s * Q.m_pad + m) * Q.ldp + n;
-    if (n + 3 < Q.N) {
-      const float4 v = __ldcs(reinterpret_cast<const float4*>(src));
-      acc[0] += v.x;
-      acc[1] += v.y;
-      acc[2] += v.z;
-      acc[3] += v.w;
-    } else {
-      for (int q = 0; q < 4 && n + q < Q.N; ++q) acc[q] += src[q];
+  if (row_ok && n < Q.N) {
+    for (int s = 0; s < Q.splits; ++s) {
+      const float* src = Q.part + ((size_t)s * Q.m_pad + m) * Q.ldp + n;
+      if (n + 3 < Q.N) {
+        const float4 v = __ldcs(reinterpret_cast<const float4*>(src));
+        acc[0] += v.x;
+        acc[1] += v.y;
+        acc[2] += v.z;
+        acc[3] += v.w;
+      } else {
+        for (int q = 0; q < 4 && n + q < Q.N; ++q) acc[q] += src[q];
+      }
+    }
+    for (int q = 0; q < 4 && n + q < Q.N; ++q) {
+      if (Q.out_f32)
+        static_cast<float*>(Q.out)[(size_t)m * Q.ldo + n + q] = acc[q];
+      else
+        static_cast<__nv_bfloat16*>(Q.out)[(size_t)m * Q.ldo + n + q] = __float2bfloat16_rn(acc[q]);
     }
   }
-  for (int q = 0; q < 4 && n + q < Q.N; ++q) {
-    if (Q.out_f32)
-      static_cast<float*>(Q.out)[(size_t)m * Q.ldo + n + q] = acc[q];
-    else
-      static_cast<__nv_bfloat16*>(Q.out)[(size_t)m * Q.ldo + n + q] = __float2bfloat16_rn(acc[q]);
+  if (Q.lse) {  // warp-uniform
+    float lm = -INFINITY, ls = 0.f;
+    for (int q = 0; q < 4; ++q)
+      if (row_ok && n + q < Q.N) lse_merge2(lm, ls, acc[q], 1.f);
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) {
+      const float m2 = __shfl_xor_sync(0xffffffffu, lm, o), s2 = __shfl_xor_sync(0xffffffffu, ls, o);
+      lse_merge2(lm, ls, m2, s2);
+    }
+    if ((e & 31) == 0 && row_ok) Q.lse[(size_t)m * Q.ld_lse + n / kLseGroup] = make_float2(lm, ls);
   }
 }
 
 }  // namespace
 
 cudaError_t launch_split_reduce(const GemmBatch& batch, cudaStream_t stream) {
-  long long total4 = 0;
-  for (int p = 0; p < batch.num_problems; ++p) {
-    const GemmProblem& Q = batch.prob[p];
-    if (Q.splits > 1) total4 += (long long)Q.M * ((Q.N + 3) / 4);
-  }
-  if (total4 == 0) return cudaSuccess;
-  return launch_kernel(split_reduce_kernel, dim3((unsigned)((total4 + 255) / 256)), dim3(256), 0, stream, 1, batch,
-                       (int)total4);
+  long long total = 0;
+  for (int p = 0; p < batch.num_problems; ++p) total += reduce_items(batch.prob[p]);
+  if (total == 0) return cudaSuccess;
+  return launch_kernel(split_reduce_kernel, dim3((unsigned)((total + 255) / 256)), dim3(256), 0, stream, 1, batch,
+                       total);
 }
 
 size_t fused_gemm_smem_bytes() { return smem_bytes<false>(); }
@@ -756,6 +819,7 @@ cudaError_t launch_fused_gemm(const GemmBatch& batch, bool b_mn_major, bool q4, 
 }
 
 int gemm_tile_m() { return kBM; }
+int gemm_lse_group() { return kLseGroup; }
 int gemm_tile_n() { return kBN; }
 int gemm_tile_k() { return kBK; }
 

@@ -72,6 +72,10 @@ struct GemmProblem {
   int m_pad;           // num_m_tiles * tile rows
   float* part;         // partials [splits * m_pad, ldp]
   int ldp;
+  // fp32 output without splits only: per row and 128-column group g, the
+  // group's (max, sum of exp(z - max)) over columns < N, at lse[row * ld_lse + g]
+  float2* lse;
+  int ld_lse;
 };
 
 // One launch: up to kMaxProblems independent fused contractions.
@@ -106,6 +110,7 @@ size_t fused_gemm_smem_bytes();
 // of the batch with splits > 1 (bf16 or fp32 per out_f32).
 cudaError_t launch_split_reduce(const GemmBatch& batch, cudaStream_t stream);
 int gemm_tile_m();
+int gemm_lse_group();  // columns of one log-sum-exp partial
 int gemm_tile_n();
 int gemm_tile_k();
 
@@ -222,10 +227,13 @@ cudaError_t launch_ce_index(const CeIndex& a, cudaStream_t stream);
 // dst[i, :] = src[idx[i], :] for i < n (rows of d bf16, d a multiple of 8).
 cudaError_t launch_gather_rows(const __nv_bfloat16* src, long long ld, const int32_t* idx, int n, int d,
                                __nv_bfloat16* dst, cudaStream_t stream);
-// Per row i < nT of the fp32 logits Z [nT, ldz]: rowloss[i] = lse - z[ycol[i]] and
-// G[i, :] = bf16(softmax - onehot), zero in columns [nJ, ldg).
-cudaError_t launch_ce_rows(const float* Z, int ldz, int nJ, const int32_t* ycol, int nT, __nv_bfloat16* G, int ldg,
-                           float* rowloss, cudaStream_t stream);
+// Per row i < nT of the fp32 logits Z [nT, ldz] with their log-sum-exp
+// partials lse_part [nT, ld_part] (one per gemm_lse_group() columns):
+// lse[i], rowloss[i] = lse - z[ycol[i]] and G[i, :] = bf16(softmax - onehot),
+// zero in columns [nJ, ldg).
+cudaError_t launch_ce_rows(const float2* lse_part, int ld_part, const float* Z, int ldz, int nJ, const int32_t* ycol,
+                           int nT, float* lse, float* rowloss, __nv_bfloat16* G, int ldg, int num_sms,
+                           cudaStream_t stream);
 // token_loss[t] (optional) and *loss = sum of rowloss in a fixed order.
 cudaError_t launch_ce_finish(const float* rowloss, int nT, const int32_t* tpos, int T, float* token_loss,
                              float* loss, cudaStream_t stream);

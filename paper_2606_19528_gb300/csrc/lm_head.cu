@@ -9,11 +9,15 @@
 //                   then compacted in parallel), each trainable target's
 //                   column in J
 //   gather_rows     rows of h (trainable positions) and of E (J) made dense
-//   ce_rows         per trainable position: log-sum-exp over J, its loss, and
-//                   G = softmax_J - onehot(target) in bf16 for the dh contraction
+//   ce_lse          per trainable position: log-sum-exp over J merged from the
+//                   logits contraction's per-group partials, and its loss
+//   ce_grad         G = softmax_J - onehot(target) in bf16 for the dh
+//                   contraction, one streaming pass over the logits
 //   ce_finish       per-position losses and their sum, in a fixed order
 //   scatter_rows    dh rows of trainable positions, zeros elsewhere
 #include <math.h>
+
+#include <algorithm>
 
 #include "common.cuh"
 #include "kernels.h"
@@ -201,19 +205,23 @@ __device__ __forceinline__ void lse_merge(float& m, float& s, float m2, float s2
   }
 }
 
-// One block per trainable position i: lse over its nJ logits, its loss, and
-// G[i, :] = bf16(exp(z - lse) - [j == ycol]) with zeros in [nJ, ldg).
-__global__ void __launch_bounds__(256) ce_rows_kernel(const float* __restrict__ Z, int ldz, int nJ,
-                                                      const int32_t* __restrict__ ycol, __nv_bfloat16* __restrict__ G,
-                                                      int ldg, float* __restrict__ rowloss) {
+// One block per trainable position i: its log-sum-exp over J from the logits
+// contraction's per-group (max, sum of exp) partials, and its loss
+// lse - z[i, ycol[i]].
+__global__ void __launch_bounds__(256) ce_lse_kernel(const float2* __restrict__ part, int ld_part, int ngroups,
+                                                     const float* __restrict__ Z, int ldz,
+                                                     const int32_t* __restrict__ ycol, float* __restrict__ lse_out,
+                                                     float* __restrict__ rowloss) {
   griddep_wait();
   griddep_launch_dependents();
   __shared__ float sm[8], ss[8];
-  __shared__ float s_lse;
   const int i = blockIdx.x;
-  const float* z = Z + (long long)i * ldz;
+  const float2* pr = part + (long long)i * ld_part;
   float m = -INFINITY, s = 0.f;
-  for (int j = threadIdx.x; j < nJ; j += blockDim.x) lse_merge(m, s, z[j], 1.f);
+  for (int g = threadIdx.x; g < ngroups; g += blockDim.x) {
+    const float2 q = pr[g];
+    lse_merge(m, s, q.x, q.y);
+  }
 #pragma unroll
   for (int o = 16; o > 0; o >>= 1) {
     const float m2 = __shfl_xor_sync(0xffffffffu, m, o), s2 = __shfl_xor_sync(0xffffffffu, s, o);
@@ -229,17 +237,41 @@ __global__ void __launch_bounds__(256) ce_rows_kernel(const float* __restrict__ 
     float M = sm[0], S = ss[0];
     for (int w = 1; w < (int)(blockDim.x >> 5); ++w) lse_merge(M, S, sm[w], ss[w]);
     const float lse = M + logf(S);
-    s_lse = lse;
-    rowloss[i] = lse - z[ycol[i]];
+    lse_out[i] = lse;
+    rowloss[i] = lse - Z[(long long)i * ldz + ycol[i]];
   }
-  __syncthreads();
-  const float lse = s_lse;
-  const int yc = ycol[i];
-  __nv_bfloat16* g = G + (long long)i * ldg;
-  for (int j = threadIdx.x; j < ldg; j += blockDim.x) {
-    float v = 0.f;
-    if (j < nJ) v = expf(z[j] - lse) - (j == yc ? 1.f : 0.f);
-    g[j] = __float2bfloat16_rn(v);
+}
+
+// G[i, :] = bf16(exp(z - lse_i) - [j == ycol_i]) with zeros in [nJ, ldg): one
+// read of the fp32 logits, 16-byte loads and 8-byte stores; work items are
+// (row, 4096-column chunk) pairs over a grid-stride loop.
+constexpr int kGradChunk = 4096;
+
+__global__ void __launch_bounds__(256) ce_grad_kernel(const float* __restrict__ Z, int ldz, int nJ,
+                                                      const int32_t* __restrict__ ycol,
+                                                      const float* __restrict__ lse_in, int nT,
+                                                      __nv_bfloat16* __restrict__ G, int ldg) {
+  griddep_wait();
+  griddep_launch_dependents();
+  const int chunks = (ldg + kGradChunk - 1) / kGradChunk;
+  const long long items = (long long)nT * chunks;
+  for (long long e = blockIdx.x; e < items; e += gridDim.x) {
+    const int i = (int)(e / chunks), c = (int)(e % chunks);
+    const float lse = lse_in[i];
+    const int yc = ycol[i];
+    const float* z = Z + (long long)i * ldz;
+    __nv_bfloat16* g = G + (long long)i * ldg;
+    const int j_end = min(ldg, (c + 1) * kGradChunk);
+#pragma unroll 4
+    for (int j = c * kGradChunk + 4 * (int)threadIdx.x; j < j_end; j += 4 * (int)blockDim.x) {
+      float4 q = make_float4(0.f, 0.f, 0.f, 0.f);
+      if (j < nJ) q = __ldcs(reinterpret_cast<const float4*>(z + j));  // ldz >= j + 4: inside the row
+      const float zv[4] = {q.x, q.y, q.z, q.w};
+      float o[4];
+#pragma unroll
+      for (int u = 0; u < 4; ++u) o[u] = j + u < nJ ? expf(zv[u] - lse) - (j + u == yc ? 1.f : 0.f) : 0.f;
+      *reinterpret_cast<uint2*>(g + j) = make_uint2(pack_bf16x2(o[0], o[1]), pack_bf16x2(o[2], o[3]));
+    }
   }
 }
 
@@ -313,10 +345,16 @@ cudaError_t launch_gather_rows(const __nv_bfloat16* src, long long ld, const int
                        src, ld, idx, n, d, dst);
 }
 
-cudaError_t launch_ce_rows(const float* Z, int ldz, int nJ, const int32_t* ycol, int nT, __nv_bfloat16* G, int ldg,
-                           float* rowloss, cudaStream_t st) {
+cudaError_t launch_ce_rows(const float2* lse_part, int ld_part, const float* Z, int ldz, int nJ, const int32_t* ycol,
+                           int nT, float* lse, float* rowloss, __nv_bfloat16* G, int ldg, int num_sms, cudaStream_t st) {
   if (nT <= 0) return cudaSuccess;
-  return launch_kernel(ce_rows_kernel, dim3(nT), dim3(256), 0, st, 1, Z, ldz, nJ, ycol, G, ldg, rowloss);
+  const int ngroups = (nJ + gemm_lse_group() - 1) / gemm_lse_group();
+  cudaError_t e = launch_kernel(ce_lse_kernel, dim3(nT), dim3(256), 0, st, 1, lse_part, ld_part, ngroups, Z, ldz,
+                                ycol, lse, rowloss);
+  if (e != cudaSuccess) return e;
+  const long long items = (long long)nT * ((ldg + kGradChunk - 1) / kGradChunk);
+  const int grid = (int)std::min<long long>(items, (long long)num_sms * 8);
+  return launch_kernel(ce_grad_kernel, dim3(grid), dim3(256), 0, st, 1, Z, ldz, nJ, ycol, lse, nT, G, ldg);
 }
 
 cudaError_t launch_ce_finish(const float* rowloss, int nT, const int32_t* tpos, int T, float* token_loss,

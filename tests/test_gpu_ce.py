@@ -79,8 +79,13 @@ def check(case, mask=True):
     return nT, nJ
 
 
-@pytest.mark.parametrize("T,d,V,k", [(300, 256, 5000, 37), (128, 512, 3000, 200), (1000, 1024, 20000, 64)],
-                         ids=["T300_d256_V5000_k37", "T128_d512_V3000_k200", "T1000_d1024_V20000_k64"])
+# the last case has few output tiles over a deep contraction (d = 3072): the
+# logits contraction is split and its log-sum-exp partials come from the split
+# reduce instead of the epilogue
+@pytest.mark.parametrize("T,d,V,k", [(300, 256, 5000, 37), (128, 512, 3000, 200), (1000, 1024, 20000, 64),
+                                     (128, 3072, 20000, 64)],
+                         ids=["T300_d256_V5000_k37", "T128_d512_V3000_k200", "T1000_d1024_V20000_k64",
+                              "T128_d3072_V20000_k64_split"])
 def test_ce_topk_parity(T, d, V, k):
     case = CeCase(T, d, V, k=k, table_width=k + 3)
     nT, nJ = check(case)
