@@ -247,11 +247,13 @@ __global__ void __launch_bounds__(kThreads, 1) rank_mma_kernel(const __grid_cons
                                  __uint_as_float(v[e + 3])));
           } else if (g < S::rows(P)) {
 #pragma unroll
-            for (int e = 0; e < 16; ++e) {
-              if constexpr (kCol)
-                col_store(P, g, j0 + e, __uint_as_float(v[e]));
-              else
-                row_store(P, g, j0 + e, __uint_as_float(v[e]));
+            for (int h = 0; h < 16; h += 8) {
+              if (j0 + h < P.rpad) {
+                if constexpr (kCol)
+                  col_store8(P, g, j0 + h, v + h);
+                else
+                  row_store8(P, g, j0 + h, v + h);
+              }
             }
           }
         }
