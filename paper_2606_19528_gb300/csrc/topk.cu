@@ -8,11 +8,16 @@
 //   normalize_rows  E~_i = bf16(E_i / ||E_i||), the sum of squares
 //                   accumulated in fp32 in index order (squares of bf16 are
 //                   exact), correctly rounded sqrt and division
-//   topk_select     radix select on an order-preserving uint32 image of the
-//                   similarities: 11-bit histograms (then 11, then 10 bits)
-//                   until the candidates at or above the chosen prefix fit in
-//                   shared memory, then a bitonic sort of the candidates on
-//                   (similarity descending, index ascending)
+//   topk_select     rows of at least 32768 tokens: a threshold from an
+//                   8192-value sample of the row, one streaming pass that
+//                   keeps every value at or above it, and a bitonic sort of
+//                   those candidates on (similarity descending, index
+//                   ascending); shorter rows, or a sample that leaves fewer
+//                   than k or more than 4096 candidates: radix select on an
+//                   order-preserving uint32 image of the similarities (11-bit
+//                   histograms, then 11, then 10 bits) until the candidates at
+//                   or above the chosen prefix fit in shared memory, then the
+//                   same sort
 #include "common.cuh"
 #include "kernels.h"
 
@@ -124,7 +129,197 @@ __device__ void find_bin(SelShared& sh, int nbins, int k_rem) {
   __syncthreads();
 }
 
-__global__ void __launch_bounds__(kSelThreads) topk_select_kernel(const float* __restrict__ S, long long lds, int V,
+// "a before b": larger key first, the lower index first on equal keys.
+__device__ __forceinline__ bool before(uint32_t ka, int ia, uint32_t kb, int ib) {
+  return ka > kb || (ka == kb && ia < ib);
+}
+
+// Sorts the n candidates in shared memory (n <= kCap) with a bitonic network
+// held in registers: the p2 >= 1024 slots (padded with keys below every real
+// one) sit at positions tid + e * 1024, e < p2 / 1024; strides below 32 are
+// exchanged by warp shuffles, 32 .. 512 through shared memory, 1024 and up
+// within the thread.  Writes the first k indices to out.
+__device__ void sort_and_write(SelShared& sh, int n, int k, int32_t* __restrict__ out) {
+  int p2 = kSelThreads;
+  while (p2 < n) p2 <<= 1;
+  const int E = p2 / kSelThreads;  // 1, 2 or 4
+  const int tid = threadIdx.x;
+  uint32_t key[4];
+  int idx[4];
+#pragma unroll
+  for (int e = 0; e < 4; ++e) {
+    const int p = tid + e * kSelThreads;
+    key[e] = e < E && p < n ? sh.ckey[p] : 0u;
+    idx[e] = e < E && p < n ? sh.cidx[p] : 0x7fffffff;
+  }
+  __syncthreads();  // the candidate arrays now serve as the exchange buffer
+  for (int size = 2; size <= p2; size <<= 1) {
+    for (int stride = size >> 1; stride > 0; stride >>= 1) {
+      if (stride >= kSelThreads) {
+        // partner slot e | (stride / 1024) of the same thread; constant indices keep the slots in registers
+        auto cex = [&](uint32_t& ka, int& ia, uint32_t& kb, int& ib, int e) {
+          const bool up = ((tid + e * kSelThreads) & size) == 0;
+          if (before(kb, ib, ka, ia) == up) {
+            const uint32_t tk = ka;
+            const int ti = ia;
+            ka = kb;
+            ia = ib;
+            kb = tk;
+            ib = ti;
+          }
+        };
+        if (stride == kSelThreads) {
+          cex(key[0], idx[0], key[1], idx[1], 0);
+          if (E == 4) cex(key[2], idx[2], key[3], idx[3], 2);
+        } else {  // stride 2048, E == 4
+          cex(key[0], idx[0], key[2], idx[2], 0);
+          cex(key[1], idx[1], key[3], idx[3], 1);
+        }
+      } else {
+        const bool via_smem = stride >= 32;
+        if (via_smem) {
+#pragma unroll
+          for (int e = 0; e < 4; ++e)
+            if (e < E) {
+              sh.ckey[tid + e * kSelThreads] = key[e];
+              sh.cidx[tid + e * kSelThreads] = idx[e];
+            }
+          __syncthreads();
+        }
+#pragma unroll
+        for (int e = 0; e < 4; ++e) {
+          if (e < E) {
+            const int p = tid + e * kSelThreads;
+            uint32_t kq;
+            int iq;
+            if (via_smem) {
+              kq = sh.ckey[p ^ stride];
+              iq = sh.cidx[p ^ stride];
+            } else {
+              kq = __shfl_xor_sync(0xffffffffu, key[e], stride);
+              iq = __shfl_xor_sync(0xffffffffu, idx[e], stride);
+            }
+            const bool up = (p & size) == 0, lo = (p & stride) == 0;
+            const bool q_first = before(kq, iq, key[e], idx[e]);
+            // an ascending run keeps the first of the pair at the lower position
+            if (lo ? q_first == up : q_first != up) {
+              key[e] = kq;
+              idx[e] = iq;
+            }
+          }
+        }
+        if (via_smem) __syncthreads();
+      }
+    }
+  }
+#pragma unroll
+  for (int e = 0; e < 4; ++e) {
+    const int p = tid + e * kSelThreads;
+    if (e < E && p < k) out[p] = idx[e];
+  }
+}
+
+// Sampled threshold for long rows: the r-th largest of kSample evenly spread
+// row values (r sized so that about kOver * k of the row's values lie at or
+// above it), found to 22 key bits by two histogram levels over the sample
+// alone; then one streaming pass appends every value at or above that
+// threshold, one ballot per 16-byte load and, for a warp with hits, one
+// shared-memory atomic.  A value left out is strictly below every candidate,
+// so when the candidates number between k and kCap they contain the exact
+// top k.  Returns false (and the caller falls back to the full radix select)
+// otherwise.
+constexpr int kSample = 8 * kSelThreads;
+constexpr int kSampleMinV = 4 * kSample;
+constexpr float kOver = 1.6f;
+
+__device__ bool sampled_select(SelShared& sh, const float* __restrict__ s, int V, int k, int32_t* __restrict__ out) {
+  const float4* s4 = reinterpret_cast<const float4*>(s);
+  const int n4 = V / 4;
+  const int lane = threadIdx.x & 31;
+  uint32_t sk[8];  // this thread's sample keys
+#pragma unroll
+  for (int u = 0; u < 2; ++u) {
+    const float4 q = __ldg(s4 + (int)(((long long)(threadIdx.x + u * kSelThreads) * n4) / (2 * kSelThreads)));
+    sk[4 * u + 0] = ord_key(q.x);
+    sk[4 * u + 1] = ord_key(q.y);
+    sk[4 * u + 2] = ord_key(q.z);
+    sk[4 * u + 3] = ord_key(q.w);
+  }
+  const int rs = min(kSample, max(1, (int)ceilf(kOver * (float)k * (float)kSample / (float)V)));
+  uint32_t prefix = 0;
+  int r_rem = rs;
+  for (int lvl = 0; lvl < 2; ++lvl) {
+    for (int b = threadIdx.x; b < 2048; b += kSelThreads) sh.hist[b] = 0;
+    __syncthreads();
+#pragma unroll
+    for (int e = 0; e < 8; ++e) {
+      if (lvl == 0)
+        atomicAdd(&sh.hist[sk[e] >> 21], 1);
+      else if ((sk[e] >> 21) == prefix)
+        atomicAdd(&sh.hist[(sk[e] >> 10) & 2047u], 1);
+    }
+    __syncthreads();
+    find_bin(sh, 2048, r_rem);
+    prefix = (lvl == 0 ? 0u : prefix << 11) | (uint32_t)sh.bin;
+    r_rem -= sh.above;
+    __syncthreads();
+  }
+  // the smallest value whose key has the chosen 22-bit prefix
+  const uint32_t key_lo = prefix << 10;
+  const float tf = __uint_as_float((key_lo & 0x80000000u) ? (key_lo & 0x7fffffffu) : ~key_lo);
+  if (threadIdx.x == 0) sh.ncand = 0;
+  __syncthreads();
+  // appends this lane's hits among its first nv values of q (positions j0 + e); whole warps call it
+  auto append4 = [&](const float4 q, int nv, int j0) {
+    const float f[4] = {q.x, q.y, q.z, q.w};
+    const int c = (nv > 0 && f[0] >= tf) + (nv > 1 && f[1] >= tf) + (nv > 2 && f[2] >= tf) + (nv > 3 && f[3] >= tf);
+    if (__ballot_sync(0xffffffffu, c > 0) == 0u) return;
+    int x = c;  // inclusive scan of the hit counts over the warp
+#pragma unroll
+    for (int o = 1; o < 32; o <<= 1) {
+      const int y = __shfl_up_sync(0xffffffffu, x, o);
+      if (lane >= o) x += y;
+    }
+    int base = 0;
+    if (lane == 31) base = atomicAdd(&sh.ncand, x);
+    int slot = __shfl_sync(0xffffffffu, base, 31) + x - c;
+#pragma unroll
+    for (int e = 0; e < 4; ++e) {
+      if (e < nv && f[e] >= tf) {
+        if (slot < kCap) {
+          sh.ckey[slot] = ord_key(f[e]);
+          sh.cidx[slot] = j0 + e;
+        }
+        ++slot;
+      }
+    }
+  };
+  // every thread runs the same iterations, so the ballots see whole warps
+  for (int base4 = 0; base4 < n4; base4 += 4 * kSelThreads) {
+    float4 q[4];
+#pragma unroll
+    for (int u = 0; u < 4; ++u) {
+      const int j4 = base4 + u * kSelThreads + (int)threadIdx.x;
+      q[u] = j4 < n4 ? __ldcs(s4 + j4) : make_float4(0.f, 0.f, 0.f, 0.f);
+    }
+#pragma unroll
+    for (int u = 0; u < 4; ++u) {
+      const int j4 = base4 + u * kSelThreads + (int)threadIdx.x;
+      append4(q[u], j4 < n4 ? 4 : 0, 4 * j4);
+    }
+  }
+  if (threadIdx.x < 32) {  // the last V mod 4 values, one warp
+    const int j = 4 * n4 + lane;
+    append4(make_float4(j < V ? s[j] : 0.f, 0.f, 0.f, 0.f), j < V ? 1 : 0, j);
+  }
+  __syncthreads();
+  const int n = sh.ncand;
+  if (n < k || n > kCap) return false;  // uniform: read after the barrier
+  sort_and_write(sh, n, k, out);
+  return true;
+}
+
+__global__ void __launch_bounds__(kSelThreads, 2) topk_select_kernel(const float* __restrict__ S, long long lds, int V,
                                                                   int k, int row0, int32_t* __restrict__ table,
                                                                   int* __restrict__ status) {
   griddep_wait();
@@ -133,6 +328,10 @@ __global__ void __launch_bounds__(kSelThreads) topk_select_kernel(const float* _
   SelShared& sh = *reinterpret_cast<SelShared*>(smem_raw);
   const int r = blockIdx.x;
   const float* s = S + (long long)r * lds;  // lds is a multiple of 4: 16-byte aligned rows
+  if (V >= kSampleMinV) {
+    if (sampled_select(sh, s, V, k, table + (long long)(row0 + r) * k)) return;
+    __syncthreads();  // the fallback reuses the shared buffers
+  }
   // levels: (shift of the level's digit, digit bits); the prefix so far selects candidates
   const int shifts[3] = {21, 10, 0}, bits[3] = {11, 11, 10};
   uint32_t prefix = 0;  // chosen digits so far, as key >> shift of the current level
@@ -146,8 +345,23 @@ __global__ void __launch_bounds__(kSelThreads) topk_select_kernel(const float* _
       const uint32_t key = ord_key(f);
       if (lvl == 0 || (key >> hi_shift) == prefix) atomicAdd(&sh.hist[(key >> sh_) & (nb - 1)], 1);
     };
-    for (int j4 = threadIdx.x; j4 < V / 4; j4 += kSelThreads) {
-      const float4 q = __ldg(reinterpret_cast<const float4*>(s) + j4);
+    const float4* s4 = reinterpret_cast<const float4*>(s);
+    const int n4 = V / 4;
+    int j4 = threadIdx.x;
+    for (; j4 + 3 * kSelThreads < n4; j4 += 4 * kSelThreads) {  // four loads in flight per thread
+      float4 q[4];
+#pragma unroll
+      for (int u = 0; u < 4; ++u) q[u] = __ldg(s4 + j4 + u * kSelThreads);
+#pragma unroll
+      for (int u = 0; u < 4; ++u) {
+        count(q[u].x);
+        count(q[u].y);
+        count(q[u].z);
+        count(q[u].w);
+      }
+    }
+    for (; j4 < n4; j4 += kSelThreads) {
+      const float4 q = __ldg(s4 + j4);
       count(q.x);
       count(q.y);
       count(q.z);
@@ -182,44 +396,34 @@ __global__ void __launch_bounds__(kSelThreads) topk_select_kernel(const float* _
       sh.cidx[slot] = j;
     }
   };
-  for (int j4 = threadIdx.x; j4 < V / 4; j4 += kSelThreads) {
-    const float4 q = __ldcs(reinterpret_cast<const float4*>(s) + j4);  // last read of the row
-    take(q.x, 4 * j4);
-    take(q.y, 4 * j4 + 1);
-    take(q.z, 4 * j4 + 2);
-    take(q.w, 4 * j4 + 3);
+  {
+    const float4* s4 = reinterpret_cast<const float4*>(s);
+    const int n4 = V / 4;
+    int j4 = threadIdx.x;
+    for (; j4 + 3 * kSelThreads < n4; j4 += 4 * kSelThreads) {
+      float4 q[4];
+#pragma unroll
+      for (int u = 0; u < 4; ++u) q[u] = __ldcs(s4 + j4 + u * kSelThreads);  // last read of the row
+#pragma unroll
+      for (int u = 0; u < 4; ++u) {
+        const int j = 4 * (j4 + u * kSelThreads);
+        take(q[u].x, j);
+        take(q[u].y, j + 1);
+        take(q[u].z, j + 2);
+        take(q[u].w, j + 3);
+      }
+    }
+    for (; j4 < n4; j4 += kSelThreads) {
+      const float4 q = __ldcs(s4 + j4);
+      take(q.x, 4 * j4);
+      take(q.y, 4 * j4 + 1);
+      take(q.z, 4 * j4 + 2);
+      take(q.w, 4 * j4 + 3);
+    }
   }
   for (int j = (V & ~3) + (int)threadIdx.x; j < V; j += kSelThreads) take(s[j], j);
   __syncthreads();
-  const int n = sh.ncand;
-  int p2 = 1;
-  while (p2 < n) p2 <<= 1;
-  for (int i = n + (int)threadIdx.x; i < p2; i += kSelThreads) {
-    sh.ckey[i] = 0u;  // below every real key
-    sh.cidx[i] = 0x7fffffff;
-  }
-  __syncthreads();
-  // bitonic sort: "a before b" when a.key > b.key, or equal keys and a.idx < b.idx
-  for (int size = 2; size <= p2; size <<= 1) {
-    for (int stride = size >> 1; stride > 0; stride >>= 1) {
-      for (int i = threadIdx.x; i < p2 / 2; i += kSelThreads) {
-        const int lo = 2 * i - (i & (stride - 1)), hi = lo + stride;
-        const bool up = (lo & size) == 0;  // this run sorted "a before b"
-        const uint32_t ka = sh.ckey[lo], kb = sh.ckey[hi];
-        const int ia = sh.cidx[lo], ib = sh.cidx[hi];
-        const bool b_first = kb > ka || (kb == ka && ib < ia);
-        if (b_first == up) {
-          sh.ckey[lo] = kb;
-          sh.ckey[hi] = ka;
-          sh.cidx[lo] = ib;
-          sh.cidx[hi] = ia;
-        }
-      }
-      __syncthreads();
-    }
-  }
-  int32_t* out = table + (long long)(row0 + r) * k;
-  for (int i = threadIdx.x; i < k; i += kSelThreads) out[i] = sh.cidx[i];
+  sort_and_write(sh, sh.ncand, k, table + (long long)(row0 + r) * k);
 }
 
 }  // namespace

@@ -65,8 +65,11 @@ def check_rows(bits, table, k, rows):
         assert np.all(np.isin(must, L)), i
 
 
-@pytest.mark.parametrize("V,d,k", [(5000, 256, 37), (1200, 64, 1024), (20000, 1024, 500)],
-                         ids=["V5000_d256_k37", "V1200_d64_k1024", "V20000_d1024_k500"])
+# V >= 32768 takes the sampled-threshold selection, smaller V the radix path
+@pytest.mark.parametrize("V,d,k", [(5000, 256, 37), (1200, 64, 1024), (20000, 1024, 500), (40000, 64, 300),
+                                   (70000, 128, 1024)],
+                         ids=["V5000_d256_k37", "V1200_d64_k1024", "V20000_d1024_k500", "V40000_d64_k300_sampled",
+                              "V70000_d128_k1024_sampled"])
 def test_topk_table_parity(V, d, k):
     bits = synth.gen_E(0, 50, V, d)
     table = run_table(bits, k)
@@ -85,3 +88,29 @@ def test_topk_argument_errors():
     with pytest.raises(lora.LoraError) as e:
         lora.lora_topk_workspace_size(5000, 16, 1025)  # k beyond the selection's capacity
     assert e.value.code == lora.LORA_EINVAL
+
+
+def test_topk_sampled_ties_and_fallback():
+    """Rows 0..1999 are one vector u, rows 2000..4999 one vector v with
+    cos(u, v) about 0.9, the rest random (V = 40000, k = 1000).  A u row's
+    sampled threshold lands on v's similarity, so 5000 values pass it (more
+    than the 4096 candidate slots) and the row falls back to the radix select;
+    a v row passes 3000 tied values and stays on the sampled path.  Identical
+    inputs give identical tensor-core sums, so the ties are exact and the
+    lower index goes first: u rows list tokens 0..999, v rows 2000..2999."""
+    V, d, k = 40000, 64, 1000
+    bits = synth.gen_E(0, 51, V, d)
+    x = synth.bf16_bits_to_f64(bits)
+    u = x[7] / np.linalg.norm(x[7])
+    w = x[11] - (x[11] @ u) * u
+    v = 0.9 * u + np.sqrt(1 - 0.81) * w / np.linalg.norm(w)
+    ub, vb = synth.to_bf16_bits(u[None, :]), synth.to_bf16_bits(v[None, :])
+    bits = bits.copy()
+    bits[0:2000] = ub
+    bits[2000:5000] = vb
+    table = run_table(bits, k)
+    for i in (0, 1, 1999):
+        assert table[i].tolist() == list(range(1000)), i
+    for i in (2000, 4999):
+        assert table[i].tolist() == list(range(2000, 3000)), i
+    check_rows(bits, table, k, np.array([5000, 12345, V - 1]))
