@@ -236,8 +236,14 @@ int lora_ce_fwd_bwd(const lora_ce_args* args, void* workspace, size_t workspace_
  * row i of `table` [V, k] int32 lists the k tokens with the largest C[i, :],
  * in descending order, the lower index first on equal similarities (row i
  * starts with i unless another token has the same direction).  The V x V
- * matrix is never formed: similarities are computed 512 rows at a time in
- * fp32 on the tensor cores and each row's top k is selected from them.
+ * matrix is never formed.  Below V = 32768 similarities are computed 512 rows
+ * at a time in fp32 on the tensor cores and each row's top k is selected from
+ * them.  From V = 32768 on, each row first gets a threshold from its
+ * similarities to 8192 evenly spread tokens, the similarity contraction keeps
+ * only the values at or above it (at most 4096 per row, in workspace), and
+ * those are sorted; rows left with fewer than k or more than 4096 such values
+ * are redone exactly on the 512-row path, which needs one synchronization of
+ * `stream` (a 4-byte read of their count) before the call returns.
  * E [V, d] bf16 (16-byte aligned), d a multiple of 8, 1 <= k <= min(V, 1024).
  * A row whose k-th similarity is shared by more candidates than the selection
  * holds (thousands of exact ties) is left unwritten and lora_read_status

@@ -261,6 +261,10 @@ void gemm_shape(GemmProblem& g, int64_t M, int64_t N, int64_t Kc, int64_t r) {
   g.ldp = 0;
   g.lse = nullptr;
   g.ld_lse = 0;
+  g.tau = nullptr;
+  g.cnt = nullptr;
+  g.cand = nullptr;
+  g.cap = 0;
 }
 
 // Appends the problem just filled in at b.prob[b.num_problems].
@@ -1164,9 +1168,12 @@ int ce_check(const lora_ce_args* a, CePlan* pl) {
 // its partials in `part` (kCeSplitFloats elements).
 // lse (fp32 output only): per-row log-sum-exp partials [M, ld_lse], written by
 // the epilogue, or by the split reduce when the contraction is split.
+// cand (fp32 output only): append mode instead of storing out (tau, cnt, cand,
+// cap as in GemmProblem); never split.
 int ce_gemm(const DeviceInfo* d, int* counter, const void* A, int64_t lda, const void* B, int64_t ldb, void* out,
             int64_t ldo, int64_t M, int64_t N, int64_t K, bool b_mn, bool f32_out, float* part, cudaStream_t st,
-            float2* lse = nullptr, int ld_lse = 0) {
+            float2* lse = nullptr, int ld_lse = 0, const float* tau = nullptr, int* cnt = nullptr,
+            uint2* cand = nullptr, int cap = 0) {
   GemmBatch b;
   init_batch(b, d);
   b.tile_counter = counter;
@@ -1179,7 +1186,10 @@ int ce_gemm(const DeviceInfo* d, int* counter, const void* A, int64_t lda, const
     return rc;
   }
   b.tmB2[0] = b.tmB[0];
-  if ((rc = make_map(&b.tmOut[0], out, N, M, ldo, f32_out ? 32 : 64, 32, f32_out)) != LORA_OK) return rc;
+  // append mode stores nothing through the output map: a valid 32 x 32 fp32 map inside cand
+  if ((rc = cand ? make_map(&b.tmOut[0], cand, 32, 32, 32, 32, 32, true)
+                 : make_map(&b.tmOut[0], out, N, M, ldo, f32_out ? 32 : 64, 32, f32_out)) != LORA_OK)
+    return rc;
   GemmProblem& g = b.prob[0];
   gemm_shape(g, M, N, K, 0);
   g.out = out;
@@ -1187,9 +1197,14 @@ int ce_gemm(const DeviceInfo* d, int* counter, const void* A, int64_t lda, const
   g.out_f32 = f32_out ? 1 : 0;
   g.lse = lse;
   g.ld_lse = ld_lse;
+  g.tau = tau;
+  g.cnt = cnt;
+  g.cand = cand;
+  g.cap = cap;
   add_problem(b);
   int sp[1];
   choose_splits(b, sp);
+  if (cand) sp[0] = 1;
   float* parts[1] = {part};
   if ((rc = apply_splits(b, sp, parts)) != LORA_OK) return rc;
   if (launch_fused_gemm(b, b_mn, false, d->num_sms, st, f32_out) != cudaSuccess) return LORA_ECUDA;
@@ -1198,11 +1213,15 @@ int ce_gemm(const DeviceInfo* d, int* counter, const void* A, int64_t lda, const
 
 
 // ------------------------------------------------------------------ top-k similarity table
-constexpr int kTopkChunk = 512;  // rows of similarities per contraction
+constexpr int kTopkChunk = 512;         // rows of materialised similarities per contraction
+constexpr int kTopkSampleRows = 8192;   // rows per sample contraction
+constexpr int kTopkAppendRows = 4096;   // rows per appending contraction
 
 struct TopkPlan {
-  size_t counters, status, en, s, part, total;
-  int chunks;
+  size_t counters, status, fail_count, cnt, en, s, part, es, zs, tau, cand, fail_rows, total;
+  int chunks;                 // materialised chunks (short rows)
+  int sblocks, achunks, fmax;  // sampled path: sample blocks, appending chunks, fallback batches at most
+  bool sampled;
   long long lds;
 };
 
@@ -1210,7 +1229,11 @@ int topk_check(const lora_bf16* E, int64_t V, int64_t d, int64_t k, TopkPlan* pl
   if (V < 1 || d < 8 || (d % 8) || k < 1 || k > V || k > topk_max_k() || V > (1ll << 24) || d > (1ll << 20))
     return LORA_EINVAL;
   if (E && !aligned16(E)) return LORA_EALIGN;
+  pl->sampled = V >= topk_sample_min_v();
   pl->chunks = (int)cdiv(V, kTopkChunk);
+  pl->sblocks = pl->sampled ? (int)cdiv(V, kTopkSampleRows) : 0;
+  pl->achunks = pl->sampled ? (int)cdiv(V, kTopkAppendRows) : 0;
+  pl->fmax = pl->sampled ? pl->chunks : 0;
   pl->lds = rup(V, 4);
   size_t off = 0;
   auto take = [&](size_t bytes) {
@@ -1218,11 +1241,23 @@ int topk_check(const lora_bf16* E, int64_t V, int64_t d, int64_t k, TopkPlan* pl
     off += up256(bytes);
     return o;
   };
-  pl->counters = take((size_t)pl->chunks * 4);
+  // zeroed at the start of a call: tile counters, status, fallback count, candidate counts
+  const int nctr = pl->sampled ? pl->sblocks + pl->achunks + pl->fmax : pl->chunks;
+  pl->counters = take((size_t)nctr * 4);
   pl->status = take(4);
+  pl->fail_count = take(4);
+  pl->cnt = take(pl->sampled ? (size_t)std::min<int64_t>(V, kTopkAppendRows) * 4 : 0);
   pl->en = take((size_t)V * d * 2);
   pl->s = take((size_t)std::min<int64_t>(V, kTopkChunk) * pl->lds * 4);
-  pl->part = take(kCeSplitFloats * 4);  // small vocabularies: few tiles per chunk
+  pl->part = take(kCeSplitFloats * 4);  // short rows: few tiles per chunk
+  pl->es = pl->zs = pl->tau = pl->cand = pl->fail_rows = 0;
+  if (pl->sampled) {
+    pl->es = take((size_t)topk_sample() * d * 2);  // later the gathered rows of a fallback batch
+    pl->zs = take((size_t)std::min<int64_t>(V, kTopkSampleRows) * topk_sample() * 4);
+    pl->tau = take((size_t)V * 4);
+    pl->cand = take((size_t)std::min<int64_t>(V, kTopkAppendRows) * topk_cap() * 8);
+    pl->fail_rows = take((size_t)V * 4);
+  }
   pl->total = off;
   return LORA_OK;
 }
@@ -1568,19 +1603,76 @@ int lora_topk_table(const lora_bf16* E, int64_t V, int64_t d, int64_t k, int32_t
   if ((rc = device_info(&dv)) != LORA_OK) return rc;
   cudaStream_t st = static_cast<cudaStream_t>(stream);
   uint8_t* ws = static_cast<uint8_t*>(workspace);
-  if (cudaMemsetAsync(ws, 0, pl.en, st) != cudaSuccess) return LORA_ECUDA;  // tile counters and status
+  if (cudaMemsetAsync(ws, 0, pl.en, st) != cudaSuccess) return LORA_ECUDA;  // counters, status, counts
   bf* en = at<bf>(ws, pl.en);
   float* S = at<float>(ws, pl.s);
-  if (launch_normalize_rows(cb(E), (int)V, (int)d, en, st) != cudaSuccess) return LORA_ECUDA;
-  for (int c = 0; c < pl.chunks; ++c) {
-    const int64_t r0 = (int64_t)c * kTopkChunk, rows = std::min<int64_t>(kTopkChunk, V - r0);
+  int* ctr = at<int>(ws, pl.counters);
+  float* part = at<float>(ws, pl.part);
+  const int D = (int)d;
+  if (launch_normalize_rows(cb(E), (int)V, D, en, st) != cudaSuccess) return LORA_ECUDA;
+  if (!pl.sampled) {
+    for (int c = 0; c < pl.chunks; ++c) {
+      const int64_t r0 = (int64_t)c * kTopkChunk, rows = std::min<int64_t>(kTopkChunk, V - r0);
+      {
+        ProfScope ps(LORA_KERNEL_GEMM_FWD, st);
+        if ((rc = ce_gemm(dv, ctr + c, en + r0 * d, d, en, d, S, pl.lds, rows, V, d, false, true, part, st)) !=
+            LORA_OK)
+          return rc;
+      }
+      if (launch_topk_select(S, pl.lds, (int)V, (int)k, (int)r0, nullptr, (int)rows, table, dv->status, st) !=
+          cudaSuccess)
+        return LORA_ECUDA;
+    }
+    return LORA_OK;
+  }
+  // sampled path: thresholds from the similarities to the sample tokens
+  bf* es = at<bf>(ws, pl.es);
+  float* zs = at<float>(ws, pl.zs);
+  float* tau = at<float>(ws, pl.tau);
+  int* cnt = at<int>(ws, pl.cnt);
+  uint2* cand = at<uint2>(ws, pl.cand);
+  int32_t* fail_rows = at<int32_t>(ws, pl.fail_rows);
+  int* fail_count = at<int>(ws, pl.fail_count);
+  const int ns = topk_sample();
+  int next = 0;
+  if (launch_topk_gather_sample(en, (int)V, D, es, dv->num_sms, st) != cudaSuccess) return LORA_ECUDA;
+  for (int b = 0; b < pl.sblocks; ++b) {
+    const int64_t r0 = (int64_t)b * kTopkSampleRows, rows = std::min<int64_t>(kTopkSampleRows, V - r0);
     {
       ProfScope ps(LORA_KERNEL_GEMM_FWD, st);
-      if ((rc = ce_gemm(dv, at<int>(ws, pl.counters) + c, en + r0 * d, d, en, d, S, pl.lds, rows, V, d, false,
-                        true, at<float>(ws, pl.part), st)) != LORA_OK)
+      if ((rc = ce_gemm(dv, ctr + next++, en + r0 * d, d, es, d, zs, ns, rows, ns, d, false, true, part, st)) !=
+          LORA_OK)
         return rc;
     }
-    if (launch_topk_select(S, pl.lds, (int)V, (int)k, (int)r0, (int)rows, table, dv->status, st) != cudaSuccess)
+    if (launch_topk_tau(zs, (int)V, (int)k, (int)rows, tau + r0, st) != cudaSuccess) return LORA_ECUDA;
+  }
+  // every similarity, keeping the values at or above the row's threshold; then the sort
+  for (int c = 0; c < pl.achunks; ++c) {
+    const int64_t r0 = (int64_t)c * kTopkAppendRows, rows = std::min<int64_t>(kTopkAppendRows, V - r0);
+    {
+      ProfScope ps(LORA_KERNEL_GEMM_FWD, st);
+      if ((rc = ce_gemm(dv, ctr + next++, en + r0 * d, d, en, d, nullptr, 0, rows, V, d, false, true, part, st,
+                        nullptr, 0, tau + r0, cnt, cand, topk_cap())) != LORA_OK)
+        return rc;
+    }
+    if (launch_topk_sort(cand, cnt, topk_cap(), (int)k, (int)r0, (int)rows, table, fail_rows, fail_count, st) !=
+        cudaSuccess)
+      return LORA_ECUDA;
+  }
+  // rows whose threshold left too few or too many candidates: the exact materialised path
+  int nf = 0;
+  if (cudaMemcpyAsync(&nf, fail_count, sizeof(int), cudaMemcpyDeviceToHost, st) != cudaSuccess ||
+      cudaStreamSynchronize(st) != cudaSuccess)
+    return LORA_ECUDA;
+  for (int f0 = 0; f0 < nf; f0 += kTopkChunk) {
+    const int n = std::min(kTopkChunk, nf - f0);
+    if (launch_gather_rows(en, d, fail_rows + f0, n, D, es, st) != cudaSuccess) return LORA_ECUDA;
+    {
+      ProfScope ps(LORA_KERNEL_GEMM_FWD, st);
+      if ((rc = ce_gemm(dv, ctr + next++, es, d, en, d, S, pl.lds, n, V, d, false, true, part, st)) != LORA_OK)
+        return rc;
+    }
+    if (launch_topk_select(S, pl.lds, (int)V, (int)k, 0, fail_rows + f0, n, table, dv->status, st) != cudaSuccess)
       return LORA_ECUDA;
   }
   return LORA_OK;

@@ -449,8 +449,51 @@ __global__ void __launch_bounds__(Cfg<kQ>::kThreads, 1) fused_lora_gemm(const __
         const int row_st = (Q.splits > 1 ? ks * Q.m_pad : 0) + row0;  // stored row of this warp's first row
         // log-sum-exp partial of this thread's row over the warp's column group
         const bool lse_on = kF32 && Q.lse != nullptr && Q.splits == 1;  // split partials: the reduce does it
+        const bool app = kF32 && Q.cand != nullptr;  // append mode (never split)
+        const float tau = app && row0 + lane < Q.M ? Q.tau[row0 + lane] : INFINITY;
         float lm = -INFINITY, ls = 0.f;
-        for (int cc = 0; cc < Cfg<kQ>::kPartCols; cc += block_cols) {
+        if (app && row0 < Q.M && n0 + h * kSeg + part * Cfg<kQ>::kPartCols < Q.N) {  // uniform across the warp
+          // append mode: a first pass over the warp's columns records this row's hits as
+          // bit masks, one atomic reserves the row's slots, a second pass writes the hits
+          constexpr int kBlocks = Cfg<kQ>::kPartCols / 32;
+          uint32_t mask[kBlocks];
+          int total = 0;
+#pragma unroll
+          for (int bk = 0; bk < kBlocks; ++bk) {
+            const int col0 = h * kSeg + part * Cfg<kQ>::kPartCols + bk * 32;
+            mask[bk] = 0u;
+            if (n0 + col0 < Q.N) {  // uniform
+              uint32_t v[32];
+              tmem_ld_32x32b_x32(tmem_base + ((uint32_t)(q * 32) << 16) + (uint32_t)col0, v);
+              tmem_ld_wait();
+              const int nv = min(32, Q.N - (n0 + col0));
+#pragma unroll
+              for (int j = 0; j < 32; ++j)
+                if (j < nv && __uint_as_float(v[j]) >= tau) mask[bk] |= 1u << j;
+              total += __popc(mask[bk]);
+            }
+          }
+          int slot = 0;
+          if (total > 0) slot = atomicAdd(Q.cnt + row0 + lane, total);
+          uint2* dst = Q.cand + (size_t)(row0 + lane) * Q.cap;
+#pragma unroll
+          for (int bk = 0; bk < kBlocks; ++bk) {
+            if (__any_sync(0xffffffffu, mask[bk] != 0u)) {  // the TMEM load is warp-wide
+              const int col0 = h * kSeg + part * Cfg<kQ>::kPartCols + bk * 32;
+              uint32_t v[32];
+              tmem_ld_32x32b_x32(tmem_base + ((uint32_t)(q * 32) << 16) + (uint32_t)col0, v);
+              tmem_ld_wait();
+#pragma unroll
+              for (int j = 0; j < 32; ++j) {
+                if ((mask[bk] >> j) & 1u) {
+                  if (slot < Q.cap) dst[slot] = make_uint2(ord_key(__uint_as_float(v[j])), (uint32_t)(n0 + col0 + j));
+                  ++slot;
+                }
+              }
+            }
+          }
+        }
+        for (int cc = 0; !app && cc < Cfg<kQ>::kPartCols; cc += block_cols) {
           const int col0 = h * kSeg + part * Cfg<kQ>::kPartCols + cc;  // tile column of this block
           if (n0 + col0 >= Q.N || row0 >= Q.M) break;     // uniform across the warp
           const uint32_t taddr = tmem_base + ((uint32_t)(q * 32) << 16) + (uint32_t)col0;

@@ -76,6 +76,13 @@ struct GemmProblem {
   // group's (max, sum of exp(z - max)) over columns < N, at lse[row * ld_lse + g]
   float2* lse;
   int ld_lse;
+  // fp32 output without splits only, instead of storing the output: every
+  // value z[row, n] >= tau[row] is appended as (order key, n) to row's list
+  // cand[row * cap ..], cnt[row] counting every hit (also past cap)
+  const float* tau;
+  int* cnt;
+  uint2* cand;
+  int cap;
 };
 
 // One launch: up to kMaxProblems independent fused contractions.
@@ -247,8 +254,21 @@ cudaError_t launch_normalize_rows(const __nv_bfloat16* E, int V, int d, __nv_bfl
 // Rows row0 .. row0 + nrows - 1 of the table from their similarities S [nrows, lds] fp32:
 // the k largest per row, descending, lower index first on ties; *status =
 // kStatusTopkTies when a row has too many candidates tied at its k-th value.
-cudaError_t launch_topk_select(const float* S, long long lds, int V, int k, int row0, int nrows, int32_t* table,
-                               int* status, cudaStream_t stream);
+// Top-k selection per row of similarities S [nrows, lds] (row r goes to table
+// row rows[r], or row0 + r when rows is null).
+cudaError_t launch_topk_select(const float* S, long long lds, int V, int k, int row0, const int32_t* rows, int nrows,
+                               int32_t* table, int* status, cudaStream_t stream);
+// Thresholds of nrows rows from their sample similarities Z [nrows, topk_sample()].
+cudaError_t launch_topk_tau(const float* Z, int V, int k, int nrows, float* tau, cudaStream_t stream);
+// Sorts each row's appended candidates into the table, or lists the row for the fallback.
+cudaError_t launch_topk_sort(const uint2* cand, int* cnt, int cap, int k, int row0, int nrows, int32_t* table,
+                             int32_t* fail_rows, int* fail_count, cudaStream_t stream);
+// Es [topk_sample(), d] = the evenly spread sample rows of En [V, d].
+cudaError_t launch_topk_gather_sample(const __nv_bfloat16* En, int V, int d, __nv_bfloat16* Es, int num_sms,
+                                      cudaStream_t stream);
+int topk_sample();        // sample tokens per row
+int topk_sample_min_v();  // shortest rows that take the sampled selection
+int topk_cap();           // candidate slots per row
 int topk_max_k();
 
 // One bounded wait on a barrier nothing arrives on (failure-detection self-check).

@@ -63,11 +63,6 @@ __global__ void normalize_rows_kernel(const __nv_bfloat16* __restrict__ E, int V
   }
 }
 
-// Order-preserving image of a float: larger value, larger key.
-__device__ __forceinline__ uint32_t ord_key(float f) {
-  const uint32_t u = __float_as_uint(f);
-  return (u & 0x80000000u) ? ~u : (u | 0x80000000u);
-}
 
 // Exclusive scan of one value per thread over the block; returns the total.
 __device__ __forceinline__ int scan_block(int v, int* excl, int* warp_tot) {
@@ -134,89 +129,106 @@ __device__ __forceinline__ bool before(uint32_t ka, int ia, uint32_t kb, int ib)
   return ka > kb || (ka == kb && ia < ib);
 }
 
-// Sorts the n candidates in shared memory (n <= kCap) with a bitonic network
-// held in registers: the p2 >= 1024 slots (padded with keys below every real
-// one) sit at positions tid + e * 1024, e < p2 / 1024; strides below 32 are
-// exchanged by warp shuffles, 32 .. 512 through shared memory, 1024 and up
-// within the thread.  Writes the first k indices to out.
-__device__ void sort_and_write(SelShared& sh, int n, int k, int32_t* __restrict__ out) {
-  int p2 = kSelThreads;
-  while (p2 < n) p2 <<= 1;
-  const int E = p2 / kSelThreads;  // 1, 2 or 4
+// Bitonic sort on (key descending, index ascending) of p2 = kT * E slots held
+// in registers: slot e of thread t is position t + e * kT.  Strides below 32
+// are exchanged by warp shuffles, 32 .. kT / 2 through the shared buffers xk,
+// xi (p2 entries), kT and up within the thread (fully unrolled, so the slots
+// stay in registers).  Every thread of the block takes part.
+template <int kT, int E>
+__device__ void bitonic_sort(uint32_t (&key)[E], int (&idx)[E], uint32_t* xk, int* xi) {
+  constexpr int p2 = kT * E;
   const int tid = threadIdx.x;
-  uint32_t key[4];
-  int idx[4];
-#pragma unroll
-  for (int e = 0; e < 4; ++e) {
-    const int p = tid + e * kSelThreads;
-    key[e] = e < E && p < n ? sh.ckey[p] : 0u;
-    idx[e] = e < E && p < n ? sh.cidx[p] : 0x7fffffff;
-  }
-  __syncthreads();  // the candidate arrays now serve as the exchange buffer
   for (int size = 2; size <= p2; size <<= 1) {
     for (int stride = size >> 1; stride > 0; stride >>= 1) {
-      if (stride >= kSelThreads) {
-        // partner slot e | (stride / 1024) of the same thread; constant indices keep the slots in registers
-        auto cex = [&](uint32_t& ka, int& ia, uint32_t& kb, int& ib, int e) {
-          const bool up = ((tid + e * kSelThreads) & size) == 0;
-          if (before(kb, ib, ka, ia) == up) {
-            const uint32_t tk = ka;
-            const int ti = ia;
-            ka = kb;
-            ia = ib;
-            kb = tk;
-            ib = ti;
+      if (stride >= kT) {
+#pragma unroll
+        for (int lg = 0; (1 << lg) < E; ++lg) {
+          if (stride == (kT << lg)) {
+#pragma unroll
+            for (int e = 0; e < E; ++e) {
+              const int f = e | (1 << lg);
+              if ((e & (1 << lg)) == 0 && f < E) {
+                const bool up = ((tid + e * kT) & size) == 0;
+                if (before(key[f], idx[f], key[e], idx[e]) == up) {
+                  const uint32_t tk = key[e];
+                  const int ti = idx[e];
+                  key[e] = key[f];
+                  idx[e] = idx[f];
+                  key[f] = tk;
+                  idx[f] = ti;
+                }
+              }
+            }
           }
-        };
-        if (stride == kSelThreads) {
-          cex(key[0], idx[0], key[1], idx[1], 0);
-          if (E == 4) cex(key[2], idx[2], key[3], idx[3], 2);
-        } else {  // stride 2048, E == 4
-          cex(key[0], idx[0], key[2], idx[2], 0);
-          cex(key[1], idx[1], key[3], idx[3], 1);
         }
       } else {
         const bool via_smem = stride >= 32;
         if (via_smem) {
 #pragma unroll
-          for (int e = 0; e < 4; ++e)
-            if (e < E) {
-              sh.ckey[tid + e * kSelThreads] = key[e];
-              sh.cidx[tid + e * kSelThreads] = idx[e];
-            }
+          for (int e = 0; e < E; ++e) {
+            xk[tid + e * kT] = key[e];
+            xi[tid + e * kT] = idx[e];
+          }
           __syncthreads();
         }
 #pragma unroll
-        for (int e = 0; e < 4; ++e) {
-          if (e < E) {
-            const int p = tid + e * kSelThreads;
-            uint32_t kq;
-            int iq;
-            if (via_smem) {
-              kq = sh.ckey[p ^ stride];
-              iq = sh.cidx[p ^ stride];
-            } else {
-              kq = __shfl_xor_sync(0xffffffffu, key[e], stride);
-              iq = __shfl_xor_sync(0xffffffffu, idx[e], stride);
-            }
-            const bool up = (p & size) == 0, lo = (p & stride) == 0;
-            const bool q_first = before(kq, iq, key[e], idx[e]);
-            // an ascending run keeps the first of the pair at the lower position
-            if (lo ? q_first == up : q_first != up) {
-              key[e] = kq;
-              idx[e] = iq;
-            }
+        for (int e = 0; e < E; ++e) {
+          const int p = tid + e * kT;
+          uint32_t kq;
+          int iq;
+          if (via_smem) {
+            kq = xk[p ^ stride];
+            iq = xi[p ^ stride];
+          } else {
+            kq = __shfl_xor_sync(0xffffffffu, key[e], stride);
+            iq = __shfl_xor_sync(0xffffffffu, idx[e], stride);
+          }
+          const bool up = (p & size) == 0, lo = (p & stride) == 0;
+          const bool q_first = before(kq, iq, key[e], idx[e]);
+          // an ascending run keeps the first of the pair at the lower position
+          if (lo ? q_first == up : q_first != up) {
+            key[e] = kq;
+            idx[e] = iq;
           }
         }
         if (via_smem) __syncthreads();
       }
     }
   }
+}
+
+// Loads n <= kT * E candidates (get(p) -> (key, index)), sorts them and writes
+// the first k indices to out; padding sorts below every real key.
+template <int kT, int E, typename Get>
+__device__ void sort_write_e(Get get, int n, int k, uint32_t* xk, int* xi, int32_t* __restrict__ out) {
+  uint32_t key[E];
+  int idx[E];
 #pragma unroll
-  for (int e = 0; e < 4; ++e) {
-    const int p = tid + e * kSelThreads;
-    if (e < E && p < k) out[p] = idx[e];
+  for (int e = 0; e < E; ++e) {
+    const int p = threadIdx.x + e * kT;
+    const uint2 v = p < n ? get(p) : make_uint2(0u, 0x7fffffffu);
+    key[e] = v.x;
+    idx[e] = (int)v.y;
   }
+  __syncthreads();  // the candidates may live in the exchange buffer
+  bitonic_sort<kT, E>(key, idx, xk, xi);
+#pragma unroll
+  for (int e = 0; e < E; ++e) {
+    const int p = threadIdx.x + e * kT;
+    if (p < k) out[p] = idx[e];
+  }
+}
+
+// Sorts the n candidates in shared memory (n <= kCap; the selection kernel's
+// 1024 threads) and writes the first k indices to out.
+__device__ void sort_and_write(SelShared& sh, int n, int k, int32_t* __restrict__ out) {
+  auto get = [&](int p) { return make_uint2(sh.ckey[p], (uint32_t)sh.cidx[p]); };
+  if (n <= kSelThreads)
+    sort_write_e<kSelThreads, 1>(get, n, k, sh.ckey, sh.cidx, out);
+  else if (n <= 2 * kSelThreads)
+    sort_write_e<kSelThreads, 2>(get, n, k, sh.ckey, sh.cidx, out);
+  else
+    sort_write_e<kSelThreads, 4>(get, n, k, sh.ckey, sh.cidx, out);
 }
 
 // Sampled threshold for long rows: the r-th largest of kSample evenly spread
@@ -232,20 +244,16 @@ constexpr int kSample = 8 * kSelThreads;
 constexpr int kSampleMinV = 4 * kSample;
 constexpr float kOver = 1.6f;
 
-__device__ bool sampled_select(SelShared& sh, const float* __restrict__ s, int V, int k, int32_t* __restrict__ out) {
-  const float4* s4 = reinterpret_cast<const float4*>(s);
-  const int n4 = V / 4;
-  const int lane = threadIdx.x & 31;
-  uint32_t sk[8];  // this thread's sample keys
-#pragma unroll
-  for (int u = 0; u < 2; ++u) {
-    const float4 q = __ldg(s4 + (int)(((long long)(threadIdx.x + u * kSelThreads) * n4) / (2 * kSelThreads)));
-    sk[4 * u + 0] = ord_key(q.x);
-    sk[4 * u + 1] = ord_key(q.y);
-    sk[4 * u + 2] = ord_key(q.z);
-    sk[4 * u + 3] = ord_key(q.w);
-  }
-  const int rs = min(kSample, max(1, (int)ceilf(kOver * (float)k * (float)kSample / (float)V)));
+// Rank of the sample value that sets the threshold: about kOver * k of a
+// row's V values are expected at or above the rs-th largest of kSample.
+__device__ __forceinline__ int sample_rank(int V, int k) {
+  return min(kSample, max(1, (int)ceilf(kOver * (float)k * (float)kSample / (float)V)));
+}
+
+// The smallest value whose order key shares the top 22 bits of the rs-th
+// largest of the block's kSample sample keys (8 per thread): two histogram
+// levels of 11 bits over the sample.
+__device__ float sample_threshold(SelShared& sh, const uint32_t* sk, int rs) {
   uint32_t prefix = 0;
   int r_rem = rs;
   for (int lvl = 0; lvl < 2; ++lvl) {
@@ -264,9 +272,24 @@ __device__ bool sampled_select(SelShared& sh, const float* __restrict__ s, int V
     r_rem -= sh.above;
     __syncthreads();
   }
-  // the smallest value whose key has the chosen 22-bit prefix
   const uint32_t key_lo = prefix << 10;
-  const float tf = __uint_as_float((key_lo & 0x80000000u) ? (key_lo & 0x7fffffffu) : ~key_lo);
+  return __uint_as_float((key_lo & 0x80000000u) ? (key_lo & 0x7fffffffu) : ~key_lo);
+}
+
+__device__ bool sampled_select(SelShared& sh, const float* __restrict__ s, int V, int k, int32_t* __restrict__ out) {
+  const float4* s4 = reinterpret_cast<const float4*>(s);
+  const int n4 = V / 4;
+  const int lane = threadIdx.x & 31;
+  uint32_t sk[8];  // this thread's sample keys, evenly spread over the row
+#pragma unroll
+  for (int u = 0; u < 2; ++u) {
+    const float4 q = __ldg(s4 + (int)(((long long)(threadIdx.x + u * kSelThreads) * n4) / (2 * kSelThreads)));
+    sk[4 * u + 0] = ord_key(q.x);
+    sk[4 * u + 1] = ord_key(q.y);
+    sk[4 * u + 2] = ord_key(q.z);
+    sk[4 * u + 3] = ord_key(q.w);
+  }
+  const float tf = sample_threshold(sh, sk, sample_rank(V, k));
   if (threadIdx.x == 0) sh.ncand = 0;
   __syncthreads();
   // appends this lane's hits among its first nv values of q (positions j0 + e); whole warps call it
@@ -320,16 +343,18 @@ __device__ bool sampled_select(SelShared& sh, const float* __restrict__ s, int V
 }
 
 __global__ void __launch_bounds__(kSelThreads, 2) topk_select_kernel(const float* __restrict__ S, long long lds, int V,
-                                                                  int k, int row0, int32_t* __restrict__ table,
+                                                                  int k, int row0, const int32_t* __restrict__ rows,
+                                                                  int32_t* __restrict__ table,
                                                                   int* __restrict__ status) {
   griddep_wait();
   griddep_launch_dependents();
   extern __shared__ uint8_t smem_raw[];
   SelShared& sh = *reinterpret_cast<SelShared*>(smem_raw);
   const int r = blockIdx.x;
+  const long long trow = rows ? rows[r] : row0 + r;  // table row of similarity row r
   const float* s = S + (long long)r * lds;  // lds is a multiple of 4: 16-byte aligned rows
   if (V >= kSampleMinV) {
-    if (sampled_select(sh, s, V, k, table + (long long)(row0 + r) * k)) return;
+    if (sampled_select(sh, s, V, k, table + trow * k)) return;
     __syncthreads();  // the fallback reuses the shared buffers
   }
   // levels: (shift of the level's digit, digit bits); the prefix so far selects candidates
@@ -423,7 +448,164 @@ __global__ void __launch_bounds__(kSelThreads, 2) topk_select_kernel(const float
   }
   for (int j = (V & ~3) + (int)threadIdx.x; j < V; j += kSelThreads) take(s[j], j);
   __syncthreads();
-  sort_and_write(sh, sh.ncand, k, table + (long long)(row0 + r) * k);
+  sort_and_write(sh, sh.ncand, k, table + trow * k);
+}
+
+// Rows of the sample similarities Z [rows, kSample]: each row's threshold,
+// the smallest sample value in the bin of a 2048-bin linear histogram over
+// [min, max] of the row's sample that holds its rs-th largest value, so that
+// between rs and rs + (that bin's count) sample values are at or above it.
+// 256 threads, 32 values each.
+constexpr int kTauThreads = 256;
+constexpr int kTauPer = kSample / kTauThreads;
+
+__global__ void __launch_bounds__(kTauThreads, 4) topk_tau_kernel(const float* __restrict__ Z, int V, int k,
+                                                                float* __restrict__ tau) {
+  griddep_wait();
+  griddep_launch_dependents();
+  __shared__ int hist[2048];
+  __shared__ float red[2][kTauThreads / 32];
+  __shared__ int s_bin, s_above;
+  const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+  const float4* z4 = reinterpret_cast<const float4*>(Z + (long long)blockIdx.x * kSample);
+  float v[kTauPer];
+#pragma unroll
+  for (int u = 0; u < kTauPer / 4; ++u) {
+    const float4 q = __ldcs(z4 + tid + u * kTauThreads);
+    v[4 * u] = q.x;
+    v[4 * u + 1] = q.y;
+    v[4 * u + 2] = q.z;
+    v[4 * u + 3] = q.w;
+  }
+  float lo = v[0], hi = v[0];
+#pragma unroll
+  for (int e = 1; e < kTauPer; ++e) {
+    lo = fminf(lo, v[e]);
+    hi = fmaxf(hi, v[e]);
+  }
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) {
+    lo = fminf(lo, __shfl_xor_sync(0xffffffffu, lo, o));
+    hi = fmaxf(hi, __shfl_xor_sync(0xffffffffu, hi, o));
+  }
+  for (int b = tid; b < 2048; b += kTauThreads) hist[b] = 0;
+  if (lane == 0) {
+    red[0][warp] = lo;
+    red[1][warp] = hi;
+  }
+  __syncthreads();
+  lo = red[0][0];
+  hi = red[1][0];
+#pragma unroll
+  for (int w = 1; w < kTauThreads / 32; ++w) {
+    lo = fminf(lo, red[0][w]);
+    hi = fmaxf(hi, red[1][w]);
+  }
+  const float scale = hi > lo ? 2048.f / (hi - lo) : 0.f;
+  auto bin_of = [&](float x) { return min(2047, max(0, (int)((x - lo) * scale))); };
+#pragma unroll
+  for (int e = 0; e < kTauPer; ++e) atomicAdd(&hist[bin_of(v[e])], 1);
+  __syncthreads();
+  // bins by descending index: thread t holds bins 2047 - 8t .. 2040 - 8t
+  const int rs = sample_rank(V, k);
+  int local = 0;
+#pragma unroll
+  for (int q = 0; q < 8; ++q) local += hist[2047 - 8 * tid - q];
+  int x = local;  // inclusive scan over the block
+#pragma unroll
+  for (int o = 1; o < 32; o <<= 1) {
+    const int y = __shfl_up_sync(0xffffffffu, x, o);
+    if (lane >= o) x += y;
+  }
+  __shared__ int wsum[kTauThreads / 32];
+  if (lane == 31) wsum[warp] = x;
+  __syncthreads();
+  int excl = x - local;
+  for (int w = 0; w < warp; ++w) excl += wsum[w];
+  if (excl < rs && rs <= excl + local) {
+    int acc = excl;
+#pragma unroll
+    for (int q = 0; q < 8; ++q) {
+      const int h = hist[2047 - 8 * tid - q];
+      if (rs <= acc + h) {
+        s_bin = 2047 - 8 * tid - q;
+        s_above = acc;
+        break;
+      }
+      acc += h;
+    }
+  }
+  __syncthreads();
+  // the smallest sample value in the chosen bin
+  const int bstar = s_bin;
+  float m = INFINITY;
+#pragma unroll
+  for (int e = 0; e < kTauPer; ++e)
+    if (bin_of(v[e]) == bstar) m = fminf(m, v[e]);
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) m = fminf(m, __shfl_xor_sync(0xffffffffu, m, o));
+  __syncthreads();
+  if (lane == 0) red[0][warp] = m;
+  __syncthreads();
+  if (tid == 0) {
+    float t = red[0][0];
+    for (int w = 1; w < kTauThreads / 32; ++w) t = fminf(t, red[0][w]);
+    tau[blockIdx.x] = t;
+  }
+}
+
+// One row of a chunk: its cnt[r] candidates (order key, token) appended by the
+// similarity contraction; with k <= n <= cap they hold the exact top k and
+// are sorted into the table (256 threads, 1 to 16 register slots each),
+// otherwise the row joins the fallback list.  The row's count is reset for the
+// next chunk.
+constexpr int kSortThreads = 256;
+
+__global__ void __launch_bounds__(kSortThreads, 4) topk_sort_kernel(const uint2* __restrict__ cand,
+                                                                   int* __restrict__ cnt, int cap, int k, int row0,
+                                                                   int32_t* __restrict__ table,
+                                                                   int32_t* __restrict__ fail_rows,
+                                                                   int* __restrict__ fail_count) {
+  griddep_wait();
+  griddep_launch_dependents();
+  __shared__ uint32_t xk[kCap];
+  __shared__ int xi[kCap];
+  const int r = blockIdx.x, tid = threadIdx.x;
+  const int n = cnt[r];
+  __syncthreads();  // every thread has read the count before it is reset
+  if (tid == 0) cnt[r] = 0;
+  if (n < k || n > cap || n > kCap) {
+    if (tid == 0) fail_rows[atomicAdd(fail_count, 1)] = row0 + r;
+    return;
+  }
+  const uint2* c = cand + (long long)r * cap;
+  auto get = [&](int p) { return c[p]; };
+  int32_t* out = table + (long long)(row0 + r) * k;
+  if (n <= kSortThreads)
+    sort_write_e<kSortThreads, 1>(get, n, k, xk, xi, out);
+  else if (n <= 2 * kSortThreads)
+    sort_write_e<kSortThreads, 2>(get, n, k, xk, xi, out);
+  else if (n <= 4 * kSortThreads)
+    sort_write_e<kSortThreads, 4>(get, n, k, xk, xi, out);
+  else if (n <= 8 * kSortThreads)
+    sort_write_e<kSortThreads, 8>(get, n, k, xk, xi, out);
+  else
+    sort_write_e<kSortThreads, 16>(get, n, k, xk, xi, out);
+}
+
+// Es[i, :] = En[floor(i * V / kSample), :]: the sample tokens, evenly spread.
+__global__ void topk_gather_sample_kernel(const __nv_bfloat16* __restrict__ En, int V, int d,
+                                          __nv_bfloat16* __restrict__ Es) {
+  griddep_wait();
+  griddep_launch_dependents();
+  const int vpr = d / 8;
+  const long long total = (long long)kSample * vpr;
+  for (long long e = blockIdx.x * (long long)blockDim.x + threadIdx.x; e < total;
+       e += (long long)gridDim.x * blockDim.x) {
+    const int i = (int)(e / vpr), v = (int)(e % vpr);
+    const long long src = (long long)i * V / kSample;
+    reinterpret_cast<uint4*>(Es + (long long)i * d)[v] = reinterpret_cast<const uint4*>(En + src * d)[v];
+  }
 }
 
 }  // namespace
@@ -432,18 +614,42 @@ cudaError_t launch_normalize_rows(const __nv_bfloat16* E, int V, int d, __nv_bfl
   return launch_kernel(normalize_rows_kernel, dim3((V + 127) / 128), dim3(128), 0, st, 1, E, V, d, En);
 }
 
-cudaError_t launch_topk_select(const float* S, long long lds, int V, int k, int row0, int nrows, int32_t* table,
-                               int* status, cudaStream_t st) {
-  static bool attr_done = false;
-  const int smem = (int)sizeof(SelShared);
-  if (!attr_done) {
-    cudaError_t e = cudaFuncSetAttribute(topk_select_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
-    if (e != cudaSuccess) return e;
-    attr_done = true;
-  }
-  return launch_kernel(topk_select_kernel, dim3(nrows), dim3(kSelThreads), smem, st, 1, S, lds, V, k, row0, table,
-                       status);
+// Sets the dynamic shared-memory size of the selection kernels once.
+cudaError_t sel_attrs() {
+  static const cudaError_t e = [] {
+    const int smem = (int)sizeof(SelShared);
+    cudaError_t r = cudaFuncSetAttribute(topk_select_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
+    return r;
+  }();
+  return e;
 }
+
+cudaError_t launch_topk_select(const float* S, long long lds, int V, int k, int row0, const int32_t* rows, int nrows,
+                               int32_t* table, int* status, cudaStream_t st) {
+  cudaError_t e = sel_attrs();
+  if (e != cudaSuccess) return e;
+  return launch_kernel(topk_select_kernel, dim3(nrows), dim3(kSelThreads), (int)sizeof(SelShared), st, 1, S, lds, V,
+                       k, row0, rows, table, status);
+}
+
+cudaError_t launch_topk_tau(const float* Z, int V, int k, int nrows, float* tau, cudaStream_t st) {
+  return launch_kernel(topk_tau_kernel, dim3(nrows), dim3(kTauThreads), 0, st, 1, Z, V, k, tau);
+}
+
+cudaError_t launch_topk_sort(const uint2* cand, int* cnt, int cap, int k, int row0, int nrows, int32_t* table,
+                             int32_t* fail_rows, int* fail_count, cudaStream_t st) {
+  return launch_kernel(topk_sort_kernel, dim3(nrows), dim3(kSortThreads), 0, st, 1, cand, cnt, cap, k, row0, table,
+                       fail_rows, fail_count);
+}
+
+cudaError_t launch_topk_gather_sample(const __nv_bfloat16* En, int V, int d, __nv_bfloat16* Es, int num_sms,
+                                      cudaStream_t st) {
+  return launch_kernel(topk_gather_sample_kernel, dim3(num_sms * 4), dim3(256), 0, st, 1, En, V, d, Es);
+}
+
+int topk_sample() { return kSample; }
+int topk_sample_min_v() { return kSampleMinV; }
+int topk_cap() { return kCap; }
 
 int topk_max_k() { return kSelThreads; }
 
