@@ -807,12 +807,27 @@ def run_gpu(args, wl):
         e1.record(stream)
         torch.cuda.synchronize()
         e2e_ms = max_over_ranks(dist, e0.elapsed_time(e1) / Ke, device)
+        # the same host-to-device copies alone: the link rate the pipelined steps are bounded by
+        c0, c1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        torch.cuda.synchronize()
+        c0.record(copy)
+        for _ in range(10):
+            with torch.cuda.stream(copy):
+                for g, t in h_x.items():
+                    xs2[g].view(torch.int16).copy_(t, non_blocking=True)
+                for d_, t in zip(dys2, h_dy):
+                    d_.view(torch.int16).copy_(t, non_blocking=True)
+        c1.record(copy)
+        torch.cuda.synchronize()
+        copy_ms = c0.elapsed_time(c1) / 10
         e2e = {"value": world * wl.T / (e2e_ms / 1e3), "unit": UNIT, "h2d_bytes_per_step": h2d_bytes,
                "d2h_bytes_per_step": d2h_bytes, "ms_per_step": e2e_ms, "steps": Ke,
-               "serial_ms_per_step": serial_ms,
+               "serial_ms_per_step": serial_ms, "h2d_only_ms_per_step": copy_ms,
+               "h2d_gbs": h2d_bytes / (copy_ms / 1e3) / 1e9,
                "note": "every step copies its x and dy from pinned host memory and its dA, dB back to pinned "
                        "host memory; the copy of step i+1's inputs (copy stream, second input buffer) "
-                       "overlaps step i; serial_ms_per_step: copies and step on one stream"}
+                       "overlaps step i; serial_ms_per_step: copies and step on one stream; h2d_only: the "
+                       "input copies alone, the host link rate that bounds the pipelined steps"}
 
     if rank != 0:
         if dist is not None:
@@ -877,7 +892,17 @@ def main(argv=None):
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--cpu-budget", type=float, default=15.0)
+    ap.add_argument("--sweep", action="store_true",
+                    help="the Llama layer over T in {256, 1024, 4096, 16384} x r in {4 .. 128} (one JSON line per "
+                         "point; device-timed steps only)")
     args = ap.parse_args(argv)
+    if args.sweep:
+        args.no_e2e = args.no_cpu_baseline = True
+        rc = 0
+        for T in workloads.SWEEP_TOKENS:
+            for r in workloads.SWEEP_RANKS:
+                rc |= run_gpu(args, workloads.llama_sweep(T, r))
+        return rc
     wl = workloads.BY_NAME[args.workload]()
     if wl.kind == "topk":
         if args.impl == "reference":

@@ -27,7 +27,7 @@ __device__ int g_status;  // first device-side error (kStatusTimeout), 0 if none
 
 constexpr int kMaxDevices = 64;
 constexpr size_t kWsHeader = 256;  // 64 tile counters, one per fused-GEMM launch of a call
-constexpr int kSideSms = 12;        // SMs the backward's rank-r work gets beside the contractions
+constexpr int kSideSms = 12;        // SMs the backward's rank-r work gets beside the contractions (r <= 32)
 constexpr long long kDefaultWaitNs = 4000000000ll;
 
 struct DeviceInfo {
@@ -757,12 +757,22 @@ bool overlap_enabled() {
   return on;
 }
 
-int side_sms_setting(int num_sms) {
+// The rank-r work grows with the rank while the contractions do not: 12 SMs up
+// to r = 32, 24 up to 64, 28 beyond (measured on the Llama layer at T = 256 ..
+// 4096); LORA_SIDE_SMS overrides.
+int side_sms_setting(int num_sms, int max_rank) {
   static const int v = [] {
     const char* e = getenv("LORA_SIDE_SMS");
-    return e ? atoi(e) : kSideSms;
+    return e ? atoi(e) : 0;
   }();
-  return std::max(2, std::min(num_sms / 4, v));
+  const int w = v > 0 ? v : (max_rank <= 32 ? kSideSms : max_rank <= 64 ? 24 : 28);
+  return std::max(2, std::min(num_sms / 4, w));
+}
+
+int max_rank_of(const lora_proj* projs, int n) {
+  int r = 0;
+  for (int i = 0; i < n; ++i) r = std::max(r, (int)projs[i].shape.rank);
+  return r;
 }
 
 struct SideCtx {
@@ -788,7 +798,7 @@ struct Overlap {
   int side_ctas = 0;
   cudaStream_t main = nullptr, side = nullptr;
   cudaEvent_t ev_fork = nullptr, ev_sv = nullptr, ev_done = nullptr;
-  int init(const DeviceInfo* d, cudaStream_t st) {
+  int init(const DeviceInfo* d, cudaStream_t st, int max_rank) {
     if (!overlap_enabled()) return LORA_OK;
     SideCtx& c = t_side.dev[d - g_dev];
     if (!c.side && cudaStreamCreateWithFlags(&c.side, cudaStreamNonBlocking) != cudaSuccess) return LORA_ECUDA;
@@ -799,7 +809,7 @@ struct Overlap {
     ev_fork = c.ev[0];
     ev_sv = c.ev[1];
     ev_done = c.ev[2];
-    side_ctas = side_sms_setting(d->num_sms);
+    side_ctas = side_sms_setting(d->num_sms, max_rank);
     on = true;
     return LORA_OK;
   }
@@ -834,7 +844,7 @@ int run_step(const lora_proj* projs, int n, int mode, void* ws, const Plan& pl, 
   // forward and backward in one call: the backward's rank-r work runs on a side
   // stream with a few SMs while the contractions use the rest
   Overlap ov;
-  if (mode == LORA_FWD_BWD && (rc = ov.init(d, st)) != LORA_OK) return rc;
+  if (mode == LORA_FWD_BWD && (rc = ov.init(d, st, max_rank_of(projs, n))) != LORA_OK) return rc;
   const int gemm_sms = ov.on ? d->num_sms - ov.side_ctas : d->num_sms;
   // backward rank-r work: B^T, su^T, sv (and sv^T), then dB and dA; on `rs`
   // with `ctas` persistent CTAs; the operands of the dx contraction go to bops
@@ -1018,7 +1028,9 @@ int plan_all(const lora_proj* projs, int n, int mode, Plan* pl, bool allow_split
   pl->split_f.assign(n, 1);
   pl->split_b.assign(n, 1);
   // a forward-and-backward call leaves the side stream's SMs out of the contractions
-  const int pairs = mode == LORA_FWD_BWD && overlap_enabled() ? (kPlanSms - side_sms_setting(kPlanSms)) / 2 : kPlanPairs;
+  const int pairs = mode == LORA_FWD_BWD && overlap_enabled()
+                        ? (kPlanSms - side_sms_setting(kPlanSms, max_rank_of(projs, n))) / 2
+                        : kPlanPairs;
   std::vector<size_t> split_need(n, 0);
   for (int dir = 0; dir < 2; ++dir) {
     if (!(mode & (dir == 0 ? LORA_FWD : LORA_BWD))) continue;
