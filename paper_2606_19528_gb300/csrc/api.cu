@@ -265,6 +265,7 @@ void gemm_shape(GemmProblem& g, int64_t M, int64_t N, int64_t Kc, int64_t r) {
   g.cnt = nullptr;
   g.cand = nullptr;
   g.cap = 0;
+  g.row_off = g.col_off = g.sym = 0;
 }
 
 // Appends the problem just filled in at b.prob[b.num_problems].
@@ -1224,6 +1225,40 @@ int ce_gemm(const DeviceInfo* d, int* counter, const void* A, int64_t lda, const
 }
 
 
+// Upper triangle of the similarities of rows [r0, r0 + rows) (a whole number of
+// 512-row blocks, at most 8, but for the last rows of V) in append mode: block
+// I contracts against tokens from 512 I on, so its first 512-column tile is
+// the diagonal block (row side only) and the others also append to the
+// columns' lists.
+int topk_sym_gemm(const DeviceInfo* d, int* counter, const bf* en, int64_t dd, int64_t V, int64_t r0, int64_t rows,
+                  const float* tau, int* cnt, uint2* cand, int cap, cudaStream_t st) {
+  GemmBatch b;
+  init_batch(b, d);
+  b.tile_counter = counter;
+  int rc;
+  for (int64_t a0 = r0; a0 < r0 + rows; a0 += 512) {
+    const int p = b.num_problems;
+    const int64_t m = std::min<int64_t>(512, r0 + rows - a0), N = V - a0;
+    if ((rc = make_map(&b.tmA[p], en + a0 * dd, dd, m, dd, 64, 128)) != LORA_OK) return rc;
+    if ((rc = make_map(&b.tmB[p], en + a0 * dd, dd, N, dd, 64, 64)) != LORA_OK) return rc;
+    b.tmA2[p] = b.tmA[p];
+    b.tmB2[p] = b.tmB[p];
+    if ((rc = make_map(&b.tmOut[p], cand, 32, 32, 32, 32, 32, true)) != LORA_OK) return rc;  // never stored through
+    GemmProblem& g = b.prob[p];
+    gemm_shape(g, m, N, dd, 0);
+    g.out_f32 = 1;
+    g.tau = tau;
+    g.cnt = cnt;
+    g.cand = cand;
+    g.cap = cap;
+    g.row_off = (int)a0;
+    g.col_off = (int)a0;
+    g.sym = 1;
+    add_problem(b);
+  }
+  return launch_fused_gemm(b, false, false, d->num_sms, st, true) == cudaSuccess ? LORA_OK : LORA_ECUDA;
+}
+
 // ------------------------------------------------------------------ top-k similarity table
 constexpr int kTopkChunk = 512;         // rows of materialised similarities per contraction
 constexpr int kTopkSampleRows = 8192;   // rows per sample contraction
@@ -1258,7 +1293,7 @@ int topk_check(const lora_bf16* E, int64_t V, int64_t d, int64_t k, TopkPlan* pl
   pl->counters = take((size_t)nctr * 4);
   pl->status = take(4);
   pl->fail_count = take(4);
-  pl->cnt = take(pl->sampled ? (size_t)std::min<int64_t>(V, kTopkAppendRows) * 4 : 0);
+  pl->cnt = take(pl->sampled ? (size_t)V * 4 : 0);
   pl->en = take((size_t)V * d * 2);
   pl->s = take((size_t)std::min<int64_t>(V, kTopkChunk) * pl->lds * 4);
   pl->part = take(kCeSplitFloats * 4);  // short rows: few tiles per chunk
@@ -1267,7 +1302,7 @@ int topk_check(const lora_bf16* E, int64_t V, int64_t d, int64_t k, TopkPlan* pl
     pl->es = take((size_t)topk_sample() * d * 2);  // later the gathered rows of a fallback batch
     pl->zs = take((size_t)std::min<int64_t>(V, kTopkSampleRows) * topk_sample() * 4);
     pl->tau = take((size_t)V * 4);
-    pl->cand = take((size_t)std::min<int64_t>(V, kTopkAppendRows) * topk_cap() * 8);
+    pl->cand = take((size_t)V * topk_cap() * 8);  // every row's list: the transposed side fills later rows
     pl->fail_rows = take((size_t)V * 4);
   }
   pl->total = off;
@@ -1658,19 +1693,16 @@ int lora_topk_table(const lora_bf16* E, int64_t V, int64_t d, int64_t k, int32_t
     }
     if (launch_topk_tau(zs, (int)V, (int)k, (int)rows, tau + r0, st) != cudaSuccess) return LORA_ECUDA;
   }
-  // every similarity, keeping the values at or above the row's threshold; then the sort
+  // the upper triangle of the similarities (C is symmetric), every value offered to both of
+  // its rows' lists against their thresholds; then each row's list is sorted
   for (int c = 0; c < pl.achunks; ++c) {
     const int64_t r0 = (int64_t)c * kTopkAppendRows, rows = std::min<int64_t>(kTopkAppendRows, V - r0);
-    {
-      ProfScope ps(LORA_KERNEL_GEMM_FWD, st);
-      if ((rc = ce_gemm(dv, ctr + next++, en + r0 * d, d, en, d, nullptr, 0, rows, V, d, false, true, part, st,
-                        nullptr, 0, tau + r0, cnt, cand, topk_cap())) != LORA_OK)
-        return rc;
-    }
-    if (launch_topk_sort(cand, cnt, topk_cap(), (int)k, (int)r0, (int)rows, table, fail_rows, fail_count, st) !=
-        cudaSuccess)
-      return LORA_ECUDA;
+    ProfScope ps(LORA_KERNEL_GEMM_FWD, st);
+    if ((rc = topk_sym_gemm(dv, ctr + next++, en, d, V, r0, rows, tau, cnt, cand, topk_cap(), st)) != LORA_OK)
+      return rc;
   }
+  if (launch_topk_sort(cand, cnt, topk_cap(), (int)k, 0, (int)V, table, fail_rows, fail_count, st) != cudaSuccess)
+    return LORA_ECUDA;
   // rows whose threshold left too few or too many candidates: the exact materialised path
   int nf = 0;
   if (cudaMemcpyAsync(&nf, fail_count, sizeof(int), cudaMemcpyDeviceToHost, st) != cudaSuccess ||

@@ -450,18 +450,23 @@ __global__ void __launch_bounds__(Cfg<kQ>::kThreads, 1) fused_lora_gemm(const __
         // log-sum-exp partial of this thread's row over the warp's column group
         const bool lse_on = kF32 && Q.lse != nullptr && Q.splits == 1;  // split partials: the reduce does it
         const bool app = kF32 && Q.cand != nullptr;  // append mode (never split)
-        const float tau = app && row0 + lane < Q.M ? Q.tau[row0 + lane] : INFINITY;
+        const float tau = app && row0 + lane < Q.M ? Q.tau[Q.row_off + row0 + lane] : INFINITY;
         float lm = -INFINITY, ls = 0.f;
         if (app && row0 < Q.M && n0 + h * kSeg + part * Cfg<kQ>::kPartCols < Q.N) {  // uniform across the warp
-          // append mode: a first pass over the warp's columns records this row's hits as
-          // bit masks, one atomic reserves the row's slots, a second pass writes the hits
+          // append mode: a first pass over the warp's columns records hits as bit masks (this
+          // thread's row; with the transposed side also lane l's column of each 32-column
+          // block, over the warp's 32 rows), one atomic per list reserves the slots, a second
+          // pass writes the hits
           constexpr int kBlocks = Cfg<kQ>::kPartCols / 32;
-          uint32_t mask[kBlocks];
+          const bool tr = Q.sym && n0 > 0;  // off the diagonal block
+          const int i_abs = Q.row_off + row0 + lane;
+          uint32_t mask[kBlocks], cmask[kBlocks];
           int total = 0;
 #pragma unroll
           for (int bk = 0; bk < kBlocks; ++bk) {
             const int col0 = h * kSeg + part * Cfg<kQ>::kPartCols + bk * 32;
             mask[bk] = 0u;
+            cmask[bk] = 0u;
             if (n0 + col0 < Q.N) {  // uniform
               uint32_t v[32];
               tmem_ld_32x32b_x32(tmem_base + ((uint32_t)(q * 32) << 16) + (uint32_t)col0, v);
@@ -471,23 +476,54 @@ __global__ void __launch_bounds__(Cfg<kQ>::kThreads, 1) fused_lora_gemm(const __
               for (int j = 0; j < 32; ++j)
                 if (j < nv && __uint_as_float(v[j]) >= tau) mask[bk] |= 1u << j;
               total += __popc(mask[bk]);
+              if (tr) {
+                const float tau_c = lane < nv ? Q.tau[Q.col_off + n0 + col0 + lane] : INFINITY;
+                const bool row_ok = row0 + lane < Q.M;
+#pragma unroll
+                for (int j = 0; j < 32; ++j) {
+                  const float t = __shfl_sync(0xffffffffu, tau_c, j);
+                  const unsigned m = __ballot_sync(0xffffffffu, row_ok && __uint_as_float(v[j]) >= t);
+                  if (lane == j) cmask[bk] = m;
+                }
+              }
             }
           }
           int slot = 0;
-          if (total > 0) slot = atomicAdd(Q.cnt + row0 + lane, total);
-          uint2* dst = Q.cand + (size_t)(row0 + lane) * Q.cap;
+          if (total > 0) slot = atomicAdd(Q.cnt + i_abs, total);
+          int cbase[kBlocks];
 #pragma unroll
           for (int bk = 0; bk < kBlocks; ++bk) {
-            if (__any_sync(0xffffffffu, mask[bk] != 0u)) {  // the TMEM load is warp-wide
+            cbase[bk] = 0;
+            if (cmask[bk] != 0u)
+              cbase[bk] = atomicAdd(Q.cnt + Q.col_off + n0 + h * kSeg + part * Cfg<kQ>::kPartCols + bk * 32 + lane,
+                                    __popc(cmask[bk]));
+          }
+          uint2* dst = Q.cand + (size_t)i_abs * Q.cap;
+#pragma unroll
+          for (int bk = 0; bk < kBlocks; ++bk) {
+            if (__any_sync(0xffffffffu, (mask[bk] | cmask[bk]) != 0u)) {  // the TMEM load is warp-wide
               const int col0 = h * kSeg + part * Cfg<kQ>::kPartCols + bk * 32;
+              const int j_abs0 = Q.col_off + n0 + col0;
               uint32_t v[32];
               tmem_ld_32x32b_x32(tmem_base + ((uint32_t)(q * 32) << 16) + (uint32_t)col0, v);
               tmem_ld_wait();
 #pragma unroll
               for (int j = 0; j < 32; ++j) {
                 if ((mask[bk] >> j) & 1u) {
-                  if (slot < Q.cap) dst[slot] = make_uint2(ord_key(__uint_as_float(v[j])), (uint32_t)(n0 + col0 + j));
+                  if (slot < Q.cap) dst[slot] = make_uint2(ord_key(__uint_as_float(v[j])), (uint32_t)(j_abs0 + j));
                   ++slot;
+                }
+              }
+              if (tr) {
+#pragma unroll
+                for (int j = 0; j < 32; ++j) {
+                  const unsigned m = __shfl_sync(0xffffffffu, cmask[bk], j);
+                  const int b0 = __shfl_sync(0xffffffffu, cbase[bk], j);
+                  if ((m >> lane) & 1u) {
+                    const int sl = b0 + __popc(m & ((1u << lane) - 1u));
+                    if (sl < Q.cap)
+                      Q.cand[(size_t)(j_abs0 + j) * Q.cap + sl] = make_uint2(ord_key(__uint_as_float(v[j])), (uint32_t)i_abs);
+                  }
                 }
               }
             }

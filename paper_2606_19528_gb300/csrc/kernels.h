@@ -76,13 +76,17 @@ struct GemmProblem {
   // group's (max, sum of exp(z - max)) over columns < N, at lse[row * ld_lse + g]
   float2* lse;
   int ld_lse;
-  // fp32 output without splits only, instead of storing the output: every
-  // value z[row, n] >= tau[row] is appended as (order key, n) to row's list
-  // cand[row * cap ..], cnt[row] counting every hit (also past cap)
+  // fp32 output without splits only, instead of storing the output: with
+  // i = row_off + m and j = col_off + n the absolute indices of z[m, n],
+  // z >= tau[i] is appended as (order key, j) to i's list cand[i * cap ..],
+  // cnt[i] counting every hit (also past cap); with sym set, tiles with
+  // n0 > 0 (off the diagonal block) also append (order key, i) to j's list
+  // when z >= tau[j]
   const float* tau;
   int* cnt;
   uint2* cand;
   int cap;
+  int row_off, col_off, sym;
 };
 
 // One launch: up to kMaxProblems independent fused contractions.
