@@ -460,6 +460,25 @@ __global__ void __launch_bounds__(Cfg<kQ>::kThreads, 1) fused_lora_gemm(const __
           constexpr int kBlocks = Cfg<kQ>::kPartCols / 32;
           const bool tr = Q.sym && n0 > 0;  // off the diagonal block
           const int i_abs = Q.row_off + row0 + lane;
+          // the transposed side reads the block column-wise from the warp's staging buffer
+          // (free in append mode): row `lane` stored as 8 16-byte chunks, chunk u at u ^ (lane mod 8)
+          auto stage_block = [&](const uint32_t(&v)[32]) {
+#pragma unroll
+            for (int u = 0; u < 8; ++u) {
+              const uint32_t a = stg + (uint32_t)lane * 128u + (uint32_t)(((u ^ (lane & 7)) & 7) << 4);
+              asm volatile("st.shared.v4.b32 [%0], {%1, %2, %3, %4};" ::"r"(a), "r"(v[4 * u]), "r"(v[4 * u + 1]),
+                           "r"(v[4 * u + 2]), "r"(v[4 * u + 3])
+                           : "memory");
+            }
+            __syncwarp();
+          };
+          auto col_value = [&](int r) {  // row r, column `lane` of the staged block
+            const uint32_t a = stg + (uint32_t)r * 128u + (uint32_t)((((lane >> 2) ^ (r & 7)) & 7) << 4) +
+                               (uint32_t)(lane & 3) * 4u;
+            float x;
+            asm volatile("ld.shared.f32 %0, [%1];" : "=f"(x) : "r"(a) : "memory");
+            return x;
+          };
           uint32_t mask[kBlocks], cmask[kBlocks];
           int total = 0;
 #pragma unroll
@@ -477,14 +496,15 @@ __global__ void __launch_bounds__(Cfg<kQ>::kThreads, 1) fused_lora_gemm(const __
                 if (j < nv && __uint_as_float(v[j]) >= tau) mask[bk] |= 1u << j;
               total += __popc(mask[bk]);
               if (tr) {
+                // lane l: which of the warp's 32 rows reach column l's threshold
+                stage_block(v);
                 const float tau_c = lane < nv ? Q.tau[Q.col_off + n0 + col0 + lane] : INFINITY;
-                const bool row_ok = row0 + lane < Q.M;
-#pragma unroll
-                for (int j = 0; j < 32; ++j) {
-                  const float t = __shfl_sync(0xffffffffu, tau_c, j);
-                  const unsigned m = __ballot_sync(0xffffffffu, row_ok && __uint_as_float(v[j]) >= t);
-                  if (lane == j) cmask[bk] = m;
-                }
+                uint32_t cm = 0u;
+#pragma unroll 8
+                for (int r = 0; r < 32; ++r)
+                  if (col_value(r) >= tau_c && row0 + r < Q.M) cm |= 1u << r;
+                cmask[bk] = cm;
+                __syncwarp();  // read before the next block is staged
               }
             }
           }
@@ -514,17 +534,19 @@ __global__ void __launch_bounds__(Cfg<kQ>::kThreads, 1) fused_lora_gemm(const __
                   ++slot;
                 }
               }
-              if (tr) {
-#pragma unroll
-                for (int j = 0; j < 32; ++j) {
-                  const unsigned m = __shfl_sync(0xffffffffu, cmask[bk], j);
-                  const int b0 = __shfl_sync(0xffffffffu, cbase[bk], j);
-                  if ((m >> lane) & 1u) {
-                    const int sl = b0 + __popc(m & ((1u << lane) - 1u));
-                    if (sl < Q.cap)
-                      Q.cand[(size_t)(j_abs0 + j) * Q.cap + sl] = make_uint2(ord_key(__uint_as_float(v[j])), (uint32_t)i_abs);
-                  }
+              if (tr && __any_sync(0xffffffffu, cmask[bk] != 0u)) {
+                // lane l writes column l's hits from the staged block
+                stage_block(v);
+                uint32_t m = cmask[bk];
+                int sl = cbase[bk];
+                uint2* cd = Q.cand + (size_t)(j_abs0 + lane) * Q.cap;
+                while (m != 0u) {
+                  const int r = __ffs(m) - 1;
+                  m &= m - 1u;
+                  if (sl < Q.cap) cd[sl] = make_uint2(ord_key(col_value(r)), (uint32_t)(Q.row_off + row0 + r));
+                  ++sl;
                 }
+                __syncwarp();  // read before the next block is staged
               }
             }
           }
