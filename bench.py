@@ -505,7 +505,7 @@ def run_gpu_ce(args, wl):
     flops = 4.0 * nT * nJ * wl.hidden  # logits and dh contractions
     sustained = peaks.get("bf16_tflops_sustained", FALLBACK_PEAKS["bf16_tflops_sustained"])
     burst = peaks.get("bf16_tflops", FALLBACK_PEAKS["bf16_tflops"])
-    gemm_tf = gemm_flops / (gemm_ms / 1e3) / 1e12 if gemm_ms > 0 else None
+    gemm_tf = flops / (gemm_ms / 1e3) / 1e12 if gemm_ms > 0 else None
     line = {
         "metric": METRIC, "value": world * wl.T / (step_ms / 1e3), "unit": UNIT, "n_gpus": world,
         "steps": K, "warmup": W, "ms_per_step": step_ms, "higher_is_better": True, "scaling": "weak",
@@ -515,7 +515,7 @@ def run_gpu_ce(args, wl):
                    "step": "lora_ce_fwd_bwd: index pass, logits of trainable positions over J, softmax CE, dh",
                    "l2": "256 MiB buffer written between timed steps (outside the step events)",
                    "parallelism": f"{world} independent replica(s), no collective"},
-        "tflops": gemm_flops / (step_ms / 1e3) / 1e12,
+        "tflops": flops / (step_ms / 1e3) / 1e12,
         "roofline": {"kernel": "fused_lora_gemm (logits and dh contractions)", "bound": "tensor",
                      "achieved": gemm_tf, "peak": sustained, "unit": "TFLOP/s",
                      "frac": gemm_tf / sustained if gemm_tf else None, "traffic": None,
@@ -606,12 +606,12 @@ def run_gpu_topk(args, wl):
     if V >= 32768:
         # the contractions performed: each row against 8192 sample tokens (thresholds), and the upper
         # triangle of C = E~ E~^T in 512-row blocks (block I against tokens from 512 I on)
-        gemm_flops = 2.0 * V * 8192 * d + sum(2.0 * min(512, V - a0) * (V - a0) * d for a0 in range(0, V, 512))
+        done_flops = 2.0 * V * 8192 * d + sum(2.0 * min(512, V - a0) * (V - a0) * d for a0 in range(0, V, 512))
     else:
-        gemm_flops = flops
+        done_flops = flops
     sustained = peaks.get("bf16_tflops_sustained", FALLBACK_PEAKS["bf16_tflops_sustained"])
     burst = peaks.get("bf16_tflops", FALLBACK_PEAKS["bf16_tflops"])
-    gemm_tf = gemm_flops / (gemm_ms / 1e3) / 1e12
+    gemm_tf = done_flops / (gemm_ms / 1e3) / 1e12
     line = {
         "metric": "top-k similarity table rows/s", "value": V / (step_ms / 1e3), "unit": "rows/s", "n_gpus": 1,
         "steps": K, "warmup": W, "ms_per_step": step_ms, "higher_is_better": True, "scaling": "strong",
@@ -622,11 +622,11 @@ def run_gpu_topk(args, wl):
                            "whose epilogue keeps each value at or above either of its rows' thresholds; then a "
                            "per-row sort",
                    "tflops_counts": "contractions performed (sample + upper triangle), not 2 V^2 d"},
-        "tflops": gemm_flops / (step_ms / 1e3) / 1e12,
+        "tflops": done_flops / (step_ms / 1e3) / 1e12,
         "roofline": {"kernel": "fused_lora_gemm (sample and similarity contractions)", "bound": "tensor",
                      "achieved": gemm_tf, "peak": sustained, "unit": "TFLOP/s", "frac": gemm_tf / sustained,
                      "traffic": None, "peak_kind": f"bf16 sustained, of {peaks_src}",
-                     "frac_of_burst": gemm_tf / burst, "flops_per_step": gemm_flops, "ms_per_step": gemm_ms},
+                     "frac_of_burst": gemm_tf / burst, "flops_per_step": done_flops, "ms_per_step": gemm_ms},
         "gpu_launches": launches, "clocks": clk, "status": lora.lora_strerror(lora.lora_read_status()),
         "e2e": None,
     }

@@ -1153,7 +1153,7 @@ int ce_check(const lora_ce_args* a, CePlan* pl) {
     return o;
   };
   pl->tiles = take(16);
-  pl->counts = take(16);
+  pl->counts = take(32);  // |T_set|, |J|, error flag, -, two last-block counters
   pl->segs = take(128 * 4);
   pl->flags = take((size_t)V);
   pl->J = take((size_t)V * 4);
@@ -1596,22 +1596,21 @@ int lora_ce_fwd_bwd(const lora_ce_args* a, void* workspace, size_t workspace_byt
     float2* lse_part = at<float2>(ws, pl.lse_part);
     const int ldz = (int)rup(nJ, 4), ldg = (int)rup(nJ, 8);
     int* tiles = at<int>(ws, pl.tiles);
-    if (launch_gather_rows(cb(a->h), D, ix.tl, nT, D, ht, st) != cudaSuccess) return LORA_ECUDA;
     // J sorted ascending with |J| = V is every token in order: E serves as E_J
     const bf* ej = cb(a->E);
-    if (nJ < V) {
-      bf* ejw = at<bf>(ws, pl.ej);
-      if (launch_gather_rows(cb(a->E), D, ix.J, nJ, D, ejw, st) != cudaSuccess) return LORA_ECUDA;
-      ej = ejw;
-    }
+    bf* ejw = at<bf>(ws, pl.ej);
+    if (launch_gather_rows2(cb(a->h), D, ix.tl, nT, ht, cb(a->E), D, ix.J, nJ < V ? nJ : 0, ejw, D, st) !=
+        cudaSuccess)
+      return LORA_ECUDA;
+    if (nJ < V) ej = ejw;
     {
       ProfScope ps(LORA_KERNEL_GEMM_FWD, st);
       if ((rc = ce_gemm(d, tiles, ht, D, ej, D, z, ldz, nT, nJ, D, false, true, at<float>(ws, pl.part), st, lse_part,
                         pl.ld_lse)) != LORA_OK)
         return rc;
     }
-    if (launch_ce_rows(lse_part, pl.ld_lse, z, ldz, nJ, ix.ycol, nT, at<float>(ws, pl.lse), rowloss, g, ldg,
-                       d->num_sms, st) != cudaSuccess)
+    if (launch_ce_rows(lse_part, pl.ld_lse, z, ldz, nJ, ix.ycol, nT, at<float>(ws, pl.lse), rowloss, ix.tpos, T,
+                       a->token_loss, a->loss, ix.counts + 5, g, ldg, d->num_sms, st) != cudaSuccess)
       return LORA_ECUDA;
     if (a->dh) {
       bf* dht = at<bf>(ws, pl.dht);
@@ -1621,7 +1620,9 @@ int lora_ce_fwd_bwd(const lora_ce_args* a, void* workspace, size_t workspace_byt
         return rc;
     }
   }
-  if (launch_ce_finish(rowloss, nT, ix.tpos, T, a->token_loss, a->loss, st) != cudaSuccess) return LORA_ECUDA;
+  // with trainable positions the log-sum-exp launch's last block has written the losses
+  if (nT == 0 && launch_ce_finish(rowloss, nT, ix.tpos, T, a->token_loss, a->loss, st) != cudaSuccess)
+    return LORA_ECUDA;
   if (a->dh && launch_scatter_rows(at<bf>(ws, pl.dht), ix.tpos, T, D, mb(a->dh), st) != cudaSuccess)
     return LORA_ECUDA;
   if (a->vocab && nJ > 0 &&

@@ -231,20 +231,27 @@ struct CeIndex {
   long long ld_topk;
   int k;
   uint8_t* flags;
-  int32_t *J, *pos, *tl, *tpos, *ycol, *counts;
+  int32_t *J, *pos, *tl, *tpos, *ycol;
+  int32_t* counts;      // [8]: |T_set|, |J|, error flag, -, two last-block counters
   int32_t* seg_counts;  // 128 per-segment counts of the vocabulary compaction
 };
 cudaError_t launch_ce_index(const CeIndex& a, cudaStream_t stream);
 // dst[i, :] = src[idx[i], :] for i < n (rows of d bf16, d a multiple of 8).
 cudaError_t launch_gather_rows(const __nv_bfloat16* src, long long ld, const int32_t* idx, int n, int d,
                                __nv_bfloat16* dst, cudaStream_t stream);
+// Two such gathers in one launch.
+cudaError_t launch_gather_rows2(const __nv_bfloat16* src_a, long long ld_a, const int32_t* idx_a, int n_a,
+                                __nv_bfloat16* dst_a, const __nv_bfloat16* src_b, long long ld_b,
+                                const int32_t* idx_b, int n_b, __nv_bfloat16* dst_b, int d, cudaStream_t stream);
 // Per row i < nT of the fp32 logits Z [nT, ldz] with their log-sum-exp
-// partials lse_part [nT, ld_part] (one per gemm_lse_group() columns):
+// partials lse_part [nT, ld_part] (one per gemm_lse_group() columns), nT >= 1:
 // lse[i], rowloss[i] = lse - z[ycol[i]] and G[i, :] = bf16(softmax - onehot),
 // zero in columns [nJ, ldg).
+// The last block also writes token_loss (optional) and *loss (as launch_ce_finish);
+// done: a zeroed counter.
 cudaError_t launch_ce_rows(const float2* lse_part, int ld_part, const float* Z, int ldz, int nJ, const int32_t* ycol,
-                           int nT, float* lse, float* rowloss, __nv_bfloat16* G, int ldg, int num_sms,
-                           cudaStream_t stream);
+                           int nT, float* lse, float* rowloss, const int32_t* tpos, int T, float* token_loss,
+                           float* loss, int* done, __nv_bfloat16* G, int ldg, int num_sms, cudaStream_t stream);
 // token_loss[t] (optional) and *loss = sum of rowloss in a fixed order.
 cudaError_t launch_ce_finish(const float* rowloss, int nT, const int32_t* tpos, int T, float* token_loss,
                              float* loss, cudaStream_t stream);

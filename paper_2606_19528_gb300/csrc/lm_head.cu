@@ -28,26 +28,43 @@ namespace {
 
 constexpr int kScanThreads = 1024;
 
-__global__ void vocab_mark_kernel(const int32_t* __restrict__ targets, const uint8_t* __restrict__ mask, int T,
-                                  const int32_t* __restrict__ topk, long long ld, int k, int V,
-                                  uint8_t* __restrict__ flags, int32_t* __restrict__ counts) {
+// One block of 128 threads per position t: if t is trainable, flags[v] = 1
+// for the k entries v of its target's table row (per 1024 entries, all loads
+// of a thread issued before its stores).
+constexpr int kMarkThreads = 128;
+
+__global__ void __launch_bounds__(kMarkThreads) vocab_mark_kernel(const int32_t* __restrict__ targets,
+                                                                  const uint8_t* __restrict__ mask, int T,
+                                                                  const int32_t* __restrict__ topk, long long ld,
+                                                                  int k, int V, uint8_t* __restrict__ flags,
+                                                                  int32_t* __restrict__ counts) {
   griddep_wait();
   griddep_launch_dependents();
-  const long long n = (long long)T * k;
-  for (long long e = blockIdx.x * (long long)blockDim.x + threadIdx.x; e < n; e += (long long)gridDim.x * blockDim.x) {
-    const int t = (int)(e / k), j = (int)(e % k);
+  for (int t = blockIdx.x; t < T; t += gridDim.x) {
     if (mask && !mask[t]) continue;
     const int y = targets[t];
     if (y < 0 || y >= V) {
-      counts[2] = 1;  // invalid target
+      if (threadIdx.x == 0) counts[2] = 1;  // invalid target
       continue;
     }
-    const int v = topk[(long long)y * ld + j];
-    if (v < 0 || v >= V) {
-      counts[2] = 1;  // invalid table entry
-      continue;
+    const int32_t* row = topk + (long long)y * ld;
+    for (int j0 = 0; j0 < k; j0 += 8 * kMarkThreads) {
+      int v[8];
+#pragma unroll
+      for (int q = 0; q < 8; ++q) {
+        const int j = j0 + threadIdx.x + q * kMarkThreads;
+        v[q] = j < k ? row[j] : 0;
+      }
+#pragma unroll
+      for (int q = 0; q < 8; ++q) {
+        if (j0 + threadIdx.x + q * kMarkThreads < k) {
+          if (v[q] < 0 || v[q] >= V)
+            counts[2] = 1;  // invalid table entry
+          else
+            flags[v[q]] = 1;
+        }
+      }
     }
-    flags[v] = 1;
   }
 }
 
@@ -127,14 +144,22 @@ __global__ void __launch_bounds__(256) vocab_count_kernel(const uint8_t* __restr
 
 // Blocks 0 .. kSegs-1: their segment of J (ascending) and pos; block kSegs:
 // the trainable positions, their inverse map and the counts.
-__global__ void __launch_bounds__(kScanThreads) compact_kernel(const uint8_t* __restrict__ flags, int V, int full,
-                                                               const int32_t* __restrict__ seg_counts,
-                                                               const uint8_t* __restrict__ mask, int T,
-                                                               int32_t* J, int32_t* pos, int32_t* tl, int32_t* tpos,
-                                                               int32_t* counts) {
-  griddep_wait();
-  griddep_launch_dependents();
-  __shared__ int s_base;
+// The last block to finish also places each trainable target in J (ycol).
+__device__ void ycol_rows(const int32_t* __restrict__ targets, const int32_t* tl, const int32_t* pos, int V,
+                          int32_t* ycol, int32_t* counts) {
+  const int nT = counts[0];
+  for (int i = threadIdx.x; i < nT; i += blockDim.x) {
+    const int y = targets[tl[i]];
+    const int c = (y >= 0 && y < V) ? pos[y] : -1;
+    if (c < 0) counts[2] = 1;  // a trainable target outside J (or out of range)
+    ycol[i] = c < 0 ? 0 : c;
+  }
+}
+
+__device__ void compact_part(const uint8_t* __restrict__ flags, int V, int full, const int32_t* __restrict__ seg_counts,
+                             const uint8_t* __restrict__ mask, int T, int32_t* J, int32_t* pos, int32_t* tl,
+                             int32_t* tpos, int32_t* counts, int* s_base_p) {
+  int& s_base = *s_base_p;
   if (blockIdx.x < kSegs) {
     const int seg = (V + kSegs - 1) / kSegs;
     const int b0 = min(V, (int)blockIdx.x * seg), b1 = min(V, b0 + seg);
@@ -166,18 +191,24 @@ __global__ void __launch_bounds__(kScanThreads) compact_kernel(const uint8_t* __
   }
 }
 
-// Column in J of each trainable position's target (after the compaction).
-__global__ void ycol_kernel(const int32_t* __restrict__ targets, const int32_t* __restrict__ tl,
-                            const int32_t* __restrict__ pos, int V, int32_t* __restrict__ ycol,
-                            int32_t* __restrict__ counts) {
+__global__ void __launch_bounds__(kScanThreads) compact_kernel(const uint8_t* __restrict__ flags, int V, int full,
+                                                               const int32_t* __restrict__ seg_counts,
+                                                               const uint8_t* __restrict__ mask, int T,
+                                                               int32_t* J, int32_t* pos, int32_t* tl, int32_t* tpos,
+                                                               int32_t* counts, const int32_t* __restrict__ targets,
+                                                               int32_t* ycol, int32_t* done) {
   griddep_wait();
   griddep_launch_dependents();
-  const int nT = counts[0];
-  for (int i = blockIdx.x * blockDim.x + threadIdx.x; i < nT; i += gridDim.x * blockDim.x) {
-    const int y = targets[tl[i]];
-    const int c = (y >= 0 && y < V) ? pos[y] : -1;
-    if (c < 0) counts[2] = 1;  // a trainable target outside J (or out of range)
-    ycol[i] = c < 0 ? 0 : c;
+  __shared__ int s_base, s_last;
+  compact_part(flags, V, full, seg_counts, mask, T, J, pos, tl, tpos, counts, &s_base);
+  // the last block to finish (every J, pos, tl written and visible) places the targets
+  __threadfence();
+  __syncthreads();
+  if (threadIdx.x == 0) s_last = atomicAdd(done, 1) == (int)gridDim.x - 1;
+  __syncthreads();
+  if (s_last) {
+    __threadfence();
+    ycol_rows(targets, tl, pos, V, ycol, counts);
   }
 }
 
@@ -195,6 +226,38 @@ __global__ void gather_rows_kernel(const __nv_bfloat16* __restrict__ src, long l
   }
 }
 
+// Two gathers in one launch (blockIdx.y selects the row set): one warp per
+// row, four 16-byte loads in flight per lane.
+__global__ void gather_rows2_kernel(const __nv_bfloat16* __restrict__ src_a, long long ld_a,
+                                    const int32_t* __restrict__ idx_a, int n_a, __nv_bfloat16* __restrict__ dst_a,
+                                    const __nv_bfloat16* __restrict__ src_b, long long ld_b,
+                                    const int32_t* __restrict__ idx_b, int n_b, __nv_bfloat16* __restrict__ dst_b,
+                                    int d) {
+  griddep_wait();
+  griddep_launch_dependents();
+  const bool b = blockIdx.y == 1;
+  const __nv_bfloat16* src = b ? src_b : src_a;
+  const long long ld = b ? ld_b : ld_a;
+  const int32_t* idx = b ? idx_b : idx_a;
+  const int n = b ? n_b : n_a;
+  __nv_bfloat16* dst = b ? dst_b : dst_a;
+  const int vpr = d / 8, lane = threadIdx.x & 31;
+  const int warps = gridDim.x * (blockDim.x >> 5);
+  for (int i = blockIdx.x * (blockDim.x >> 5) + (threadIdx.x >> 5); i < n; i += warps) {
+    const uint4* s = reinterpret_cast<const uint4*>(src + (long long)idx[i] * ld);
+    uint4* o = reinterpret_cast<uint4*>(dst + (long long)i * d);
+    for (int v0 = lane; v0 < vpr; v0 += 4 * 32) {
+      uint4 q[4];
+#pragma unroll
+      for (int u = 0; u < 4; ++u)
+        if (v0 + u * 32 < vpr) q[u] = __ldg(s + v0 + u * 32);
+#pragma unroll
+      for (int u = 0; u < 4; ++u)
+        if (v0 + u * 32 < vpr) o[v0 + u * 32] = q[u];
+    }
+  }
+}
+
 // Combine two (max, sum of exp(x - max)) pairs.
 __device__ __forceinline__ void lse_merge(float& m, float& s, float m2, float s2) {
   if (m2 > m) {
@@ -205,13 +268,33 @@ __device__ __forceinline__ void lse_merge(float& m, float& s, float m2, float s2
   }
 }
 
+// Per-position losses (zeros off the trainable set) and their sum in a fixed
+// order (fp64), by one block of 256 threads.
+__device__ void finish_body(const float* rowloss, int nT, const int32_t* tpos, int T, float* token_loss,
+                            float* loss) {
+  __shared__ double part[256];
+  if (token_loss)
+    for (int t = threadIdx.x; t < T; t += blockDim.x) token_loss[t] = tpos[t] >= 0 ? rowloss[tpos[t]] : 0.f;
+  double acc = 0.0;
+  for (int i = threadIdx.x; i < nT; i += blockDim.x) acc += (double)rowloss[i];
+  part[threadIdx.x] = acc;
+  __syncthreads();
+  for (int w = blockDim.x / 2; w > 0; w >>= 1) {
+    if ((int)threadIdx.x < w) part[threadIdx.x] += part[threadIdx.x + w];
+    __syncthreads();
+  }
+  if (threadIdx.x == 0) *loss = (float)part[0];
+}
+
 // One block per trainable position i: its log-sum-exp over J from the logits
 // contraction's per-group (max, sum of exp) partials, and its loss
 // lse - z[i, ycol[i]].
 __global__ void __launch_bounds__(256) ce_lse_kernel(const float2* __restrict__ part, int ld_part, int ngroups,
                                                      const float* __restrict__ Z, int ldz,
                                                      const int32_t* __restrict__ ycol, float* __restrict__ lse_out,
-                                                     float* __restrict__ rowloss) {
+                                                     float* rowloss, const int32_t* __restrict__ tpos, int T,
+                                                     float* __restrict__ token_loss, float* __restrict__ loss,
+                                                     int* __restrict__ done) {
   griddep_wait();
   griddep_launch_dependents();
   __shared__ float sm[8], ss[8];
@@ -239,6 +322,16 @@ __global__ void __launch_bounds__(256) ce_lse_kernel(const float2* __restrict__ 
     const float lse = M + logf(S);
     lse_out[i] = lse;
     rowloss[i] = lse - Z[(long long)i * ldz + ycol[i]];
+  }
+  // the last block to finish (every rowloss written and visible) sums the losses
+  __shared__ int s_last;
+  __threadfence();
+  __syncthreads();
+  if (threadIdx.x == 0) s_last = atomicAdd(done, 1) == (int)gridDim.x - 1;
+  __syncthreads();
+  if (s_last) {
+    __threadfence();
+    finish_body(rowloss, (int)gridDim.x, tpos, T, token_loss, loss);
   }
 }
 
@@ -275,24 +368,12 @@ __global__ void __launch_bounds__(256) ce_grad_kernel(const float* __restrict__ 
   }
 }
 
-// Per-position losses (zeros off the trainable set) and their sum in a fixed order.
 __global__ void __launch_bounds__(256) ce_finish_kernel(const float* __restrict__ rowloss, int nT,
                                                         const int32_t* __restrict__ tpos, int T,
                                                         float* __restrict__ token_loss, float* __restrict__ loss) {
   griddep_wait();
   griddep_launch_dependents();
-  __shared__ double part[256];
-  if (token_loss)
-    for (int t = threadIdx.x; t < T; t += blockDim.x) token_loss[t] = tpos[t] >= 0 ? rowloss[tpos[t]] : 0.f;
-  double acc = 0.0;
-  for (int i = threadIdx.x; i < nT; i += blockDim.x) acc += (double)rowloss[i];
-  part[threadIdx.x] = acc;
-  __syncthreads();
-  for (int w = blockDim.x / 2; w > 0; w >>= 1) {
-    if ((int)threadIdx.x < w) part[threadIdx.x] += part[threadIdx.x + w];
-    __syncthreads();
-  }
-  if (threadIdx.x == 0) *loss = (float)part[0];
+  finish_body(rowloss, nT, tpos, T, token_loss, loss);
 }
 
 __global__ void scatter_rows_kernel(const __nv_bfloat16* __restrict__ src, const int32_t* __restrict__ tpos, int T,
@@ -322,20 +403,26 @@ int grid_for(long long n, int threads, int cap) {
 cudaError_t launch_ce_index(const CeIndex& a, cudaStream_t st) {
   cudaError_t e;
   if (a.topk) {
-    const long long n = (long long)a.T * a.k;
-    e = launch_kernel(vocab_mark_kernel, dim3(grid_for(n, 256, 4096)), dim3(256), 0, st, 1, a.targets, a.mask, a.T,
-                      a.topk, a.ld_topk, a.k, a.V, a.flags, a.counts);
+    e = launch_kernel(vocab_mark_kernel, dim3(std::min(a.T, 65535)), dim3(kMarkThreads), 0, st, 1, a.targets,
+                      a.mask, a.T, a.topk, a.ld_topk, a.k, a.V, a.flags, a.counts);
     if (e != cudaSuccess) return e;
   }
   const int full = a.topk ? 0 : 1;
   e = launch_kernel(vocab_count_kernel, dim3(kSegs), dim3(256), 0, st, 1, (const uint8_t*)a.flags, a.V, full,
                     a.seg_counts);
   if (e != cudaSuccess) return e;
-  e = launch_kernel(compact_kernel, dim3(kSegs + 1), dim3(kScanThreads), 0, st, 1, (const uint8_t*)a.flags, a.V,
-                    full, (const int32_t*)a.seg_counts, a.mask, a.T, a.J, a.pos, a.tl, a.tpos, a.counts);
-  if (e != cudaSuccess) return e;
-  return launch_kernel(ycol_kernel, dim3(grid_for(a.T, 256, 64)), dim3(256), 0, st, 1, a.targets,
-                       (const int32_t*)a.tl, (const int32_t*)a.pos, a.V, a.ycol, a.counts);
+  return launch_kernel(compact_kernel, dim3(kSegs + 1), dim3(kScanThreads), 0, st, 1, (const uint8_t*)a.flags, a.V,
+                       full, (const int32_t*)a.seg_counts, a.mask, a.T, a.J, a.pos, a.tl, a.tpos, a.counts, a.targets,
+                       a.ycol, a.counts + 4);
+}
+
+cudaError_t launch_gather_rows2(const __nv_bfloat16* src_a, long long ld_a, const int32_t* idx_a, int n_a,
+                                __nv_bfloat16* dst_a, const __nv_bfloat16* src_b, long long ld_b,
+                                const int32_t* idx_b, int n_b, __nv_bfloat16* dst_b, int d, cudaStream_t st) {
+  if (n_b <= 0) return launch_gather_rows(src_a, ld_a, idx_a, n_a, d, dst_a, st);
+  if (n_a <= 0) return launch_gather_rows(src_b, ld_b, idx_b, n_b, d, dst_b, st);
+  return launch_kernel(gather_rows2_kernel, dim3(grid_for(std::max(n_a, n_b), 8, 4096), 2), dim3(256), 0, st, 1,
+                       src_a, ld_a, idx_a, n_a, dst_a, src_b, ld_b, idx_b, n_b, dst_b, d);
 }
 
 cudaError_t launch_gather_rows(const __nv_bfloat16* src, long long ld, const int32_t* idx, int n, int d,
@@ -346,11 +433,12 @@ cudaError_t launch_gather_rows(const __nv_bfloat16* src, long long ld, const int
 }
 
 cudaError_t launch_ce_rows(const float2* lse_part, int ld_part, const float* Z, int ldz, int nJ, const int32_t* ycol,
-                           int nT, float* lse, float* rowloss, __nv_bfloat16* G, int ldg, int num_sms, cudaStream_t st) {
+                           int nT, float* lse, float* rowloss, const int32_t* tpos, int T, float* token_loss,
+                           float* loss, int* done, __nv_bfloat16* G, int ldg, int num_sms, cudaStream_t st) {
   if (nT <= 0) return cudaSuccess;
   const int ngroups = (nJ + gemm_lse_group() - 1) / gemm_lse_group();
   cudaError_t e = launch_kernel(ce_lse_kernel, dim3(nT), dim3(256), 0, st, 1, lse_part, ld_part, ngroups, Z, ldz,
-                                ycol, lse, rowloss);
+                                ycol, lse, rowloss, tpos, T, token_loss, loss, done);
   if (e != cudaSuccess) return e;
   const long long items = (long long)nT * ((ldg + kGradChunk - 1) / kGradChunk);
   const int grid = (int)std::min<long long>(items, (long long)num_sms * 8);
