@@ -242,14 +242,15 @@ inline int64_t rup(int64_t x, int64_t m) { return (x + m - 1) / m * m; }
 // ------------------------------------------------------------------ fused-contraction problems
 // Output [M, N] over a contraction of Kc base columns plus an r-wide adapter
 // slab; one contraction pass, output written directly (no split).
-void gemm_shape(GemmProblem& g, int64_t M, int64_t N, int64_t Kc, int64_t r) {
+// tile_n: the launch's tile width (gemm_tile_n(), or gemm_tile_n_f32() for fp32 output).
+void gemm_shape(GemmProblem& g, int64_t M, int64_t N, int64_t Kc, int64_t r, int tile_n = 0) {
   g.ldo = (int)N;
   g.out_f32 = 0;
   g.M = (int)M;
   g.N = (int)N;
   g.Kmain = (int)Kc;
   g.r = (int)r;
-  g.num_n_tiles = cdiv(N, gemm_tile_n());
+  g.num_n_tiles = cdiv(N, tile_n > 0 ? tile_n : gemm_tile_n());
   g.num_m_tiles = cdiv(M, gemm_tile_m());
   g.m_fast = N >= M ? 1 : 0;  // the weight operand at least as large as the activation operand
   g.kb_main = cdiv(Kc, gemm_tile_k());
@@ -1204,7 +1205,7 @@ int ce_gemm(const DeviceInfo* d, int* counter, const void* A, int64_t lda, const
                  : make_map(&b.tmOut[0], out, N, M, ldo, f32_out ? 32 : 64, 32, f32_out)) != LORA_OK)
     return rc;
   GemmProblem& g = b.prob[0];
-  gemm_shape(g, M, N, K, 0);
+  gemm_shape(g, M, N, K, 0, f32_out ? gemm_tile_n_f32() : 0);
   g.out = out;
   g.ldo = (int)ldo;
   g.out_f32 = f32_out ? 1 : 0;
@@ -1236,16 +1237,16 @@ int topk_sym_gemm(const DeviceInfo* d, int* counter, const bf* en, int64_t dd, i
   init_batch(b, d);
   b.tile_counter = counter;
   int rc;
-  for (int64_t a0 = r0; a0 < r0 + rows; a0 += 512) {
+  for (int64_t a0 = r0; a0 < r0 + rows; a0 += kSymRows) {
     const int p = b.num_problems;
-    const int64_t m = std::min<int64_t>(512, r0 + rows - a0), N = V - a0;
+    const int64_t m = std::min<int64_t>(kSymRows, r0 + rows - a0), N = V - a0;
     if ((rc = make_map(&b.tmA[p], en + a0 * dd, dd, m, dd, 64, 128)) != LORA_OK) return rc;
     if ((rc = make_map(&b.tmB[p], en + a0 * dd, dd, N, dd, 64, 64)) != LORA_OK) return rc;
     b.tmA2[p] = b.tmA[p];
     b.tmB2[p] = b.tmB[p];
     if ((rc = make_map(&b.tmOut[p], cand, 32, 32, 32, 32, 32, true)) != LORA_OK) return rc;  // never stored through
     GemmProblem& g = b.prob[p];
-    gemm_shape(g, m, N, dd, 0);
+    gemm_shape(g, m, N, dd, 0, gemm_tile_n_f32());
     g.out_f32 = 1;
     g.tau = tau;
     g.cnt = cnt;

@@ -66,7 +66,7 @@ constexpr uint32_t kEpiStage = 32 * 128;          // per-warp output block: 32 r
 constexpr uint32_t kTmemCols = 512;
 constexpr int kConvWarps = 4;                     // 4-bit weights: dequantizing warps per CTA
 
-constexpr int kMaxStages = 4;
+constexpr int kMaxStages = 6;
 constexpr uint32_t kStageBytes = kAHalf + 2 * kBSeg;  // bf16 weights: activation + weight boxes
 constexpr uint32_t kQCodes = 8192;                    // 4-bit block: 256 weight rows x 64 codes
 constexpr uint32_t kQSlot = kQCodes + 4096;           // + (s, b) boxes
@@ -105,8 +105,8 @@ struct __align__(8) Ctl {
   uint64_t wfull[kWStages];        // even CTA, 4-bit: both CTAs' weight tile dequantized (or loaded)
   uint64_t convd[kWStages];        // both CTAs, 4-bit: this CTA's dequantizing warps finished a weight tile
   uint64_t wempty[kWStages];       // both CTAs, 4-bit: the pair's MMAs finished reading a weight tile
-  uint64_t tfull;                  // both CTAs: accumulator complete
-  uint64_t tempty[2];              // even CTA: both CTAs' epilogues drained a segment
+  uint64_t tfull[2];               // both CTAs: accumulator (buffer) complete
+  uint64_t tempty[2];              // even CTA: both CTAs' epilogues drained a segment (buffer)
   uint64_t tile_full[kTileRing];   // both CTAs: tile id written
   uint64_t tile_empty[kTileRing];  // even CTA: every consumer of both CTAs read the slot
   uint64_t drain;                  // both CTAs: every MMA of the pair completed
@@ -122,6 +122,7 @@ constexpr size_t smem_bytes() {
 
 // Problem p, first row m0 and first column n0 of tile t, its split ks and
 // that split's contraction blocks [kb0, kb1).
+template <int kTileN = kBN>
 __device__ __forceinline__ void decode_tile(const GemmBatch& b, int t, int& p, int& m0, int& n0, int& ks, int& kb0,
                                             int& kb1) {
   p = 0;
@@ -135,10 +136,10 @@ __device__ __forceinline__ void decode_tile(const GemmBatch& b, int t, int& p, i
   kb1 = min(Q.kb_total, kb0 + Q.kb_split);
   if (Q.m_fast) {
     m0 = (local % Q.num_m_tiles) * kBM;
-    n0 = (local / Q.num_m_tiles) * kBN;
+    n0 = (local / Q.num_m_tiles) * kTileN;
   } else {
     m0 = (local / Q.num_n_tiles) * kBM;
-    n0 = (local % Q.num_n_tiles) * kBN;
+    n0 = (local % Q.num_n_tiles) * kTileN;
   }
 }
 
@@ -204,7 +205,19 @@ __device__ __forceinline__ void dequant_stage(uint32_t slot, uint32_t wdst, int 
 
 template <bool kBMn, bool kQ, bool kF32 = false>
 __global__ void __launch_bounds__(Cfg<kQ>::kThreads, 1) fused_lora_gemm(const __grid_constant__ GemmBatch b) {
-  constexpr int kStages = Cfg<kQ>::kStages;
+  // fp32 output: 256 x 256 tiles whose accumulator alternates between two TMEM
+  // buffers, so one tile's epilogue overlaps the next tile's contraction (the
+  // appending and log-sum-exp epilogues are long); a 6-deep ring of 32 KB stages
+  constexpr bool kNarrow = kF32;
+  static_assert(!kNarrow || (!kQ && !kBMn), "fp32 output is the plain forward form");
+  constexpr int kSegs = kNarrow ? 1 : 2;  // 256-column segments per tile
+  constexpr int kTileN = kSegs * kSeg;
+  constexpr int kStages = kNarrow ? 6 : Cfg<kQ>::kStages;
+  constexpr uint32_t kStageB = kNarrow ? kAHalf + kBSeg : kStageBytes;
+  static_assert(kStages <= kMaxStages && (!kNarrow || kStages * kStageB <= Cfg<kQ>::kRing), "ring");
+  auto a_addr_of = [&](uint32_t bs, int st) {
+    return kQ ? Cfg<kQ>::a_addr(bs, st) : bs + (uint32_t)st * kStageB;
+  };
   extern __shared__ uint8_t smem_raw[];
   const uint32_t raw = smem_u32(smem_raw);
   const uint32_t base = (raw + 1023u) & ~1023u;
@@ -233,7 +246,8 @@ __global__ void __launch_bounds__(Cfg<kQ>::kThreads, 1) fused_lora_gemm(const __
       mbar_init(smem_u32(&ctl->convd[w]), kConvWarps);
       mbar_init(smem_u32(&ctl->wempty[w]), 1);
     }
-    mbar_init(smem_u32(&ctl->tfull), 1);
+    mbar_init(smem_u32(&ctl->tfull[0]), 1);
+    mbar_init(smem_u32(&ctl->tfull[1]), 1);
     for (int h = 0; h < 2; ++h) mbar_init(smem_u32(&ctl->tempty[h]), 2 * kEpi);
     for (int k = 0; k < kTileRing; ++k) {
       mbar_init(smem_u32(&ctl->tile_full[k]), 1);
@@ -298,14 +312,14 @@ __global__ void __launch_bounds__(Cfg<kQ>::kThreads, 1) fused_lora_gemm(const __
           break;
         }
         int p, m0, n0, ks, kb0, kb1;
-        decode_tile(b, t, p, m0, n0, ks, kb0, kb1);
+        decode_tile<kTileN>(b, t, p, m0, n0, ks, kb0, kb1);
         const GemmProblem& Q = b.prob[p];
         const int my_m = m0 + c * kHalf;
         const bool a_mine = my_m < Q.M;
         // weight box (segment h, pair position cc, j): columns n0 + 256 h + 128 cc + 64 j
         auto box_ok = [&](int h, int cc, int j) { return n0 + h * kSeg + cc * kHalf + j * 64 < Q.N; };
         uint32_t boxes = 0;
-        for (int h = 0; h < 2; ++h)
+        for (int h = 0; h < kSegs; ++h)
           for (int cc = 0; cc < 2; ++cc)
             for (int j = 0; j < 2; ++j) boxes += box_ok(h, cc, j) ? 1u : 0u;
         // bytes landing in this pair per stage (signalled on the even CTA)
@@ -322,7 +336,7 @@ __global__ void __launch_bounds__(Cfg<kQ>::kThreads, 1) fused_lora_gemm(const __
           const bool w_tma = !kQ;
           if (c == 0) mbar_arrive_expect_tx(smem_u32(&ctl->full[stage]), w_tma ? tx_pair : tx_a);
           const uint32_t bar = full_pl + (uint32_t)stage * 8u;
-          const uint32_t a_dst = Cfg<kQ>::a_addr(base, stage);
+          const uint32_t a_dst = a_addr_of(base, stage);
           const uint32_t b_dst = a_dst + kAHalf;
           const int kc = main ? kb * kBK : (kb - Q.kb_main) * kBK;
           const CUtensorMap* ta = main ? &b.tmA[p] : &b.tmA2[p];
@@ -330,7 +344,7 @@ __global__ void __launch_bounds__(Cfg<kQ>::kThreads, 1) fused_lora_gemm(const __
           if (a_mine) tma_load_2d_pair(a_dst, ta, bar, kc, my_m);
           if (w_tma) {
 #pragma unroll
-            for (int h = 0; h < 2; ++h) {
+            for (int h = 0; h < kSegs; ++h) {
 #pragma unroll
               for (int j = 0; j < 2; ++j) {
                 if (!box_ok(h, c, j)) continue;
@@ -367,11 +381,13 @@ __global__ void __launch_bounds__(Cfg<kQ>::kThreads, 1) fused_lora_gemm(const __
           break;
         }
         int p, m0, n0, ks, kb0, kb1;
-        decode_tile(b, t, p, m0, n0, ks, kb0, kb1);
+        decode_tile<kTileN>(b, t, p, m0, n0, ks, kb0, kb1);
         const GemmProblem& Q = b.prob[p];
-        const int nseg = Q.N - n0 > kSeg ? 2 : 1;  // segments holding any column < N
-        // segment h is free once both epilogues drained it for the previous tile
-        const uint32_t drained_par = (uint32_t)((it & 1) ^ 1);
+        const int nseg = kNarrow ? 1 : (Q.N - n0 > kSeg ? 2 : 1);  // segments holding any column < N
+        // accumulator buffer of this tile; a segment (buffer) is free once both epilogues drained
+        // it for its previous tile (the previous tile, or with two buffers the one before)
+        const int buf = kNarrow ? (it & 1) : 0;
+        const uint32_t drained_par = kNarrow ? (uint32_t)(((it >> 1) & 1) ^ 1) : (uint32_t)((it & 1) ^ 1);
         for (int kb = kb0; kb < kb1; ++kb) {
           if (!mbar_wait(smem_u32(&ctl->full[stage]), phase, wc, abort_flag)) {
             ok = false;
@@ -383,19 +399,19 @@ __global__ void __launch_bounds__(Cfg<kQ>::kThreads, 1) fused_lora_gemm(const __
             break;
           }
           tc_fence_after();
-          const uint32_t a_addr = Cfg<kQ>::a_addr(base, stage);
+          const uint32_t a_addr = a_addr_of(base, stage);
           const uint32_t b_addr = kQ ? Cfg<kQ>::w_tile(base, wt) : a_addr + kAHalf;
           const int nk = kb < Q.kb_main ? kBK / 16 : min(kBK / 16, (Q.r - (kb - Q.kb_main) * kBK + 15) / 16);
-          for (int h = 0; h < 2; ++h) {
+          for (int h = 0; h < kSegs; ++h) {
             if (kb == kb0) {
-              if (!mbar_wait_cluster(smem_u32(&ctl->tempty[h]), drained_par, wc, abort_flag)) {
+              if (!mbar_wait_cluster(smem_u32(&ctl->tempty[buf + h]), drained_par, wc, abort_flag)) {
                 ok = false;
                 break;
               }
               tc_fence_after();
             }
             if (h >= nseg) continue;
-            const uint32_t d_tmem = tmem_base + (uint32_t)(h * kSeg);
+            const uint32_t d_tmem = tmem_base + (uint32_t)((buf + h) * kSeg);
             const uint32_t bseg = b_addr + (uint32_t)h * kBSeg;
             for (int k = 0; k < nk; ++k) {
               const uint64_t adesc = sw128_desc(a_addr + k * 32, 16, 1024);
@@ -413,7 +429,7 @@ __global__ void __launch_bounds__(Cfg<kQ>::kThreads, 1) fused_lora_gemm(const __
           }
         }
         if (!ok) break;
-        umma_commit_pair_mc(smem_u32(&ctl->tfull), pair_mask);
+        umma_commit_pair_mc(smem_u32(&ctl->tfull[buf]), pair_mask);
       }
       // completes in both CTAs of the pair once every MMA issued above has finished
       umma_commit_pair_mc(smem_u32(&ctl->drain), pair_mask);
@@ -433,15 +449,17 @@ __global__ void __launch_bounds__(Cfg<kQ>::kThreads, 1) fused_lora_gemm(const __
       if (lane == 0) mbar_arrive_cluster(tile_empty_root + (uint32_t)slot * 8u);
       if (t < 0) break;
       int p, m0, n0, ks, kb0, kb1;
-      decode_tile(b, t, p, m0, n0, ks, kb0, kb1);
+      decode_tile<kTileN>(b, t, p, m0, n0, ks, kb0, kb1);
       const GemmProblem& Q = b.prob[p];
-      bool ok = mbar_wait_cluster(smem_u32(&ctl->tfull), (uint32_t)(it & 1), wc, abort_flag);
+      const int buf = kNarrow ? (it & 1) : 0;  // accumulator buffer of this tile
+      const uint32_t tpar = kNarrow ? (uint32_t)((it >> 1) & 1) : (uint32_t)(it & 1);
+      bool ok = mbar_wait_cluster(smem_u32(&ctl->tfull[buf]), tpar, wc, abort_flag);
       ok = __all_sync(0xffffffffu, ok);
       if (!ok) break;
       tc_fence_after();
       const int row0 = m0 + c * kHalf + q * 32;  // first of this warp's 32 rows
       const uint32_t stg = epi_base + (uint32_t)(warp - 2) * kEpiStage;
-      for (int h = 0; h < 2; ++h) {
+      for (int h = 0; h < kSegs; ++h) {
         // a staged block is 32 rows x 128 bytes: 64 bf16 columns, or 32 fp32 columns
         // (fp32 output, or the partial of one split of the contraction)
         const bool f32 = kF32 || Q.splits > 1;
@@ -458,7 +476,7 @@ __global__ void __launch_bounds__(Cfg<kQ>::kThreads, 1) fused_lora_gemm(const __
           // block, over the warp's 32 rows), one atomic per list reserves the slots, a second
           // pass writes the hits
           constexpr int kBlocks = Cfg<kQ>::kPartCols / 32;
-          const bool tr = Q.sym && n0 > 0;  // off the diagonal block
+          const bool tr = Q.sym && n0 >= kSymRows;  // off the diagonal block
           const int i_abs = Q.row_off + row0 + lane;
           // the transposed side reads the block column-wise from the warp's staging buffer
           // (free in append mode): row `lane` stored as 8 16-byte chunks, chunk u at u ^ (lane mod 8)
@@ -488,7 +506,7 @@ __global__ void __launch_bounds__(Cfg<kQ>::kThreads, 1) fused_lora_gemm(const __
             cmask[bk] = 0u;
             if (n0 + col0 < Q.N) {  // uniform
               uint32_t v[32];
-              tmem_ld_32x32b_x32(tmem_base + ((uint32_t)(q * 32) << 16) + (uint32_t)col0, v);
+              tmem_ld_32x32b_x32(tmem_base + ((uint32_t)(q * 32) << 16) + (uint32_t)(buf * kSeg + col0), v);
               tmem_ld_wait();
               const int nv = min(32, Q.N - (n0 + col0));
 #pragma unroll
@@ -525,7 +543,7 @@ __global__ void __launch_bounds__(Cfg<kQ>::kThreads, 1) fused_lora_gemm(const __
               const int col0 = h * kSeg + part * Cfg<kQ>::kPartCols + bk * 32;
               const int j_abs0 = Q.col_off + n0 + col0;
               uint32_t v[32];
-              tmem_ld_32x32b_x32(tmem_base + ((uint32_t)(q * 32) << 16) + (uint32_t)col0, v);
+              tmem_ld_32x32b_x32(tmem_base + ((uint32_t)(q * 32) << 16) + (uint32_t)(buf * kSeg + col0), v);
               tmem_ld_wait();
 #pragma unroll
               for (int j = 0; j < 32; ++j) {
@@ -554,7 +572,7 @@ __global__ void __launch_bounds__(Cfg<kQ>::kThreads, 1) fused_lora_gemm(const __
         for (int cc = 0; !app && cc < Cfg<kQ>::kPartCols; cc += block_cols) {
           const int col0 = h * kSeg + part * Cfg<kQ>::kPartCols + cc;  // tile column of this block
           if (n0 + col0 >= Q.N || row0 >= Q.M) break;     // uniform across the warp
-          const uint32_t taddr = tmem_base + ((uint32_t)(q * 32) << 16) + (uint32_t)col0;
+          const uint32_t taddr = tmem_base + ((uint32_t)(q * 32) << 16) + (uint32_t)(buf * kSeg + col0);
           uint32_t v[32], w[32];
           tmem_ld_32x32b_x32(taddr, v);
           if (!f32) tmem_ld_32x32b_x32(taddr + 32u, w);
@@ -611,7 +629,7 @@ __global__ void __launch_bounds__(Cfg<kQ>::kThreads, 1) fused_lora_gemm(const __
         }
         tc_fence_before();
         __syncwarp();
-        if (lane == 0) mbar_arrive_cluster(tempty_pl + (uint32_t)h * 8u);
+        if (lane == 0) mbar_arrive_cluster(tempty_pl + (uint32_t)(buf + h) * 8u);
       }
     }
     // the output must be written before the CTA exits
@@ -922,6 +940,7 @@ cudaError_t launch_fused_gemm(const GemmBatch& batch, bool b_mn_major, bool q4, 
 int gemm_tile_m() { return kBM; }
 int gemm_lse_group() { return kLseGroup; }
 int gemm_tile_n() { return kBN; }
+int gemm_tile_n_f32() { return kSeg; }
 int gemm_tile_k() { return kBK; }
 
 }  // namespace lora

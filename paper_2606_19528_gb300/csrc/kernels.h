@@ -89,6 +89,10 @@ struct GemmProblem {
   int row_off, col_off, sym;
 };
 
+// Rows of each problem of the symmetric top-k contraction: its columns start at
+// the problem's first row, so tiles with n0 < kSymRows form the diagonal block.
+constexpr int kSymRows = 512;
+
 // One launch: up to kMaxProblems independent fused contractions.
 //  tmA  [M, Kmain] K-major (x or dy)        tmA2 [M, r] K-major (su or sv)
 //  forward:  tmB  W [N, Kmain] K-major       tmB2 B [N, r] K-major
@@ -121,6 +125,7 @@ size_t fused_gemm_smem_bytes();
 // of the batch with splits > 1 (bf16 or fp32 per out_f32).
 cudaError_t launch_split_reduce(const GemmBatch& batch, cudaStream_t stream);
 int gemm_tile_m();
+int gemm_tile_n_f32();  // tile columns of the fp32-output form (two accumulator buffers)
 int gemm_lse_group();  // columns of one log-sum-exp partial
 int gemm_tile_n();
 int gemm_tile_k();
