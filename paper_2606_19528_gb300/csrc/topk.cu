@@ -124,21 +124,26 @@ __device__ void find_bin(SelShared& sh, int nbins, int k_rem) {
   __syncthreads();
 }
 
-// "a before b": larger key first, the lower index first on equal keys.
-__device__ __forceinline__ bool before(uint32_t ka, int ia, uint32_t kb, int ib) {
-  return ka > kb || (ka == kb && ia < ib);
+// A candidate as one 64-bit value, larger first: the order key above, the
+// complement of the index below (equal keys: the lower index first).
+__device__ __forceinline__ uint64_t pack_cand(uint32_t key, int idx) {
+  return ((uint64_t)key << 32) | (uint32_t)(0xffffffffu - (uint32_t)idx);
 }
+__device__ __forceinline__ int cand_index(uint64_t v) { return (int)(0xffffffffu - (uint32_t)v); }
 
-// Bitonic sort on (key descending, index ascending) of p2 = kT * E slots held
-// in registers: slot e of thread t is position t + e * kT.  Strides below 32
-// are exchanged by warp shuffles, 32 .. kT / 2 through the shared buffers xk,
-// xi (p2 entries), kT and up within the thread (fully unrolled, so the slots
-// stay in registers).  Every thread of the block takes part.
+// Bitonic sort, descending, of p2 = kT * E packed candidates held in
+// registers: slot e of thread t is position t + e * kT.  Strides below 32 are
+// exchanged by warp shuffles, 32 .. kT / 2 through the shared buffer x (p2
+// entries), kT and up within the thread (fully unrolled, so the slots stay in
+// registers).  Every thread of the block takes part.
 template <int kT, int E>
-__device__ void bitonic_sort(uint32_t (&key)[E], int (&idx)[E], uint32_t* xk, int* xi) {
+__device__ void bitonic_sort(uint64_t (&v)[E], uint64_t* x) {
   constexpr int p2 = kT * E;
   const int tid = threadIdx.x;
+  // fully unrolled: every stage's exchange form and masks are compile-time constants
+#pragma unroll
   for (int size = 2; size <= p2; size <<= 1) {
+#pragma unroll
     for (int stride = size >> 1; stride > 0; stride >>= 1) {
       if (stride >= kT) {
 #pragma unroll
@@ -149,13 +154,10 @@ __device__ void bitonic_sort(uint32_t (&key)[E], int (&idx)[E], uint32_t* xk, in
               const int f = e | (1 << lg);
               if ((e & (1 << lg)) == 0 && f < E) {
                 const bool up = ((tid + e * kT) & size) == 0;
-                if (before(key[f], idx[f], key[e], idx[e]) == up) {
-                  const uint32_t tk = key[e];
-                  const int ti = idx[e];
-                  key[e] = key[f];
-                  idx[e] = idx[f];
-                  key[f] = tk;
-                  idx[f] = ti;
+                if ((v[f] > v[e]) == up) {
+                  const uint64_t t = v[e];
+                  v[e] = v[f];
+                  v[f] = t;
                 }
               }
             }
@@ -165,31 +167,17 @@ __device__ void bitonic_sort(uint32_t (&key)[E], int (&idx)[E], uint32_t* xk, in
         const bool via_smem = stride >= 32;
         if (via_smem) {
 #pragma unroll
-          for (int e = 0; e < E; ++e) {
-            xk[tid + e * kT] = key[e];
-            xi[tid + e * kT] = idx[e];
-          }
+          for (int e = 0; e < E; ++e) x[tid + e * kT] = v[e];
           __syncthreads();
         }
 #pragma unroll
         for (int e = 0; e < E; ++e) {
           const int p = tid + e * kT;
-          uint32_t kq;
-          int iq;
-          if (via_smem) {
-            kq = xk[p ^ stride];
-            iq = xi[p ^ stride];
-          } else {
-            kq = __shfl_xor_sync(0xffffffffu, key[e], stride);
-            iq = __shfl_xor_sync(0xffffffffu, idx[e], stride);
-          }
+          const uint64_t q = via_smem ? x[p ^ stride] : __shfl_xor_sync(0xffffffffu, v[e], stride);
           const bool up = (p & size) == 0, lo = (p & stride) == 0;
-          const bool q_first = before(kq, iq, key[e], idx[e]);
+          const bool q_first = q > v[e];
           // an ascending run keeps the first of the pair at the lower position
-          if (lo ? q_first == up : q_first != up) {
-            key[e] = kq;
-            idx[e] = iq;
-          }
+          if (lo ? q_first == up : q_first != up) v[e] = q;
         }
         if (via_smem) __syncthreads();
       }
@@ -198,24 +186,26 @@ __device__ void bitonic_sort(uint32_t (&key)[E], int (&idx)[E], uint32_t* xk, in
 }
 
 // Loads n <= kT * E candidates (get(p) -> (key, index)), sorts them and writes
-// the first k indices to out; padding sorts below every real key.
+// the first k indices to out; padding sorts below every real candidate.
 template <int kT, int E, typename Get>
-__device__ void sort_write_e(Get get, int n, int k, uint32_t* xk, int* xi, int32_t* __restrict__ out) {
-  uint32_t key[E];
-  int idx[E];
+__device__ void sort_write_e(Get get, int n, int k, uint64_t* x, int32_t* __restrict__ out) {
+  uint64_t v[E];
 #pragma unroll
   for (int e = 0; e < E; ++e) {
     const int p = threadIdx.x + e * kT;
-    const uint2 v = p < n ? get(p) : make_uint2(0u, 0x7fffffffu);
-    key[e] = v.x;
-    idx[e] = (int)v.y;
+    if (p < n) {
+      const uint2 c = get(p);
+      v[e] = pack_cand(c.x, (int)c.y);
+    } else {
+      v[e] = 0ull;
+    }
   }
   __syncthreads();  // the candidates may live in the exchange buffer
-  bitonic_sort<kT, E>(key, idx, xk, xi);
+  bitonic_sort<kT, E>(v, x);
 #pragma unroll
   for (int e = 0; e < E; ++e) {
     const int p = threadIdx.x + e * kT;
-    if (p < k) out[p] = idx[e];
+    if (p < k) out[p] = cand_index(v[e]);
   }
 }
 
@@ -223,12 +213,13 @@ __device__ void sort_write_e(Get get, int n, int k, uint32_t* xk, int* xi, int32
 // 1024 threads) and writes the first k indices to out.
 __device__ void sort_and_write(SelShared& sh, int n, int k, int32_t* __restrict__ out) {
   auto get = [&](int p) { return make_uint2(sh.ckey[p], (uint32_t)sh.cidx[p]); };
+  uint64_t* x = reinterpret_cast<uint64_t*>(sh.ckey);  // ckey and cidx together: 4096 x 8 bytes
   if (n <= kSelThreads)
-    sort_write_e<kSelThreads, 1>(get, n, k, sh.ckey, sh.cidx, out);
+    sort_write_e<kSelThreads, 1>(get, n, k, x, out);
   else if (n <= 2 * kSelThreads)
-    sort_write_e<kSelThreads, 2>(get, n, k, sh.ckey, sh.cidx, out);
+    sort_write_e<kSelThreads, 2>(get, n, k, x, out);
   else
-    sort_write_e<kSelThreads, 4>(get, n, k, sh.ckey, sh.cidx, out);
+    sort_write_e<kSelThreads, 4>(get, n, k, x, out);
 }
 
 // Sampled threshold for long rows: the r-th largest of kSample evenly spread
@@ -465,7 +456,7 @@ __global__ void __launch_bounds__(kTauThreads, 4) topk_tau_kernel(const float* _
   griddep_launch_dependents();
   __shared__ int hist[2048];
   __shared__ float red[2][kTauThreads / 32];
-  __shared__ int s_bin, s_above;
+  __shared__ int s_bin;
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
   const float4* z4 = reinterpret_cast<const float4*>(Z + (long long)blockIdx.x * kSample);
   float v[kTauPer];
@@ -529,7 +520,6 @@ __global__ void __launch_bounds__(kTauThreads, 4) topk_tau_kernel(const float* _
       const int h = hist[2047 - 8 * tid - q];
       if (rs <= acc + h) {
         s_bin = 2047 - 8 * tid - q;
-        s_above = acc;
         break;
       }
       acc += h;
@@ -568,8 +558,7 @@ __global__ void __launch_bounds__(kSortThreads, 4) topk_sort_kernel(const uint2*
                                                                    int* __restrict__ fail_count) {
   griddep_wait();
   griddep_launch_dependents();
-  __shared__ uint32_t xk[kCap];
-  __shared__ int xi[kCap];
+  __shared__ uint64_t xs[kCap];
   const int r = blockIdx.x, tid = threadIdx.x;
   const int n = cnt[r];
   __syncthreads();  // every thread has read the count before it is reset
@@ -582,15 +571,15 @@ __global__ void __launch_bounds__(kSortThreads, 4) topk_sort_kernel(const uint2*
   auto get = [&](int p) { return c[p]; };
   int32_t* out = table + (long long)(row0 + r) * k;
   if (n <= kSortThreads)
-    sort_write_e<kSortThreads, 1>(get, n, k, xk, xi, out);
+    sort_write_e<kSortThreads, 1>(get, n, k, xs, out);
   else if (n <= 2 * kSortThreads)
-    sort_write_e<kSortThreads, 2>(get, n, k, xk, xi, out);
+    sort_write_e<kSortThreads, 2>(get, n, k, xs, out);
   else if (n <= 4 * kSortThreads)
-    sort_write_e<kSortThreads, 4>(get, n, k, xk, xi, out);
+    sort_write_e<kSortThreads, 4>(get, n, k, xs, out);
   else if (n <= 8 * kSortThreads)
-    sort_write_e<kSortThreads, 8>(get, n, k, xk, xi, out);
+    sort_write_e<kSortThreads, 8>(get, n, k, xs, out);
   else
-    sort_write_e<kSortThreads, 16>(get, n, k, xk, xi, out);
+    sort_write_e<kSortThreads, 16>(get, n, k, xs, out);
 }
 
 // Es[i, :] = En[floor(i * V / kSample), :]: the sample tokens, evenly spread.
