@@ -736,6 +736,43 @@ def run_gpu(args, wl):
     torch.cuda.synchronize()
     brk_ms, brk_launches = lora.lora_profile_end()
 
+    # ---------------- comparison (never the metric): the same forward and backward written as a
+    # composition of torch.matmul calls (cuBLAS, bf16 in, fp32 accumulate), same buffers, same L2 flush
+    composition = None
+    if wl.layers == 1 and not wl.q4 and rank == 0:
+        s = wl.scale
+
+        def torch_step():
+            for e in L.p:
+                x, W, A, B, dy = e["x"], e["W"], e["A"], e["B"], e["dy"]
+                u = x @ A.t()
+                su = u * s
+                e["y"].copy_(x @ W.t() + su @ B.t())
+                sv = (dy @ B) * s
+                e["dx"].copy_(dy @ W + sv @ A)
+                e["dB"].copy_((dy.t() @ su).float())
+                e["dA"].copy_((sv.t() @ x).float())
+
+        for _ in range(3):
+            torch_step()
+        torch.cuda.synchronize()
+        cev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in range(20)]
+        for a, b in cev:
+            flush.zero_()
+            a.record(stream)
+            torch_step()
+            b.record(stream)
+        torch.cuda.synchronize()
+        comp_ms = sum(a.elapsed_time(b) for a, b in cev) / len(cev)
+        composition = {"ms_per_step": comp_ms, "value": wl.T / (comp_ms / 1e3), "unit": UNIT,
+                       "library_speedup": comp_ms / step_ms,
+                       "note": "torch.matmul (cuBLAS) bf16 composition of the same forward and backward over the "
+                               "same device buffers (u = x A^T, y = x W^T + s u B^T, v = dy B, dx = dy W + s v A, "
+                               "dB = s dy^T u, dA = s v^T x), L2 flushed between steps; a comparison, not the "
+                               "measured path"}
+        L.step(lora, stream)  # leave the library's outputs in the buffers
+        torch.cuda.synchronize()
+
     # ---------------- end-to-end: host inputs (pinned) -> device -> step -> gradients back to host
     e2e = None
     if not args.no_e2e:
@@ -879,6 +916,7 @@ def run_gpu(args, wl):
         "clocks": clk,
         "status": lora.lora_strerror(status),
         "e2e": e2e,
+        "cublas_composition": composition,
     }
     if world == 1 and not args.no_cpu_baseline:
         line["cpu_baseline"] = cpu_baseline(wl, budget_s=args.cpu_budget)
