@@ -1266,7 +1266,7 @@ constexpr int kTopkSampleRows = 8192;   // rows per sample contraction
 constexpr int kTopkAppendRows = 4096;   // rows per appending contraction
 
 struct TopkPlan {
-  size_t counters, status, fail_count, cnt, en, s, part, es, zs, tau, cand, fail_rows, total;
+  size_t counters, status, fail_count, big_count, cnt, en, s, part, es, zs, tau, cand, fail_rows, big_rows, total;
   int chunks;                 // materialised chunks (short rows)
   int sblocks, achunks, fmax;  // sampled path: sample blocks, appending chunks, fallback batches at most
   bool sampled;
@@ -1294,17 +1294,19 @@ int topk_check(const lora_bf16* E, int64_t V, int64_t d, int64_t k, TopkPlan* pl
   pl->counters = take((size_t)nctr * 4);
   pl->status = take(4);
   pl->fail_count = take(4);
+  pl->big_count = take(4);
   pl->cnt = take(pl->sampled ? (size_t)V * 4 : 0);
   pl->en = take((size_t)V * d * 2);
   pl->s = take((size_t)std::min<int64_t>(V, kTopkChunk) * pl->lds * 4);
   pl->part = take(kCeSplitFloats * 4);  // short rows: few tiles per chunk
-  pl->es = pl->zs = pl->tau = pl->cand = pl->fail_rows = 0;
+  pl->es = pl->zs = pl->tau = pl->cand = pl->fail_rows = pl->big_rows = 0;
   if (pl->sampled) {
     pl->es = take((size_t)topk_sample() * d * 2);  // later the gathered rows of a fallback batch
     pl->zs = take((size_t)std::min<int64_t>(V, kTopkSampleRows) * topk_sample() * 4);
     pl->tau = take((size_t)V * 4);
     pl->cand = take((size_t)V * topk_cap() * 8);  // every row's list: the transposed side fills later rows
     pl->fail_rows = take((size_t)V * 4);
+    pl->big_rows = take((size_t)V * 4);
   }
   pl->total = off;
   return LORA_OK;
@@ -1703,7 +1705,8 @@ int lora_topk_table(const lora_bf16* E, int64_t V, int64_t d, int64_t k, int32_t
     if ((rc = topk_sym_gemm(dv, ctr + next++, en, d, V, r0, rows, tau, cnt, cand, topk_cap(), st)) != LORA_OK)
       return rc;
   }
-  if (launch_topk_sort(cand, cnt, topk_cap(), (int)k, 0, (int)V, table, fail_rows, fail_count, st) != cudaSuccess)
+  if (launch_topk_sort(cand, cnt, topk_cap(), (int)k, 0, (int)V, table, at<int32_t>(ws, pl.big_rows),
+                       at<int>(ws, pl.big_count), fail_rows, fail_count, dv->num_sms, st) != cudaSuccess)
     return LORA_ECUDA;
   // rows whose threshold left too few or too many candidates: the exact materialised path
   int nf = 0;

@@ -276,9 +276,11 @@ cudaError_t launch_topk_select(const float* S, long long lds, int V, int k, int 
                                int32_t* table, int* status, cudaStream_t stream);
 // Thresholds of nrows rows from their sample similarities Z [nrows, topk_sample()].
 cudaError_t launch_topk_tau(const float* Z, int V, int k, int nrows, float* tau, cudaStream_t stream);
-// Sorts each row's appended candidates into the table, or lists the row for the fallback.
+// Sorts each row's appended candidates into the table (a warp per row, a block for
+// lists over 1024: big_rows / big_count, a zeroed count), or lists the row for the fallback.
 cudaError_t launch_topk_sort(const uint2* cand, int* cnt, int cap, int k, int row0, int nrows, int32_t* table,
-                             int32_t* fail_rows, int* fail_count, cudaStream_t stream);
+                             int32_t* big_rows, int* big_count, int32_t* fail_rows, int* fail_count, int num_sms,
+                             cudaStream_t stream);
 // Es [topk_sample(), d] = the evenly spread sample rows of En [V, d].
 cudaError_t launch_topk_gather_sample(const __nv_bfloat16* En, int V, int d, __nv_bfloat16* Es, int num_sms,
                                       cudaStream_t stream);

@@ -18,6 +18,8 @@
 //                   histograms, then 11, then 10 bits) until the candidates at
 //                   or above the chosen prefix fit in shared memory, then the
 //                   same sort
+#include <algorithm>
+
 #include "common.cuh"
 #include "kernels.h"
 
@@ -139,7 +141,7 @@ __device__ __forceinline__ int cand_index(uint64_t v) { return (int)(0xffffffffu
 template <int kT, int E>
 __device__ void bitonic_sort(uint64_t (&v)[E], uint64_t* x) {
   constexpr int p2 = kT * E;
-  const int tid = threadIdx.x;
+  const int tid = kT == 32 ? (int)(threadIdx.x & 31) : (int)threadIdx.x;  // kT = 32: one warp, no barrier
   // fully unrolled: every stage's exchange form and masks are compile-time constants
 #pragma unroll
   for (int size = 2; size <= p2; size <<= 1) {
@@ -189,10 +191,11 @@ __device__ void bitonic_sort(uint64_t (&v)[E], uint64_t* x) {
 // the first k indices to out; padding sorts below every real candidate.
 template <int kT, int E, typename Get>
 __device__ void sort_write_e(Get get, int n, int k, uint64_t* x, int32_t* __restrict__ out) {
+  const int tid = kT == 32 ? (int)(threadIdx.x & 31) : (int)threadIdx.x;
   uint64_t v[E];
 #pragma unroll
   for (int e = 0; e < E; ++e) {
-    const int p = threadIdx.x + e * kT;
+    const int p = tid + e * kT;
     if (p < n) {
       const uint2 c = get(p);
       v[e] = pack_cand(c.x, (int)c.y);
@@ -200,11 +203,11 @@ __device__ void sort_write_e(Get get, int n, int k, uint64_t* x, int32_t* __rest
       v[e] = 0ull;
     }
   }
-  __syncthreads();  // the candidates may live in the exchange buffer
+  if (kT > 32) __syncthreads();  // the candidates may live in the exchange buffer
   bitonic_sort<kT, E>(v, x);
 #pragma unroll
   for (int e = 0; e < E; ++e) {
-    const int p = threadIdx.x + e * kT;
+    const int p = tid + e * kT;
     if (p < k) out[p] = cand_index(v[e]);
   }
 }
@@ -544,42 +547,67 @@ __global__ void __launch_bounds__(kTauThreads, 4) topk_tau_kernel(const float* _
   }
 }
 
-// One row of a chunk: its cnt[r] candidates (order key, token) appended by the
-// similarity contraction; with k <= n <= cap they hold the exact top k and
-// are sorted into the table (256 threads, 1 to 16 register slots each),
-// otherwise the row joins the fallback list.  The row's count is reset for the
-// next chunk.
+// Each row's cnt[r] candidates (order key, token) appended by the similarity
+// contraction; with k <= n <= cap they hold the exact top k.  One warp per row
+// sorts lists of up to 1024 in registers (32 lanes x up to 32 slots: shuffles
+// below stride 32, in-thread swaps above, no barrier); longer lists go to a
+// list for the block sort below; rows outside [k, cap] join the fallback list.
+constexpr int kWarpSortMax = 1024;
 constexpr int kSortThreads = 256;
 
-__global__ void __launch_bounds__(kSortThreads, 4) topk_sort_kernel(const uint2* __restrict__ cand,
-                                                                   int* __restrict__ cnt, int cap, int k, int row0,
-                                                                   int32_t* __restrict__ table,
-                                                                   int32_t* __restrict__ fail_rows,
-                                                                   int* __restrict__ fail_count) {
+__global__ void __launch_bounds__(kSortThreads, 2) topk_sort_warp_kernel(
+    const uint2* __restrict__ cand, const int* __restrict__ cnt, int cap, int k, int row0, int nrows,
+    int32_t* __restrict__ table, int32_t* __restrict__ big_rows, int* __restrict__ big_count,
+    int32_t* __restrict__ fail_rows, int* __restrict__ fail_count) {
   griddep_wait();
   griddep_launch_dependents();
-  __shared__ uint64_t xs[kCap];
-  const int r = blockIdx.x, tid = threadIdx.x;
+  const int r = blockIdx.x * (kSortThreads / 32) + (int)(threadIdx.x >> 5), lane = threadIdx.x & 31;
+  if (r >= nrows) return;  // whole warps
   const int n = cnt[r];
-  __syncthreads();  // every thread has read the count before it is reset
-  if (tid == 0) cnt[r] = 0;
   if (n < k || n > cap || n > kCap) {
-    if (tid == 0) fail_rows[atomicAdd(fail_count, 1)] = row0 + r;
+    if (lane == 0) fail_rows[atomicAdd(fail_count, 1)] = row0 + r;
+    return;
+  }
+  if (n > kWarpSortMax) {
+    if (lane == 0) big_rows[atomicAdd(big_count, 1)] = r;
     return;
   }
   const uint2* c = cand + (long long)r * cap;
   auto get = [&](int p) { return c[p]; };
   int32_t* out = table + (long long)(row0 + r) * k;
-  if (n <= kSortThreads)
-    sort_write_e<kSortThreads, 1>(get, n, k, xs, out);
-  else if (n <= 2 * kSortThreads)
-    sort_write_e<kSortThreads, 2>(get, n, k, xs, out);
-  else if (n <= 4 * kSortThreads)
-    sort_write_e<kSortThreads, 4>(get, n, k, xs, out);
-  else if (n <= 8 * kSortThreads)
-    sort_write_e<kSortThreads, 8>(get, n, k, xs, out);
+  if (n <= 128)
+    sort_write_e<32, 4>(get, n, k, nullptr, out);
+  else if (n <= 256)
+    sort_write_e<32, 8>(get, n, k, nullptr, out);
+  else if (n <= 512)
+    sort_write_e<32, 16>(get, n, k, nullptr, out);
   else
-    sort_write_e<kSortThreads, 16>(get, n, k, xs, out);
+    sort_write_e<32, 32>(get, n, k, nullptr, out);
+}
+
+// The rows the warp sort listed (more than 1024 candidates): one block of 256
+// threads per row (up to 16 register slots each), rows taken from the list.
+__global__ void __launch_bounds__(kSortThreads, 4) topk_sort_kernel(const uint2* __restrict__ cand,
+                                                                   const int* __restrict__ cnt, int cap, int k,
+                                                                   int row0, const int32_t* __restrict__ big_rows,
+                                                                   const int* __restrict__ big_count,
+                                                                   int32_t* __restrict__ table) {
+  griddep_wait();
+  griddep_launch_dependents();
+  __shared__ uint64_t xs[kCap];
+  const int nbig = *big_count;
+  for (int i = blockIdx.x; i < nbig; i += gridDim.x) {
+    const int r = big_rows[i];
+    const int n = cnt[r];  // kWarpSortMax < n <= kCap
+    const uint2* c = cand + (long long)r * cap;
+    auto get = [&](int p) { return c[p]; };
+    int32_t* out = table + (long long)(row0 + r) * k;
+    if (n <= 8 * kSortThreads)
+      sort_write_e<kSortThreads, 8>(get, n, k, xs, out);
+    else
+      sort_write_e<kSortThreads, 16>(get, n, k, xs, out);
+    __syncthreads();  // the exchange buffer is free for the next row
+  }
 }
 
 // Es[i, :] = En[floor(i * V / kSample), :]: the sample tokens, evenly spread.
@@ -626,9 +654,15 @@ cudaError_t launch_topk_tau(const float* Z, int V, int k, int nrows, float* tau,
 }
 
 cudaError_t launch_topk_sort(const uint2* cand, int* cnt, int cap, int k, int row0, int nrows, int32_t* table,
-                             int32_t* fail_rows, int* fail_count, cudaStream_t st) {
-  return launch_kernel(topk_sort_kernel, dim3(nrows), dim3(kSortThreads), 0, st, 1, cand, cnt, cap, k, row0, table,
-                       fail_rows, fail_count);
+                             int32_t* big_rows, int* big_count, int32_t* fail_rows, int* fail_count, int num_sms,
+                             cudaStream_t st) {
+  const int per = kSortThreads / 32;
+  cudaError_t e = launch_kernel(topk_sort_warp_kernel, dim3((nrows + per - 1) / per), dim3(kSortThreads), 0, st, 1,
+                                cand, (const int*)cnt, cap, k, row0, nrows, table, big_rows, big_count, fail_rows,
+                                fail_count);
+  if (e != cudaSuccess) return e;
+  return launch_kernel(topk_sort_kernel, dim3(std::min(nrows, 4 * num_sms)), dim3(kSortThreads), 0, st, 1, cand,
+                       (const int*)cnt, cap, k, row0, (const int32_t*)big_rows, (const int*)big_count, table);
 }
 
 cudaError_t launch_topk_gather_sample(const __nv_bfloat16* En, int V, int d, __nv_bfloat16* Es, int num_sms,
