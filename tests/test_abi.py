@@ -103,3 +103,35 @@ def test_ce_and_topk_sizes_and_arguments(lib):
     assert t >= 128256 * 3072 * 2 + 512 * 128256 * 4  # normalised rows plus one chunk of similarities
     for V, d, k in ((100, 12, 5), (100, 16, 101), (5000, 16, 1025), (0, 16, 1)):
         assert lib.lora_topk_workspace_size(V, d, k, ctypes.byref(n_bad)) == lora.LORA_EINVAL
+
+
+def test_topk_workspace_switches_to_the_sampled_layout(lib):
+    """Rows of at least 32768 tokens take the sampled selection, whose
+    candidate lists (4096 slots of 8 bytes per row) live in the workspace;
+    shorter rows only need the normalised rows and one 512-row chunk of
+    similarities."""
+    d, k = 256, 100
+    below = lora.lora_topk_workspace_size(32767, d, k)
+    at = lora.lora_topk_workspace_size(32768, d, k)
+    assert below < 32767 * d * 2 + 512 * 32768 * 4 + 400 * 2 ** 20
+    assert at >= 32768 * 4096 * 8 + 32768 * d * 2
+    assert at - below > 32768 * 4096 * 8 - 2 ** 20
+
+
+def test_ce_full_vocabulary_reads_the_embedding_in_place(lib):
+    """Without a top-k table J is the whole vocabulary and E is used where it
+    lies: the workspace carries no gathered copy of it (V x d bf16)."""
+    T, d, V = 256, 1024, 50000
+    full = lora.lora_ce_workspace_size(lora.make_ce_args(T, d, V, 256, 256, 256, 256))
+    reduced = lora.lora_ce_workspace_size(lora.make_ce_args(T, d, V, 256, 256, 256, 256, topk=256, ld_topk=8, k=8))
+    assert reduced - full >= V * d * 2 - 2 ** 16
+
+
+def test_forward_and_backward_plan_their_splits_for_the_contractions_sms(lib):
+    """A forward-and-backward call gives the side stream some SMs, so its
+    contractions plan their splits for fewer CTA pairs than a forward-only
+    call; both still size their own partials (few output tiles split)."""
+    st = lora.make_shape(256, 3072, 8192, 16, 2.0)
+    fwd = lora.lora_workspace_size(st, lora.LORA_FWD)
+    both = lora.lora_workspace_size(st, lora.LORA_FWD_BWD)
+    assert fwd > 0 and both > fwd
