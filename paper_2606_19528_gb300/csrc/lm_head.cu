@@ -5,15 +5,17 @@
 // J and the hidden-state gradient.
 //   vocab_mark      J = union of the trainable targets' first k top-k entries
 //   vocab_count,    J and the trainable positions as ascending lists and
-//   compact, ycol   their inverse maps (128 vocabulary segments counted,
-//                   then compacted in parallel), each trainable target's
-//                   column in J
-//   gather_rows     rows of h (trainable positions) and of E (J) made dense
+//   compact         their inverse maps (128 vocabulary segments counted, then
+//                   compacted in parallel); the last block places each
+//                   trainable target in J
+//   gather_rows(2)  rows of h (trainable positions) and of E (J) made dense
 //   ce_lse          per trainable position: log-sum-exp over J merged from the
-//                   logits contraction's per-group partials, and its loss
+//                   logits contraction's per-group partials, and its loss; the
+//                   last block writes the per-position losses and their sum
+//                   in a fixed order
 //   ce_grad         G = softmax_J - onehot(target) in bf16 for the dh
 //                   contraction, one streaming pass over the logits
-//   ce_finish       per-position losses and their sum, in a fixed order
+//   ce_finish       the losses when no position is trainable
 //   scatter_rows    dh rows of trainable positions, zeros elsewhere
 #include <math.h>
 

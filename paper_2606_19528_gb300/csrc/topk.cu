@@ -2,22 +2,26 @@
 // Approximation", "Choosing the Reduced Vocabulary Set"): token vectors are
 // normalised, C = E~ E~^T holds the cosine similarities, and row i of the
 // table lists the k most similar tokens in descending order (lower index
-// first on ties).  The V x V matrix is never formed: rows are processed in
-// chunks; a tcgen05 contraction (fused_gemm.cu, fp32 output) writes one
-// chunk's similarities, and one CTA per row selects its top k from them.
-//   normalize_rows  E~_i = bf16(E_i / ||E_i||), the sum of squares
-//                   accumulated in fp32 in index order (squares of bf16 are
-//                   exact), correctly rounded sqrt and division
-//   topk_select     rows of at least 32768 tokens: a threshold from an
-//                   8192-value sample of the row, one streaming pass that
-//                   keeps every value at or above it, and a bitonic sort of
-//                   those candidates on (similarity descending, index
-//                   ascending); shorter rows, or a sample that leaves fewer
-//                   than k or more than 4096 candidates: radix select on an
-//                   order-preserving uint32 image of the similarities (11-bit
-//                   histograms, then 11, then 10 bits) until the candidates at
-//                   or above the chosen prefix fit in shared memory, then the
-//                   same sort
+// first on ties).  The V x V matrix is never formed.
+//   normalize_rows      E~_i = bf16(E_i / ||E_i||), the sum of squares
+//                       accumulated in fp32 in index order (squares of bf16
+//                       are exact), correctly rounded sqrt and division
+// Rows shorter than 32768 tokens (the host runs 512-row chunks):
+//   topk_select         per row of a chunk's fp32 similarities (tcgen05
+//                       contraction in fused_gemm.cu): radix select on an
+//                       order-preserving uint32 image (11-bit histograms,
+//                       then 11, then 10 bits) until the candidates at or
+//                       above the chosen prefix fit in shared memory, then a
+//                       sort on (similarity descending, index ascending); it
+//                       also serves the longer rows' fallback
+// Rows of at least 32768 tokens:
+//   topk_gather_sample  8192 evenly spread tokens
+//   topk_tau            each row's threshold from its similarities to them
+//   (fused_gemm.cu)     the upper triangle of C, each value appended to the
+//                       candidate lists of both its rows when it reaches
+//                       their thresholds
+//   topk_sort_warp,     each row's candidates sorted: a warp per list of up
+//   topk_sort           to 1024 in registers, a block for longer lists
 #include <algorithm>
 
 #include "common.cuh"
