@@ -98,6 +98,14 @@ def test_ce_full_vocab_parity():
     assert nJ == 4000
 
 
+def test_ce_table_covering_the_whole_vocabulary():
+    """A top-k table whose rows cover every token makes J the whole
+    vocabulary: E is read in place although a table was given."""
+    case = CeCase(128, 256, 600, k=600, frac=0.5)
+    nT, nJ = check(case)
+    assert nJ == 600
+
+
 def test_ce_logits_masking_identity():
     """Full vocabulary: the logits and losses of a trainable position do not
     depend on which other positions are trainable, so the masked call's

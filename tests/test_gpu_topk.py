@@ -66,10 +66,10 @@ def check_rows(bits, table, k, rows):
 
 
 # V >= 32768 takes the sampled-threshold selection, smaller V the radix path
-@pytest.mark.parametrize("V,d,k", [(5000, 256, 37), (1200, 64, 1024), (20000, 1024, 500), (40000, 64, 300),
-                                   (70000, 128, 1024)],
-                         ids=["V5000_d256_k37", "V1200_d64_k1024", "V20000_d1024_k500", "V40000_d64_k300_sampled",
-                              "V70000_d128_k1024_sampled"])
+@pytest.mark.parametrize("V,d,k", [(5000, 256, 37), (1200, 64, 1024), (20000, 1024, 500), (32767, 64, 64),
+                                   (32768, 64, 64), (40000, 64, 300), (70000, 128, 1024)],
+                         ids=["V5000_d256_k37", "V1200_d64_k1024", "V20000_d1024_k500", "V32767_d64_k64",
+                              "V32768_d64_k64_sampled", "V40000_d64_k300_sampled", "V70000_d128_k1024_sampled"])
 def test_topk_table_parity(V, d, k):
     bits = synth.gen_E(0, 50, V, d)
     table = run_table(bits, k)
