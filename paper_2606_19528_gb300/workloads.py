@@ -143,6 +143,11 @@ def llama_topk_table() -> Workload:
                     topk=500)
 
 
+def topk_table_small() -> Workload:
+    """A 40000-token table at d = 3072, k = 500: the sampled path on a few GB of device memory."""
+    return Workload("topk_table_V40000_k500", 13, 0, 1, 1.0, [], kind="topk", vocab=40000, hidden=3072, topk=500)
+
+
 BY_NAME = {
     "single": single_small,
     "single_B0": lambda: single_small(True),
@@ -154,6 +159,7 @@ BY_NAME = {
     "lm_head_ce": llama_lm_head_ce,
     "lm_head_ce_full": llama_lm_head_ce_full,
     "topk_table": llama_topk_table,
+    "topk_table_small": topk_table_small,
     "llama_layer_q4": llama_layer_T2048_q4,
     "llama_layer_T256": llama_layer_T256,
     "llama_layer_T256_q4": lambda: llama_layer_T256(True),
