@@ -27,7 +27,6 @@ __device__ int g_status;  // first device-side error (kStatusTimeout), 0 if none
 
 constexpr int kMaxDevices = 64;
 constexpr size_t kWsHeader = 256;  // 64 tile counters, one per fused-GEMM launch of a call
-constexpr int kSideSms = 12;        // SMs the backward's rank-r work gets beside the contractions (r <= 32)
 constexpr long long kDefaultWaitNs = 4000000000ll;
 
 struct DeviceInfo {
@@ -759,22 +758,39 @@ bool overlap_enabled() {
   return on;
 }
 
-// The rank-r work grows with the rank while the contractions do not: 12 SMs up
-// to r = 32, 24 up to 64, 28 beyond (measured on the Llama layer at T = 256 ..
-// 4096); LORA_SIDE_SMS overrides.
-int side_sms_setting(int num_sms, int max_rank) {
+// Width of the side stream.  Its rank-r kernels stream x and dy once more
+// (about 2T(2N + K) bytes a projection, HBM- and issue-bound, with more work per
+// byte as r grows) and move adapter-sized data whatever T is (B and its
+// transpose, dA and dB in fp32: ~18 bytes per r(K + N) in effect), while the
+// contractions beside them are compute-bound (4TKN FLOPs, 4-bit weights ~1.3x
+// slower per FLOP); both finish together when
+//   w / (SMs - w) = kSideBalance x sum [2T(2N + K)(1 + r / 144) + 18 r(K + N)] / sum 4TKN q.
+// kSideBalance gives the Llama-3.2-3B layer 12 SMs at r = 16; the same rule
+// gives the measured best widths of the Qwen-2.5-3B layer (16 at r = 16, 20
+// at r = 64, T = 4096) and of the Llama layer at r = 64 (16 at T = 4096, 28
+// at T = 256).  Rounded to an even count so the contractions keep whole CTA
+// pairs; LORA_SIDE_SMS overrides.
+constexpr double kSideBalance = 194.3;
+constexpr double kSideAdapterBytes = 17.9;
+
+int side_sms_setting(int num_sms, const lora_proj* projs, int n) {
   static const int v = [] {
     const char* e = getenv("LORA_SIDE_SMS");
     return e ? atoi(e) : 0;
   }();
-  const int w = v > 0 ? v : (max_rank <= 32 ? kSideSms : max_rank <= 64 ? 24 : 28);
+  int w = v;
+  if (w <= 0) {
+    double bytes = 0.0, flops = 0.0;
+    for (int i = 0; i < n; ++i) {
+      const lora_shape& sh = projs[i].shape;
+      bytes += 2.0 * sh.T * (2.0 * sh.d_out + sh.d_in) * (1.0 + sh.rank / 144.0) +
+               kSideAdapterBytes * sh.rank * (double)(sh.d_in + sh.d_out);
+      flops += 4.0 * sh.T * (double)sh.d_in * sh.d_out * (is_q4(projs[i]) ? 1.3 : 1.0);
+    }
+    const double c = flops > 0.0 ? kSideBalance * bytes / flops : 0.0;
+    w = 2 * (int)std::lround(num_sms * c / (1.0 + c) / 2.0);
+  }
   return std::max(2, std::min(num_sms / 4, w));
-}
-
-int max_rank_of(const lora_proj* projs, int n) {
-  int r = 0;
-  for (int i = 0; i < n; ++i) r = std::max(r, (int)projs[i].shape.rank);
-  return r;
 }
 
 struct SideCtx {
@@ -800,7 +816,7 @@ struct Overlap {
   int side_ctas = 0;
   cudaStream_t main = nullptr, side = nullptr;
   cudaEvent_t ev_fork = nullptr, ev_sv = nullptr, ev_done = nullptr;
-  int init(const DeviceInfo* d, cudaStream_t st, int max_rank) {
+  int init(const DeviceInfo* d, cudaStream_t st, const lora_proj* projs, int n) {
     if (!overlap_enabled()) return LORA_OK;
     SideCtx& c = t_side.dev[d - g_dev];
     if (!c.side && cudaStreamCreateWithFlags(&c.side, cudaStreamNonBlocking) != cudaSuccess) return LORA_ECUDA;
@@ -811,7 +827,7 @@ struct Overlap {
     ev_fork = c.ev[0];
     ev_sv = c.ev[1];
     ev_done = c.ev[2];
-    side_ctas = side_sms_setting(d->num_sms, max_rank);
+    side_ctas = side_sms_setting(d->num_sms, projs, n);
     on = true;
     return LORA_OK;
   }
@@ -846,7 +862,7 @@ int run_step(const lora_proj* projs, int n, int mode, void* ws, const Plan& pl, 
   // forward and backward in one call: the backward's rank-r work runs on a side
   // stream with a few SMs while the contractions use the rest
   Overlap ov;
-  if (mode == LORA_FWD_BWD && (rc = ov.init(d, st, max_rank_of(projs, n))) != LORA_OK) return rc;
+  if (mode == LORA_FWD_BWD && (rc = ov.init(d, st, projs, n)) != LORA_OK) return rc;
   const int gemm_sms = ov.on ? d->num_sms - ov.side_ctas : d->num_sms;
   // backward rank-r work: B^T, su^T, sv (and sv^T), then dB and dA; on `rs`
   // with `ctas` persistent CTAs; the operands of the dx contraction go to bops
@@ -1031,7 +1047,7 @@ int plan_all(const lora_proj* projs, int n, int mode, Plan* pl, bool allow_split
   pl->split_b.assign(n, 1);
   // a forward-and-backward call leaves the side stream's SMs out of the contractions
   const int pairs = mode == LORA_FWD_BWD && overlap_enabled()
-                        ? (kPlanSms - side_sms_setting(kPlanSms, max_rank_of(projs, n))) / 2
+                        ? (kPlanSms - side_sms_setting(kPlanSms, projs, n)) / 2
                         : kPlanPairs;
   std::vector<size_t> split_need(n, 0);
   for (int dir = 0; dir < 2; ++dir) {
