@@ -292,6 +292,42 @@ def barrier(dist, device=None):
             dist.barrier()
 
 
+KERNEL_PASS_NOTE = ("launch durations from CUDA events around each launch of this kernel over a second pass of "
+                    "the same K steps, run right after the timed region; the timed region itself records "
+                    "events around whole steps only, because an event between two launches stops "
+                    "programmatic dependent launch there")
+
+
+def timed_passes(torch, lora, step, K, stream, flush=None, kinds=(0, 1)):
+    """The timed region, then the kernel pass.
+
+    Timed region: K steps with events around each step only (L2 flushed
+    between steps when `flush` is given).  Kernel pass: the same K steps
+    with the library's events around every launch of `kinds`.  Returns
+    (per-step ms of the timed region, {kind: device ms per step} of the
+    kernel pass, library launches inside the timed region)."""
+    ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in range(K)]
+    torch.cuda.synchronize()
+    launches0 = lora.lora_launch_count()
+    for i in range(K):
+        if flush is not None:
+            flush.zero_()
+        ev[i][0].record(stream)
+        step()
+        ev[i][1].record(stream)
+    torch.cuda.synchronize()
+    launches = lora.lora_launch_count() - launches0
+    step_ms = [a.elapsed_time(b) for a, b in ev]
+    lora.lora_profile_begin(kinds)
+    for _ in range(K):
+        if flush is not None:
+            flush.zero_()
+        step()
+    torch.cuda.synchronize()
+    kern_ms, _ = lora.lora_profile_end()
+    return step_ms, {k: v / K for k, v in kern_ms.items()}, launches
+
+
 # ----------------------------------------------------------------------------- GPU arm
 
 class LayerOnDevice:
@@ -459,26 +495,17 @@ def run_gpu_ce(args, wl):
     gpu_id = str(getattr(props, "uuid", local))
     if gpu_id and not gpu_id.startswith("GPU-") and len(gpu_id) == 36:
         gpu_id = "GPU-" + gpu_id
-    ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in range(K)]
     clocks = ClockSampler(gpu_id) if rank == 0 else None
     barrier(dist, device)
     torch.cuda.synchronize()
     if clocks:
         clocks.start()
         time.sleep(0.3)
-    launches0 = lora.lora_launch_count()
-    lora.lora_profile_begin((lora.LORA_KERNEL_GEMM_FWD, lora.LORA_KERNEL_GEMM_BWD))
-    for i in range(K):
-        flush.zero_()
-        ev[i][0].record(stream)
-        step()
-        ev[i][1].record(stream)
-    torch.cuda.synchronize()
-    kern_ms, _ = lora.lora_profile_end()
-    launches = lora.lora_launch_count() - launches0
+    steps_ms, kern_ms, launches = timed_passes(torch, lora, step, K, stream, flush,
+                                               (lora.LORA_KERNEL_GEMM_FWD, lora.LORA_KERNEL_GEMM_BWD))
     barrier(dist, device)
     clk = clocks.stop() if clocks else None
-    step_ms = max_over_ranks(dist, sum(a.elapsed_time(b) for a, b in ev) / K, device)
+    step_ms = max_over_ranks(dist, sum(steps_ms) / K, device)
 
     # end to end: h, targets and mask from pinned host memory, loss back, every step
     h_h = torch.from_numpy(np.ascontiguousarray(h).view(np.int16)).pin_memory()
@@ -501,7 +528,7 @@ def run_gpu_ce(args, wl):
         if dist is not None:
             dist.destroy_process_group()
         return 0
-    gemm_ms = (kern_ms["gemm_fwd"] + kern_ms["gemm_bwd"]) / K
+    gemm_ms = kern_ms["gemm_fwd"] + kern_ms["gemm_bwd"]
     flops = 4.0 * nT * nJ * wl.hidden  # logits and dh contractions
     sustained = peaks.get("bf16_tflops_sustained", FALLBACK_PEAKS["bf16_tflops_sustained"])
     burst = peaks.get("bf16_tflops", FALLBACK_PEAKS["bf16_tflops"])
@@ -520,7 +547,8 @@ def run_gpu_ce(args, wl):
                      "achieved": gemm_tf, "peak": sustained, "unit": "TFLOP/s",
                      "frac": gemm_tf / sustained if gemm_tf else None, "traffic": None,
                      "peak_kind": f"bf16 sustained, of {peaks_src}", "frac_of_burst": gemm_tf / burst if gemm_tf else None,
-                     "flops_per_step": flops, "ms_per_step": gemm_ms},
+                     "flops_per_step": flops, "ms_per_step": gemm_ms,
+                     "timing": KERNEL_PASS_NOTE},
         "gpu_launches": launches,
         "clocks": clk,
         "status": lora.lora_strerror(lora.lora_read_status()),
@@ -589,19 +617,10 @@ def run_gpu_topk(args, wl):
     clocks = ClockSampler(gpu_id)
     clocks.start()
     time.sleep(0.3)
-    ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in range(K)]
-    launches0 = lora.lora_launch_count()
-    lora.lora_profile_begin((lora.LORA_KERNEL_GEMM_FWD,))
-    for i in range(K):
-        ev[i][0].record(stream)
-        step()
-        ev[i][1].record(stream)
-    torch.cuda.synchronize()
-    kern_ms, _ = lora.lora_profile_end()
-    launches = lora.lora_launch_count() - launches0
+    steps_ms, kern_ms, launches = timed_passes(torch, lora, step, K, stream, None, (lora.LORA_KERNEL_GEMM_FWD,))
     clk = clocks.stop()
-    step_ms = sum(a.elapsed_time(b) for a, b in ev) / K
-    gemm_ms = kern_ms["gemm_fwd"] / K
+    step_ms = sum(steps_ms) / K
+    gemm_ms = kern_ms["gemm_fwd"]
     flops = 2.0 * V * V * d
     if V >= 32768:
         # the contractions performed: each row against 8192 sample tokens (thresholds), and the upper
@@ -626,7 +645,8 @@ def run_gpu_topk(args, wl):
         "roofline": {"kernel": "fused_lora_gemm (sample and similarity contractions)", "bound": "tensor",
                      "achieved": gemm_tf, "peak": sustained, "unit": "TFLOP/s", "frac": gemm_tf / sustained,
                      "traffic": None, "peak_kind": f"bf16 sustained, of {peaks_src}",
-                     "frac_of_burst": gemm_tf / burst, "flops_per_step": done_flops, "ms_per_step": gemm_ms},
+                     "frac_of_burst": gemm_tf / burst, "flops_per_step": done_flops, "ms_per_step": gemm_ms,
+                     "timing": KERNEL_PASS_NOTE},
         "gpu_launches": launches, "clocks": clk, "status": lora.lora_strerror(lora.lora_read_status()),
         "e2e": None,
     }
@@ -701,30 +721,20 @@ def run_gpu(args, wl):
     if gpu_id and not gpu_id.startswith("GPU-") and len(gpu_id) == 36:
         gpu_id = "GPU-" + gpu_id
 
-    # ---------------- timed region: device-resident inputs, L2 flushed between steps
-    ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in range(K)]
+    # ---------------- timed region: device-resident inputs, L2 flushed between steps;
+    # then the kernel pass (events around the fused-GEMM launches)
     clocks = ClockSampler(gpu_id) if rank == 0 else None
     barrier(dist, device)
     torch.cuda.synchronize()
     if clocks:
         clocks.start()
         time.sleep(0.3)
-    launches0 = lora.lora_launch_count()
-    # only the fused-GEMM launches are bracketed with events here, so that the
-    # other launches follow one another with programmatic dependent launch
-    lora.lora_profile_begin((lora.LORA_KERNEL_GEMM_FWD, lora.LORA_KERNEL_GEMM_BWD))
-    for i in range(K):
-        flush.zero_()
-        ev[i][0].record(stream)
-        L.step(lora, stream)
-        ev[i][1].record(stream)
-    torch.cuda.synchronize()
-    kern_ms, kern_launches = lora.lora_profile_end()
-    launches = lora.lora_launch_count() - launches0
+    steps_ms, kern_ms, launches = timed_passes(torch, lora, lambda: L.step(lora, stream), K, stream, flush,
+                                               (lora.LORA_KERNEL_GEMM_FWD, lora.LORA_KERNEL_GEMM_BWD))
     barrier(dist, device)
     clk = clocks.stop() if clocks else None
     status = lora.lora_read_status()
-    step_ms_local = sum(a.elapsed_time(b) for a, b in ev) / K
+    step_ms_local = sum(steps_ms) / K
     step_ms = max_over_ranks(dist, step_ms_local, device)
 
     # ---------------- per-kind breakdown: a separate pass with events around every launch group
@@ -880,7 +890,7 @@ def run_gpu(args, wl):
     flops = wl.flops()
     tflops = flops / (step_ms / 1e3) / 1e12
     f_fwd, f_bwd = gemm_flops(wl)
-    gemm_ms = (kern_ms["gemm_fwd"] + kern_ms["gemm_bwd"]) / K
+    gemm_ms = kern_ms["gemm_fwd"] + kern_ms["gemm_bwd"]
     gemm_tflops = (f_fwd + f_bwd) / (gemm_ms / 1e3) / 1e12
     sustained = peaks.get("bf16_tflops_sustained", FALLBACK_PEAKS["bf16_tflops_sustained"])
     burst = peaks.get("bf16_tflops", FALLBACK_PEAKS["bf16_tflops"])
@@ -910,7 +920,8 @@ def run_gpu(args, wl):
                      "traffic_unit": "bytes per step (forward + backward launch), ncu dram__bytes_read+write",
                      "peak_kind": f"bf16 sustained, of {peaks_src}",
                      "frac_of_burst": gemm_tflops / burst,
-                     "flops_per_step": f_fwd + f_bwd, "ms_per_step": gemm_ms},
+                     "flops_per_step": f_fwd + f_bwd, "ms_per_step": gemm_ms,
+                     "timing": KERNEL_PASS_NOTE},
         "kernels": per_kernel,
         "gpu_launches": launches,
         "clocks": clk,
