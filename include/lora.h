@@ -276,8 +276,9 @@ int lora_set_wait_limit_ns(int64_t ns);
 enum {
   LORA_KERNEL_GEMM_FWD = 0, /* fused [x | su] . [W | B]^T contraction */
   LORA_KERNEL_GEMM_BWD = 1, /* fused [dy | sv] . [W ; A] contraction */
-  LORA_KERNEL_ROWPROJ = 2,  /* su = s x A^T, sv = s dy B (with their split reductions) */
-  LORA_KERNEL_COLPROJ = 3,  /* dB = dy^T su, dA = sv^T x (with their split reductions) */
+  LORA_KERNEL_ROWPROJ = 2,  /* su = s x A^T; the pass over dy: sv = s dy B, and dB = dy^T su where fused
+                               (r <= 16); with their partial sums */
+  LORA_KERNEL_COLPROJ = 3,  /* dA = sv^T x, and dB = dy^T su where not fused; with their partial sums */
   LORA_KERNEL_PAD = 4,      /* zero-padded copies for ranks that are not multiples of 8 */
   LORA_KERNEL_KINDS = 5
 };

@@ -642,6 +642,187 @@ int launch_cols(const std::vector<ColSpec>& specs, const Arena& ar, const Device
   return LORA_OK;
 }
 
+// ------------------------------------------------------------------ fused pass over dy
+// sv = s dy B and dB = dy^T su of one projection in one read of dy.
+struct DySpec {
+  const bf* dy;
+  int T, N, r;
+  float scale;
+  const bf* bt;   // B^T [pad8(r), N]
+  const bf* sut;  // su^T [pad8(r), T]
+  bf* sv;         // [T, pad8(r)]
+  bf* svT;        // [pad8(r), T]
+  float* dB;      // [N, r]
+};
+
+struct DyCut {
+  int tt, groups, bpu, pieces;
+};
+
+constexpr int kDyTile = 128;  // tokens per tile and columns per block of the fused pass
+
+size_t dy_sv_floats(int T, int rpad, int pieces) { return pieces > 1 ? (size_t)pieces * T * rpad : 0; }
+size_t dy_db_floats(int N, int rpad, int groups) { return groups > 1 ? (size_t)groups * N * rpad : 0; }
+
+// Token groups TMEM forces on a projection: each holds at most tiles_max tiles.
+int dy_need_groups(int T, int tiles_max) { return cdiv(cdiv(T, kDyTile), tiles_max); }
+
+// A projection takes the fused pass up to r = 16: beyond, the B^T and su^T
+// boxes every stage carries (4 x 64 x r bf16 beside 32 KB of dy) make the one
+// issuing thread's copies the limit, and the two separate passes are faster
+// (Llama-3.2-3B layer, T = 2048, r = 32: 773 against 569 us; Qwen-2.5-3B
+// layer, T = 4096, r = 64: 1254 against 944 us).  It also needs the partials
+// of its fewest token groups to stay within a quarter of its dy bytes.
+bool dy_fusable(int T, int N, int r) {
+  const int rpad = rank_pad16(r);
+  return rpad <= 16 && dy_db_floats(N, rpad, dy_need_groups(T, dy_tiles_max(rpad))) * 4 <= (size_t)T * N * 2 / 4;
+}
+
+// The cut of a projection for (gmul, pmul): gmul x the necessary token groups
+// and pmul column pieces, trimmed (pieces first) until the partials fit within
+// those of the necessary groups plus an eighth of the projection's dy bytes.
+DyCut dy_cut(int T, int N, int rpad, int tiles_max, int gmul, int pmul) {
+  const int tiles = cdiv(T, kDyTile), blocks = cdiv(N, kDyTile);
+  const int need = dy_need_groups(T, tiles_max);
+  int groups = std::min(tiles, std::min(need * gmul, std::max(need, kDyMaxCut)));
+  int pieces = std::min(blocks, std::min(pmul, kDyMaxCut));
+  const size_t cap = dy_db_floats(N, rpad, need) + (size_t)T * N / 16;
+  while (pieces > 1 && dy_sv_floats(T, rpad, pieces) + dy_db_floats(N, rpad, groups) > cap) --pieces;
+  while (groups > need && dy_sv_floats(T, rpad, pieces) + dy_db_floats(N, rpad, groups) > cap) --groups;
+  DyCut c;
+  c.tt = cdiv(tiles, groups);
+  c.groups = cdiv(tiles, c.tt);
+  c.bpu = cdiv(blocks, pieces);
+  c.pieces = cdiv(blocks, c.bpu);
+  return c;
+}
+
+size_t dy_cut_floats(const DySpec& s, const DyCut& c) {
+  const int rpad = rank_pad16(s.r);
+  return dy_sv_floats(s.T, rpad, c.pieces) + dy_db_floats(s.N, rpad, c.groups);
+}
+
+// Cost of a batch's cuts on `ctas` persistent CTAs, in stage times (one
+// 128 x 128 tile of dy): the units go round-robin in unit order, each costs its
+// stages plus a fixed fill and its read-outs; partials add their traffic and
+// the reduce launch.
+double dy_cost(const std::vector<DySpec>& specs, size_t i0, size_t i1, const std::vector<DyCut>& cuts, int ctas) {
+  std::vector<double> load(ctas, 0.0);
+  long long u = 0;
+  double part = 0.0;
+  for (size_t i = i0; i < i1; ++i) {
+    const DySpec& s = specs[i];
+    const DyCut& c = cuts[i - i0];
+    const int tiles = cdiv(s.T, kDyTile), blocks = cdiv(s.N, kDyTile), rpad = rank_pad16(s.r);
+    for (int g = 0; g < c.groups; ++g) {
+      const int nt = std::min(tiles, (g + 1) * c.tt) - g * c.tt;
+      for (int q = 0; q < c.pieces; ++q, ++u) {
+        const int nb = std::min(blocks, (q + 1) * c.bpu) - q * c.bpu;
+        load[u % ctas] += nb * nt + 2.0 + nt * rpad / 64.0 + nb * rpad / 64.0;
+      }
+    }
+    part += (double)dy_cut_floats(s, c);
+  }
+  const double make = *std::max_element(load.begin(), load.end());
+  return part > 0 ? make + 4.0 + part * 8.0 / 32768.0 / ctas : make;
+}
+
+// The cuts of a batch (rank class of its largest rank) that cost least on `ctas` CTAs.
+std::vector<DyCut> dy_choose(const std::vector<DySpec>& specs, size_t i0, size_t i1, int ctas) {
+  int rmax = 16;
+  for (size_t i = i0; i < i1; ++i) rmax = std::max(rmax, rank_pad16(specs[i].r));
+  const int tmax = dy_tiles_max(rmax);
+  std::vector<DyCut> best, cur(i1 - i0);
+  double best_cost = 0.0;
+  for (int gmul : {1, 2, 4, 8})
+    for (int pmul : {1, 2, 4, 8}) {
+      for (size_t i = i0; i < i1; ++i) cur[i - i0] = dy_cut(specs[i].T, specs[i].N, rank_pad16(specs[i].r), tmax, gmul, pmul);
+      const double c = dy_cost(specs, i0, i1, cur, ctas);
+      if (best.empty() || c < best_cost - 1e-9) {
+        best = cur;
+        best_cost = c;
+      }
+    }
+  return best;
+}
+
+// Partial floats a batch may need whatever the CTA count (the largest over every candidate cut).
+size_t dy_worst_floats(const std::vector<DySpec>& specs, size_t i0, size_t i1) {
+  int rmax = 16;
+  for (size_t i = i0; i < i1; ++i) rmax = std::max(rmax, rank_pad16(specs[i].r));
+  const int tmax = dy_tiles_max(rmax);
+  size_t worst = 0;
+  for (int gmul : {1, 2, 4, 8})
+    for (int pmul : {1, 2, 4, 8}) {
+      size_t f = 0;
+      for (size_t i = i0; i < i1; ++i)
+        f += dy_cut_floats(specs[i], dy_cut(specs[i].T, specs[i].N, rank_pad16(specs[i].r), tmax, gmul, pmul));
+      worst = std::max(worst, f);
+    }
+  return worst;
+}
+
+size_t dy_plan_floats(const std::vector<DySpec>& specs) {
+  size_t f = 0;
+  for (size_t i0 = 0; i0 < specs.size(); i0 += kMaxRankProblems)
+    f += dy_worst_floats(specs, i0, std::min(specs.size(), i0 + kMaxRankProblems));
+  return f;
+}
+
+// The fused passes over dy on `ctas` persistent CTAs (one per SM), then their reduce.
+int launch_dy_pass(const std::vector<DySpec>& specs, const Arena& ar, const DeviceInfo* d, int ctas, cudaStream_t st) {
+  size_t pf = 0;
+  int rc;
+  for (size_t i0 = 0; i0 < specs.size(); i0 += kMaxRankProblems) {
+    const size_t i1 = std::min(specs.size(), i0 + kMaxRankProblems);
+    const std::vector<DyCut> cuts = dy_choose(specs, i0, i1, ctas);
+    DyBatch b;
+    memset(&b, 0, sizeof(b));
+    for (size_t i = i0; i < i1; ++i) {
+      const DySpec& s = specs[i];
+      const DyCut& c = cuts[i - i0];
+      DyProb& p = b.p[b.n++];
+      const int r8 = rank_pad8(s.r);
+      if ((rc = make_map(&p.tmDy, s.dy, s.N, s.T, s.N, 64, kDyTile)) != LORA_OK) return rc;
+      if ((rc = make_map(&p.tmBt, s.bt, s.N, s.r, s.N, 64, r8)) != LORA_OK) return rc;
+      if ((rc = make_map(&p.tmSuT, s.sut, s.T, s.r, s.T, 64, r8)) != LORA_OK) return rc;
+      p.T = s.T;
+      p.N = s.N;
+      p.r = s.r;
+      p.rpad = rank_pad16(s.r);
+      p.scale = s.scale;
+      p.sv = s.sv;
+      p.ld_sv = r8;
+      p.svT = s.svT;
+      p.dB = s.dB;
+      p.tiles = cdiv(s.T, kDyTile);
+      p.tt = c.tt;
+      p.groups = c.groups;
+      p.blocks = cdiv(s.N, kDyTile);
+      p.bpu = c.bpu;
+      p.pieces = c.pieces;
+      p.unit_begin = b.units;
+      b.units += c.groups * c.pieces;
+      if (c.pieces > 1) {
+        p.sv_part = (long long)pf;
+        pf += dy_sv_floats(s.T, p.rpad, c.pieces);
+        b.red_sv += s.T * r8;
+      }
+      if (c.groups > 1) {
+        p.db_part = (long long)pf;
+        pf += dy_db_floats(s.N, p.rpad, c.groups);
+        b.red_db += s.N * s.r;
+      }
+    }
+    if (pf > ar.n_partials) return LORA_EWORKSPACE;  // planning bound violated
+    b.partials = ar.partials;
+    b.status = d->status;
+    b.limit_ns = g_wait_limit_ns;
+    if (launch_dy(b, ctas, st) != cudaSuccess) return LORA_ECUDA;
+  }
+  return LORA_OK;
+}
+
 Arena arena(void* ws, const Plan& pl, int phase) {
   return Arena{at<float>(ws, pl.part_off[phase]), pl.n_partials[phase]};
 }
@@ -758,39 +939,67 @@ bool overlap_enabled() {
   return on;
 }
 
-// Width of the side stream.  Its rank-r kernels stream x and dy once more
-// (about 2T(2N + K) bytes a projection, HBM- and issue-bound, with more work per
-// byte as r grows) and move adapter-sized data whatever T is (B and its
-// transpose, dA and dB in fp32: ~18 bytes per r(K + N) in effect), while the
-// contractions beside them are compute-bound (4TKN FLOPs, 4-bit weights ~1.3x
-// slower per FLOP); both finish together when
-//   w / (SMs - w) = kSideBalance x sum [2T(2N + K)(1 + r / 144) + 18 r(K + N)] / sum 4TKN q.
-// kSideBalance gives the Llama-3.2-3B layer 12 SMs at r = 16; the same rule
-// gives the measured best widths of the Qwen-2.5-3B layer (16 at r = 16, 20
-// at r = 64, T = 4096) and of the Llama layer at r = 64 (16 at T = 4096, 28
-// at T = 256).  Rounded to an even count so the contractions keep whole CTA
-// pairs; LORA_SIDE_SMS overrides.
-constexpr double kSideBalance = 194.3;
-constexpr double kSideAdapterBytes = 17.9;
+// Widths of the side stream in its two phases.  Beside the forward
+// contraction (2TKN FLOPs per projection, compute-bound, 4-bit weights ~1.3x
+// slower per FLOP) it transposes B and su and reads dy once: the fused pass
+// (sv and dB, r <= 16) or the sv pass; the dx contraction waits for sv.
+// Beside the dx contraction it runs dA = sv^T x (2TK bytes per distinct x) and,
+// where the pass over dy was not fused, dB (dy read again, 0.6 x as costly
+// per byte).  The rank-r kernels are issue-bound, costlier per byte as r
+// grows.  Each phase gets the share of SMs that ends it with the contraction
+// beside it:
+//   w / (SMs - w) = kappa x side bytes of the phase / contraction FLOPs,
+// side bytes = 2T(...)(1 + r / 144) + an adapter-sized term (transposes,
+// partial sums, fp32 gradients).  kappa1 gives the Llama-3.2-3B layer at
+// r = 16 12 SMs, kappa2 8 SMs, the measured best pair at T = 2048; the same
+// constants give 16 / 8 for the Qwen-2.5-3B layer at r = 16 (best measured
+// 16-18 / 8) and 22 / 20 at r = 64 (best 16-20 / 20-24).  Rounded to even
+// counts so the contractions keep whole CTA pairs; LORA_SIDE_SMS and
+// LORA_SIDE_SMS2 override.
+constexpr double kSideKappa1 = 290.0;
+constexpr double kSideKappa2 = 245.0;
+constexpr double kSideAdapter1 = 12.0;  // bytes per r N
+constexpr double kSideAdapter2 = 8.0;   // bytes per r K
+constexpr double kSideSecondPass = 0.6;  // the unfused dB pass over dy: its kernel streams faster per byte
 
-int side_sms_setting(int num_sms, const lora_proj* projs, int n) {
-  static const int v = [] {
-    const char* e = getenv("LORA_SIDE_SMS");
-    return e ? atoi(e) : 0;
-  }();
-  int w = v;
-  if (w <= 0) {
-    double bytes = 0.0, flops = 0.0;
-    for (int i = 0; i < n; ++i) {
-      const lora_shape& sh = projs[i].shape;
-      bytes += 2.0 * sh.T * (2.0 * sh.d_out + sh.d_in) * (1.0 + sh.rank / 144.0) +
-               kSideAdapterBytes * sh.rank * (double)(sh.d_in + sh.d_out);
-      flops += 4.0 * sh.T * (double)sh.d_in * sh.d_out * (is_q4(projs[i]) ? 1.3 : 1.0);
+struct SideWidths {
+  int w1 = 0, w2 = 0;
+};
+
+int env_int(const char* name) {
+  const char* e = getenv(name);
+  return e ? atoi(e) : 0;
+}
+
+bool dy_fusable(int T, int N, int r);
+
+SideWidths side_widths(int num_sms, const lora_proj* projs, int n) {
+  static const int v1 = env_int("LORA_SIDE_SMS"), v2 = env_int("LORA_SIDE_SMS2");
+  double b1 = 0.0, b2 = 0.0, flops = 0.0;
+  std::vector<const void*> xs;
+  for (int i = 0; i < n; ++i) {
+    const lora_shape& sh = projs[i].shape;
+    const double T = (double)sh.T, K = (double)sh.d_in, N = (double)sh.d_out, r = (double)sh.rank;
+    const double fr = 1.0 + r / 144.0;
+    b1 += 2.0 * T * N * fr + kSideAdapter1 * r * N;
+    b2 += kSideAdapter2 * r * K;
+    if (!dy_fusable((int)sh.T, (int)sh.d_out, (int)sh.rank)) b2 += kSideSecondPass * 2.0 * T * N * fr;
+    // dA reads each distinct x once (shapes without pointers: once per projection)
+    const void* x = projs[i].x;
+    if (x == nullptr || std::find(xs.begin(), xs.end(), x) == xs.end()) {
+      b2 += 2.0 * T * K * fr;
+      if (x != nullptr) xs.push_back(x);
     }
-    const double c = flops > 0.0 ? kSideBalance * bytes / flops : 0.0;
-    w = 2 * (int)std::lround(num_sms * c / (1.0 + c) / 2.0);
+    flops += 2.0 * T * K * N * (is_q4(projs[i]) ? 1.3 : 1.0);
   }
-  return std::max(2, std::min(num_sms / 4, w));
+  auto width = [&](double kappa, double bytes) {
+    const double c = flops > 0.0 ? kappa * bytes / flops : 0.0;
+    return 2 * (int)std::lround(num_sms * c / (1.0 + c) / 2.0);
+  };
+  SideWidths w;
+  w.w1 = std::max(2, std::min(num_sms / 4, v1 > 0 ? v1 : width(kSideKappa1, b1)));
+  w.w2 = std::max(2, std::min(num_sms / 4, v2 > 0 ? v2 : width(kSideKappa2, b2)));
+  return w;
 }
 
 struct SideCtx {
@@ -813,7 +1022,8 @@ thread_local ThreadSide t_side;
 
 struct Overlap {
   bool on = false, forked = false, joined = false;
-  int side_ctas = 0;
+  int side_ctas = 0;   // beside the forward contraction
+  int side_ctas2 = 0;  // beside the dx contraction
   cudaStream_t main = nullptr, side = nullptr;
   cudaEvent_t ev_fork = nullptr, ev_sv = nullptr, ev_done = nullptr;
   int init(const DeviceInfo* d, cudaStream_t st, const lora_proj* projs, int n) {
@@ -827,7 +1037,9 @@ struct Overlap {
     ev_fork = c.ev[0];
     ev_sv = c.ev[1];
     ev_done = c.ev[2];
-    side_ctas = side_sms_setting(d->num_sms, projs, n);
+    const SideWidths w = side_widths(d->num_sms, projs, n);
+    side_ctas = w.w1;
+    side_ctas2 = w.w2;
     on = true;
     return LORA_OK;
   }
@@ -863,15 +1075,22 @@ int run_step(const lora_proj* projs, int n, int mode, void* ws, const Plan& pl, 
   // stream with a few SMs while the contractions use the rest
   Overlap ov;
   if (mode == LORA_FWD_BWD && (rc = ov.init(d, st, projs, n)) != LORA_OK) return rc;
-  const int gemm_sms = ov.on ? d->num_sms - ov.side_ctas : d->num_sms;
+  const int gemm_sms = ov.on ? d->num_sms - ov.side_ctas : d->num_sms;      // forward contraction
+  const int gemm_sms_b = ov.on ? d->num_sms - ov.side_ctas2 : d->num_sms;  // dx contraction
   // backward rank-r work: B^T, su^T, sv (and sv^T), then dB and dA; on `rs`
   // with `ctas` persistent CTAs; the operands of the dx contraction go to bops
   std::vector<Operands> bops(n);
-  auto bwd_rank = [&](cudaStream_t rs, int ctas) -> int {
+  // ctas: CTAs of the transposes and the passes over dy; ctas2: of dA (and the
+  // second pass over dy where it is not fused)
+  auto bwd_rank = [&](cudaStream_t rs, int ctas, int ctas2) -> int {
     int rc;
     std::vector<RowSpec> rows;
     std::vector<ColSpec> cols;
+    std::vector<DySpec> dys;
     std::vector<bf*> sut(n), svt(n);
+    std::vector<char> fused(n);
+    for (int i = 0; i < n; ++i)
+      fused[i] = dy_fusable((int)projs[i].shape.T, (int)projs[i].shape.d_out, (int)projs[i].shape.rank);
     std::vector<Operands>& ops = bops;
     TransposeJobs tj;
     memset(&tj, 0, sizeof(tj));
@@ -903,18 +1122,24 @@ int run_step(const lora_proj* projs, int n, int mode, void* ws, const Plan& pl, 
         if ((rc = transpose(cb(p.B), N, r, bt)) != LORA_OK) return rc;
         if ((rc = transpose(cb(p.su), T, r, sut[i])) != LORA_OK) return rc;
         bf* sv = at<bf>(W_(i), plans[i].sv);
-        add_row_block(rows, cb(p.dy), N, T, N, p.shape.scale, bt, N, r, sv, r8, nullptr, 0, svt[i], false);
+        if (fused[i])
+          dys.push_back(DySpec{cb(p.dy), T, N, r, p.shape.scale, bt, sut[i], sv, svt[i], p.dB});
+        else
+          add_row_block(rows, cb(p.dy), N, T, N, p.shape.scale, bt, N, r, sv, r8, nullptr, 0, svt[i], false);
         ops[i].s_in = sv;
         ops[i].ld_s = r8;
       }
       if (launch_transposes(tj, rs) != cudaSuccess) return LORA_ECUDA;
     }
     {
+      // sv (and dB where fused) before the event the dx contraction waits for
       ProfScope ps(LORA_KERNEL_ROWPROJ, rs);
+      if ((rc = launch_dy_pass(dys, arena(ws, pl, kPhBwdRows), d, ctas, rs)) != LORA_OK) return rc;
       if ((rc = launch_rows(rows, arena(ws, pl, kPhBwdRows), d, ctas, rs)) != LORA_OK) return rc;
     }
     if (ov.on && cudaEventRecord(ov.ev_sv, rs) != cudaSuccess) return LORA_ECUDA;
     for (int i = 0; i < n; ++i) {
+      if (fused[i]) continue;
       const lora_proj& p = projs[i];
       const int T = (int)p.shape.T, N = (int)p.shape.d_out, r = (int)p.shape.rank;
       add_col_block(cols, cb(p.dy), N, T, N, sut[i], T, r, p.dB, 1, false);
@@ -926,7 +1151,7 @@ int run_step(const lora_proj* projs, int n, int mode, void* ws, const Plan& pl, 
     }
     {
       ProfScope ps(LORA_KERNEL_COLPROJ, rs);
-      if ((rc = launch_cols(cols, arena(ws, pl, kPhBwdCols), d, ctas, rs)) != LORA_OK) return rc;
+      if ((rc = launch_cols(cols, arena(ws, pl, kPhBwdCols), d, ctas2, rs)) != LORA_OK) return rc;
     }
     return LORA_OK;
   };
@@ -964,7 +1189,7 @@ int run_step(const lora_proj* projs, int n, int mode, void* ws, const Plan& pl, 
     }
     // the backward's rank-r work needs su only: it may start now, beside the forward contractions
     if (ov.on && (rc = ov.fork()) != LORA_OK) return rc;
-    if (ov.on && (rc = bwd_rank(ov.side, ov.side_ctas)) != LORA_OK) return rc;
+    if (ov.on && (rc = bwd_rank(ov.side, ov.side_ctas, ov.side_ctas2)) != LORA_OK) return rc;
     // one launch per batch of bf16-weight, then of 4-bit-weight problems;
     // heavier problems first so that the tile walk ends balanced
     for (int q4 = 0; q4 < 2; ++q4) {
@@ -992,7 +1217,7 @@ int run_step(const lora_proj* projs, int n, int mode, void* ws, const Plan& pl, 
     }
   }
   if (mode & LORA_BWD) {
-    if (!ov.on && (rc = bwd_rank(st, d->num_sms)) != LORA_OK) return rc;
+    if (!ov.on && (rc = bwd_rank(st, d->num_sms, d->num_sms)) != LORA_OK) return rc;
     // the dx contraction reads sv: with the side stream, wait for it
     if (ov.on && (rc = ov.wait_sv()) != LORA_OK) return rc;
     std::vector<Operands>& ops = bops;
@@ -1015,7 +1240,7 @@ int run_step(const lora_proj* projs, int n, int mode, void* ws, const Plan& pl, 
         }
         if ((rc = apply_splits(b, sp, parts)) != LORA_OK) return rc;
         ProfScope ps(LORA_KERNEL_GEMM_BWD, st);
-        if (launch_fused_gemm(b, true, q4 != 0, gemm_sms, st) != cudaSuccess) return LORA_ECUDA;
+        if (launch_fused_gemm(b, true, q4 != 0, gemm_sms_b, st) != cudaSuccess) return LORA_ECUDA;
         if (launch_split_reduce(b, st) != cudaSuccess) return LORA_ECUDA;
       }
     }
@@ -1031,6 +1256,8 @@ int plan_all(const lora_proj* projs, int n, int mode, Plan* pl, bool allow_split
   const int tile = rank_mma_tile();
   auto upt = [&](int64_t len) { return (size_t)cdiv(cdiv(len, 64), kMinUnitChunks); };
   auto tiles = [&](int64_t len) { return (size_t)cdiv(len, tile); };
+  std::vector<DySpec> dy_shapes;  // the fused passes over dy, in the order the backward forms them
+  size_t rows_bwd = 0;
   for (int i = 0; i < n; ++i) {
     int rc = check_shape(&projs[i].shape);
     if (rc != LORA_OK) return rc;
@@ -1038,17 +1265,27 @@ int plan_all(const lora_proj* projs, int n, int mode, Plan* pl, bool allow_split
     const size_t r16 = (size_t)rank_pad16((int)s.rank);
     if ((mode & LORA_FWD) && upt(s.d_in) > 1) pl->n_partials[kPhFwdRows] += tiles(s.T) * upt(s.d_in) * tile * r16;
     if (mode & LORA_BWD) {
-      if (upt(s.d_out) > 1) pl->n_partials[kPhBwdRows] += tiles(s.T) * upt(s.d_out) * tile * r16;
-      if (upt(s.T) > 1) pl->n_partials[kPhBwdCols] += (tiles(s.d_out) + tiles(s.d_in)) * upt(s.T) * tile * r16;
+      const bool fused = dy_fusable((int)s.T, (int)s.d_out, (int)s.rank);
+      if (fused)
+        dy_shapes.push_back(DySpec{nullptr, (int)s.T, (int)s.d_out, (int)s.rank, s.scale, nullptr, nullptr, nullptr,
+                                   nullptr, nullptr});
+      else if (upt(s.d_out) > 1)
+        rows_bwd += tiles(s.T) * upt(s.d_out) * tile * r16;
+      if (upt(s.T) > 1) pl->n_partials[kPhBwdCols] += ((fused ? 0 : tiles(s.d_out)) + tiles(s.d_in)) * upt(s.T) * tile * r16;
     }
   }
+  // the fused passes over dy and the remaining row products run one after the other: one arena
+  pl->n_partials[kPhBwdRows] = std::max(rows_bwd, dy_plan_floats(dy_shapes));
   // split contractions: batches as run_step forms them (every projection counted for the backward)
   pl->split_f.assign(n, 1);
   pl->split_b.assign(n, 1);
   // a forward-and-backward call leaves the side stream's SMs out of the contractions
-  const int pairs = mode == LORA_FWD_BWD && overlap_enabled()
-                        ? (kPlanSms - side_sms_setting(kPlanSms, projs, n)) / 2
-                        : kPlanPairs;
+  int pairs_dir[2] = {kPlanPairs, kPlanPairs};
+  if (mode == LORA_FWD_BWD && overlap_enabled()) {
+    const SideWidths w = side_widths(kPlanSms, projs, n);
+    pairs_dir[0] = (kPlanSms - w.w1) / 2;
+    pairs_dir[1] = (kPlanSms - w.w2) / 2;
+  }
   std::vector<size_t> split_need(n, 0);
   for (int dir = 0; dir < 2; ++dir) {
     if (!(mode & (dir == 0 ? LORA_FWD : LORA_BWD))) continue;
@@ -1071,7 +1308,7 @@ int plan_all(const lora_proj* projs, int n, int mode, Plan* pl, bool allow_split
           add_problem(b);
         }
         int sp[kMaxProblems];
-        choose_splits(b, sp, pairs);
+        choose_splits(b, sp, pairs_dir[dir]);
         if (!allow_split)
           for (int q = 0; q < b.num_problems; ++q) sp[q] = 1;
         for (int q = 0; q < b.num_problems; ++q) {

@@ -202,6 +202,47 @@ struct ColBatch {
   long long limit_ns;
 };
 
+// The backward's two products over dy in one pass (one problem per projection):
+//   sv = s dy B   [T, r]   (bf16 into sv [T, ld_sv] and sv^T [pad8(r), T], zero columns / rows past r)
+//   dB = dy^T su  [N, r]   (fp32)
+// B and su come transposed (B^T [pad8(r), N], su^T [pad8(r), T], zero rows
+// past r).  A work unit is (token group g, column piece q): the column blocks
+// of q (128 columns each) in turn, and for each the group's 128-token tiles;
+// the group's sv accumulators stay in TMEM across the unit.  A projection cut
+// into several pieces writes fp32 sv partials [piece][T][rpad]; one cut into
+// several groups writes fp32 dB partials [group][N][rpad]; the dy reduce pass
+// sums them in order.
+constexpr int kDyMaxCut = 8;  // most pieces / groups of one projection
+struct DyProb {
+  CUtensorMap tmDy;   // dy [T, N]: box 64 columns x 128 tokens, 128-byte swizzle
+  CUtensorMap tmBt;   // B^T [r, N]: box 64 columns x pad8(r) rows
+  CUtensorMap tmSuT;  // su^T [r, T]: box 64 tokens x pad8(r) rows
+  int T, N, r, rpad;  // rpad: r rounded up to 16 (the MMA's N)
+  float scale;
+  __nv_bfloat16* sv;  // [T, ld_sv]
+  int ld_sv;
+  __nv_bfloat16* svT;  // [pad8(r), T]
+  float* dB;           // [N, r]
+  int tiles, tt, groups;     // 128-token tiles, tiles per group, groups
+  int blocks, bpu, pieces;   // 128-column blocks, blocks per piece, pieces
+  int unit_begin;
+  long long sv_part, db_part;  // partial offsets (pieces > 1 / groups > 1)
+};
+struct DyBatch {
+  DyProb p[kMaxRankProblems];
+  int n, units;
+  float* partials;
+  int red_sv, red_db;  // elements of the reduce pass: sum of T x pad8(r) (pieces > 1), N x r (groups > 1)
+  int* status;
+  long long limit_ns;
+};
+// Largest token tiles per group for a padded rank (TMEM: sv accumulators of
+// the group plus two dB accumulators).
+int dy_tiles_max(int rpad);
+// Stages of 128 tokens x 128 columns one CTA pipelines for a padded rank.
+int dy_stages(int rpad);
+cudaError_t launch_dy(const DyBatch& b, int ctas, cudaStream_t stream);
+
 // Output rows (tokens of a row product, columns of a column product) per tile.
 int rank_mma_tile();
 // Rank-r products on the tensor cores, then their partial-sum pass when needed;

@@ -1,10 +1,11 @@
 // Rank-r products of the LoRA linear on the 5th-generation tensor cores.
 // Row products, out[t, j] = scale * sum_c X[t, c] * W[j, c]:
 //   su = s x A^T      (forward; x [T, K], A [r, K])
-//   sv = s dy B       (backward; dy [T, N], B given transposed, B^T [r, N])
+//   sv = s dy B       (backward, r > 16; dy [T, N], B given transposed, B^T [r, N])
 // Column products, out[c, j] = sum_t X[t, c] * S[t, j] (S given transposed):
-//   dB = dy^T su      (dy [T, N], su^T [r, T])
+//   dB = dy^T su      (backward, r > 16; dy [T, N], su^T [r, T])
 //   dA = sv^T x       (x [T, K], sv^T [r, T])
+// (Up to r = 16 the backward's sv and dB come from one fused pass over dy.)
 // One problem per activation X, with the rank side the concatenation of
 // every projection reading X (q, k and v share x).  Each is a skinny
 // contraction that streams the tall X once: an output tile is 128 rows of X's
@@ -20,9 +21,11 @@
 // outputs, or fp32 partials when a tile's reduction spans several work units
 // (summed in unit order by a second pass, so results never depend on
 // scheduling).  Two accumulators let the read-back of one unit overlap the
-// next unit's loads and MMAs.  The tensor core makes the MMA work
-// negligible, so the kernel streams X at the rate TMA and HBM allow.  Every
-// wait is bounded.
+// next unit's loads and MMAs.  The MMAs are tiny (N = rank), but each reads
+// its 4 KB X tile from shared memory, ~64 cycles apiece: with the copies'
+// issue cost that bounds the rate one CTA streams X at (~45-60 GB/s), so
+// these kernels fill the HBM bandwidth only on many SMs.  Every wait is
+// bounded.
 #include "rank_store.cuh"
 
 namespace lora {
