@@ -806,12 +806,12 @@ int launch_dy_pass(const std::vector<DySpec>& specs, const Arena& ar, const Devi
       if (c.pieces > 1) {
         p.sv_part = (long long)pf;
         pf += dy_sv_floats(s.T, p.rpad, c.pieces);
-        b.red_sv += s.T * r8;
+        b.red_sv += s.T * (r8 / 8);
       }
       if (c.groups > 1) {
         p.db_part = (long long)pf;
         pf += dy_db_floats(s.N, p.rpad, c.groups);
-        b.red_db += s.N * s.r;
+        b.red_db += s.N * ((s.r + 3) / 4);
       }
     }
     if (pf > ar.n_partials) return LORA_EWORKSPACE;  // planning bound violated

@@ -232,7 +232,7 @@ struct DyBatch {
   DyProb p[kMaxRankProblems];
   int n, units;
   float* partials;
-  int red_sv, red_db;  // elements of the reduce pass: sum of T x pad8(r) (pieces > 1), N x r (groups > 1)
+  int red_sv, red_db;  // items of the reduce pass: T x pad8(r) / 8 (pieces > 1), N x ceil(r / 4) (groups > 1)
   int* status;
   long long limit_ns;
 };

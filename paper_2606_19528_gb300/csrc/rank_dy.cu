@@ -362,7 +362,9 @@ __global__ void __launch_bounds__(kThreads, 1) rank_dy_kernel(const __grid_const
 
 // Sums the partials of the projections cut into several pieces (sv: in piece
 // order, then bf16 of scale * sum into sv and sv^T) or token groups (dB: in
-// group order).  One thread per output element.
+// group order).  A thread takes 8 rank columns of one token's sv (threads in
+// turn take consecutive tokens, so the sv^T stores coalesce) or 4 of one dB
+// row, and issues the loads of every piece before it sums them.
 __global__ void __launch_bounds__(256) dy_reduce_kernel(const __grid_constant__ DyBatch b) {
   griddep_wait();
   const long long total = (long long)b.red_sv + b.red_db;
@@ -374,33 +376,56 @@ __global__ void __launch_bounds__(256) dy_reduce_kernel(const __grid_constant__ 
       for (; pi < b.n; ++pi) {
         const DyProb& P = b.p[pi];
         if (P.pieces <= 1) continue;
-        const long long n = (long long)P.T * pad8(P.r);
+        const long long n = (long long)P.T * (pad8(P.r) / 8);
         if (e < n) break;
         e -= n;
       }
       const DyProb& P = b.p[pi];
-      const int r8 = pad8(P.r);
-      const int t = (int)(e / r8), j = (int)(e % r8);
-      float s = 0.f;
-      for (int q = 0; q < P.pieces; ++q) s += __ldcg(b.partials + P.sv_part + ((size_t)q * P.T + t) * P.rpad + j);
-      const __nv_bfloat16 o = __float2bfloat16_rn(j < P.r ? P.scale * s : 0.f);
-      if (j < P.ld_sv) P.sv[(size_t)t * P.ld_sv + j] = o;
-      P.svT[(size_t)j * P.T + t] = o;
+      const int j = (int)(e / P.T) * 8, t = (int)(e % P.T);
+      const float* src = b.partials + P.sv_part + (size_t)t * P.rpad + j;
+      const size_t step = (size_t)P.T * P.rpad;
+      float4 lo[kDyMaxCut], hi[kDyMaxCut];
+#pragma unroll
+      for (int q = 0; q < kDyMaxCut; ++q) {
+        if (q < P.pieces) {
+          lo[q] = __ldcg(reinterpret_cast<const float4*>(src + q * step));
+          hi[q] = __ldcg(reinterpret_cast<const float4*>(src + q * step + 4));
+        }
+      }
+      float v[8] = {0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f};
+#pragma unroll
+      for (int q = 0; q < kDyMaxCut; ++q) {
+        if (q < P.pieces) {
+          v[0] += lo[q].x, v[1] += lo[q].y, v[2] += lo[q].z, v[3] += lo[q].w;
+          v[4] += hi[q].x, v[5] += hi[q].y, v[6] += hi[q].z, v[7] += hi[q].w;
+        }
+      }
+      sv_store8(P, t, j, v);
     } else {
       e -= b.red_sv;
       int pi = 0;
       for (; pi < b.n; ++pi) {
         const DyProb& P = b.p[pi];
         if (P.groups <= 1) continue;
-        const long long n = (long long)P.N * P.r;
+        const long long n = (long long)P.N * ((P.r + 3) / 4);
         if (e < n) break;
         e -= n;
       }
       const DyProb& P = b.p[pi];
-      const int c = (int)(e / P.r), j = (int)(e % P.r);
-      float s = 0.f;
-      for (int g = 0; g < P.groups; ++g) s += __ldcg(b.partials + P.db_part + ((size_t)g * P.N + c) * P.rpad + j);
-      P.dB[(size_t)c * P.r + j] = s;
+      const int jq = (P.r + 3) / 4;
+      const int c = (int)(e / jq), j = (int)(e % jq) * 4;
+      const float* src = b.partials + P.db_part + (size_t)c * P.rpad + j;
+      const size_t step = (size_t)P.N * P.rpad;
+      float4 s = make_float4(0.f, 0.f, 0.f, 0.f);
+      for (int g = 0; g < P.groups; ++g) {
+        const float4 a = __ldcg(reinterpret_cast<const float4*>(src + g * step));
+        s.x += a.x, s.y += a.y, s.z += a.z, s.w += a.w;
+      }
+      float* d = P.dB + (size_t)c * P.r + j;
+      const float o[4] = {s.x, s.y, s.z, s.w};
+#pragma unroll
+      for (int k = 0; k < 4; ++k)
+        if (j + k < P.r) d[k] = o[k];
     }
   }
   griddep_launch_dependents();
@@ -447,7 +472,7 @@ cudaError_t launch_dy(const DyBatch& b, int ctas, cudaStream_t st) {
   }
   if (e != cudaSuccess || (long long)b.red_sv + b.red_db <= 0) return e;
   const long long total = (long long)b.red_sv + b.red_db;
-  const int blocks = (int)std::min<long long>((total + 255) / 256, 4LL * ctas);
+  const int blocks = (int)std::min<long long>((total + 255) / 256, 8LL * ctas);
   return launch_kernel(dy_reduce_kernel, dim3(blocks), dim3(256), 0, st, 1, b);
 }
 
