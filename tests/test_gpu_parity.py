@@ -229,6 +229,33 @@ def test_stack_equals_single_calls():
         assert G.rel_fro(G.host_f64(q.dB), G.host_f64(ps[i].dB)) < 1e-6, pr.name
 
 
+def test_stack_mixed_ranks_fused_and_two_pass():
+    """One call whose projections take both backward paths over dy: r <= 16
+    the fused pass (sv and dB in one read), r > 16 the two separate passes,
+    sharing one partial arena in turn; ragged T and N, projections sharing x.
+    Every output against the oracle; the backward-only call (all SMs, other
+    cuts) agrees with the two-stream call to fp32 rounding."""
+    T, s = 648, 2.0
+    shapes = [(520, 392, 16), (520, 136, 32), (520, 264, 3), (392, 520, 64), (136, 1032, 8)]
+    groups = [0, 0, 0, 1, 2]
+    ps, xs = [], {}
+    for i, ((K, N, r), g) in enumerate(zip(shapes, groups)):
+        bits = gen_proj(21, i, 0, T, K, N, r, s, group=g)
+        p = G.DevProj(*bits, s, share_x=xs.get(g))
+        xs.setdefault(g, p.x)
+        ps.append(p)
+    G.run_stack(ps)
+    for p in ps:
+        check_full(p)
+    first = [(p.dA.clone(), p.dB.clone(), p.dx.clone()) for p in ps]
+    G.run_stack(ps, lora.LORA_FWD)
+    G.run_stack(ps, lora.LORA_BWD)
+    for p, (dA, dB, dx) in zip(ps, first):
+        assert G.rel_fro(G.host_f64(p.dA), G.host_f64(dA)) < 1e-6
+        assert G.rel_fro(G.host_f64(p.dB), G.host_f64(dB)) < 1e-6
+        assert G.rel_fro(G.host_f64(p.dx), G.host_f64(dx)) < 2e-3
+
+
 SWEEP = [(T, r) for T in workloads.SWEEP_TOKENS for r in workloads.SWEEP_RANKS]
 
 
