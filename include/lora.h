@@ -42,6 +42,16 @@
  *    (argument errors), or kernels may already be enqueued (LORA_ECUDA).
  *    Device-side bounded waits that expire set a status word readable with
  *    lora_read_status (LORA_ETIMEOUT); they never trap.
+ *
+ * Environment (read once per process; for measurement, never needed):
+ *   LORA_PDL=0        launch without programmatic dependent launch;
+ *   LORA_OVERLAP=0    run a forward-and-backward call on the caller's stream
+ *                     alone (no side stream for the backward's rank-r work);
+ *   LORA_SIDE_SMS=n   SMs of the side stream beside the forward contraction,
+ *   LORA_SIDE_SMS2=n  and beside the backward-dx contraction (2 .. SMs / 4;
+ *                     default: the balance rule of the implementation).
+ * A workspace size reported with one setting may not cover a call made with
+ * another: query the size in the process that makes the calls.
  */
 #ifndef LORA_GB300_H_
 #define LORA_GB300_H_

@@ -239,8 +239,6 @@ struct DyBatch {
 // Largest token tiles per group for a padded rank (TMEM: sv accumulators of
 // the group plus two dB accumulators).
 int dy_tiles_max(int rpad);
-// Stages of 128 tokens x 128 columns one CTA pipelines for a padded rank.
-int dy_stages(int rpad);
 cudaError_t launch_dy(const DyBatch& b, int ctas, cudaStream_t stream);
 
 // Output rows (tokens of a row product, columns of a column product) per tile.

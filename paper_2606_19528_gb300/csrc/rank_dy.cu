@@ -450,15 +450,6 @@ int rank_class(int rpad) { return rpad <= 16 ? 16 : rpad <= 32 ? 32 : rpad <= 64
 
 int dy_tiles_max(int rpad) { return (int)kTmemCols / rank_class(rpad) - 2; }
 
-int dy_stages(int rpad) {
-  switch (rank_class(rpad)) {
-    case 16: return DyRing<16>::kStages;
-    case 32: return DyRing<32>::kStages;
-    case 64: return DyRing<64>::kStages;
-    default: return DyRing<128>::kStages;
-  }
-}
-
 cudaError_t launch_dy(const DyBatch& b, int ctas, cudaStream_t st) {
   if (b.n <= 0 || b.units <= 0 || ctas <= 0) return cudaSuccess;
   int rmax = 16;
