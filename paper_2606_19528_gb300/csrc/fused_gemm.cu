@@ -911,13 +911,9 @@ size_t fused_gemm_smem_bytes() { return smem_bytes<false>(); }
 template <bool kBMn, bool kQ, bool kF32>
 cudaError_t launch_variant(const GemmBatch& batch, int pairs, cudaStream_t stream) {
   constexpr size_t smem = smem_bytes<kQ>();
-  static bool attr_done = false;
-  if (!attr_done) {
-    cudaError_t e = cudaFuncSetAttribute(fused_lora_gemm<kBMn, kQ, kF32>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                         (int)smem);
-    if (e != cudaSuccess) return e;
-    attr_done = true;
-  }
+  static std::atomic<unsigned long long> attr_done{0};
+  const cudaError_t e = set_smem_once(fused_lora_gemm<kBMn, kQ, kF32>, (int)smem, attr_done);
+  if (e != cudaSuccess) return e;
   return launch_kernel(fused_lora_gemm<kBMn, kQ, kF32>, dim3((unsigned)(2 * pairs)), dim3(Cfg<kQ>::kThreads), smem,
                        stream, 2, batch);
 }

@@ -7,6 +7,8 @@
 #include <stddef.h>
 #include <stdint.h>
 
+#include <atomic>
+
 namespace lora {
 
 // Counts one kernel launch (defined with the C ABI).
@@ -45,6 +47,21 @@ cudaError_t launch_kernel(void (*kernel)(KArgs...), dim3 grid, dim3 block, size_
   const cudaError_t e = cudaLaunchKernelEx(&cfg, kernel, static_cast<Args&&>(args)...);
   note_launch();
   return e != cudaSuccess ? e : cudaGetLastError();
+}
+
+// Raises `kernel`'s dynamic shared-memory limit to `smem` bytes on the
+// current device, once per device (the attribute belongs to the device's copy
+// of the kernel); `done` is the kernel's bit set of devices already raised.
+template <typename... KArgs>
+cudaError_t set_smem_once(void (*kernel)(KArgs...), int smem, std::atomic<unsigned long long>& done) {
+  int dev = 0;
+  cudaError_t e = cudaGetDevice(&dev);
+  if (e != cudaSuccess) return e;
+  const unsigned long long bit = 1ull << (dev & 63);
+  if (done.load(std::memory_order_acquire) & bit) return cudaSuccess;
+  e = cudaFuncSetAttribute(kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
+  if (e == cudaSuccess) done.fetch_or(bit, std::memory_order_acq_rel);
+  return e;
 }
 
 // ---------------------------------------------------------------- fused GEMM

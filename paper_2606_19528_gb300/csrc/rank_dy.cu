@@ -434,12 +434,9 @@ __global__ void __launch_bounds__(256) dy_reduce_kernel(const __grid_constant__ 
 template <int R>
 cudaError_t launch_dy_r(const DyBatch& b, int ctas, cudaStream_t st) {
   constexpr int smem = (int)dy_smem_bytes<R>();
-  static bool attr_done = false;
-  if (!attr_done) {
-    cudaError_t e = cudaFuncSetAttribute(rank_dy_kernel<R>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
-    if (e != cudaSuccess) return e;
-    attr_done = true;
-  }
+  static std::atomic<unsigned long long> attr_done{0};
+  const cudaError_t e = set_smem_once(rank_dy_kernel<R>, smem, attr_done);
+  if (e != cudaSuccess) return e;
   const int grid = b.units < ctas ? b.units : ctas;
   return launch_kernel(rank_dy_kernel<R>, dim3(grid), dim3(kThreads), smem, st, 1, b);
 }

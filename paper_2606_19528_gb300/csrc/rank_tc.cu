@@ -293,12 +293,9 @@ __global__ void __launch_bounds__(kThreads, 1) rank_mma_kernel(const __grid_cons
 template <int R, bool kCol>
 cudaError_t launch_r(const typename Side<kCol>::Batch& b, int ctas, cudaStream_t st) {
   constexpr int smem = (int)tc_smem_bytes<R>();
-  static bool attr_done = false;
-  if (!attr_done) {
-    cudaError_t e = cudaFuncSetAttribute(rank_mma_kernel<R, kCol>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
-    if (e != cudaSuccess) return e;
-    attr_done = true;
-  }
+  static std::atomic<unsigned long long> attr_done{0};
+  const cudaError_t e = set_smem_once(rank_mma_kernel<R, kCol>, smem, attr_done);
+  if (e != cudaSuccess) return e;
   const int grid = b.units < ctas ? b.units : ctas;
   return launch_kernel(rank_mma_kernel<R, kCol>, dim3(grid), dim3(kThreads), smem, st, 1, b);
 }

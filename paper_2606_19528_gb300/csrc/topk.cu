@@ -635,14 +635,10 @@ cudaError_t launch_normalize_rows(const __nv_bfloat16* E, int V, int d, __nv_bfl
   return launch_kernel(normalize_rows_kernel, dim3((V + 127) / 128), dim3(128), 0, st, 1, E, V, d, En);
 }
 
-// Sets the dynamic shared-memory size of the selection kernels once.
+// Sets the dynamic shared-memory size of the selection kernel (once per device).
 cudaError_t sel_attrs() {
-  static const cudaError_t e = [] {
-    const int smem = (int)sizeof(SelShared);
-    cudaError_t r = cudaFuncSetAttribute(topk_select_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
-    return r;
-  }();
-  return e;
+  static std::atomic<unsigned long long> attr_done{0};
+  return set_smem_once(topk_select_kernel, (int)sizeof(SelShared), attr_done);
 }
 
 cudaError_t launch_topk_select(const float* S, long long lds, int V, int k, int row0, const int32_t* rows, int nrows,
