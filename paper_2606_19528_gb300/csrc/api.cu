@@ -727,8 +727,18 @@ double dy_cost(const std::vector<DySpec>& specs, size_t i0, size_t i1, const std
   return part > 0 ? make + 4.0 + part * 8.0 / 32768.0 / ctas : make;
 }
 
-// The cuts of a batch (rank class of its largest rank) that cost least on `ctas` CTAs.
+// The cuts of a batch (rank class of its largest rank) that cost least on
+// `ctas` CTAs.  Choices are cached per shape set.
 std::vector<DyCut> dy_choose(const std::vector<DySpec>& specs, size_t i0, size_t i1, int ctas) {
+  static std::mutex mu;
+  static std::map<std::vector<long long>, std::vector<DyCut>> cache;
+  std::vector<long long> key{ctas};
+  for (size_t i = i0; i < i1; ++i) key.insert(key.end(), {specs[i].T, specs[i].N, specs[i].r});
+  {
+    std::lock_guard<std::mutex> lk(mu);
+    auto it = cache.find(key);
+    if (it != cache.end()) return it->second;
+  }
   int rmax = 16;
   for (size_t i = i0; i < i1; ++i) rmax = std::max(rmax, rank_pad16(specs[i].r));
   const int tmax = dy_tiles_max(rmax);
@@ -743,6 +753,9 @@ std::vector<DyCut> dy_choose(const std::vector<DySpec>& specs, size_t i0, size_t
         best_cost = c;
       }
     }
+  std::lock_guard<std::mutex> lk(mu);
+  if (cache.size() > 4096) cache.clear();
+  cache.emplace(key, best);
   return best;
 }
 

@@ -380,6 +380,7 @@ __global__ void __launch_bounds__(256) dy_reduce_kernel(const __grid_constant__ 
         if (e < n) break;
         e -= n;
       }
+      if (pi >= b.n) continue;  // unreachable with consistent counts
       const DyProb& P = b.p[pi];
       const int j = (int)(e / P.T) * 8, t = (int)(e % P.T);
       const float* src = b.partials + P.sv_part + (size_t)t * P.rpad + j;
@@ -411,6 +412,7 @@ __global__ void __launch_bounds__(256) dy_reduce_kernel(const __grid_constant__ 
         if (e < n) break;
         e -= n;
       }
+      if (pi >= b.n) continue;  // unreachable with consistent counts
       const DyProb& P = b.p[pi];
       const int jq = (P.r + 3) / 4;
       const int c = (int)(e / jq), j = (int)(e % jq) * 4;
