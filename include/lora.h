@@ -28,7 +28,13 @@
  *    the caller, row-major and dense (leading dimension = row length), and
  *    16-byte aligned; the library never allocates or frees memory;
  *  - T, d_in and d_out are multiples of 8 (16-byte rows for the tensor-memory
- *    accelerator), 1 <= rank <= 128, scale finite;
+ *    accelerator), 0 <= rank <= 128, scale finite;
+ *  - rank 0 is a frozen projection without an adapter: the forward computes
+ *    y = x W^T and the backward dx = dy W only; A, B, su, dA and dB are
+ *    neither read nor written and may be NULL.  The paper adapts only the q
+ *    and v projections of each layer (hyper-parameter table), so the other
+ *    projections of a layer are such frozen linears, still on the backward
+ *    path through dx;
  *  - calls are asynchronous on `stream` (a cudaStream_t; NULL = legacy
  *    default stream); return LORA_OK once every kernel is enqueued;
  *  - inputs may alias each other (e.g. q, k and v passing one x); outputs
@@ -39,7 +45,9 @@
  *    initialisation and are garbage afterwards; calls that run concurrently
  *    need separate workspaces;
  *  - errors: a negative LORA_E* code is returned and nothing is enqueued
- *    (argument errors), or kernels may already be enqueued (LORA_ECUDA).
+ *    (argument errors), or kernels may already be enqueued (LORA_ECUDA);
+ *    lora_last_error() repeats the code the calling thread's latest call
+ *    returned.
  *    Device-side bounded waits that expire set a status word readable with
  *    lora_read_status (LORA_ETIMEOUT); they never trap.
  *
@@ -100,9 +108,9 @@ int lora_linear_fwd(const lora_shape* shape, const lora_bf16* x, const lora_bf16
                     const lora_bf16* A, const lora_bf16* B, lora_bf16* y, lora_bf16* su,
                     void* workspace, size_t workspace_bytes, void* stream);
 
-/* Forward of one LoRA linear exactly as lora_linear_fwd computes it, but
- * with no workspace argument, for callers that cannot allocate device memory
- * when they call: an operator running inside another framework's execution
+/* Forward of one LoRA linear as lora_linear_fwd computes it, but with no
+ * workspace argument, for callers that cannot allocate device memory when
+ * they call: an operator running inside another framework's execution
  * callback, where allocating is not allowed, or a latency-bound path that
  * cannot afford the device-wide synchronisation cudaMalloc and cudaFree
  * cause.  Its scratch is one fixed array of 4 MiB in device memory that the
@@ -113,8 +121,13 @@ int lora_linear_fwd(const lora_shape* shape, const lora_bf16* x, const lora_bf16
  * array's device address; make that first call before any stream capture.
  * All calls share the array and leave their scratch in it: calls that
  * overlap on the GPU (for example on two streams at once) race and give
- * wrong results.  Nothing is allocated.  The paper has no counterpart of
- * this entry point.  Returns as lora_linear_fwd, or LORA_ESCRATCH. */
+ * wrong results.  Nothing is allocated.  Its contraction always runs in one
+ * pass: where lora_linear_fwd splits the contraction of a forward with few
+ * output tiles (fewer than 76, e.g. 512 tokens x d_out 3072) into fp32
+ * partial sums, the two results differ by the bf16 rounding of differently
+ * ordered fp32 sums; with 76 or more output tiles of 256 x 512 they are
+ * identical bit for bit.  The paper has no counterpart of this entry point.
+ * Returns as lora_linear_fwd (argument errors first), or LORA_ESCRATCH. */
 int lora_linear_fwd_noalloc(const lora_shape* shape, const lora_bf16* x, const lora_bf16* W,
                             const lora_bf16* A, const lora_bf16* B, lora_bf16* y, lora_bf16* su,
                             void* stream);
@@ -312,6 +325,15 @@ int lora_profile_end(double* ms, int64_t* launches);
 
 /* Static message for a LORA_* code. */
 const char* lora_strerror(int code);
+
+/* The code the calling thread's most recent library call returned (every
+ * entry point that returns a LORA_* code records it, successes included, in
+ * thread-local storage; lora_strerror, lora_version, lora_launch_count and
+ * lora_last_error itself do not).  Device-side codes of kernels that already
+ * ran are not included: lora_read_status reports those.  LORA_OK before any
+ * call.  For callers that keep only a success flag across a layer of their
+ * own; each call also returns its code directly. */
+int lora_last_error(void);
 
 /* Library version, major * 10000 + minor * 100 + patch. */
 int lora_version(void);

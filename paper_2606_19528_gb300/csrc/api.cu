@@ -173,7 +173,7 @@ int check_shape(const lora_shape* s) {
   if (s->T < 8 || s->d_in < 8 || s->d_out < 8) return LORA_EINVAL;
   if ((s->T % 8) || (s->d_in % 8) || (s->d_out % 8)) return LORA_EINVAL;
   if (s->T > (1ll << 30) || s->d_in > (1ll << 20) || s->d_out > (1ll << 20)) return LORA_EINVAL;
-  if (s->rank < 1 || s->rank > 128) return LORA_EINVAL;
+  if (s->rank < 0 || s->rank > 128) return LORA_EINVAL;  // rank 0: frozen projection, no adapter
   if (!isfinite(s->scale)) return LORA_EINVAL;
   return LORA_OK;
 }
@@ -849,7 +849,9 @@ int add_fwd_problem(GemmBatch& b, const lora_proj& p, const Operands& o) {
   // activation boxes: one CTA's 128 rows x 64 contraction elements; weight
   // boxes: 64 rows x 64 (two per CTA)
   if ((rc = make_map(&b.tmA[i], p.x, K, T, K, 64, 128)) != LORA_OK) return rc;
-  if ((rc = make_map(&b.tmA2[i], o.s_in, r, T, o.ld_s, 64, 128)) != LORA_OK) return rc;
+  // rank 0: no adapter slab (kb_total = kb_main), so the slab maps are never read
+  if ((rc = r > 0 ? make_map(&b.tmA2[i], o.s_in, r, T, o.ld_s, 64, 128) : (b.tmA2[i] = b.tmA[i], LORA_OK)) != LORA_OK)
+    return rc;
   if (is_q4(p)) {
     // 4-bit W: a box is 64 rows x 64 codes (32 bytes); (s, b) boxes are 128 rows x 4 groups
     if ((rc = make_map_plain(&b.tmQ[i], CU_TENSOR_MAP_DATA_TYPE_UINT8, 1, p.Wq.codes, K / 2, N, K / 2, 32, 64)) !=
@@ -861,7 +863,8 @@ int add_fwd_problem(GemmBatch& b, const lora_proj& p, const Operands& o) {
   } else if ((rc = make_map(&b.tmB[i], p.W, K, N, K, 64, 64)) != LORA_OK) {
     return rc;
   }
-  if ((rc = make_map(&b.tmB2[i], o.B, r, N, o.ld_b, 64, 64)) != LORA_OK) return rc;
+  if ((rc = r > 0 ? make_map(&b.tmB2[i], o.B, r, N, o.ld_b, 64, 64) : (b.tmB2[i] = b.tmA[i], LORA_OK)) != LORA_OK)
+    return rc;
   if ((rc = make_map(&b.tmOut[i], p.y, N, T, N, 64, 32)) != LORA_OK) return rc;
   GemmProblem& g = b.prob[i];
   gemm_shape(g, T, N, K, r);
@@ -877,7 +880,8 @@ int add_bwd_problem(GemmBatch& b, const lora_proj& p, const Operands& o) {
   const int64_t T = s.T, K = s.d_in, N = s.d_out, r = s.rank;
   int rc;
   if ((rc = make_map(&b.tmA[i], p.dy, N, T, N, 64, 128)) != LORA_OK) return rc;
-  if ((rc = make_map(&b.tmA2[i], o.s_in, r, T, o.ld_s, 64, 128)) != LORA_OK) return rc;
+  if ((rc = r > 0 ? make_map(&b.tmA2[i], o.s_in, r, T, o.ld_s, 64, 128) : (b.tmA2[i] = b.tmA[i], LORA_OK)) != LORA_OK)
+    return rc;
   // W [N, K] read MN-major: inner dimension K (the GEMM's output columns), rows = contraction
   if (is_q4(p)) {
     // 4-bit W: a box is 64 rows x 128 codes (64 bytes); (s, b) boxes are 64 rows x 4 groups
@@ -890,7 +894,8 @@ int add_bwd_problem(GemmBatch& b, const lora_proj& p, const Operands& o) {
   } else if ((rc = make_map(&b.tmB[i], p.W, K, N, K, 64, 64)) != LORA_OK) {
     return rc;
   }
-  if ((rc = make_map(&b.tmB2[i], p.A, K, r, K, 64, 64)) != LORA_OK) return rc;
+  if ((rc = r > 0 ? make_map(&b.tmB2[i], p.A, K, r, K, 64, 64) : (b.tmB2[i] = b.tmA[i], LORA_OK)) != LORA_OK)
+    return rc;
   if ((rc = make_map(&b.tmOut[i], p.dx, K, T, K, 64, 32)) != LORA_OK) return rc;
   GemmProblem& g = b.prob[i];
   gemm_shape(g, T, K, N, r);
@@ -917,8 +922,10 @@ int check_weight(const lora_proj& p) {
   return LORA_OK;
 }
 
+// A frozen projection (rank 0) has no adapter: A, B, su, dA and dB are neither read nor written.
 int check_fwd_ptrs(const lora_proj& p) {
-  if (!p.x || !p.A || !p.B || !p.y) return LORA_ENULL;
+  if (!p.x || !p.y) return LORA_ENULL;
+  if (p.shape.rank > 0 && (!p.A || !p.B)) return LORA_ENULL;
   const void* ps[] = {p.x, p.W, p.A, p.B, p.y, p.su};
   for (const void* q : ps)
     if (q && !aligned16(q)) return LORA_EALIGN;
@@ -926,7 +933,8 @@ int check_fwd_ptrs(const lora_proj& p) {
 }
 
 int check_bwd_ptrs(const lora_proj& p) {
-  if (!p.dy || !p.x || !p.A || !p.B || !p.su || !p.dA || !p.dB) return LORA_ENULL;
+  if (!p.dy || !p.x) return LORA_ENULL;
+  if (p.shape.rank > 0 && (!p.A || !p.B || !p.su || !p.dA || !p.dB)) return LORA_ENULL;
   const void* ps[] = {p.dy, p.x, p.W, p.A, p.B, p.su, p.dx, p.dA, p.dB};
   for (const void* q : ps)
     if (q && !aligned16(q)) return LORA_EALIGN;
@@ -993,6 +1001,8 @@ SideWidths side_widths(int num_sms, const lora_proj* projs, int n) {
   for (int i = 0; i < n; ++i) {
     const lora_shape& sh = projs[i].shape;
     const double T = (double)sh.T, K = (double)sh.d_in, N = (double)sh.d_out, r = (double)sh.rank;
+    flops += 2.0 * T * K * N * (is_q4(projs[i]) ? 1.3 : 1.0);
+    if (sh.rank == 0) continue;  // a frozen projection puts no work on the side stream
     const double fr = 1.0 + r / 144.0;
     b1 += 2.0 * T * N * fr + kSideAdapter1 * r * N;
     b2 += kSideAdapter2 * r * K;
@@ -1003,7 +1013,6 @@ SideWidths side_widths(int num_sms, const lora_proj* projs, int n) {
       b2 += 2.0 * T * K * fr;
       if (x != nullptr) xs.push_back(x);
     }
-    flops += 2.0 * T * K * N * (is_q4(projs[i]) ? 1.3 : 1.0);
   }
   auto width = [&](double kappa, double bytes) {
     const double c = flops > 0.0 ? kappa * bytes / flops : 0.0;
@@ -1013,6 +1022,13 @@ SideWidths side_widths(int num_sms, const lora_proj* projs, int n) {
   w.w1 = std::max(2, std::min(num_sms / 4, v1 > 0 ? v1 : width(kSideKappa1, b1)));
   w.w2 = std::max(2, std::min(num_sms / 4, v2 > 0 ? v2 : width(kSideKappa2, b2)));
   return w;
+}
+
+// Whether any projection has an adapter (rank > 0): frozen ones have no rank-r work.
+bool any_adapter(const lora_proj* projs, int n) {
+  for (int i = 0; i < n; ++i)
+    if (projs[i].shape.rank > 0) return true;
+  return false;
 }
 
 struct SideCtx {
@@ -1040,7 +1056,7 @@ struct Overlap {
   cudaStream_t main = nullptr, side = nullptr;
   cudaEvent_t ev_fork = nullptr, ev_sv = nullptr, ev_done = nullptr;
   int init(const DeviceInfo* d, cudaStream_t st, const lora_proj* projs, int n) {
-    if (!overlap_enabled()) return LORA_OK;
+    if (!overlap_enabled() || !any_adapter(projs, n)) return LORA_OK;
     SideCtx& c = t_side.dev[d - g_dev];
     if (!c.side && cudaStreamCreateWithFlags(&c.side, cudaStreamNonBlocking) != cudaSuccess) return LORA_ECUDA;
     for (cudaEvent_t& e : c.ev)
@@ -1103,7 +1119,8 @@ int run_step(const lora_proj* projs, int n, int mode, void* ws, const Plan& pl, 
     std::vector<bf*> sut(n), svt(n);
     std::vector<char> fused(n);
     for (int i = 0; i < n; ++i)
-      fused[i] = dy_fusable((int)projs[i].shape.T, (int)projs[i].shape.d_out, (int)projs[i].shape.rank);
+      fused[i] = projs[i].shape.rank > 0 &&
+                 dy_fusable((int)projs[i].shape.T, (int)projs[i].shape.d_out, (int)projs[i].shape.rank);
     std::vector<Operands>& ops = bops;
     TransposeJobs tj;
     memset(&tj, 0, sizeof(tj));
@@ -1129,6 +1146,7 @@ int run_step(const lora_proj* projs, int n, int mode, void* ws, const Plan& pl, 
       for (int i = 0; i < n; ++i) {
         const lora_proj& p = projs[i];
         const int T = (int)p.shape.T, N = (int)p.shape.d_out, r = (int)p.shape.rank, r8 = rank_pad8(r);
+        if (r == 0) continue;  // frozen: dx = dy W only
         bf* bt = at<bf>(W_(i), plans[i].bt);
         sut[i] = at<bf>(W_(i), plans[i].sut);
         svt[i] = at<bf>(W_(i), plans[i].svt);
@@ -1152,7 +1170,7 @@ int run_step(const lora_proj* projs, int n, int mode, void* ws, const Plan& pl, 
     }
     if (ov.on && cudaEventRecord(ov.ev_sv, rs) != cudaSuccess) return LORA_ECUDA;
     for (int i = 0; i < n; ++i) {
-      if (fused[i]) continue;
+      if (fused[i] || projs[i].shape.rank == 0) continue;
       const lora_proj& p = projs[i];
       const int T = (int)p.shape.T, N = (int)p.shape.d_out, r = (int)p.shape.rank;
       add_col_block(cols, cb(p.dy), N, T, N, sut[i], T, r, p.dB, 1, false);
@@ -1160,7 +1178,7 @@ int run_step(const lora_proj* projs, int n, int mode, void* ws, const Plan& pl, 
     for (int i = 0; i < n; ++i) {
       const lora_proj& p = projs[i];
       const int T = (int)p.shape.T, K = (int)p.shape.d_in, r = (int)p.shape.rank;
-      add_col_block(cols, cb(p.x), K, T, K, svt[i], T, r, p.dA, 0, true);
+      if (r > 0) add_col_block(cols, cb(p.x), K, T, K, svt[i], T, r, p.dA, 0, true);
     }
     {
       ProfScope ps(LORA_KERNEL_COLPROJ, rs);
@@ -1178,6 +1196,7 @@ int run_step(const lora_proj* projs, int n, int mode, void* ws, const Plan& pl, 
         const int T = (int)p.shape.T, K = (int)p.shape.d_in, N = (int)p.shape.d_out, r = (int)p.shape.rank;
         const int r8 = rank_pad8(r);
         const bool pad = (r % 8) != 0;
+        if (r == 0) continue;  // frozen: y = x W^T only
         bf* su_gemm = (p.su && !pad) ? mb(p.su) : at<bf>(W_(i), plans[i].su_pad);
         const int ld_gemm = (p.su && !pad) ? r : r8;
         bf* su_user2 = (p.su && pad) ? mb(p.su) : nullptr;
@@ -1276,6 +1295,7 @@ int plan_all(const lora_proj* projs, int n, int mode, Plan* pl, bool allow_split
     if (rc != LORA_OK) return rc;
     const lora_shape& s = projs[i].shape;
     const size_t r16 = (size_t)rank_pad16((int)s.rank);
+    if (s.rank == 0) continue;  // frozen projection: no rank-r work
     if ((mode & LORA_FWD) && upt(s.d_in) > 1) pl->n_partials[kPhFwdRows] += tiles(s.T) * upt(s.d_in) * tile * r16;
     if (mode & LORA_BWD) {
       const bool fused = dy_fusable((int)s.T, (int)s.d_out, (int)s.rank);
@@ -1582,6 +1602,13 @@ int topk_check(const lora_bf16* E, int64_t V, int64_t d, int64_t k, TopkPlan* pl
 
 void note_launch() { g_launches.fetch_add(1, std::memory_order_relaxed); }
 
+// Code the calling thread's most recent entry point returned (lora_last_error).
+thread_local int t_last_error = LORA_OK;
+inline int rec(int rc) {
+  t_last_error = rc;
+  return rc;
+}
+
 bool pdl_enabled() {
   static const bool on = [] {
     const char* e = getenv("LORA_PDL");
@@ -1596,7 +1623,9 @@ using namespace lora;
 
 extern "C" {
 
-int lora_version(void) { return 200; }
+int lora_version(void) { return 300; }
+
+int lora_last_error(void) { return t_last_error; }
 
 const char* lora_strerror(int code) {
   switch (code) {
@@ -1616,51 +1645,52 @@ const char* lora_strerror(int code) {
 int lora_set_wait_limit_ns(int64_t ns) {
   std::lock_guard<std::mutex> lk(g_mu);
   g_wait_limit_ns = ns > 0 ? (long long)ns : kDefaultWaitNs;
-  return LORA_OK;
+  return rec(LORA_OK);
 }
 
 int lora_workspace_size(const lora_shape* shape, int mode, size_t* bytes) {
-  if (!shape || !bytes) return LORA_ENULL;
-  if (mode < LORA_FWD || mode > LORA_FWD_BWD) return LORA_EINVAL;
+  if (!shape || !bytes) return rec(LORA_ENULL);
+  if (mode < LORA_FWD || mode > LORA_FWD_BWD) return rec(LORA_EINVAL);
   lora_proj p;
   memset(&p, 0, sizeof(p));
   p.shape = *shape;
-  return lora_stack_workspace_size(&p, 1, mode, bytes);
+  return rec(lora_stack_workspace_size(&p, 1, mode, bytes));
 }
 
 int lora_stack_workspace_size(const lora_proj* projs, int n_proj, int mode, size_t* bytes) {
-  if (!projs || !bytes) return LORA_ENULL;
-  if (n_proj < 1 || n_proj > 64 || mode < LORA_FWD || mode > LORA_FWD_BWD) return LORA_EINVAL;
+  if (!projs || !bytes) return rec(LORA_ENULL);
+  if (n_proj < 1 || n_proj > 64 || mode < LORA_FWD || mode > LORA_FWD_BWD) return rec(LORA_EINVAL);
   Plan pl;
   int rc = plan_all(projs, n_proj, mode, &pl);
-  if (rc != LORA_OK) return rc;
+  if (rc != LORA_OK) return rec(rc);
   *bytes = pl.total;
-  return LORA_OK;
+  return rec(LORA_OK);
 }
 
 int lora_stack_step(const lora_proj* projs, int n_proj, int mode, void* workspace, size_t workspace_bytes,
                     void* stream) {
-  if (!projs) return LORA_ENULL;
-  if (n_proj < 1 || n_proj > 64 || mode < LORA_FWD || mode > LORA_FWD_BWD) return LORA_EINVAL;
+  if (!projs) return rec(LORA_ENULL);
+  if (n_proj < 1 || n_proj > 64 || mode < LORA_FWD || mode > LORA_FWD_BWD) return rec(LORA_EINVAL);
   DeviceInfo* d = nullptr;
   int rc = device_info(&d);
-  if (rc != LORA_OK) return rc;
+  if (rc != LORA_OK) return rec(rc);
   Plan pl;
-  if ((rc = plan_all(projs, n_proj, mode, &pl)) != LORA_OK) return rc;
+  if ((rc = plan_all(projs, n_proj, mode, &pl)) != LORA_OK) return rec(rc);
   const size_t need = pl.total;
   for (int i = 0; i < n_proj; ++i) {
-    if ((mode & LORA_FWD) && (rc = check_fwd_ptrs(projs[i])) != LORA_OK) return rc;
-    if ((mode & LORA_BWD) && (rc = check_bwd_ptrs(projs[i])) != LORA_OK) return rc;
-    if (mode == LORA_FWD_BWD && !projs[i].su) return LORA_ENULL;  // the backward needs the saved su
+    if ((mode & LORA_FWD) && (rc = check_fwd_ptrs(projs[i])) != LORA_OK) return rec(rc);
+    if ((mode & LORA_BWD) && (rc = check_bwd_ptrs(projs[i])) != LORA_OK) return rec(rc);
+    if (mode == LORA_FWD_BWD && projs[i].shape.rank > 0 && !projs[i].su)
+      return rec(LORA_ENULL);  // the backward needs the saved su
   }
-  if ((rc = check_ws(workspace, workspace_bytes, need)) != LORA_OK) return rc;
-  return run_step(projs, n_proj, mode, workspace, pl, d, static_cast<cudaStream_t>(stream));
+  if ((rc = check_ws(workspace, workspace_bytes, need)) != LORA_OK) return rec(rc);
+  return rec(run_step(projs, n_proj, mode, workspace, pl, d, static_cast<cudaStream_t>(stream)));
 }
 
 int lora_linear_fwd(const lora_shape* shape, const lora_bf16* x, const lora_bf16* W, const lora_bf16* A,
                     const lora_bf16* B, lora_bf16* y, lora_bf16* su, void* workspace, size_t workspace_bytes,
                     void* stream) {
-  if (!shape) return LORA_ENULL;
+  if (!shape) return rec(LORA_ENULL);
   lora_proj p;
   memset(&p, 0, sizeof(p));
   p.shape = *shape;
@@ -1670,13 +1700,13 @@ int lora_linear_fwd(const lora_shape* shape, const lora_bf16* x, const lora_bf16
   p.B = B;
   p.y = y;
   p.su = su;
-  return lora_stack_step(&p, 1, LORA_FWD, workspace, workspace_bytes, stream);
+  return rec(lora_stack_step(&p, 1, LORA_FWD, workspace, workspace_bytes, stream));
 }
 
 int lora_linear_bwd(const lora_shape* shape, const lora_bf16* dy, const lora_bf16* x, const lora_bf16* W,
                     const lora_bf16* A, const lora_bf16* B, const lora_bf16* su, lora_bf16* dx, float* dA,
                     float* dB, void* workspace, size_t workspace_bytes, void* stream) {
-  if (!shape) return LORA_ENULL;
+  if (!shape) return rec(LORA_ENULL);
   lora_proj p;
   memset(&p, 0, sizeof(p));
   p.shape = *shape;
@@ -1689,13 +1719,13 @@ int lora_linear_bwd(const lora_shape* shape, const lora_bf16* dy, const lora_bf1
   p.dx = dx;
   p.dA = dA;
   p.dB = dB;
-  return lora_stack_step(&p, 1, LORA_BWD, workspace, workspace_bytes, stream);
+  return rec(lora_stack_step(&p, 1, LORA_BWD, workspace, workspace_bytes, stream));
 }
 
 int lora_linear_fwd_q4(const lora_shape* shape, const lora_bf16* x, const lora_q4_weight* Wq, const lora_bf16* A,
                        const lora_bf16* B, lora_bf16* y, lora_bf16* su, void* workspace, size_t workspace_bytes,
                        void* stream) {
-  if (!shape || !Wq) return LORA_ENULL;
+  if (!shape || !Wq) return rec(LORA_ENULL);
   lora_proj p;
   memset(&p, 0, sizeof(p));
   p.shape = *shape;
@@ -1705,14 +1735,14 @@ int lora_linear_fwd_q4(const lora_shape* shape, const lora_bf16* x, const lora_q
   p.B = B;
   p.y = y;
   p.su = su;
-  if (!p.Wq.codes || !p.Wq.params) return LORA_ENULL;
-  return lora_stack_step(&p, 1, LORA_FWD, workspace, workspace_bytes, stream);
+  if (!p.Wq.codes || !p.Wq.params) return rec(LORA_ENULL);
+  return rec(lora_stack_step(&p, 1, LORA_FWD, workspace, workspace_bytes, stream));
 }
 
 int lora_linear_bwd_q4(const lora_shape* shape, const lora_bf16* dy, const lora_bf16* x, const lora_q4_weight* Wq,
                        const lora_bf16* A, const lora_bf16* B, const lora_bf16* su, lora_bf16* dx, float* dA,
                        float* dB, void* workspace, size_t workspace_bytes, void* stream) {
-  if (!shape || !Wq) return LORA_ENULL;
+  if (!shape || !Wq) return rec(LORA_ENULL);
   lora_proj p;
   memset(&p, 0, sizeof(p));
   p.shape = *shape;
@@ -1725,8 +1755,8 @@ int lora_linear_bwd_q4(const lora_shape* shape, const lora_bf16* dy, const lora_
   p.dx = dx;
   p.dA = dA;
   p.dB = dB;
-  if (!p.Wq.codes || !p.Wq.params) return LORA_ENULL;
-  return lora_stack_step(&p, 1, LORA_BWD, workspace, workspace_bytes, stream);
+  if (!p.Wq.codes || !p.Wq.params) return rec(LORA_ENULL);
+  return rec(lora_stack_step(&p, 1, LORA_BWD, workspace, workspace_bytes, stream));
 }
 
 int64_t lora_launch_count(void) { return (int64_t)g_launches.load(); }
@@ -1737,14 +1767,14 @@ int lora_profile_begin_kinds(uint32_t kind_mask) {
   g_prof.next = 0;
   g_prof.mask = kind_mask;
   g_prof.on = true;
-  return LORA_OK;
+  return rec(LORA_OK);
 }
 
 int lora_profile_begin(void) { return lora_profile_begin_kinds((1u << LORA_KERNEL_KINDS) - 1u); }
 
 int lora_profile_end(double* ms, int64_t* launches) {
   std::lock_guard<std::mutex> lk(g_prof_mu);
-  if (!g_prof.on) return LORA_EINVAL;
+  if (!g_prof.on) return rec(LORA_EINVAL);
   double acc[LORA_KERNEL_KINDS] = {0};
   int64_t cnt[LORA_KERNEL_KINDS] = {0};
   int rc = LORA_OK;
@@ -1764,26 +1794,26 @@ int lora_profile_end(double* ms, int64_t* launches) {
   g_prof.recs.clear();
   g_prof.next = 0;
   g_prof.on = false;
-  return rc;
+  return rec(rc);
 }
 
 int lora_stack_ckpt_workspace_size(const lora_proj* projs, int n_layers, int n_per_layer, size_t* bytes) {
-  if (!bytes) return LORA_ENULL;
+  if (!bytes) return rec(LORA_ENULL);
   size_t sb = 0, wb = 0;
   const int rc = ckpt_layout(projs, n_layers, n_per_layer, &sb, &wb);
-  if (rc != LORA_OK) return rc;
+  if (rc != LORA_OK) return rec(rc);
   *bytes = sb + wb;
-  return LORA_OK;
+  return rec(LORA_OK);
 }
 
 int lora_stack_ckpt(const lora_proj* projs, int n_layers, int n_per_layer, void* workspace, size_t workspace_bytes,
                     void* stream) {
   size_t sb = 0, wb = 0;
   int rc = ckpt_layout(projs, n_layers, n_per_layer, &sb, &wb);
-  if (rc != LORA_OK) return rc;
-  if ((rc = check_ws(workspace, workspace_bytes, sb + wb)) != LORA_OK) return rc;
+  if (rc != LORA_OK) return rec(rc);
+  if ((rc = check_ws(workspace, workspace_bytes, sb + wb)) != LORA_OK) return rec(rc);
   DeviceInfo* d = nullptr;
-  if ((rc = device_info(&d)) != LORA_OK) return rc;
+  if ((rc = device_info(&d)) != LORA_OK) return rec(rc);
   uint8_t* su_scratch = static_cast<uint8_t*>(workspace);
   void* step_ws = su_scratch + sb;
   std::vector<lora_proj> layer;
@@ -1791,44 +1821,44 @@ int lora_stack_ckpt(const lora_proj* projs, int n_layers, int n_per_layer, void*
   for (int l = 0; l < n_layers; ++l) {
     layer_copy(projs + (size_t)l * n_per_layer, n_per_layer, su_scratch, &layer);
     for (const lora_proj& p : layer) {
-      if ((rc = check_fwd_ptrs(p)) != LORA_OK) return rc;
-      if ((rc = check_bwd_ptrs(p)) != LORA_OK) return rc;
+      if ((rc = check_fwd_ptrs(p)) != LORA_OK) return rec(rc);
+      if ((rc = check_bwd_ptrs(p)) != LORA_OK) return rec(rc);
     }
   }
   // Stage I: every layer's forward, saving nothing
   for (int l = 0; l < n_layers; ++l) {
     layer_copy(projs + (size_t)l * n_per_layer, n_per_layer, nullptr, &layer);
-    if ((rc = lora_stack_step(layer.data(), n_per_layer, LORA_FWD, step_ws, wb, stream)) != LORA_OK) return rc;
+    if ((rc = lora_stack_step(layer.data(), n_per_layer, LORA_FWD, step_ws, wb, stream)) != LORA_OK) return rec(rc);
   }
   // Stage III: from the last layer back, re-run its forward saving su, then its backward
   for (int l = n_layers - 1; l >= 0; --l) {
     layer_copy(projs + (size_t)l * n_per_layer, n_per_layer, su_scratch, &layer);
-    if ((rc = lora_stack_step(layer.data(), n_per_layer, LORA_FWD_BWD, step_ws, wb, stream)) != LORA_OK) return rc;
+    if ((rc = lora_stack_step(layer.data(), n_per_layer, LORA_FWD_BWD, step_ws, wb, stream)) != LORA_OK) return rec(rc);
   }
-  return LORA_OK;
+  return rec(LORA_OK);
 }
 
 int lora_ce_workspace_size(const lora_ce_args* args, size_t* bytes) {
-  if (!bytes) return LORA_ENULL;
+  if (!bytes) return rec(LORA_ENULL);
   CePlan pl;
   const int rc = ce_check(args, &pl);
-  if (rc != LORA_OK) return rc;
+  if (rc != LORA_OK) return rec(rc);
   *bytes = pl.total;
-  return LORA_OK;
+  return rec(LORA_OK);
 }
 
 int lora_ce_fwd_bwd(const lora_ce_args* a, void* workspace, size_t workspace_bytes, void* stream) {
   CePlan pl;
   int rc = ce_check(a, &pl);
-  if (rc != LORA_OK) return rc;
-  if ((rc = check_ws(workspace, workspace_bytes, pl.total)) != LORA_OK) return rc;
+  if (rc != LORA_OK) return rec(rc);
+  if ((rc = check_ws(workspace, workspace_bytes, pl.total)) != LORA_OK) return rec(rc);
   DeviceInfo* d = nullptr;
-  if ((rc = device_info(&d)) != LORA_OK) return rc;
+  if ((rc = device_info(&d)) != LORA_OK) return rec(rc);
   cudaStream_t st = static_cast<cudaStream_t>(stream);
   const int T = (int)a->T, V = (int)a->V, D = (int)a->d;
   uint8_t* ws = static_cast<uint8_t*>(workspace);
   // tile counters, counts and vocabulary flags start at zero
-  if (cudaMemsetAsync(ws, 0, pl.flags + (size_t)V, st) != cudaSuccess) return LORA_ECUDA;
+  if (cudaMemsetAsync(ws, 0, pl.flags + (size_t)V, st) != cudaSuccess) return rec(LORA_ECUDA);
   CeIndex ix;
   ix.targets = a->targets;
   ix.mask = a->mask;
@@ -1845,13 +1875,13 @@ int lora_ce_fwd_bwd(const lora_ce_args* a, void* workspace, size_t workspace_byt
   ix.ycol = at<int32_t>(ws, pl.ycol);
   ix.counts = at<int32_t>(ws, pl.counts);
   ix.seg_counts = at<int32_t>(ws, pl.segs);
-  if (launch_ce_index(ix, st) != cudaSuccess) return LORA_ECUDA;
+  if (launch_ce_index(ix, st) != cudaSuccess) return rec(LORA_ECUDA);
   // |T_set| and |J| size the contractions
   int32_t counts[3] = {0, 0, 0};
   if (cudaMemcpyAsync(counts, ix.counts, sizeof(counts), cudaMemcpyDeviceToHost, st) != cudaSuccess ||
       cudaStreamSynchronize(st) != cudaSuccess)
-    return LORA_ECUDA;
-  if (counts[2]) return LORA_EINVAL;
+    return rec(LORA_ECUDA);
+  if (counts[2]) return rec(LORA_EINVAL);
   const int nT = counts[0], nJ = counts[1];
   if (a->counts) {
     a->counts[0] = nT;
@@ -1870,63 +1900,63 @@ int lora_ce_fwd_bwd(const lora_ce_args* a, void* workspace, size_t workspace_byt
     bf* ejw = at<bf>(ws, pl.ej);
     if (launch_gather_rows2(cb(a->h), D, ix.tl, nT, ht, cb(a->E), D, ix.J, nJ < V ? nJ : 0, ejw, D, st) !=
         cudaSuccess)
-      return LORA_ECUDA;
+      return rec(LORA_ECUDA);
     if (nJ < V) ej = ejw;
     {
       ProfScope ps(LORA_KERNEL_GEMM_FWD, st);
       if ((rc = ce_gemm(d, tiles, ht, D, ej, D, z, ldz, nT, nJ, D, false, true, at<float>(ws, pl.part), st, lse_part,
                         pl.ld_lse)) != LORA_OK)
-        return rc;
+        return rec(rc);
     }
     if (launch_ce_rows(lse_part, pl.ld_lse, z, ldz, nJ, ix.ycol, nT, at<float>(ws, pl.lse), rowloss, ix.tpos, T,
                        a->token_loss, a->loss, ix.counts + 5, g, ldg, d->num_sms, st) != cudaSuccess)
-      return LORA_ECUDA;
+      return rec(LORA_ECUDA);
     if (a->dh) {
       bf* dht = at<bf>(ws, pl.dht);
       ProfScope ps(LORA_KERNEL_GEMM_BWD, st);
       if ((rc = ce_gemm(d, tiles + 1, g, ldg, ej, D, dht, D, nT, D, nJ, true, false, at<float>(ws, pl.part), st)) !=
           LORA_OK)
-        return rc;
+        return rec(rc);
     }
   }
   // with trainable positions the log-sum-exp launch's last block has written the losses
   if (nT == 0 && launch_ce_finish(rowloss, nT, ix.tpos, T, a->token_loss, a->loss, st) != cudaSuccess)
-    return LORA_ECUDA;
+    return rec(LORA_ECUDA);
   if (a->dh && launch_scatter_rows(at<bf>(ws, pl.dht), ix.tpos, T, D, mb(a->dh), st) != cudaSuccess)
-    return LORA_ECUDA;
+    return rec(LORA_ECUDA);
   if (a->vocab && nJ > 0 &&
       cudaMemcpyAsync(a->vocab, ix.J, (size_t)nJ * 4, cudaMemcpyDeviceToDevice, st) != cudaSuccess)
-    return LORA_ECUDA;
-  return LORA_OK;
+    return rec(LORA_ECUDA);
+  return rec(LORA_OK);
 }
 
 int lora_topk_workspace_size(int64_t V, int64_t d, int64_t k, size_t* bytes) {
-  if (!bytes) return LORA_ENULL;
+  if (!bytes) return rec(LORA_ENULL);
   TopkPlan pl;
   const int rc = topk_check(nullptr, V, d, k, &pl);
-  if (rc != LORA_OK) return rc;
+  if (rc != LORA_OK) return rec(rc);
   *bytes = pl.total;
-  return LORA_OK;
+  return rec(LORA_OK);
 }
 
 int lora_topk_table(const lora_bf16* E, int64_t V, int64_t d, int64_t k, int32_t* table, void* workspace,
                     size_t workspace_bytes, void* stream) {
-  if (!E || !table) return LORA_ENULL;
+  if (!E || !table) return rec(LORA_ENULL);
   TopkPlan pl;
   int rc = topk_check(E, V, d, k, &pl);
-  if (rc != LORA_OK) return rc;
-  if ((rc = check_ws(workspace, workspace_bytes, pl.total)) != LORA_OK) return rc;
+  if (rc != LORA_OK) return rec(rc);
+  if ((rc = check_ws(workspace, workspace_bytes, pl.total)) != LORA_OK) return rec(rc);
   DeviceInfo* dv = nullptr;
-  if ((rc = device_info(&dv)) != LORA_OK) return rc;
+  if ((rc = device_info(&dv)) != LORA_OK) return rec(rc);
   cudaStream_t st = static_cast<cudaStream_t>(stream);
   uint8_t* ws = static_cast<uint8_t*>(workspace);
-  if (cudaMemsetAsync(ws, 0, pl.en, st) != cudaSuccess) return LORA_ECUDA;  // counters, status, counts
+  if (cudaMemsetAsync(ws, 0, pl.en, st) != cudaSuccess) return rec(LORA_ECUDA);  // counters, status, counts
   bf* en = at<bf>(ws, pl.en);
   float* S = at<float>(ws, pl.s);
   int* ctr = at<int>(ws, pl.counters);
   float* part = at<float>(ws, pl.part);
   const int D = (int)d;
-  if (launch_normalize_rows(cb(E), (int)V, D, en, st) != cudaSuccess) return LORA_ECUDA;
+  if (launch_normalize_rows(cb(E), (int)V, D, en, st) != cudaSuccess) return rec(LORA_ECUDA);
   if (!pl.sampled) {
     for (int c = 0; c < pl.chunks; ++c) {
       const int64_t r0 = (int64_t)c * kTopkChunk, rows = std::min<int64_t>(kTopkChunk, V - r0);
@@ -1934,13 +1964,13 @@ int lora_topk_table(const lora_bf16* E, int64_t V, int64_t d, int64_t k, int32_t
         ProfScope ps(LORA_KERNEL_GEMM_FWD, st);
         if ((rc = ce_gemm(dv, ctr + c, en + r0 * d, d, en, d, S, pl.lds, rows, V, d, false, true, part, st)) !=
             LORA_OK)
-          return rc;
+          return rec(rc);
       }
       if (launch_topk_select(S, pl.lds, (int)V, (int)k, (int)r0, nullptr, (int)rows, table, dv->status, st) !=
           cudaSuccess)
-        return LORA_ECUDA;
+        return rec(LORA_ECUDA);
     }
-    return LORA_OK;
+    return rec(LORA_OK);
   }
   // sampled path: thresholds from the similarities to the sample tokens
   bf* es = at<bf>(ws, pl.es);
@@ -1952,16 +1982,16 @@ int lora_topk_table(const lora_bf16* E, int64_t V, int64_t d, int64_t k, int32_t
   int* fail_count = at<int>(ws, pl.fail_count);
   const int ns = topk_sample();
   int next = 0;
-  if (launch_topk_gather_sample(en, (int)V, D, es, dv->num_sms, st) != cudaSuccess) return LORA_ECUDA;
+  if (launch_topk_gather_sample(en, (int)V, D, es, dv->num_sms, st) != cudaSuccess) return rec(LORA_ECUDA);
   for (int b = 0; b < pl.sblocks; ++b) {
     const int64_t r0 = (int64_t)b * kTopkSampleRows, rows = std::min<int64_t>(kTopkSampleRows, V - r0);
     {
       ProfScope ps(LORA_KERNEL_GEMM_FWD, st);
       if ((rc = ce_gemm(dv, ctr + next++, en + r0 * d, d, es, d, zs, ns, rows, ns, d, false, true, part, st)) !=
           LORA_OK)
-        return rc;
+        return rec(rc);
     }
-    if (launch_topk_tau(zs, (int)V, (int)k, (int)rows, tau + r0, st) != cudaSuccess) return LORA_ECUDA;
+    if (launch_topk_tau(zs, (int)V, (int)k, (int)rows, tau + r0, st) != cudaSuccess) return rec(LORA_ECUDA);
   }
   // the upper triangle of the similarities (C is symmetric), every value offered to both of
   // its rows' lists against their thresholds; then each row's list is sorted
@@ -1969,50 +1999,50 @@ int lora_topk_table(const lora_bf16* E, int64_t V, int64_t d, int64_t k, int32_t
     const int64_t r0 = (int64_t)c * kTopkAppendRows, rows = std::min<int64_t>(kTopkAppendRows, V - r0);
     ProfScope ps(LORA_KERNEL_GEMM_FWD, st);
     if ((rc = topk_sym_gemm(dv, ctr + next++, en, d, V, r0, rows, tau, cnt, cand, topk_cap(), st)) != LORA_OK)
-      return rc;
+      return rec(rc);
   }
   if (launch_topk_sort(cand, cnt, topk_cap(), (int)k, 0, (int)V, table, at<int32_t>(ws, pl.big_rows),
                        at<int>(ws, pl.big_count), fail_rows, fail_count, dv->num_sms, st) != cudaSuccess)
-    return LORA_ECUDA;
+    return rec(LORA_ECUDA);
   // rows whose threshold left too few or too many candidates: the exact materialised path
   int nf = 0;
   if (cudaMemcpyAsync(&nf, fail_count, sizeof(int), cudaMemcpyDeviceToHost, st) != cudaSuccess ||
       cudaStreamSynchronize(st) != cudaSuccess)
-    return LORA_ECUDA;
+    return rec(LORA_ECUDA);
   for (int f0 = 0; f0 < nf; f0 += kTopkChunk) {
     const int n = std::min(kTopkChunk, nf - f0);
-    if (launch_gather_rows(en, d, fail_rows + f0, n, D, es, st) != cudaSuccess) return LORA_ECUDA;
+    if (launch_gather_rows(en, d, fail_rows + f0, n, D, es, st) != cudaSuccess) return rec(LORA_ECUDA);
     {
       ProfScope ps(LORA_KERNEL_GEMM_FWD, st);
       if ((rc = ce_gemm(dv, ctr + next++, es, d, en, d, S, pl.lds, n, V, d, false, true, part, st)) != LORA_OK)
-        return rc;
+        return rec(rc);
     }
     if (launch_topk_select(S, pl.lds, (int)V, (int)k, 0, fail_rows + f0, n, table, dv->status, st) != cudaSuccess)
-      return LORA_ECUDA;
+      return rec(LORA_ECUDA);
   }
-  return LORA_OK;
+  return rec(LORA_OK);
 }
 
 int lora_wait_selftest(int64_t limit_ns, void* stream) {
-  if (limit_ns < 1000 || limit_ns > 1000000000ll) return LORA_EINVAL;
+  if (limit_ns < 1000 || limit_ns > 1000000000ll) return rec(LORA_EINVAL);
   DeviceInfo* d = nullptr;
   int rc = device_info(&d);
-  if (rc != LORA_OK) return rc;
+  if (rc != LORA_OK) return rec(rc);
   return launch_wait_probe(d->status, limit_ns, static_cast<cudaStream_t>(stream)) == cudaSuccess ? LORA_OK
                                                                                                     : LORA_ECUDA;
 }
 
 int lora_read_status(void* stream, int* status, int reset) {
-  if (!status) return LORA_ENULL;
-  if (cudaStreamSynchronize(static_cast<cudaStream_t>(stream)) != cudaSuccess) return LORA_ECUDA;
+  if (!status) return rec(LORA_ENULL);
+  if (cudaStreamSynchronize(static_cast<cudaStream_t>(stream)) != cudaSuccess) return rec(LORA_ECUDA);
   int v = 0;
-  if (cudaMemcpyFromSymbol(&v, g_status, sizeof(int)) != cudaSuccess) return LORA_ECUDA;
+  if (cudaMemcpyFromSymbol(&v, g_status, sizeof(int)) != cudaSuccess) return rec(LORA_ECUDA);
   if (reset) {
     const int z = 0;
-    if (cudaMemcpyToSymbol(g_status, &z, sizeof(int)) != cudaSuccess) return LORA_ECUDA;
+    if (cudaMemcpyToSymbol(g_status, &z, sizeof(int)) != cudaSuccess) return rec(LORA_ECUDA);
   }
   *status = v == 0 ? LORA_OK : v == kStatusTopkTies ? LORA_EINVAL : LORA_ETIMEOUT;
-  return LORA_OK;
+  return rec(LORA_OK);
 }
 
 }  // extern "C"
@@ -2041,10 +2071,10 @@ void* g_noalloc_addr[kMaxDevices] = {};
 extern "C" int lora_linear_fwd_noalloc(const lora_shape* shape, const lora_bf16* x, const lora_bf16* W,
                                        const lora_bf16* A, const lora_bf16* B, lora_bf16* y, lora_bf16* su,
                                        void* stream) {
-  if (!shape) return LORA_ENULL;
+  if (!shape) return rec(LORA_ENULL);
   DeviceInfo* d = nullptr;
   int rc = device_info(&d);
-  if (rc != LORA_OK) return rc;
+  if (rc != LORA_OK) return rec(rc);
   lora_proj p;
   memset(&p, 0, sizeof(p));
   p.shape = *shape;
@@ -2055,22 +2085,22 @@ extern "C" int lora_linear_fwd_noalloc(const lora_shape* shape, const lora_bf16*
   p.y = y;
   p.su = su;
   Plan pl;
-  if ((rc = plan_all(&p, 1, LORA_FWD, &pl, false)) != LORA_OK) return rc;
-  if (pl.total > kNoAllocScratchBytes) return LORA_ESCRATCH;
-  if ((rc = check_fwd_ptrs(p)) != LORA_OK) return rc;
+  if ((rc = plan_all(&p, 1, LORA_FWD, &pl, false)) != LORA_OK) return rec(rc);
+  if ((rc = check_fwd_ptrs(p)) != LORA_OK) return rec(rc);  // argument errors first, as lora_stack_step
+  if (pl.total > kNoAllocScratchBytes) return rec(LORA_ESCRATCH);
   int dev = 0;
-  if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= kMaxDevices) return LORA_ECUDA;
+  if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= kMaxDevices) return rec(LORA_ECUDA);
   void* scratch = nullptr;
   {
     // first call on this device (with it current): find the array's device address
     std::lock_guard<std::mutex> lk(g_noalloc_mu);
     if (g_noalloc_addr[dev] == nullptr) {
       void* a = nullptr;
-      if (cudaGetSymbolAddress(&a, g_noalloc_scratch) != cudaSuccess || a == nullptr) return LORA_ECUDA;
+      if (cudaGetSymbolAddress(&a, g_noalloc_scratch) != cudaSuccess || a == nullptr) return rec(LORA_ECUDA);
       g_noalloc_addr[dev] = a;
     }
     scratch = g_noalloc_addr[dev];
   }
   // run_step clears the part of the scratch that must start at zero
-  return run_step(&p, 1, LORA_FWD, scratch, pl, d, static_cast<cudaStream_t>(stream));
+  return rec(run_step(&p, 1, LORA_FWD, scratch, pl, d, static_cast<cudaStream_t>(stream)));
 }

@@ -96,6 +96,7 @@ struct Cfg {
 };
 constexpr int kTileRing = 4;  // tile ids handed from the scheduler to the other roles
 constexpr long long kDrainNs = 1000000000ll;
+constexpr long long kAbortDrainNs = 10000000ll;  // 10 ms per armed stage on the abort path
 
 struct __align__(8) Ctl {
   uint64_t full[kMaxStages];       // even CTA: both CTAs' parts of a stage landed
@@ -113,6 +114,8 @@ struct __align__(8) Ctl {
   int tile_id[kTileRing];
   uint32_t tmem_base;
   int abort;
+  int fills;   // ring stages this CTA's producer armed (expect_tx on the even CTA's barriers)
+  int qfills;  // 4-bit: code slots this CTA's code producer armed
 };
 
 template <bool kQ>
@@ -256,6 +259,8 @@ __global__ void __launch_bounds__(Cfg<kQ>::kThreads, 1) fused_lora_gemm(const __
     }
     mbar_init(smem_u32(&ctl->drain), 1);
     ctl->abort = 0;
+    ctl->fills = 0;
+    ctl->qfills = 0;
     fence_mbar_init();
   }
   if (warp == 0 && lane == 0) {
@@ -290,6 +295,7 @@ __global__ void __launch_bounds__(Cfg<kQ>::kThreads, 1) fused_lora_gemm(const __
       const uint32_t full_pl = mapa_shared(smem_u32(&ctl->full[0]), 0);
       int stage = 0;
       uint32_t phase = 0;
+      int fills = 0;
       for (int it = 0;; ++it) {
         const int slot = it % kTileRing;
         const uint32_t par = (uint32_t)((it / kTileRing) & 1);
@@ -335,6 +341,7 @@ __global__ void __launch_bounds__(Cfg<kQ>::kThreads, 1) fused_lora_gemm(const __
           // with 4-bit weights the dequantizing warps fill the weight tiles
           const bool w_tma = !kQ;
           if (c == 0) mbar_arrive_expect_tx(smem_u32(&ctl->full[stage]), w_tma ? tx_pair : tx_a);
+          ++fills;
           const uint32_t bar = full_pl + (uint32_t)stage * 8u;
           const uint32_t a_dst = a_addr_of(base, stage);
           const uint32_t b_dst = a_dst + kAHalf;
@@ -360,6 +367,7 @@ __global__ void __launch_bounds__(Cfg<kQ>::kThreads, 1) fused_lora_gemm(const __
         }
         if (!ok) break;
       }
+      ctl->fills = fills;
     }
   } else if (warp == 1) {
     // ------------------------------------------------------------ MMA issuer (even CTA)
@@ -737,6 +745,7 @@ __global__ void __launch_bounds__(Cfg<kQ>::kThreads, 1) fused_lora_gemm(const __
     if (lane == 0) {
       int qs = 0;
       uint32_t qpar = 0;
+      int qfills = 0;
       for (int it = 0;; ++it) {
         const int slot = it % kTileRing;
         if (!mbar_wait_cluster(smem_u32(&ctl->tile_full[slot]), (uint32_t)((it / kTileRing) & 1), wc, abort_flag))
@@ -768,6 +777,7 @@ __global__ void __launch_bounds__(Cfg<kQ>::kThreads, 1) fused_lora_gemm(const __
           const uint32_t codes = Cfg<kQ>::q_slot(base, qs);
           const uint32_t params = codes + kQCodes;
           mbar_arrive_expect_tx(qbar, tx_q);
+          ++qfills;
           for (int h = 0; h < 2; ++h) {
             const int colh = n0 + h * kSeg + c * kHalf;
             if (!box_ok(h, 0)) continue;
@@ -788,6 +798,7 @@ __global__ void __launch_bounds__(Cfg<kQ>::kThreads, 1) fused_lora_gemm(const __
         }
         if (!ok) break;
       }
+      ctl->qfills = qfills;
     }
   }
 
@@ -799,7 +810,20 @@ __global__ void __launch_bounds__(Cfg<kQ>::kThreads, 1) fused_lora_gemm(const __
     if (!mbar_wait_drain(smem_u32(&ctl->drain), 0, b.limit_ns > kDrainNs ? b.limit_ns : kDrainNs))
       atomicCAS(b.status, 0, kStatusTimeout);
     if (*abort_flag) {
-      // a wait gave up: give copies still in flight time to land (bounded)
+      // A wait gave up, so copies may still be in flight into this CTA's ring.  The barriers
+      // armed here track them: wait (bounded, kAbortDrainNs each) until the last fill of every
+      // ring stage (even CTA: both CTAs' operand boxes) and of every code slot (4-bit) has
+      // landed.  Copies that signal the peer's barriers, or that were issued for a fill that was
+      // never armed, are not observable here: a fixed 50 us margin follows for those.
+      const int nf = ctl->fills, nq = ctl->qfills;
+      if (c == 0)
+        for (int i = nf - 1; i >= 0 && i >= nf - kStages; --i)
+          if (!mbar_wait_drain(smem_u32(&ctl->full[i % kStages]), (uint32_t)((i / kStages) & 1), kAbortDrainNs))
+            atomicCAS(b.status, 0, kStatusTimeout);
+      if (kQ)
+        for (int i = nq - 1; i >= 0 && i >= nq - kQStages; --i)
+          if (!mbar_wait_drain(smem_u32(&ctl->qfull[i % kQStages]), (uint32_t)((i / kQStages) & 1), kAbortDrainNs))
+            atomicCAS(b.status, 0, kStatusTimeout);
       const uint64_t t0 = global_timer_ns();
       while (global_timer_ns() - t0 < 50000ull) {
       }

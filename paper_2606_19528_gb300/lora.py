@@ -36,7 +36,8 @@ EXPORTS = ("lora_workspace_size", "lora_linear_fwd", "lora_linear_fwd_noalloc", 
            "lora_stack_step", "lora_stack_ckpt_workspace_size", "lora_stack_ckpt", "lora_ce_workspace_size",
            "lora_ce_fwd_bwd", "lora_topk_workspace_size", "lora_topk_table", "lora_wait_selftest",
            "lora_read_status", "lora_set_wait_limit_ns", "lora_launch_count",
-           "lora_profile_begin", "lora_profile_begin_kinds", "lora_profile_end", "lora_strerror", "lora_version")
+           "lora_profile_begin", "lora_profile_begin_kinds", "lora_profile_end", "lora_strerror", "lora_version",
+           "lora_last_error")
 
 LORA_KERNEL_GEMM_FWD = 0
 LORA_KERNEL_GEMM_BWD = 1
@@ -112,6 +113,7 @@ def library(path: str = _LIB_PATH) -> ctypes.CDLL:
         lib.lora_strerror.argtypes = [i32]
         lib.lora_strerror.restype = ctypes.c_char_p
         lib.lora_version.argtypes = []
+        lib.lora_last_error.argtypes = []
         for name in EXPORTS:
             if name != "lora_strerror":
                 getattr(lib, name).restype = i32
@@ -317,3 +319,8 @@ def lora_strerror(code: int) -> str:
 
 def lora_version() -> int:
     return library().lora_version()
+
+
+def lora_last_error() -> int:
+    """The code this thread's most recent library call returned (include/lora.h)."""
+    return int(library().lora_last_error())

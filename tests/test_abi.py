@@ -135,3 +135,42 @@ def test_forward_and_backward_plan_their_splits_for_the_contractions_sms(lib):
     fwd = lora.lora_workspace_size(st, lora.LORA_FWD)
     both = lora.lora_workspace_size(st, lora.LORA_FWD_BWD)
     assert fwd > 0 and both > fwd
+
+
+def test_last_error_follows_the_threads_latest_call(lib):
+    """lora_last_error repeats the code of the calling thread's latest call,
+    successes included, and is per thread."""
+    import threading
+    n = ctypes.c_size_t(0)
+    assert lib.lora_workspace_size(None, 1, ctypes.byref(n)) == lora.LORA_ENULL
+    assert lora.lora_last_error() == lora.LORA_ENULL
+    st = lora.make_shape(128, 256, 256, 8, 2.0)
+    assert lib.lora_workspace_size(ctypes.byref(st), 9, ctypes.byref(n)) == lora.LORA_EINVAL
+    assert lora.lora_last_error() == lora.LORA_EINVAL
+    seen = []
+    t = threading.Thread(target=lambda: seen.append(lora.lora_last_error()))
+    t.start()
+    t.join()
+    assert seen == [lora.LORA_OK], "another thread's calls do not show"
+    assert lib.lora_workspace_size(ctypes.byref(st), 1, ctypes.byref(n)) == lora.LORA_OK
+    assert lora.lora_last_error() == lora.LORA_OK
+    lora.lora_strerror(-1)  # does not record
+    assert lora.lora_last_error() == lora.LORA_OK
+
+
+def test_frozen_projection_plans_no_rank_work(lib):
+    """Rank 0 is a frozen projection: no adapter, so its workspace holds no
+    rank-r scratch, only the tile counters (and split partials where its
+    contraction splits); a negative rank is rejected."""
+    big = lora.make_shape(4096, 3072, 3072, 0, 1.0)  # 96 tiles: no split
+    assert lora.lora_workspace_size(big, lora.LORA_FWD_BWD) <= 4096
+    adapted = lora.lora_workspace_size(lora.make_shape(4096, 3072, 3072, 16, 2.0), lora.LORA_FWD_BWD)
+    assert adapted > 4 * 4096 * 16 * 2
+    n = ctypes.c_size_t(0)
+    bad = lora.make_shape(128, 256, 256, -1, 1.0)
+    assert lib.lora_workspace_size(ctypes.byref(bad), 3, ctypes.byref(n)) == lora.LORA_EINVAL
+    # a layer adapting q and v only: the frozen projections add nothing beyond their split partials
+    layer = [lora.make_proj(lora.make_shape(4096, 3072, 3072, r, 2.0)) for r in (16, 0, 16, 0)]
+    two = [lora.make_proj(lora.make_shape(4096, 3072, 3072, 16, 2.0)) for _ in range(2)]
+    assert lora.lora_stack_workspace_size(layer, lora.LORA_FWD_BWD) == lora.lora_stack_workspace_size(
+        two, lora.LORA_FWD_BWD)

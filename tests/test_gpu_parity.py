@@ -107,21 +107,55 @@ def test_single_small_T128():
     check_full(p)
 
 
-def test_init_invariant_B0():
-    """B = 0: dA is exactly zero, and y and dx do not depend on the rank of
-    the (all-zero) adapter slab: runs with r = 8 and r = 16 agree bit for bit."""
+def run_frozen(x_bits, W_bits, dy_bits):
+    """The same contraction kernel with no adapter slab at all (rank 0: a
+    frozen projection): y = x W^T and dx = dy W.  Returns (y, dx)."""
+    T, K = x_bits.shape
+    N = W_bits.shape[0]
+    x, W, dy = G.dev_bf16(x_bits), G.dev_bf16(W_bits), G.dev_bf16(dy_bits)
+    y = torch.full((T, N), float("nan"), dtype=torch.bfloat16, device="cuda")
+    dx = torch.full((T, K), float("nan"), dtype=torch.bfloat16, device="cuda")
+    st = lora.make_shape(T, K, N, 0, 1.0)
+    ws = G.workspace(lora.lora_workspace_size(st, lora.LORA_FWD_BWD))
+    lora.lora_linear_fwd(st, x, W, None, None, y, None, ws, ws.numel())
+    lora.lora_linear_bwd(st, dy, x, W, None, None, None, dx, None, None, ws, ws.numel())
+    torch.cuda.synchronize()
+    assert lora.lora_read_status() == lora.LORA_OK
+    return y, dx
+
+
+@pytest.mark.parametrize("T,K,N", [(128, 256, 256), (264, 200, 520), (512, 3072, 1024)])
+def test_init_invariant_B0(T, K, N):
+    """B = 0 (LoRA initialisation): dA is exactly zero, and y and dx are bit
+    for bit those of the same contraction with the adapter slab skipped
+    (rank 0): the slab adds exact zeros to the fp32 accumulator.  Ranks 8 and
+    16 (slabs of one 64-deep block, different fill) and a padded rank 3; the
+    first shape is the single-projection workload with its B = 0 twin."""
     wl = workloads.single_small(zero_B=True)
-    pr = wl.projs[0]
-    outs = []
-    for r in (8, 16):
-        x, W, A, B, dy = gen_proj(wl.cfg, 0, 0, wl.T, pr.d_in, pr.d_out, r, wl.scale, zero_B=True)
+    x, W, _, _, dy = gen_proj(wl.cfg, 0, 0, T, K, N, 8, wl.scale, zero_B=True)
+    y0, dx0 = run_frozen(x, W, dy)
+    for r in (8, 16, 3):
+        _, _, A, B, _ = gen_proj(wl.cfg, 0, 0, T, K, N, r, 16.0 / r, zero_B=True)
         p = G.DevProj(x, W, A, B, dy, 16.0 / r)
         G.run_single(p)
         assert not torch.any(p.dA != 0), "dA must be exactly 0 when B = 0"
         check_full(p)
-        outs.append((p.y.clone(), p.dx.clone()))
-    assert torch.equal(outs[0][0].view(torch.int16), outs[1][0].view(torch.int16))
-    assert torch.equal(outs[0][1].view(torch.int16), outs[1][1].view(torch.int16))
+        assert torch.equal(p.y.view(torch.int16), y0.view(torch.int16)), r
+        assert torch.equal(p.dx.view(torch.int16), dx0.view(torch.int16)), r
+
+
+def test_frozen_projection_against_oracle():
+    """Rank 0 is a frozen linear: y = x W^T and dx = dy W against the oracle
+    (whose adapter terms are empty), ragged tiles in every dimension."""
+    T, K, N = 264, 1032, 392
+    x, W, _, _, dy = gen_proj(30, 0, 0, T, K, N, 1, 1.0)
+    y, dx = run_frozen(x, W, dy)
+    xf, Wf, dyf = (synth.bf16_bits_to_f64(b) for b in (x, W, dy))
+    A0, B0 = np.zeros((0, K)), np.zeros((N, 0))
+    y_want, _ = oracle.lora_forward(xf, Wf, A0, B0, 1.0)
+    dx_want, _, _, _ = oracle.lora_backward(dyf, xf, Wf, A0, B0, 1.0)
+    assert G.rel_fro(G.host_f64(y), y_want) <= G.TOL_Y
+    assert G.rel_fro(G.host_f64(dx), dx_want) <= G.TOL_DX
 
 
 # --------------------------------------------------------------- ragged shapes
@@ -198,12 +232,54 @@ def build_layer(wl, layer=0, seed=0):
 
 @pytest.mark.parametrize("name", ["llama_layer", "qwen_layer"])
 def test_layer_stack(name):
+    """The Llama-3.2-3B-shaped layer at T = 2048, r = 16 and the
+    Qwen-2.5-3B-shaped layer at T = 4096, r = 64, in the launch
+    configuration the benchmark times (one forward-and-backward call, side
+    stream): every element of y, su, dx, dA and dB against the fp64 oracle."""
     wl = workloads.BY_NAME[name]()
     ps = build_layer(wl)
     G.run_stack(ps)
-    rows = G.sample_rows(wl.T, 64, 11)
     for p in ps:
-        check_sampled(p, rows)
+        check_full(p)
+        for t in (p.y, p.su, p.dx, p.dA, p.dB):
+            assert not torch.isnan(t).any(), "an output element was never written"
+
+
+def test_layer_adapting_q_and_v_only():
+    """The paper's own setting: adapters on q and v only (hyper-parameter
+    table), the other five projections frozen (rank 0) but still on the
+    backward path through dx.  One call over the Llama-shaped layer at
+    T = 512: the adapted projections against the oracle in full, the frozen
+    ones as y = x W^T and dx = dy W, and dA / dB of the frozen ones untouched."""
+    T, r, s = 512, 16, 2.0
+    ps, xs, frozen = [], {}, []
+    for i, pr in enumerate(workloads.llama_layer()):
+        rr = r if pr.name in ("q", "v") else 0
+        bits = gen_proj(31, i, 0, T, pr.d_in, pr.d_out, max(rr, 1), s, group=pr.group)
+        if rr == 0:
+            bits = (bits[0], bits[1], np.zeros((0, pr.d_in), np.uint16), np.zeros((pr.d_out, 0), np.uint16),
+                    bits[4])
+        p = G.DevProj(*bits, s, share_x=xs.get(pr.group))
+        xs.setdefault(pr.group, p.x)
+        ps.append(p)
+        frozen.append(rr == 0)
+    projs = []
+    for p, fz in zip(ps, frozen):
+        if fz:
+            projs.append(lora.make_proj(p.shape, x=p.x, W=p.W, dy=p.dy, y=p.y, dx=p.dx))
+        else:
+            projs.append(p.proj())
+    ws = G.workspace(lora.lora_stack_workspace_size(projs, lora.LORA_FWD_BWD))
+    lora.lora_stack_step(projs, lora.LORA_FWD_BWD, ws, ws.numel())
+    torch.cuda.synchronize()
+    assert lora.lora_read_status() == lora.LORA_OK
+    for p, fz in zip(ps, frozen):
+        if not fz:
+            check_full(p)
+            continue
+        x, W, dy = (p.f64(k) for k in ("x", "W", "dy"))
+        assert G.rel_fro(G.host_f64(p.y), x @ W.T) <= G.TOL_Y
+        assert G.rel_fro(G.host_f64(p.dx), dy @ W) <= G.TOL_DX
 
 
 def test_stack_equals_single_calls():
@@ -317,6 +393,14 @@ def test_argument_errors():
     with pytest.raises(lora.LoraError) as e:
         lora.lora_linear_bwd(st, p.dy, p.x, p.W, p.A, p.B, None, p.dx, p.dA, p.dB, ws, need)
     assert e.value.code == lora.LORA_ENULL
+    assert lora.lora_last_error() == lora.LORA_ENULL
+    lora.lora_linear_fwd(st, p.x, p.W, p.A, p.B, p.y, p.su, ws, need)
+    assert lora.lora_last_error() == lora.LORA_OK
+    torch.cuda.synchronize()
+    p.y.fill_(float("nan"))
+    with pytest.raises(lora.LoraError) as e:
+        lora.lora_linear_fwd(st, p.x, p.W, None, p.B, p.y, p.su, ws, need)  # rank 8 needs A
+    assert e.value.code == lora.LORA_ENULL
     torch.cuda.synchronize()
     assert torch.isnan(p.y).all(), "a rejected call must enqueue nothing"
 
@@ -335,3 +419,47 @@ def test_bounded_wait_expires_and_context_survives():
     p = G.DevProj(*gen_proj(0, 7, 0, 128, 256, 256, 8, s), s)
     G.run_single(p)
     check_full(p)
+
+
+# --------------------------------------------------------------- data-parallel sharding identity
+
+def test_token_shards_sum_to_the_unsharded_gradients():
+    """The token sharding of a data-parallel step, run one shard after the
+    other on one GPU: each shard's y, su and dx are the matching rows of the
+    unsharded call's (within rounding: the contractions may split
+    differently), and the shards' dA and dB summed through the all-reduce
+    hook (here a local sum of the shards' buffers) equal the unsharded
+    gradients to fp32 rounding; both against the oracle."""
+    from paper_2606_19528_gb300 import shard
+    T, K, N, r, s, world = 1032, 1024, 768, 16, 2.0, 3
+    bits = gen_proj(32, 0, 0, T, K, N, r, s)
+    full = G.DevProj(*bits, s)
+    G.run_single(full)
+    check_full(full)
+    x, W, A, B, dy = bits
+    parts = []
+    for rank in range(world):
+        t0, t1 = shard.token_slice(T, rank, world)
+        p = G.DevProj(x[t0:t1], W, A, B, dy[t0:t1], s)
+        G.run_single(p)
+        for n in ("y", "su", "dx"):
+            assert G.rel_fro(G.host_f64(getattr(p, n)), G.host_f64(getattr(full, n))[t0:t1]) <= 2e-3, (rank, n)
+        parts.append(p)
+    grads = [[p.dA.clone(), p.dB.clone()] for p in parts]
+
+    def hook_for(rank):
+        def hook(buf):  # sums the packed buffers of every shard, as an all-reduce would
+            packed = [torch.cat([g.reshape(-1) for g in gs]) for gs in grads]
+            buf.copy_(torch.stack(packed).sum(0))
+        return hook
+
+    summed = [[g.clone() for g in gs] for gs in grads]
+    for rank in range(world):
+        shard.sum_adapter_grads(summed[rank], hook_for(rank))
+    for rank in range(world):
+        assert G.rel_fro(G.host_f64(summed[rank][0]), G.host_f64(full.dA)) < 1e-6
+        assert G.rel_fro(G.host_f64(summed[rank][1]), G.host_f64(full.dB)) < 1e-6
+        assert torch.equal(summed[rank][0], summed[0][0]) and torch.equal(summed[rank][1], summed[0][1])
+    dA, dB = oracle.lora_adapter_grads(full.f64("dy"), full.f64("x"), full.f64("A"), full.f64("B"), s)
+    assert G.rel_fro(G.host_f64(summed[0][0]), dA) <= G.TOL_GRAD
+    assert G.rel_fro(G.host_f64(summed[0][1]), dB) <= G.TOL_GRAD
