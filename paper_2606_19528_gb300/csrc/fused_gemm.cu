@@ -585,6 +585,21 @@ __global__ void __launch_bounds__(Cfg<kQ>::kThreads, 1) fused_lora_gemm(const __
           tmem_ld_32x32b_x32(taddr, v);
           if (!f32) tmem_ld_32x32b_x32(taddr + 32u, w);
           tmem_ld_wait();
+          if (Q.splits > 1) {
+            // fp32 partial of one split: each thread stores its row's 32 values (one 128-byte
+            // line) straight from registers into the tile-padded partial buffer, kept in L2
+            // for the reduce; no staging, so consecutive blocks' stores overlap
+            if (row0 + lane < Q.M) {
+              float* dst = Q.part + ((size_t)row_st + lane) * Q.ldp + n0 + col0;
+#pragma unroll
+              for (int k = 0; k < 8; ++k)
+                if (n0 + col0 + 4 * k < Q.N)
+                  __stcg(reinterpret_cast<float4*>(dst + 4 * k),
+                         make_float4(__uint_as_float(v[4 * k]), __uint_as_float(v[4 * k + 1]),
+                                     __uint_as_float(v[4 * k + 2]), __uint_as_float(v[4 * k + 3])));
+            }
+            continue;
+          }
           if (lse_on) {
             const int nv = min(32, Q.N - (n0 + col0));  // valid columns of the block, >= 1
             float bm = __uint_as_float(v[0]);
