@@ -439,10 +439,10 @@ def test_token_shards_sum_to_the_unsharded_gradients():
     unsharded call's (within rounding: the contractions may split
     differently), and the shards' dA and dB summed through the all-reduce
     hook (here a local sum of the shards' buffers) equal the unsharded
-    gradients up to the bf16 rounding of sv (its fp32 sums over d_out are cut
+    gradients up to the bf16 rounding of sv and su (their fp32 sums are cut
     differently for a shard, so an element may round to the neighbouring
-    bf16 value, ~1e-5 relative in dA) and fp32 rounding; both against the
-    oracle."""
+    bf16 value, ~1e-5 relative in dA and dB) and fp32 rounding; both against
+    the oracle."""
     from paper_2606_19528_gb300 import shard
     T, K, N, r, s, world = 1032, 1024, 768, 16, 2.0, 3
     bits = gen_proj(32, 0, 0, T, K, N, r, s)
@@ -471,7 +471,7 @@ def test_token_shards_sum_to_the_unsharded_gradients():
         shard.sum_adapter_grads(summed[rank], hook_for(rank))
     for rank in range(world):
         assert G.rel_fro(G.host_f64(summed[rank][0]), G.host_f64(full.dA)) < 1e-4
-        assert G.rel_fro(G.host_f64(summed[rank][1]), G.host_f64(full.dB)) < 1e-6
+        assert G.rel_fro(G.host_f64(summed[rank][1]), G.host_f64(full.dB)) < 1e-4
         assert torch.equal(summed[rank][0], summed[0][0]) and torch.equal(summed[rank][1], summed[0][1])
     dA, dB = oracle.lora_adapter_grads(full.f64("dy"), full.f64("x"), full.f64("A"), full.f64("B"), s)
     assert G.rel_fro(G.host_f64(summed[0][0]), dA) <= G.TOL_GRAD
