@@ -365,6 +365,38 @@ void choose_splits(const GemmBatch& b, int* splits, int pairs = kPlanPairs) {
   cache.emplace(key, best);
 }
 
+// Cluster split for launches with too few output tiles to fill the GPU: when
+// the batch's 256 x 512 tiles number fewer than the launch's CTA pairs and
+// its 256 x 256 tiles, two pairs each, fit on them (and all at once on the
+// device), each tile goes to a cluster of two CTA pairs that contract one half
+// of its blocks each and sum the halves through distributed shared memory: no
+// fp32 partials in memory and no reduce launch.  Problems of fewer than
+// kCsMinBlocks blocks are not worth cutting.  Rewrites the batch's tile list
+// for 256-column tiles and returns true when it applies.
+constexpr int kCsMinBlocks = 8;
+
+bool use_cluster_split(GemmBatch& b, bool b_mn, int pairs) {
+  long long wide = 0, narrow = 0;
+  for (int p = 0; p < b.num_problems; ++p) {
+    const GemmProblem& g = b.prob[p];
+    if (g.kb_total < kCsMinBlocks || g.out_f32) return false;
+    wide += (long long)g.num_m_tiles * g.num_n_tiles;
+    narrow += (long long)g.num_m_tiles * cdiv(g.N, gemm_tile_n_f32());
+  }
+  if (wide == 0 || wide >= pairs || 2 * narrow > pairs) return false;
+  if (narrow > gemm_cs_max_clusters(b_mn)) return false;
+  b.total_tiles = 0;
+  for (int p = 0; p < b.num_problems; ++p) {
+    GemmProblem& g = b.prob[p];
+    g.num_n_tiles = cdiv(g.N, gemm_tile_n_f32());
+    g.splits = 1;
+    g.kb_split = g.kb_total;
+    g.tile_begin = b.total_tiles;
+    b.total_tiles += g.num_m_tiles * g.num_n_tiles;
+  }
+  return true;
+}
+
 // fp32 partial elements of a problem cut into `sp` splits.
 size_t split_floats(const GemmProblem& g, int sp) {
   return sp > 1 ? up256((size_t)sp * g.m_pad * (size_t)rup(g.N, 4) * 4) / 4 : 0;
@@ -1241,8 +1273,12 @@ int run_step(const lora_proj* projs, int n, int mode, void* ws, const Plan& pl, 
           sp[i - i0] = pl.split_f[order[i]];
           parts[i - i0] = at<float>(ws, pl.split_off[order[i]]);
         }
-        if ((rc = apply_splits(b, sp, parts)) != LORA_OK) return rc;
         ProfScope ps(LORA_KERNEL_GEMM_FWD, st);
+        if (q4 == 0 && use_cluster_split(b, false, gemm_sms / 2)) {
+          if (launch_fused_gemm_cs(b, false, st) != cudaSuccess) return LORA_ECUDA;
+          continue;
+        }
+        if ((rc = apply_splits(b, sp, parts)) != LORA_OK) return rc;
         if (launch_fused_gemm(b, false, q4 != 0, gemm_sms, st) != cudaSuccess) return LORA_ECUDA;
         if (launch_split_reduce(b, st) != cudaSuccess) return LORA_ECUDA;
       }
@@ -1270,8 +1306,12 @@ int run_step(const lora_proj* projs, int n, int mode, void* ws, const Plan& pl, 
           sp[i - i0] = pl.split_b[order[i]];
           parts[i - i0] = at<float>(ws, pl.split_off[order[i]]);
         }
-        if ((rc = apply_splits(b, sp, parts)) != LORA_OK) return rc;
         ProfScope ps(LORA_KERNEL_GEMM_BWD, st);
+        if (q4 == 0 && use_cluster_split(b, true, gemm_sms_b / 2)) {
+          if (launch_fused_gemm_cs(b, true, st) != cudaSuccess) return LORA_ECUDA;
+          continue;
+        }
+        if ((rc = apply_splits(b, sp, parts)) != LORA_OK) return rc;
         if (launch_fused_gemm(b, true, q4 != 0, gemm_sms_b, st) != cudaSuccess) return LORA_ECUDA;
         if (launch_split_reduce(b, st) != cudaSuccess) return LORA_ECUDA;
       }

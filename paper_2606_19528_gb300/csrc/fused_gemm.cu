@@ -124,10 +124,12 @@ constexpr size_t smem_bytes() {
 }
 
 // Problem p, first row m0 and first column n0 of tile t, its split ks and
-// that split's contraction blocks [kb0, kb1).
+// that split's contraction blocks [kb0, kb1).  cs_half >= 0 (cluster split):
+// the tile is unsplit in the list and the pair takes half cs_half of its
+// contraction blocks (the first half rounded up).
 template <int kTileN = kBN>
 __device__ __forceinline__ void decode_tile(const GemmBatch& b, int t, int& p, int& m0, int& n0, int& ks, int& kb0,
-                                            int& kb1) {
+                                            int& kb1, int cs_half = -1) {
   p = 0;
   while (p + 1 < b.num_problems && t >= b.prob[p + 1].tile_begin) ++p;
   const GemmProblem& Q = b.prob[p];
@@ -137,6 +139,11 @@ __device__ __forceinline__ void decode_tile(const GemmBatch& b, int t, int& p, i
   local -= ks * per;
   kb0 = ks * Q.kb_split;
   kb1 = min(Q.kb_total, kb0 + Q.kb_split);
+  if (cs_half >= 0) {
+    const int L = (Q.kb_total + 1) / 2;
+    kb0 = cs_half * L;
+    kb1 = min(Q.kb_total, kb0 + L);
+  }
   if (Q.m_fast) {
     m0 = (local % Q.num_m_tiles) * kBM;
     n0 = (local / Q.num_m_tiles) * kTileN;
@@ -206,13 +213,19 @@ __device__ __forceinline__ void dequant_stage(uint32_t slot, uint32_t wdst, int 
   }
 }
 
-template <bool kBMn, bool kQ, bool kF32 = false>
+template <bool kBMn, bool kQ, bool kF32 = false, bool kCS = false>
 __global__ void __launch_bounds__(Cfg<kQ>::kThreads, 1) fused_lora_gemm(const __grid_constant__ GemmBatch b) {
   // fp32 output: 256 x 256 tiles whose accumulator alternates between two TMEM
   // buffers, so one tile's epilogue overlaps the next tile's contraction (the
-  // appending and log-sum-exp epilogues are long); a 6-deep ring of 32 KB stages
-  constexpr bool kNarrow = kF32;
-  static_assert(!kNarrow || (!kQ && !kBMn), "fp32 output is the plain forward form");
+  // appending and log-sum-exp epilogues are long); a 6-deep ring of 32 KB stages.
+  // kCS (cluster split, bf16 output): clusters of two CTA pairs, one 256 x 256
+  // tile per cluster; pair j contracts half j of the tile's blocks, then the
+  // halves are summed through distributed shared memory (each pair finishes
+  // and stores its own 128 columns): no fp32 partials in global memory, no
+  // reduce launch.  For launches with too few tiles to fill the GPU.
+  constexpr bool kNarrow = kF32 || kCS;
+  static_assert(!kNarrow || !kQ, "256 x 256 tiles: bf16 weights only");
+  static_assert(!kF32 || (!kBMn && !kCS), "fp32 output is the plain forward form");
   constexpr int kSegs = kNarrow ? 1 : 2;  // 256-column segments per tile
   constexpr int kTileN = kSegs * kSeg;
   constexpr int kStages = kNarrow ? 6 : Cfg<kQ>::kStages;
@@ -231,7 +244,11 @@ __global__ void __launch_bounds__(Cfg<kQ>::kThreads, 1) fused_lora_gemm(const __
 
   const int warp = threadIdx.x >> 5;
   const int lane = threadIdx.x & 31;
-  const int c = (int)cluster_ctarank();  // position within the pair (0: issues the MMAs)
+  const uint32_t crank = cluster_ctarank();
+  const int c = (int)(crank & 1u);  // position within the pair (0: issues the MMAs)
+  const uint32_t pb = crank & ~1u;  // cluster rank of the pair's even CTA (0 but for kCS)
+  const int cs_half = kCS ? (int)((crank >> 1) & 1u) : -1;  // kCS: which half of the contraction
+  const int cs_tile = kCS ? (int)(blockIdx.x >> 2) : 0;     // kCS: the cluster's one tile
   const WaitCtl wc{b.status, b.limit_ns};
 
   if (threadIdx.x == 0) {
@@ -287,12 +304,12 @@ __global__ void __launch_bounds__(Cfg<kQ>::kThreads, 1) fused_lora_gemm(const __
   cluster_sync_all();  // both CTAs' barriers exist before any cross-CTA arrival
   griddep_wait();      // the previous grid's outputs (su, sv, tile counter) are ready
   const uint32_t tmem_base = ctl->tmem_base;
-  const uint32_t tile_empty_root = mapa_shared(smem_u32(&ctl->tile_empty[0]), 0);
+  const uint32_t tile_empty_root = mapa_shared(smem_u32(&ctl->tile_empty[0]), pb);
 
   if (warp == 0) {
     // ------------------------------------------------------------ scheduler + producer
     if (lane == 0) {
-      const uint32_t full_pl = mapa_shared(smem_u32(&ctl->full[0]), 0);
+      const uint32_t full_pl = mapa_shared(smem_u32(&ctl->full[0]), pb);
       int stage = 0;
       uint32_t phase = 0;
       int fills = 0;
@@ -300,14 +317,16 @@ __global__ void __launch_bounds__(Cfg<kQ>::kThreads, 1) fused_lora_gemm(const __
         const int slot = it % kTileRing;
         const uint32_t par = (uint32_t)((it / kTileRing) & 1);
         int t;
-        if (c == 0) {
+        if (kCS) {
+          t = it == 0 ? cs_tile : -1;  // one tile, no scheduler
+        } else if (c == 0) {
           if (!mbar_wait_cluster(smem_u32(&ctl->tile_empty[slot]), par ^ 1u, wc, abort_flag)) break;
           t = atomicAdd(b.tile_counter, 1);
           if (t >= b.total_tiles) t = -1;
           ctl->tile_id[slot] = t;
-          st_cluster_u32(mapa_shared(smem_u32(&ctl->tile_id[slot]), 1), (uint32_t)t);
+          st_cluster_u32(mapa_shared(smem_u32(&ctl->tile_id[slot]), pb + 1), (uint32_t)t);
           mbar_arrive(smem_u32(&ctl->tile_full[slot]));
-          mbar_arrive_cluster(mapa_shared(smem_u32(&ctl->tile_full[slot]), 1));
+          mbar_arrive_cluster(mapa_shared(smem_u32(&ctl->tile_full[slot]), pb + 1));
         } else {
           if (!mbar_wait_cluster(smem_u32(&ctl->tile_full[slot]), par, wc, abort_flag)) break;
           t = *reinterpret_cast<volatile int*>(&ctl->tile_id[slot]);
@@ -318,7 +337,7 @@ __global__ void __launch_bounds__(Cfg<kQ>::kThreads, 1) fused_lora_gemm(const __
           break;
         }
         int p, m0, n0, ks, kb0, kb1;
-        decode_tile<kTileN>(b, t, p, m0, n0, ks, kb0, kb1);
+        decode_tile<kTileN>(b, t, p, m0, n0, ks, kb0, kb1, cs_half);
         const GemmProblem& Q = b.prob[p];
         const int my_m = m0 + c * kHalf;
         const bool a_mine = my_m < Q.M;
@@ -373,23 +392,28 @@ __global__ void __launch_bounds__(Cfg<kQ>::kThreads, 1) fused_lora_gemm(const __
     // ------------------------------------------------------------ MMA issuer (even CTA)
     if (c == 0 && lane == 0) {
       constexpr uint32_t idesc = idesc_bf16_f32(kBM, kSeg, 0, kBMn ? 1 : 0);
-      constexpr uint16_t pair_mask = 0x3;
+      const uint16_t pair_mask = (uint16_t)(0x3u << pb);
       int stage = 0;
       uint32_t phase = 0;
       uint32_t wseq = 0;  // 4-bit: contraction blocks so far (weight tile wseq % 2)
       bool ok = true;
       for (int it = 0; ok; ++it) {
         const int slot = it % kTileRing;
-        if (!mbar_wait_cluster(smem_u32(&ctl->tile_full[slot]), (uint32_t)((it / kTileRing) & 1), wc, abort_flag))
-          break;
-        const int t = *reinterpret_cast<volatile int*>(&ctl->tile_id[slot]);
-        mbar_arrive_cluster(tile_empty_root + (uint32_t)slot * 8u);
+        int t;
+        if (kCS) {
+          t = it == 0 ? cs_tile : -1;
+        } else {
+          if (!mbar_wait_cluster(smem_u32(&ctl->tile_full[slot]), (uint32_t)((it / kTileRing) & 1), wc, abort_flag))
+            break;
+          t = *reinterpret_cast<volatile int*>(&ctl->tile_id[slot]);
+          mbar_arrive_cluster(tile_empty_root + (uint32_t)slot * 8u);
+        }
         if (t < 0) {
           griddep_launch_dependents();  // no tile left for this pair
           break;
         }
         int p, m0, n0, ks, kb0, kb1;
-        decode_tile<kTileN>(b, t, p, m0, n0, ks, kb0, kb1);
+        decode_tile<kTileN>(b, t, p, m0, n0, ks, kb0, kb1, cs_half);
         const GemmProblem& Q = b.prob[p];
         const int nseg = kNarrow ? 1 : (Q.N - n0 > kSeg ? 2 : 1);  // segments holding any column < N
         // accumulator buffer of this tile; a segment (buffer) is free once both epilogues drained
@@ -442,11 +466,17 @@ __global__ void __launch_bounds__(Cfg<kQ>::kThreads, 1) fused_lora_gemm(const __
       // completes in both CTAs of the pair once every MMA issued above has finished
       umma_commit_pair_mc(smem_u32(&ctl->drain), pair_mask);
     }
+  } else if (kCS && warp < 2 + kEpi) {
+    // ------------------------------------------------------------ epilogue, cluster split: wait for the
+    // pair's accumulator; the exchange of the halves follows below, after every role
+    bool ok = mbar_wait_cluster(smem_u32(&ctl->tfull[0]), 0u, wc, abort_flag);
+    ok = __all_sync(0xffffffffu, ok);
+    tc_fence_after();
   } else if (warp < 2 + kEpi) {
     // ------------------------------------------------------------ epilogue (both CTAs)
     const int q = warp & 3;                 // TMEM lane quadrant this warp may access
     const int part = (warp - 2) >> 2;       // which kPartCols columns of each segment
-    const uint32_t tempty_pl = mapa_shared(smem_u32(&ctl->tempty[0]), 0);
+    const uint32_t tempty_pl = mapa_shared(smem_u32(&ctl->tempty[0]), pb);
     for (int it = 0;; ++it) {
       const int slot = it % kTileRing;
       bool got = mbar_wait_cluster(smem_u32(&ctl->tile_full[slot]), (uint32_t)((it / kTileRing) & 1), wc, abort_flag);
@@ -585,21 +615,6 @@ __global__ void __launch_bounds__(Cfg<kQ>::kThreads, 1) fused_lora_gemm(const __
           tmem_ld_32x32b_x32(taddr, v);
           if (!f32) tmem_ld_32x32b_x32(taddr + 32u, w);
           tmem_ld_wait();
-          if (Q.splits > 1) {
-            // fp32 partial of one split: each thread stores its row's 32 values (one 128-byte
-            // line) straight from registers into the tile-padded partial buffer, kept in L2
-            // for the reduce; no staging, so consecutive blocks' stores overlap
-            if (row0 + lane < Q.M) {
-              float* dst = Q.part + ((size_t)row_st + lane) * Q.ldp + n0 + col0;
-#pragma unroll
-              for (int k = 0; k < 8; ++k)
-                if (n0 + col0 + 4 * k < Q.N)
-                  __stcg(reinterpret_cast<float4*>(dst + 4 * k),
-                         make_float4(__uint_as_float(v[4 * k]), __uint_as_float(v[4 * k + 1]),
-                                     __uint_as_float(v[4 * k + 2]), __uint_as_float(v[4 * k + 3])));
-            }
-            continue;
-          }
           if (lse_on) {
             const int nv = min(32, Q.N - (n0 + col0));  // valid columns of the block, >= 1
             float bm = __uint_as_float(v[0]);
@@ -817,6 +832,95 @@ __global__ void __launch_bounds__(Cfg<kQ>::kThreads, 1) fused_lora_gemm(const __
     }
   }
 
+  if constexpr (kCS) {
+    // ------------------------------------------------------------ cluster split: sum the two halves
+    // Every thread of the cluster's four CTAs passes both cluster barriers.  After the first, both
+    // pairs' contractions are complete, so every CTA's ring is idle and serves as the receive
+    // buffer: 128 rows x 128 fp32 columns, 16-byte chunk kc of row r at chunk kc ^ (r mod 8) (no
+    // bank conflicts for a warp's 32 rows).  The warps over the other pair's half of the columns
+    // send their values to the same-position CTA of that pair; after the second barrier the warps
+    // over this pair's half add what arrived (fp32, two terms: the same sum whichever pair adds),
+    // round to bf16 and store.
+    cluster_sync_all();
+    if (warp >= 2 && warp < 2 + kEpi && !*abort_flag) {
+      int p, m0, n0, ks, kb0, kb1;
+      decode_tile<kTileN>(b, cs_tile, p, m0, n0, ks, kb0, kb1, cs_half);
+      const GemmProblem& Q = b.prob[p];
+      const int q = warp & 3, part = (warp - 2) >> 2;
+      const uint32_t row = (uint32_t)(q * 32 + lane);
+      const uint32_t tl = tmem_base + ((uint32_t)(q * 32) << 16);
+      auto chunk = [&](uint32_t kc) { return row * 512u + (((kc ^ row) & 7u) | (kc & ~7u)) * 16u; };
+      if (part != cs_half) {
+        const uint32_t peer = crank ^ 2u;  // the same position in the other pair
+        for (int blk = 0; blk < 4; ++blk) {
+          const int col = part * kHalf + blk * 32;
+          if (n0 + col >= Q.N) break;  // uniform: the owner stores nothing there either
+          uint32_t v[32];
+          tmem_ld_32x32b_x32(tl + (uint32_t)col, v);
+          tmem_ld_wait();
+#pragma unroll
+          for (int k = 0; k < 8; ++k)
+            st_cluster_v4(mapa_shared(base + chunk((uint32_t)(blk * 8 + k)), peer), v[4 * k], v[4 * k + 1],
+                          v[4 * k + 2], v[4 * k + 3]);
+        }
+      }
+    }
+    cluster_sync_all();
+    if (warp >= 2 && warp < 2 + kEpi && !*abort_flag) {
+      int p, m0, n0, ks, kb0, kb1;
+      decode_tile<kTileN>(b, cs_tile, p, m0, n0, ks, kb0, kb1, cs_half);
+      const GemmProblem& Q = b.prob[p];
+      const int q = warp & 3, part = (warp - 2) >> 2;
+      const uint32_t row = (uint32_t)(q * 32 + lane);
+      const uint32_t tl = tmem_base + ((uint32_t)(q * 32) << 16);
+      auto chunk = [&](uint32_t kc) { return row * 512u + (((kc ^ row) & 7u) | (kc & ~7u)) * 16u; };
+      const int row0 = m0 + c * kHalf + q * 32;
+      const uint32_t stg = epi_base + (uint32_t)(warp - 2) * kEpiStage;
+      if (part == cs_half) {
+        for (int u = 0; u < 2; ++u) {
+          const int col = part * kHalf + u * 64;
+          if (n0 + col >= Q.N || row0 >= Q.M) break;  // uniform
+          uint32_t v[32], w[32];
+          tmem_ld_32x32b_x32(tl + (uint32_t)col, v);
+          tmem_ld_32x32b_x32(tl + (uint32_t)col + 32u, w);
+          tmem_ld_wait();
+#pragma unroll
+          for (int k = 0; k < 16; ++k) {
+            uint32_t o[4];
+            asm volatile("ld.shared.v4.b32 {%0, %1, %2, %3}, [%4];"
+                         : "=r"(o[0]), "=r"(o[1]), "=r"(o[2]), "=r"(o[3])
+                         : "r"(base + chunk((uint32_t)(u * 16 + k)))
+                         : "memory");
+            uint32_t* d = k < 8 ? &v[4 * k] : &w[4 * (k - 8)];
+#pragma unroll
+            for (int e = 0; e < 4; ++e) d[e] = __float_as_uint(__uint_as_float(d[e]) + __uint_as_float(o[e]));
+          }
+          if (lane == 0) bulk_wait_read0();  // the previous store has read the staging block
+          __syncwarp();
+          const uint32_t rbase = stg + (uint32_t)lane * 128u;
+#pragma unroll
+          for (int k = 0; k < 8; ++k) {
+            const uint32_t* src = k < 4 ? &v[k * 8] : &w[(k - 4) * 8];
+            const uint32_t a = pack_bf16x2(__uint_as_float(src[0]), __uint_as_float(src[1]));
+            const uint32_t b2 = pack_bf16x2(__uint_as_float(src[2]), __uint_as_float(src[3]));
+            const uint32_t c2 = pack_bf16x2(__uint_as_float(src[4]), __uint_as_float(src[5]));
+            const uint32_t d2 = pack_bf16x2(__uint_as_float(src[6]), __uint_as_float(src[7]));
+            const uint32_t dst = rbase + (uint32_t)(((k ^ (lane & 7)) & 7) << 4);
+            asm volatile("st.shared.v4.b32 [%0], {%1, %2, %3, %4};" ::"r"(dst), "r"(a), "r"(b2), "r"(c2), "r"(d2)
+                         : "memory");
+          }
+          fence_proxy_async_smem();
+          __syncwarp();
+          if (lane == 0) {
+            tma_store_2d(&b.tmOut[p], stg, n0 + col, row0);
+            bulk_commit();
+          }
+        }
+      }
+      if (lane == 0) bulk_wait0();
+    }
+  }
+
   // ------------------------------------------------------------ teardown
   tc_fence_before();
   __syncthreads();
@@ -947,14 +1051,60 @@ cudaError_t launch_split_reduce(const GemmBatch& batch, cudaStream_t stream) {
 
 size_t fused_gemm_smem_bytes() { return smem_bytes<false>(); }
 
-template <bool kBMn, bool kQ, bool kF32>
+template <bool kBMn, bool kQ, bool kF32, bool kCS = false>
 cudaError_t launch_variant(const GemmBatch& batch, int pairs, cudaStream_t stream) {
   constexpr size_t smem = smem_bytes<kQ>();
   static std::atomic<unsigned long long> attr_done{0};
-  const cudaError_t e = set_smem_once(fused_lora_gemm<kBMn, kQ, kF32>, (int)smem, attr_done);
+  const cudaError_t e = set_smem_once(fused_lora_gemm<kBMn, kQ, kF32, kCS>, (int)smem, attr_done);
   if (e != cudaSuccess) return e;
-  return launch_kernel(fused_lora_gemm<kBMn, kQ, kF32>, dim3((unsigned)(2 * pairs)), dim3(Cfg<kQ>::kThreads), smem,
-                       stream, 2, batch);
+  // kCS: one tile per cluster of two pairs; otherwise persistent pairs
+  const unsigned grid = kCS ? (unsigned)(4 * batch.total_tiles) : (unsigned)(2 * pairs);
+  return launch_kernel(fused_lora_gemm<kBMn, kQ, kF32, kCS>, dim3(grid), dim3(Cfg<kQ>::kThreads), smem, stream,
+                       kCS ? 4 : 2, batch);
+}
+
+// Clusters of four of the cluster-split kernel that can run at once on this
+// device (0 if the query fails), cached per device and majorness.
+template <bool kBMn>
+int cs_max_clusters() {
+  static std::atomic<int> cache[64][1];
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 64) return 0;
+  int v = cache[dev][0].load(std::memory_order_acquire);
+  if (v != 0) return v > 0 ? v : 0;
+  constexpr size_t smem = smem_bytes<false>();
+  static std::atomic<unsigned long long> attr_done{0};
+  int n = -1;
+  if (set_smem_once(fused_lora_gemm<kBMn, false, false, true>, (int)smem, attr_done) == cudaSuccess) {
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = dim3(4 * 64);
+    cfg.blockDim = dim3(Cfg<false>::kThreads);
+    cfg.dynamicSmemBytes = smem;
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeClusterDimension;
+    attr[0].val.clusterDim.x = 4;
+    attr[0].val.clusterDim.y = 1;
+    attr[0].val.clusterDim.z = 1;
+    cfg.attrs = attr;
+    cfg.numAttrs = 1;
+    int k = 0;
+    if (cudaOccupancyMaxActiveClusters(&k, fused_lora_gemm<kBMn, false, false, true>, &cfg) == cudaSuccess && k > 0)
+      n = k;
+    else
+      cudaGetLastError();
+  }
+  cache[dev][0].store(n, std::memory_order_release);
+  return n > 0 ? n : 0;
+}
+
+int gemm_cs_max_clusters(bool b_mn_major) {
+  return b_mn_major ? cs_max_clusters<true>() : cs_max_clusters<false>();
+}
+
+cudaError_t launch_fused_gemm_cs(const GemmBatch& batch, bool b_mn_major, cudaStream_t stream) {
+  if (batch.total_tiles <= 0) return cudaSuccess;
+  return b_mn_major ? launch_variant<true, false, false, true>(batch, 0, stream)
+                    : launch_variant<false, false, false, true>(batch, 0, stream);
 }
 
 cudaError_t launch_fused_gemm(const GemmBatch& batch, bool b_mn_major, bool q4, int num_sms, cudaStream_t stream,

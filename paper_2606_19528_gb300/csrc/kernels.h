@@ -138,6 +138,14 @@ struct GemmBatch {
 cudaError_t launch_fused_gemm(const GemmBatch& batch, bool b_mn_major, bool q4, int num_sms, cudaStream_t stream,
                               bool f32_out = false);
 size_t fused_gemm_smem_bytes();
+// Cluster split (bf16 weights and output, either majorness): one 256 x 256
+// tile per cluster of two CTA pairs, each pair contracting half of the tile's
+// blocks, the halves summed through distributed shared memory.  The batch
+// lists each tile once (num_n_tiles over gemm_tile_n_f32() columns, splits 1);
+// the grid is 4 CTAs per tile, all resident at once when the tile count is at
+// most gemm_cs_max_clusters().
+cudaError_t launch_fused_gemm_cs(const GemmBatch& batch, bool b_mn_major, cudaStream_t stream);
+int gemm_cs_max_clusters(bool b_mn_major);
 // out = sum over s of the split partials, in split order, for every problem
 // of the batch with splits > 1 (bf16 or fp32 per out_f32).
 cudaError_t launch_split_reduce(const GemmBatch& batch, cudaStream_t stream);

@@ -113,8 +113,11 @@ def test_q4_single_parity(T, K, N, r):
 def test_q4_equals_bf16_path_on_dequantized_weight():
     """The tensor core sees the same bf16 operands either way (bf16(s q + b),
     rounded once), and the 4-bit kernel keeps the bf16 kernel's tile order and
-    contraction order: y, su and dx agree bit for bit, dA and dB too."""
-    T, K, N, r = 512, 1024, 1536, 16
+    contraction order: y, su and dx agree bit for bit, dA and dB too.  The
+    shape has 80 output tiles either way, so neither path cuts its
+    contractions (the bf16 path cuts few-tile contractions between cluster
+    pairs, the 4-bit path into fp32 partials)."""
+    T, K, N, r = 2048, 5120, 5120, 16
     p = gen_q4_proj(21, 0, 0, T, K, N, r, 2.0)
     run_q4_single(p)
     q = G.DevProj(*(p.bits[k] for k in ("x", "W", "A", "B", "dy")), p.s)
