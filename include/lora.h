@@ -117,17 +117,20 @@ int lora_linear_fwd(const lora_shape* shape, const lora_bf16* x, const lora_bf16
  * library owns; every GPU that loads the library keeps it until the process
  * exits.  Shapes whose forward needs more scratch than that are rejected
  * with LORA_ESCRATCH before anything is enqueued (roughly when tokens x
- * d_in x rank reaches 2^29; 4096 tokens x d_in 4096 at rank 16 fit).  The first call on a device looks up the
- * array's device address; make that first call before any stream capture.
+ * d_in x rank reaches 2^29; 4096 tokens x d_in 4096 at rank 16 fit).  The
+ * first call on a device looks up the array's device address; make that
+ * first call before any stream capture.
  * All calls share the array and leave their scratch in it: calls that
  * overlap on the GPU (for example on two streams at once) race and give
- * wrong results.  Nothing is allocated.  Its contraction always runs in one
- * pass: where lora_linear_fwd splits the contraction of a forward with few
- * output tiles (fewer than 76, e.g. 512 tokens x d_out 3072) into fp32
- * partial sums, the two results differ by the bf16 rounding of differently
- * ordered fp32 sums; with 76 or more output tiles of 256 x 512 they are
- * identical bit for bit.  The paper has no counterpart of this entry point.
- * Returns as lora_linear_fwd (argument errors first), or LORA_ESCRATCH. */
+ * wrong results.  Nothing is allocated.  It never stores fp32 partial sums
+ * of a contraction: lora_linear_fwd may cut the contraction of a forward
+ * with few output tiles (fewer than 76 of 256 x 512) into fp32 partials in
+ * its workspace when the two CTA pairs of a cluster cannot share it, and
+ * there the two results differ by the bf16 rounding of differently ordered
+ * fp32 sums; everywhere else (76 or more tiles, or a contraction shared
+ * within clusters, as for 512 tokens x d_out 3072) they are identical bit
+ * for bit.  The paper has no counterpart of this entry point.  Returns as
+ * lora_linear_fwd (argument errors first), or LORA_ESCRATCH. */
 int lora_linear_fwd_noalloc(const lora_shape* shape, const lora_bf16* x, const lora_bf16* W,
                             const lora_bf16* A, const lora_bf16* B, lora_bf16* y, lora_bf16* su,
                             void* stream);

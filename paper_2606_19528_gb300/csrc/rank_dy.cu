@@ -209,6 +209,11 @@ __global__ void __launch_bounds__(kThreads, 1) rank_dy_kernel(const __grid_const
       int di = 0;  // dB accumulators used so far
       int ui = 0;  // units so far
       bool ok = true;
+      // operand descriptors of stage 0 (dy K-major for sv, MN-major for dB; B^T, su^T)
+      const uint64_t desc_sv_a = sw128_desc(base, 16, 1024);
+      const uint64_t desc_sv_b = sw128_desc(base + kDyBytes, 16, 1024);
+      const uint64_t desc_db_a = sw128_desc(base, kBox, 1024);
+      const uint64_t desc_db_b = sw128_desc(base + kDyBytes + 2 * G::kSideBox, 16, 1024);
       for (int u = blockIdx.x; u < b.units && ok; u += gridDim.x, ++ui) {
         const DyUnit w = dy_unit(b, u);
         const DyProb& P = b.p[w.pi];
@@ -231,23 +236,28 @@ __global__ void __launch_bounds__(kThreads, 1) rank_dy_kernel(const __grid_const
               break;
             }
             tc_fence_after();
-            const uint32_t xs = base + (uint32_t)stage * G::kStageBytes;
-            const uint32_t bt = xs + kDyBytes, st = bt + 2 * G::kSideBox;
+            // descriptors of this stage's operands; the steps below only move their start
+            // addresses (the address field holds addr >> 4 in its low 14 bits, so adding
+            // offset >> 4 within shared memory never carries out of it)
+            const uint32_t soff = (uint32_t)stage * (G::kStageBytes >> 4);
+            const uint64_t a_sv = desc_sv_a + soff, b_sv = desc_sv_b + soff;
+            const uint64_t a_db = desc_db_a + soff, b_db = desc_db_b + soff;
             const uint32_t d_sv = tmem_base + (uint32_t)(j * R);
+            const uint32_t acc_sv = blk != w.blk0 ? 1u : 0u, acc_db = j != 0 ? 1u : 0u;
 #pragma unroll
             for (int k = 0; k < 8; ++k) {
               // sv: 16 columns of dy per step (K-major, box k / 4) against the same columns of B^T
               const uint32_t bx = (uint32_t)(k >> 2), kk = (uint32_t)(k & 3) * 32u;
-              umma_bf16(d_sv, sw128_desc(xs + bx * kBox + kk, 16, 1024), sw128_desc(bt + bx * G::kSideBox + kk, 16, 1024),
-                        idesc_sv, (blk != w.blk0 || k != 0) ? 1u : 0u);
+              umma_bf16(d_sv, a_sv + ((bx * kBox + kk) >> 4), b_sv + ((bx * G::kSideBox + kk) >> 4), idesc_sv,
+                        k != 0 ? 1u : acc_sv);
             }
 #pragma unroll
             for (int k = 0; k < 8; ++k) {
               // dB: 16 tokens of dy per step (MN-major: the two 64-column boxes kBox apart)
               // against the same tokens of su^T
               const uint32_t bx = (uint32_t)(k >> 2), kk = (uint32_t)(k & 3) * 32u;
-              umma_bf16(d_db, sw128_desc(xs + (uint32_t)k * 2048u, kBox, 1024),
-                        sw128_desc(st + bx * G::kSideBox + kk, 16, 1024), idesc_db, (j != 0 || k != 0) ? 1u : 0u);
+              umma_bf16(d_db, a_db + (((uint32_t)k * 2048u) >> 4), b_db + ((bx * G::kSideBox + kk) >> 4), idesc_db,
+                        k != 0 ? 1u : acc_db);
             }
             issued_any = true;
             umma_commit(smem_u32(&ctl->empty[stage]));

@@ -183,6 +183,10 @@ __global__ void __launch_bounds__(kThreads, 1) rank_mma_kernel(const __grid_cons
       uint32_t phase = 0;
       int it = 0;
       bool ok = true;
+      // stage 0's operand descriptors: X (K-major rows, or MN-major with the boxes kXHalf apart)
+      // and the rank side after it
+      const uint64_t desc_a = kCol ? sw128_desc(base, kXHalf, 1024) : sw128_desc(base, 16, 1024);
+      const uint64_t desc_b = sw128_desc(base + kXBytes, 16, 1024);
       for (int u = blockIdx.x; u < b.units && ok; u += gridDim.x, ++it) {
         int pi, tile, piece;
         decode_unit(b, u, pi, tile, piece);
@@ -200,13 +204,15 @@ __global__ void __launch_bounds__(kThreads, 1) rank_mma_kernel(const __grid_cons
             break;
           }
           tc_fence_after();
-          const uint32_t xs = base + (uint32_t)stage * G::kStageBytes;
-          const uint32_t ws = xs + kXBytes;
+          // this stage's descriptors: stage 0's with the start address moved (addr >> 4 in the
+          // low 14 bits of the descriptor; shared-memory offsets never carry out of them)
+          const uint32_t soff = (uint32_t)stage * (G::kStageBytes >> 4);
+          const uint64_t ad = desc_a + soff, bd = desc_b + soff;
 #pragma unroll
           for (int k = 0; k < kChunk / 16; ++k) {
             // MN-major A: 16 reduction rows of 128 B per step, the two 64-wide boxes 8 KB apart
-            const uint64_t adesc = kCol ? sw128_desc(xs + k * 2048, kXHalf, 1024) : sw128_desc(xs + k * 32, 16, 1024);
-            umma_bf16(d_tmem, adesc, sw128_desc(ws + k * 32, 16, 1024), idesc, (ch | k) != 0 ? 1u : 0u);
+            umma_bf16(d_tmem, ad + (uint32_t)(kCol ? k * 128 : k * 2), bd + (uint32_t)(k * 2), idesc,
+                      (ch | k) != 0 ? 1u : 0u);
           }
           issued_any = true;
           umma_commit(smem_u32(&ctl->empty[stage]));
