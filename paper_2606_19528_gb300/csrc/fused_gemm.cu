@@ -111,6 +111,7 @@ struct __align__(8) Ctl {
   uint64_t tile_full[kTileRing];   // both CTAs: tile id written
   uint64_t tile_empty[kTileRing];  // even CTA: every consumer of both CTAs read the slot
   uint64_t drain;                  // both CTAs: every MMA of the pair completed
+  uint64_t xchg;                   // kCS: the other pair's half of the accumulator arrived
   int tile_id[kTileRing];
   uint32_t tmem_base;
   int abort;
@@ -275,6 +276,7 @@ __global__ void __launch_bounds__(Cfg<kQ>::kThreads, 1) fused_lora_gemm(const __
       mbar_init(smem_u32(&ctl->tile_empty[k]), 2 + 2 * kEpi + (kQ ? 2 * kConvWarps + 4 : 0));
     }
     mbar_init(smem_u32(&ctl->drain), 1);
+    mbar_init(smem_u32(&ctl->xchg), 1);
     ctl->abort = 0;
     ctl->fills = 0;
     ctl->qfills = 0;
@@ -834,13 +836,14 @@ __global__ void __launch_bounds__(Cfg<kQ>::kThreads, 1) fused_lora_gemm(const __
 
   if constexpr (kCS) {
     // ------------------------------------------------------------ cluster split: sum the two halves
-    // Every thread of the cluster's four CTAs passes both cluster barriers.  After the first, both
-    // pairs' contractions are complete, so every CTA's ring is idle and serves as the receive
-    // buffer: 128 rows x 128 fp32 columns, 16-byte chunk kc of row r at chunk kc ^ (r mod 8) (no
-    // bank conflicts for a warp's 32 rows).  The warps over the other pair's half of the columns
-    // send their values to the same-position CTA of that pair; after the second barrier the warps
-    // over this pair's half add what arrived (fp32, two terms: the same sum whichever pair adds),
-    // round to bf16 and store.
+    // After the cluster barrier both pairs' contractions are complete, so every CTA's ring is idle:
+    // its first 64 KB receive the other pair's values for this CTA's rows and this pair's 128 columns,
+    // the next 64 KB stage the values this CTA sends.  Layout of both: 128 rows x 128 fp32 columns,
+    // 16-byte chunk kc of row r at chunk kc ^ (r mod 8) (a warp's 32 rows hit every bank group once).
+    // The warps over the other pair's columns stage their rows and send them with one bulk copy per
+    // warp (16 KB) to the same-position CTA of the other pair, completing on its barrier `xchg`; the
+    // warps over this pair's columns wait for the 64 KB to arrive, add them (fp32, two terms: the same
+    // sum whichever pair adds), round to bf16 and store.
     cluster_sync_all();
     if (warp >= 2 && warp < 2 + kEpi && !*abort_flag) {
       int p, m0, n0, ks, kb0, kb1;
@@ -849,35 +852,34 @@ __global__ void __launch_bounds__(Cfg<kQ>::kThreads, 1) fused_lora_gemm(const __
       const int q = warp & 3, part = (warp - 2) >> 2;
       const uint32_t row = (uint32_t)(q * 32 + lane);
       const uint32_t tl = tmem_base + ((uint32_t)(q * 32) << 16);
+      constexpr uint32_t kRecv = 0, kSend = 128u * 512u;  // offsets in the ring
       auto chunk = [&](uint32_t kc) { return row * 512u + (((kc ^ row) & 7u) | (kc & ~7u)) * 16u; };
       if (part != cs_half) {
-        const uint32_t peer = crank ^ 2u;  // the same position in the other pair
         for (int blk = 0; blk < 4; ++blk) {
-          const int col = part * kHalf + blk * 32;
-          if (n0 + col >= Q.N) break;  // uniform: the owner stores nothing there either
           uint32_t v[32];
-          tmem_ld_32x32b_x32(tl + (uint32_t)col, v);
+          tmem_ld_32x32b_x32(tl + (uint32_t)(part * kHalf + blk * 32), v);
           tmem_ld_wait();
 #pragma unroll
           for (int k = 0; k < 8; ++k)
-            st_cluster_v4(mapa_shared(base + chunk((uint32_t)(blk * 8 + k)), peer), v[4 * k], v[4 * k + 1],
-                          v[4 * k + 2], v[4 * k + 3]);
+            asm volatile("st.shared.v4.b32 [%0], {%1, %2, %3, %4};" ::"r"(base + kSend + chunk((uint32_t)(blk * 8 + k))),
+                         "r"(v[4 * k]), "r"(v[4 * k + 1]), "r"(v[4 * k + 2]), "r"(v[4 * k + 3])
+                         : "memory");
         }
-      }
-    }
-    cluster_sync_all();
-    if (warp >= 2 && warp < 2 + kEpi && !*abort_flag) {
-      int p, m0, n0, ks, kb0, kb1;
-      decode_tile<kTileN>(b, cs_tile, p, m0, n0, ks, kb0, kb1, cs_half);
-      const GemmProblem& Q = b.prob[p];
-      const int q = warp & 3, part = (warp - 2) >> 2;
-      const uint32_t row = (uint32_t)(q * 32 + lane);
-      const uint32_t tl = tmem_base + ((uint32_t)(q * 32) << 16);
-      auto chunk = [&](uint32_t kc) { return row * 512u + (((kc ^ row) & 7u) | (kc & ~7u)) * 16u; };
-      const int row0 = m0 + c * kHalf + q * 32;
-      const uint32_t stg = epi_base + (uint32_t)(warp - 2) * kEpiStage;
-      if (part == cs_half) {
-        for (int u = 0; u < 2; ++u) {
+        fence_proxy_async_smem();  // the bulk copy reads what these threads wrote
+        __syncwarp();
+        if (lane == 0) {
+          const uint32_t peer = crank ^ 2u;  // the same position in the other pair
+          const uint32_t rows = (uint32_t)(q * 32) * 512u;
+          bulk_copy_to_peer(mapa_shared(base + kRecv + rows, peer), base + kSend + rows, 32u * 512u,
+                            mapa_shared(smem_u32(&ctl->xchg), peer));
+        }
+      } else {
+        if (q == 0 && lane == 0) mbar_arrive_expect_tx(smem_u32(&ctl->xchg), 128u * 512u);
+        bool got = mbar_wait(smem_u32(&ctl->xchg), 0u, wc, abort_flag);
+        got = __all_sync(0xffffffffu, got);
+        const int row0 = m0 + c * kHalf + q * 32;
+        const uint32_t stg = epi_base + (uint32_t)(warp - 2) * kEpiStage;
+        for (int u = 0; got && u < 2; ++u) {
           const int col = part * kHalf + u * 64;
           if (n0 + col >= Q.N || row0 >= Q.M) break;  // uniform
           uint32_t v[32], w[32];
@@ -889,7 +891,7 @@ __global__ void __launch_bounds__(Cfg<kQ>::kThreads, 1) fused_lora_gemm(const __
             uint32_t o[4];
             asm volatile("ld.shared.v4.b32 {%0, %1, %2, %3}, [%4];"
                          : "=r"(o[0]), "=r"(o[1]), "=r"(o[2]), "=r"(o[3])
-                         : "r"(base + chunk((uint32_t)(u * 16 + k)))
+                         : "r"(base + kRecv + chunk((uint32_t)(u * 16 + k)))
                          : "memory");
             uint32_t* d = k < 8 ? &v[4 * k] : &w[4 * (k - 8)];
 #pragma unroll
@@ -916,8 +918,8 @@ __global__ void __launch_bounds__(Cfg<kQ>::kThreads, 1) fused_lora_gemm(const __
             bulk_commit();
           }
         }
+        if (lane == 0) bulk_wait0();
       }
-      if (lane == 0) bulk_wait0();
     }
   }
 
