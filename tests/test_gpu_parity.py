@@ -476,3 +476,38 @@ def test_token_shards_sum_to_the_unsharded_gradients():
     dA, dB = oracle.lora_adapter_grads(full.f64("dy"), full.f64("x"), full.f64("A"), full.f64("B"), s)
     assert G.rel_fro(G.host_f64(summed[0][0]), dA) <= G.TOL_GRAD
     assert G.rel_fro(G.host_f64(summed[0][1]), dB) <= G.TOL_GRAD
+
+
+# --------------------------------------------------------------- contractions with few output tiles
+
+# Shapes whose forward and backward contractions have few output tiles, so that each 256 x 256 tile is
+# shared by the two CTA pairs of a cluster (halves of the contraction summed in distributed shared
+# memory): ragged tokens and columns, the smallest depth the library cuts this way (8 blocks: the
+# backward of the first shape, 392 + 24 deep), a rank that pads, and a frozen projection.
+CS_SHAPES = [(264, 520, 392, 24), (136, 1032, 520, 3), (512, 3072, 3072, 16), (392, 2056, 1544, 0)]
+
+
+@pytest.mark.parametrize("T,K,N,r", CS_SHAPES, ids=[f"T{t}_K{k}_N{n}_r{r}" for t, k, n, r in CS_SHAPES])
+def test_few_tile_contractions(T, K, N, r):
+    """Every output against the oracle, and a second call bit for bit equal to the first (the two halves
+    are added in one fp32 operation, whichever pair adds them)."""
+    s = 2.0
+    if r == 0:
+        x, W, _, _, dy = gen_proj(33, 0, 0, T, K, N, 1, s)
+        y, dx = run_frozen(x, W, dy)
+        xf, Wf, dyf = (synth.bf16_bits_to_f64(b) for b in (x, W, dy))
+        assert G.rel_fro(G.host_f64(y), xf @ Wf.T) <= G.TOL_Y
+        assert G.rel_fro(G.host_f64(dx), dyf @ Wf) <= G.TOL_DX
+        y2, dx2 = run_frozen(x, W, dy)
+        assert torch.equal(y.view(torch.int16), y2.view(torch.int16))
+        assert torch.equal(dx.view(torch.int16), dx2.view(torch.int16))
+        return
+    bits = gen_proj(33, r, 0, T, K, N, r, s)
+    p = G.DevProj(*bits, s)
+    G.run_single(p)
+    check_full(p)
+    q = G.DevProj(*bits, s)
+    G.run_single(q)
+    for n in ("y", "su", "dx"):
+        assert torch.equal(getattr(p, n).view(torch.int16), getattr(q, n).view(torch.int16)), n
+    assert torch.equal(p.dA, q.dA) and torch.equal(p.dB, q.dB)
