@@ -1138,17 +1138,20 @@ int run_step(const lora_proj* projs, int n, int mode, void* ws, const Plan& pl, 
   int next_counter = 0;
   if (cudaMemsetAsync(ws, 0, pl.zero_bytes, st) != cudaSuccess) return LORA_ECUDA;
   // forward and backward in one call: the backward's rank-r work runs on a side
-  // stream with a few SMs while the contractions use the rest
+  // stream with a few SMs while the contractions use the rest; a backward alone
+  // computes sv (which the dx contraction reads) first on every SM, then dA (and
+  // dB where the pass over dy is not fused) on the side stream beside the dx
+  // contraction
   Overlap ov;
-  if (mode == LORA_FWD_BWD && (rc = ov.init(d, st, projs, n)) != LORA_OK) return rc;
+  if ((mode & LORA_BWD) && (rc = ov.init(d, st, projs, n)) != LORA_OK) return rc;
   const int gemm_sms = ov.on ? d->num_sms - ov.side_ctas : d->num_sms;      // forward contraction
   const int gemm_sms_b = ov.on ? d->num_sms - ov.side_ctas2 : d->num_sms;  // dx contraction
   // backward rank-r work: B^T, su^T, sv (and sv^T), then dB and dA; on `rs`
   // with `ctas` persistent CTAs; the operands of the dx contraction go to bops
   std::vector<Operands> bops(n);
-  // ctas: CTAs of the transposes and the passes over dy; ctas2: of dA (and the
-  // second pass over dy where it is not fused)
-  auto bwd_rank = [&](cudaStream_t rs, int ctas, int ctas2) -> int {
+  // ctas: CTAs of the transposes and the passes over dy, on rs; ctas2: of dA (and
+  // the second pass over dy where it is not fused), on rs2 (after rs's first phase)
+  auto bwd_rank = [&](cudaStream_t rs, int ctas, cudaStream_t rs2, int ctas2) -> int {
     int rc;
     std::vector<RowSpec> rows;
     std::vector<ColSpec> cols;
@@ -1205,7 +1208,9 @@ int run_step(const lora_proj* projs, int n, int mode, void* ws, const Plan& pl, 
       if ((rc = launch_dy_pass(dys, arena(ws, pl, kPhBwdRows), d, ctas, rs)) != LORA_OK) return rc;
       if ((rc = launch_rows(rows, arena(ws, pl, kPhBwdRows), d, ctas, rs)) != LORA_OK) return rc;
     }
-    if (ov.on && cudaEventRecord(ov.ev_sv, rs) != cudaSuccess) return LORA_ECUDA;
+    // sv is complete: the dx contraction may start (on the main stream: at once, or after this event)
+    if (ov.on && rs != ov.main && cudaEventRecord(ov.ev_sv, rs) != cudaSuccess) return LORA_ECUDA;
+    if (ov.on && rs == ov.main && rs2 != rs && (rc = ov.fork()) != LORA_OK) return rc;
     for (int i = 0; i < n; ++i) {
       if (fused[i] || projs[i].shape.rank == 0) continue;
       const lora_proj& p = projs[i];
@@ -1218,8 +1223,8 @@ int run_step(const lora_proj* projs, int n, int mode, void* ws, const Plan& pl, 
       if (r > 0) add_col_block(cols, cb(p.x), K, T, K, svt[i], T, r, p.dA, 0, true);
     }
     {
-      ProfScope ps(LORA_KERNEL_COLPROJ, rs);
-      if ((rc = launch_cols(cols, arena(ws, pl, kPhBwdCols), d, ctas2, rs)) != LORA_OK) return rc;
+      ProfScope ps(LORA_KERNEL_COLPROJ, rs2);
+      if ((rc = launch_cols(cols, arena(ws, pl, kPhBwdCols), d, ctas2, rs2)) != LORA_OK) return rc;
     }
     return LORA_OK;
   };
@@ -1258,7 +1263,7 @@ int run_step(const lora_proj* projs, int n, int mode, void* ws, const Plan& pl, 
     }
     // the backward's rank-r work needs su only: it may start now, beside the forward contractions
     if (ov.on && (rc = ov.fork()) != LORA_OK) return rc;
-    if (ov.on && (rc = bwd_rank(ov.side, ov.side_ctas, ov.side_ctas2)) != LORA_OK) return rc;
+    if (ov.on && (rc = bwd_rank(ov.side, ov.side_ctas, ov.side, ov.side_ctas2)) != LORA_OK) return rc;
     // one launch per batch of bf16-weight, then of 4-bit-weight problems;
     // heavier problems first so that the tile walk ends balanced
     for (int q4 = 0; q4 < 2; ++q4) {
@@ -1290,9 +1295,11 @@ int run_step(const lora_proj* projs, int n, int mode, void* ws, const Plan& pl, 
     }
   }
   if (mode & LORA_BWD) {
-    if (!ov.on && (rc = bwd_rank(st, d->num_sms, d->num_sms)) != LORA_OK) return rc;
-    // the dx contraction reads sv: with the side stream, wait for it
-    if (ov.on && (rc = ov.wait_sv()) != LORA_OK) return rc;
+    if (mode == LORA_BWD && (rc = bwd_rank(st, d->num_sms, ov.on ? ov.side : st, ov.on ? ov.side_ctas2 : d->num_sms)) !=
+                                LORA_OK)
+      return rc;
+    // the dx contraction reads sv: when the side stream computed it, wait for it
+    if (mode == LORA_FWD_BWD && ov.on && (rc = ov.wait_sv()) != LORA_OK) return rc;
     std::vector<Operands>& ops = bops;
     for (int q4 = 0; q4 < 2; ++q4) {
       std::vector<int> order;
@@ -1357,11 +1364,12 @@ int plan_all(const lora_proj* projs, int n, int mode, Plan* pl, bool allow_split
   // split contractions: batches as run_step forms them (every projection counted for the backward)
   pl->split_f.assign(n, 1);
   pl->split_b.assign(n, 1);
-  // a forward-and-backward call leaves the side stream's SMs out of the contractions
+  // the side stream's SMs are left out of the contractions they run beside: the
+  // forward's in a forward-and-backward call, the dx contraction's in any call with a backward
   int pairs_dir[2] = {kPlanPairs, kPlanPairs};
-  if (mode == LORA_FWD_BWD && overlap_enabled()) {
+  if ((mode & LORA_BWD) && overlap_enabled() && any_adapter(projs, n)) {
     const SideWidths w = side_widths(kPlanSms, projs, n);
-    pairs_dir[0] = (kPlanSms - w.w1) / 2;
+    if (mode == LORA_FWD_BWD) pairs_dir[0] = (kPlanSms - w.w1) / 2;
     pairs_dir[1] = (kPlanSms - w.w2) / 2;
   }
   std::vector<size_t> split_need(n, 0);

@@ -113,10 +113,13 @@ def test_q4_single_parity(T, K, N, r):
 def test_q4_equals_bf16_path_on_dequantized_weight():
     """The tensor core sees the same bf16 operands either way (bf16(s q + b),
     rounded once), and the 4-bit kernel keeps the bf16 kernel's tile order and
-    contraction order: y, su and dx agree bit for bit, dA and dB too.  The
-    shape has 80 output tiles either way, so neither path cuts its
-    contractions (the bf16 path cuts few-tile contractions between cluster
-    pairs, the 4-bit path into fp32 partials)."""
+    contraction order: y, su and dx agree bit for bit.  The shape has 80
+    output tiles either way, so neither path cuts its contractions (the bf16
+    path cuts few-tile contractions between cluster pairs, the 4-bit path into
+    fp32 partials).  dA and dB come from the rank-r kernels on the side stream,
+    whose width follows the contraction beside it (4-bit contractions are
+    weighted as slower), so their sums over 2048 tokens may be cut
+    differently: equal to the fp32 rounding of such sums (~1e-6 relative)."""
     T, K, N, r = 2048, 5120, 5120, 16
     p = gen_q4_proj(21, 0, 0, T, K, N, r, 2.0)
     run_q4_single(p)
@@ -125,7 +128,7 @@ def test_q4_equals_bf16_path_on_dequantized_weight():
     for n in ("y", "su", "dx"):
         assert torch.equal(getattr(p, n).view(torch.int16), getattr(q, n).view(torch.int16)), n
     for n in ("dA", "dB"):
-        assert torch.equal(getattr(p, n), getattr(q, n)), n
+        assert G.rel_fro(G.host_f64(getattr(p, n)), G.host_f64(getattr(q, n))) < 1e-5, n
 
 
 def test_q4_layer_stack_mixed():
