@@ -95,6 +95,7 @@ struct Cfg {
   }
 };
 constexpr int kTileRing = 4;  // tile ids handed from the scheduler to the other roles
+constexpr int kDefer = 2;     // wide tiles: blocks whose segment-0 MMAs precede the first segment-1 MMA
 constexpr long long kDrainNs = 1000000000ll;
 constexpr long long kAbortDrainNs = 10000000ll;  // 10 ms per armed stage on the abort path
 
@@ -422,7 +423,53 @@ __global__ void __launch_bounds__(Cfg<kQ>::kThreads, 1) fused_lora_gemm(const __
         // it for its previous tile (the previous tile, or with two buffers the one before)
         const int buf = kNarrow ? (it & 1) : 0;
         const uint32_t drained_par = kNarrow ? (uint32_t)(((it >> 1) & 1) ^ 1) : (uint32_t)((it & 1) ^ 1);
-        for (int kb = kb0; kb < kb1; ++kb) {
+        int kb = kb0;
+        if (!kQ && kSegs == 2) {
+          // Start of a wide tile: segment 0's MMAs of the first kDefer blocks go first, and only then
+          // does the issuer need segment 1's accumulator (the epilogue drains segment 0 first).  Each
+          // segment still accumulates its blocks in order, so the sums are unchanged.
+          const int nd = min(kDefer, kb1 - kb0);
+          int dst[kDefer];
+          for (int i = 0; i < nd && ok; ++i, ++kb) {
+            if (!mbar_wait(smem_u32(&ctl->full[stage]), phase, wc, abort_flag) ||
+                (i == 0 && !mbar_wait_cluster(smem_u32(&ctl->tempty[buf]), drained_par, wc, abort_flag))) {
+              ok = false;
+              break;
+            }
+            tc_fence_after();
+            dst[i] = stage;
+            const uint32_t a_addr = a_addr_of(base, stage);
+            const int nk = kb < Q.kb_main ? kBK / 16 : min(kBK / 16, (Q.r - (kb - Q.kb_main) * kBK + 15) / 16);
+            for (int k = 0; k < nk; ++k) {
+              const uint64_t bdesc = kBMn ? sw128_desc(a_addr + kAHalf + k * 2048, kBox, 1024)
+                                          : sw128_desc(a_addr + kAHalf + k * 32, 16, 1024);
+              umma_bf16_pair(tmem_base + (uint32_t)(buf * kSeg), sw128_desc(a_addr + k * 32, 16, 1024), bdesc, idesc,
+                             (kb != kb0 || k != 0) ? 1u : 0u);
+            }
+            if (++stage == kStages) {
+              stage = 0;
+              phase ^= 1u;
+            }
+          }
+          if (ok && !mbar_wait_cluster(smem_u32(&ctl->tempty[buf + 1]), drained_par, wc, abort_flag)) ok = false;
+          if (!ok) break;
+          tc_fence_after();
+          for (int i = 0; i < nd; ++i) {
+            const int kbi = kb0 + i;
+            const uint32_t a_addr = a_addr_of(base, dst[i]);
+            const int nk = kbi < Q.kb_main ? kBK / 16 : min(kBK / 16, (Q.r - (kbi - Q.kb_main) * kBK + 15) / 16);
+            if (nseg > 1) {
+              const uint32_t bseg = a_addr + kAHalf + kBSeg;
+              for (int k = 0; k < nk; ++k) {
+                const uint64_t bdesc = kBMn ? sw128_desc(bseg + k * 2048, kBox, 1024) : sw128_desc(bseg + k * 32, 16, 1024);
+                umma_bf16_pair(tmem_base + (uint32_t)((buf + 1) * kSeg), sw128_desc(a_addr + k * 32, 16, 1024), bdesc,
+                               idesc, (kbi != kb0 || k != 0) ? 1u : 0u);
+              }
+            }
+            umma_commit_pair_mc(smem_u32(&ctl->empty[dst[i]]), pair_mask);
+          }
+        }
+        for (; kb < kb1; ++kb) {
           if (!mbar_wait(smem_u32(&ctl->full[stage]), phase, wc, abort_flag)) {
             ok = false;
             break;
@@ -608,6 +655,51 @@ __global__ void __launch_bounds__(Cfg<kQ>::kThreads, 1) fused_lora_gemm(const __
               }
             }
           }
+        }
+        // bf16 output of a whole contraction: the warp's 128 columns of the segment are read and
+        // rounded to bf16 in registers first, and the segment is released to the next tile's MMAs at
+        // once; the staging and the stores follow (the MMAs of the next tile no longer wait for them)
+        if (!kQ && !kF32 && Q.splits == 1 && Cfg<kQ>::kPartCols == 128) {
+          const int c00 = h * kSeg + part * Cfg<kQ>::kPartCols;  // tile column of the warp's first block
+          const uint32_t ta = tmem_base + ((uint32_t)(q * 32) << 16) + (uint32_t)(buf * kSeg + c00);
+          uint32_t pk[2][32];  // [block][bf16 pair]: 64 columns per block
+#pragma unroll
+          for (int u = 0; u < 2; ++u) {
+            uint32_t v[32], w[32];
+            tmem_ld_32x32b_x32(ta + (uint32_t)(64 * u), v);
+            tmem_ld_32x32b_x32(ta + (uint32_t)(64 * u) + 32u, w);
+            tmem_ld_wait();
+#pragma unroll
+            for (int e = 0; e < 16; ++e) {
+              pk[u][e] = pack_bf16x2(__uint_as_float(v[2 * e]), __uint_as_float(v[2 * e + 1]));
+              pk[u][16 + e] = pack_bf16x2(__uint_as_float(w[2 * e]), __uint_as_float(w[2 * e + 1]));
+            }
+          }
+          tc_fence_before();
+          __syncwarp();
+          if (lane == 0) mbar_arrive_cluster(tempty_pl + (uint32_t)(buf + h) * 8u);
+#pragma unroll
+          for (int u = 0; u < 2; ++u) {
+            const int col0 = c00 + 64 * u;
+            if (n0 + col0 >= Q.N || row0 >= Q.M) break;  // uniform across the warp
+            if (lane == 0) bulk_wait_read0();            // the previous store has read the staging block
+            __syncwarp();
+            const uint32_t rbase = stg + (uint32_t)lane * 128u;
+#pragma unroll
+            for (int k = 0; k < 8; ++k) {
+              const uint32_t dst = rbase + (uint32_t)(((k ^ (lane & 7)) & 7) << 4);
+              asm volatile("st.shared.v4.b32 [%0], {%1, %2, %3, %4};" ::"r"(dst), "r"(pk[u][4 * k]),
+                           "r"(pk[u][4 * k + 1]), "r"(pk[u][4 * k + 2]), "r"(pk[u][4 * k + 3])
+                           : "memory");
+            }
+            fence_proxy_async_smem();
+            __syncwarp();
+            if (lane == 0) {
+              tma_store_2d(&b.tmOut[p], stg, n0 + col0, row_st);
+              bulk_commit();
+            }
+          }
+          continue;
         }
         for (int cc = 0; !app && cc < Cfg<kQ>::kPartCols; cc += block_cols) {
           const int col0 = h * kSeg + part * Cfg<kQ>::kPartCols + cc;  // tile column of this block
