@@ -1,4 +1,4 @@
-"""GPU tests of the forward-and-backward call's two-stream schedule (the
+"""GPU tests of the two-stream schedule of calls with a backward (the
 backward's rank-r work on a side stream joined by events): a call captured
 into a CUDA graph and replayed, and calls from two host threads on their own
 streams at the same time, give bit-identical results to the plain call."""
@@ -90,3 +90,31 @@ def test_two_host_threads_at_once():
     assert not errors, errors
     for ps, want in zip(layers, wants):
         assert same(snapshot(ps), want) is None
+
+
+def test_graph_capture_of_a_backward_only_call():
+    """A backward-only call also forks: sv on the caller's stream, then dA (and
+    dB) on the side stream beside the dx contraction.  Captured and replayed,
+    it matches the plain call bit for bit."""
+    wl = workloads.llama_sweep(256, 16)
+    ps = build_layer(wl, seed=9)
+    projs = [p.proj() for p in ps]
+    ws = G.workspace(lora.lora_stack_workspace_size(projs, lora.LORA_FWD_BWD))
+    side = torch.cuda.Stream()
+    with torch.cuda.stream(side):
+        lora.lora_stack_step(projs, lora.LORA_FWD, ws, ws.numel(), side)
+        lora.lora_stack_step(projs, lora.LORA_BWD, ws, ws.numel(), side)
+    torch.cuda.synchronize()
+    want = snapshot(ps)
+    bwd_outs = ("dx", "dA", "dB")
+    for p in ps:
+        for n in bwd_outs:
+            getattr(p, n).fill_(float("nan"))
+    g = torch.cuda.CUDAGraph()
+    with torch.cuda.graph(g, stream=side):
+        lora.lora_stack_step(projs, lora.LORA_BWD, ws, ws.numel(), side)
+    torch.cuda.synchronize()
+    g.replay()
+    torch.cuda.synchronize()
+    assert same(snapshot(ps), want) is None
+    assert lora.lora_read_status() == lora.LORA_OK
