@@ -1295,8 +1295,9 @@ int run_step(const lora_proj* projs, int n, int mode, void* ws, const Plan& pl, 
     }
   }
   if (mode & LORA_BWD) {
-    if (mode == LORA_BWD && (rc = bwd_rank(st, d->num_sms, ov.on ? ov.side : st, ov.on ? ov.side_ctas2 : d->num_sms)) !=
-                                LORA_OK)
+    // (a forward-and-backward call without the side stream runs it here too, on every SM)
+    if (!(mode == LORA_FWD_BWD && ov.on) &&
+        (rc = bwd_rank(st, d->num_sms, ov.on ? ov.side : st, ov.on ? ov.side_ctas2 : d->num_sms)) != LORA_OK)
       return rc;
     // the dx contraction reads sv: when the side stream computed it, wait for it
     if (mode == LORA_FWD_BWD && ov.on && (rc = ov.wait_sv()) != LORA_OK) return rc;

@@ -1,7 +1,12 @@
 """GPU tests of the two-stream schedule of calls with a backward (the
 backward's rank-r work on a side stream joined by events): a call captured
 into a CUDA graph and replayed, and calls from two host threads on their own
-streams at the same time, give bit-identical results to the plain call."""
+streams at the same time, give bit-identical results to the plain call; with
+the side stream switched off (LORA_OVERLAP=0) the same call runs every step
+on one stream and still matches the oracle."""
+import os
+import subprocess
+import sys
 import threading
 
 import pytest
@@ -118,3 +123,30 @@ def test_graph_capture_of_a_backward_only_call():
     torch.cuda.synchronize()
     assert same(snapshot(ps), want) is None
     assert lora.lora_read_status() == lora.LORA_OK
+
+
+ONE_STREAM = r"""
+import sys
+from paper_2606_19528_gb300 import lora, workloads
+from tests import gpu_util as G
+from tests.test_gpu_parity import build_layer, check_full
+wl = workloads.llama_sweep(256, 16)
+ps = build_layer(wl, seed=7)
+G.run_stack(ps)
+for p in ps:
+    check_full(p)
+print("one-stream call ok")
+"""
+
+
+def test_forward_and_backward_call_without_the_side_stream():
+    """LORA_OVERLAP=0 (read once per process, hence a child process): the
+    backward's rank-r work runs on the call's stream after the forward, on
+    every SM; every output of the Llama-shaped layer at T = 256 against the
+    oracle."""
+    root = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+    env = dict(os.environ, LORA_OVERLAP="0")
+    r = subprocess.run([sys.executable, "-c", ONE_STREAM], cwd=root, env=env, capture_output=True, text=True,
+                       timeout=600)
+    assert r.returncode == 0, r.stdout[-2000:] + r.stderr[-4000:]
+    assert "one-stream call ok" in r.stdout
