@@ -37,11 +37,11 @@
 //
 // 4-bit weights (Algorithm 1's on-the-fly dequantization, W = s * W_q + b with
 // one (s, b) per output row and 64-wide group along d_in): three decoupled
-// rings per CTA.  Warp 0 streams the activation boxes (4 deep); warp 10
+// rings per CTA.  Warp 0 streams the activation boxes (3 deep); warp 10
 // streams this CTA's codes and (s, b) pairs by TMA (a quarter of the bf16
-// weight bytes, 4 deep); warps 6..9 dequantize a block with packed bf16
+// weight bytes, 2 deep); warps 6..9 dequantize a block with packed bf16
 // FMAs straight into the 128-byte-swizzled operand layout the tensor core
-// reads, in a ring of 3 bf16 weight tiles, releasing the code slot at once;
+// reads, in a ring of 4 bf16 weight tiles, releasing the code slot at once;
 // warp 11 relays "tile dequantized" to the MMA issuer (one cluster-scope
 // arrive per block and CTA, kept off the dequantizing warps' path); the MMA
 // waits for an activation stage and a weight tile.  Each ring has a
@@ -70,18 +70,21 @@ constexpr int kMaxStages = 6;
 constexpr uint32_t kStageBytes = kAHalf + 2 * kBSeg;  // bf16 weights: activation + weight boxes
 constexpr uint32_t kQCodes = 8192;                    // 4-bit block: 256 weight rows x 64 codes
 constexpr uint32_t kQSlot = kQCodes + 4096;           // + (s, b) boxes
-constexpr int kQStages = 4;                           // 4-bit: code slots
-constexpr int kWStages = 3;                           // 4-bit: dequantized bf16 weight tiles
+constexpr int kQStages = 2;                           // 4-bit: code slots
+constexpr int kWStages = 4;                           // 4-bit: dequantized bf16 weight tiles
 constexpr uint32_t kWTile = 2 * kBSeg;
 
 // Shared-memory layout and warps of the bf16-weight (kQ false) and
 // 4-bit-weight (kQ true) kernels.  bf16: 4 stages of [activation | weight],
-// 8 epilogue warps; 4-bit: 4 activation boxes, 3 bf16 weight tiles, 4 code
+// 8 epilogue warps; 4-bit: 3 activation boxes, 4 bf16 weight tiles, 2 code
 // slots, 4 epilogue warps (its tiles take longer, so one warp per TMEM lane
-// quadrant drains in time) and 4 dequantizing warps.
+// quadrant drains in time) and 4 dequantizing warps.  (4-bit, Llama-shaped
+// layer: 4 weight tiles against 3 took T = 256 from 154 to 149 us and T = 2048
+// from 731 to 720 us; 2 weight tiles cost 15-30 %; the code ring's depth, 2 to
+// 8, changed nothing.)
 template <bool kQ>
 struct Cfg {
-  static constexpr int kStages = 4;  // activation ring
+  static constexpr int kStages = kQ ? 3 : 4;  // activation ring
   static constexpr int kEpi = kQ ? 4 : kEpiWarps;
   static constexpr int kParts = kEpi / 4;          // epilogue warps per TMEM lane quadrant
   static constexpr int kPartCols = kSeg / kParts;  // columns of a segment per epilogue warp
