@@ -23,9 +23,11 @@
 // 2 x 128 columns of the weight operand, and holds its 128 x 512 half of the
 // fp32 accumulator in all 512 columns of its tensor memory.  The wide tile
 // halves the shared-memory traffic per FLOP of a 256 x 256 tile, which keeps
-// the operand feed ahead of the tensor pipe.  The epilogue drains segment 0
-// first and releases it, so the next tile's first MMAs overlap the drain of
-// segment 1.  Within a problem, consecutive tiles walk M when the weight
+// the operand feed ahead of the tensor pipe.  The segments of a tile are
+// signalled complete one after the other (the last two blocks issue segment
+// 0's MMAs first), and the epilogue drains and releases segment 0 first, so
+// the drain of segment 0 overlaps segment 1's last MMAs and the next tile's
+// first MMAs overlap the drain of segment 1.  Within a problem, consecutive tiles walk M when the weight
 // operand is the larger one, so each weight tile is read from DRAM once.
 //   warp 0      tile scheduler (even CTA) and TMA producer (both CTAs):
 //               4-stage shared-memory ring of 48 KB, 128-byte swizzle
@@ -99,6 +101,7 @@ struct Cfg {
 };
 constexpr int kTileRing = 4;  // tile ids handed from the scheduler to the other roles
 constexpr int kDefer = 2;     // wide tiles: blocks whose segment-0 MMAs precede the first segment-1 MMA
+constexpr int kEndDefer = 2;  // wide tiles: last blocks whose segment-0 MMAs precede their segment-1 MMAs
 constexpr long long kDrainNs = 1000000000ll;
 constexpr long long kAbortDrainNs = 10000000ll;  // 10 ms per armed stage on the abort path
 
@@ -443,12 +446,11 @@ __global__ void __launch_bounds__(Cfg<kQ>::kThreads, 1) fused_lora_gemm(const __
             dst[i] = stage;
             const uint32_t a_addr = a_addr_of(base, stage);
             const int nk = kb < Q.kb_main ? kBK / 16 : min(kBK / 16, (Q.r - (kb - Q.kb_main) * kBK + 15) / 16);
-            for (int k = 0; k < nk; ++k) {
-              const uint64_t bdesc = kBMn ? sw128_desc(a_addr + kAHalf + k * 2048, kBox, 1024)
-                                          : sw128_desc(a_addr + kAHalf + k * 32, 16, 1024);
-              umma_bf16_pair(tmem_base + (uint32_t)(buf * kSeg), sw128_desc(a_addr + k * 32, 16, 1024), bdesc, idesc,
-                             (kb != kb0 || k != 0) ? 1u : 0u);
-            }
+            const uint64_t ad = sw128_desc(a_addr, 16, 1024);
+            const uint64_t bd = kBMn ? sw128_desc(a_addr + kAHalf, kBox, 1024) : sw128_desc(a_addr + kAHalf, 16, 1024);
+            for (int k = 0; k < nk; ++k)
+              umma_bf16_pair(tmem_base + (uint32_t)(buf * kSeg), ad + (uint64_t)(2 * k),
+                             bd + (uint64_t)((kBMn ? 128 : 2) * k), idesc, (kb != kb0 || k != 0) ? 1u : 0u);
             if (++stage == kStages) {
               stage = 0;
               phase ^= 1u;
@@ -462,17 +464,19 @@ __global__ void __launch_bounds__(Cfg<kQ>::kThreads, 1) fused_lora_gemm(const __
             const uint32_t a_addr = a_addr_of(base, dst[i]);
             const int nk = kbi < Q.kb_main ? kBK / 16 : min(kBK / 16, (Q.r - (kbi - Q.kb_main) * kBK + 15) / 16);
             if (nseg > 1) {
-              const uint32_t bseg = a_addr + kAHalf + kBSeg;
-              for (int k = 0; k < nk; ++k) {
-                const uint64_t bdesc = kBMn ? sw128_desc(bseg + k * 2048, kBox, 1024) : sw128_desc(bseg + k * 32, 16, 1024);
-                umma_bf16_pair(tmem_base + (uint32_t)((buf + 1) * kSeg), sw128_desc(a_addr + k * 32, 16, 1024), bdesc,
-                               idesc, (kbi != kb0 || k != 0) ? 1u : 0u);
-              }
+              const uint64_t ad = sw128_desc(a_addr, 16, 1024);
+              const uint64_t bd = kBMn ? sw128_desc(a_addr + kAHalf + kBSeg, kBox, 1024)
+                                       : sw128_desc(a_addr + kAHalf + kBSeg, 16, 1024);
+              for (int k = 0; k < nk; ++k)
+                umma_bf16_pair(tmem_base + (uint32_t)((buf + 1) * kSeg), ad + (uint64_t)(2 * k),
+                               bd + (uint64_t)((kBMn ? 128 : 2) * k), idesc, (kbi != kb0 || k != 0) ? 1u : 0u);
             }
             umma_commit_pair_mc(smem_u32(&ctl->empty[dst[i]]), pair_mask);
           }
         }
-        for (; kb < kb1; ++kb) {
+        // wide bf16 tiles with both segments: the last kEndDefer blocks are issued below
+        const int kb_end = (!kQ && kSegs == 2 && nseg == 2 && kb1 - kb >= kEndDefer) ? kb1 - kEndDefer : kb1;
+        for (; kb < kb_end; ++kb) {
           if (!mbar_wait(smem_u32(&ctl->full[stage]), phase, wc, abort_flag)) {
             ok = false;
             break;
@@ -532,7 +536,48 @@ __global__ void __launch_bounds__(Cfg<kQ>::kThreads, 1) fused_lora_gemm(const __
           }
         }
         if (!ok) break;
-        umma_commit_pair_mc(smem_u32(&ctl->tfull[buf]), pair_mask);
+        if (kSegs == 2) {
+          // End of a wide tile: segment 0's MMAs of the last blocks go first and segment 0 is signalled
+          // complete before segment 1, so its drain overlaps segment 1's last MMAs.  Each segment still
+          // accumulates its blocks in order.
+          int dst2[kEndDefer];
+          const int ne = kQ ? 0 : kb1 - kb;
+          for (int i = 0; i < ne && ok; ++i, ++kb) {
+            if (!mbar_wait(smem_u32(&ctl->full[stage]), phase, wc, abort_flag)) {
+              ok = false;
+              break;
+            }
+            tc_fence_after();
+            dst2[i] = stage;
+            const uint32_t a_addr = a_addr_of(base, stage);
+            const int nk = kb < Q.kb_main ? kBK / 16 : min(kBK / 16, (Q.r - (kb - Q.kb_main) * kBK + 15) / 16);
+            const uint64_t ad = sw128_desc(a_addr, 16, 1024);
+            const uint64_t bd = kBMn ? sw128_desc(a_addr + kAHalf, kBox, 1024) : sw128_desc(a_addr + kAHalf, 16, 1024);
+            for (int k = 0; k < nk; ++k)
+              umma_bf16_pair(tmem_base, ad + (uint64_t)(2 * k), bd + (uint64_t)((kBMn ? 128 : 2) * k), idesc, 1u);
+            if (++stage == kStages) {
+              stage = 0;
+              phase ^= 1u;
+            }
+          }
+          if (!ok) break;
+          umma_commit_pair_mc(smem_u32(&ctl->tfull[0]), pair_mask);
+          for (int i = 0; i < ne; ++i) {
+            const int kbi = kb1 - ne + i;
+            const uint32_t a_addr = a_addr_of(base, dst2[i]);
+            const int nk = kbi < Q.kb_main ? kBK / 16 : min(kBK / 16, (Q.r - (kbi - Q.kb_main) * kBK + 15) / 16);
+            const uint64_t ad = sw128_desc(a_addr, 16, 1024);
+            const uint64_t bd = kBMn ? sw128_desc(a_addr + kAHalf + kBSeg, kBox, 1024)
+                                     : sw128_desc(a_addr + kAHalf + kBSeg, 16, 1024);
+            for (int k = 0; k < nk; ++k)
+              umma_bf16_pair(tmem_base + (uint32_t)kSeg, ad + (uint64_t)(2 * k), bd + (uint64_t)((kBMn ? 128 : 2) * k),
+                             idesc, 1u);
+            umma_commit_pair_mc(smem_u32(&ctl->empty[dst2[i]]), pair_mask);
+          }
+          umma_commit_pair_mc(smem_u32(&ctl->tfull[1]), pair_mask);
+        } else {
+          umma_commit_pair_mc(smem_u32(&ctl->tfull[buf]), pair_mask);
+        }
       }
       // completes in both CTAs of the pair once every MMA issued above has finished
       umma_commit_pair_mc(smem_u32(&ctl->drain), pair_mask);
@@ -562,13 +607,23 @@ __global__ void __launch_bounds__(Cfg<kQ>::kThreads, 1) fused_lora_gemm(const __
       const GemmProblem& Q = b.prob[p];
       const int buf = kNarrow ? (it & 1) : 0;  // accumulator buffer of this tile
       const uint32_t tpar = kNarrow ? (uint32_t)((it >> 1) & 1) : (uint32_t)(it & 1);
-      bool ok = mbar_wait_cluster(smem_u32(&ctl->tfull[buf]), tpar, wc, abort_flag);
+      // wide tiles signal each segment's accumulator complete on its own (tfull[h])
+      bool ok = kSegs == 2 || mbar_wait_cluster(smem_u32(&ctl->tfull[buf]), tpar, wc, abort_flag);
       ok = __all_sync(0xffffffffu, ok);
       if (!ok) break;
       tc_fence_after();
       const int row0 = m0 + c * kHalf + q * 32;  // first of this warp's 32 rows
       const uint32_t stg = epi_base + (uint32_t)(warp - 2) * kEpiStage;
       for (int h = 0; h < kSegs; ++h) {
+        if (kSegs == 2) {
+          bool okh = mbar_wait_cluster(smem_u32(&ctl->tfull[h]), tpar, wc, abort_flag);
+          okh = __all_sync(0xffffffffu, okh);
+          if (!okh) {
+            ok = false;
+            break;
+          }
+          tc_fence_after();
+        }
         // a staged block is 32 rows x 128 bytes: 64 bf16 columns, or 32 fp32 columns
         // (fp32 output, or the partial of one split of the contraction)
         const bool f32 = kF32 || Q.splits > 1;
@@ -785,6 +840,7 @@ __global__ void __launch_bounds__(Cfg<kQ>::kThreads, 1) fused_lora_gemm(const __
         __syncwarp();
         if (lane == 0) mbar_arrive_cluster(tempty_pl + (uint32_t)(buf + h) * 8u);
       }
+      if (!ok) break;
     }
     // the output must be written before the CTA exits
     if (lane == 0) bulk_wait0();
