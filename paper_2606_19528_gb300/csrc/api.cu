@@ -224,6 +224,10 @@ struct Plan {
   std::vector<size_t> split_off;
   size_t zero_bytes = 0;  // [0, zero_bytes) is cleared at the start of a call
   size_t total = 0;
+  // the fused passes over dy cut for the whole device, as a backward call cuts them, even where a
+  // side stream runs them on a few SMs (the checkpointed stack, whose re-forward-and-backward calls
+  // must sum sv and dB exactly as the saved schedule's backward calls)
+  bool dy_cut_device = false;
 };
 
 template <typename T>
@@ -717,13 +721,16 @@ bool dy_fusable(int T, int N, int r) {
 
 // The cut of a projection for (gmul, pmul): gmul x the necessary token groups
 // and pmul column pieces, trimmed (pieces first) until the partials fit within
-// those of the necessary groups plus an eighth of the projection's dy bytes.
+// those of the necessary groups plus an eighth of the projection's dy bytes,
+// or kDyPartialFloor floats for a small projection (whose few units would
+// otherwise leave the side stream's SMs idle; 4 MB of partials cost ~1 us).
+constexpr size_t kDyPartialFloor = size_t(1) << 20;
 DyCut dy_cut(int T, int N, int rpad, int tiles_max, int gmul, int pmul) {
   const int tiles = cdiv(T, kDyTile), blocks = cdiv(N, kDyTile);
   const int need = dy_need_groups(T, tiles_max);
   int groups = std::min(tiles, std::min(need * gmul, std::max(need, kDyMaxCut)));
   int pieces = std::min(blocks, std::min(pmul, kDyMaxCut));
-  const size_t cap = dy_db_floats(N, rpad, need) + (size_t)T * N / 16;
+  const size_t cap = dy_db_floats(N, rpad, need) + std::max((size_t)T * N / 16, kDyPartialFloor);
   while (pieces > 1 && dy_sv_floats(T, rpad, pieces) + dy_db_floats(N, rpad, groups) > cap) --pieces;
   while (groups > need && dy_sv_floats(T, rpad, pieces) + dy_db_floats(N, rpad, groups) > cap) --groups;
   DyCut c;
@@ -819,13 +826,15 @@ size_t dy_plan_floats(const std::vector<DySpec>& specs) {
   return f;
 }
 
-// The fused passes over dy on `ctas` persistent CTAs (one per SM), then their reduce.
-int launch_dy_pass(const std::vector<DySpec>& specs, const Arena& ar, const DeviceInfo* d, int ctas, cudaStream_t st) {
+// The fused passes over dy on `ctas` persistent CTAs (one per SM), then their reduce; the cuts are
+// the cheapest ones for `plan_ctas` CTAs (the cut decides how sv and dB are summed).
+int launch_dy_pass(const std::vector<DySpec>& specs, const Arena& ar, const DeviceInfo* d, int ctas, int plan_ctas,
+                   cudaStream_t st) {
   size_t pf = 0;
   int rc;
   for (size_t i0 = 0; i0 < specs.size(); i0 += kMaxRankProblems) {
     const size_t i1 = std::min(specs.size(), i0 + kMaxRankProblems);
-    const std::vector<DyCut> cuts = dy_choose(specs, i0, i1, ctas);
+    const std::vector<DyCut> cuts = dy_choose(specs, i0, i1, plan_ctas);
     DyBatch b;
     memset(&b, 0, sizeof(b));
     for (size_t i = i0; i < i1; ++i) {
@@ -1058,6 +1067,31 @@ SideWidths side_widths(int num_sms, const lora_proj* projs, int n) {
   SideWidths w;
   w.w1 = std::max(2, std::min(num_sms / 4, v1 > 0 ? v1 : width(kSideKappa1, b1)));
   w.w2 = std::max(2, std::min(num_sms / 4, v2 > 0 ? v2 : width(kSideKappa2, b2)));
+  // A contraction with few output tiles runs as a cluster split, four CTAs per 256 x 256 tile, and leaves
+  // the other SMs idle: the side stream takes them (the split still fits beside it).
+  auto cs_sms = [&](bool bwd, int side) {
+    long long wide = 0, narrow = 0;
+    for (int i = 0; i < n; ++i) {
+      if (is_q4(projs[i])) return 0;  // 4-bit weights keep the wide tiles
+      const lora_shape& sh = projs[i].shape;
+      const int out = bwd ? sh.d_in : sh.d_out, depth = bwd ? sh.d_out : sh.d_in;
+      const int kb = cdiv(depth, 64) + (sh.rank > 0 ? cdiv(sh.rank, 64) : 0);
+      if (kb < kCsMinBlocks || kb > kCsMaxBlocks) return 0;
+      wide += (long long)cdiv(sh.T, 256) * cdiv(out, gemm_tile_n());
+      narrow += (long long)cdiv(sh.T, 256) * cdiv(out, gemm_tile_n_f32());
+    }
+    const int pairs = (num_sms - side) / 2;
+    if (wide == 0 || wide >= pairs || 2 * narrow > pairs || narrow > gemm_cs_max_clusters(bwd)) return 0;
+    return (int)(4 * narrow);
+  };
+  if (v1 <= 0) {
+    const int used = cs_sms(false, w.w1);
+    if (used > 0) w.w1 = std::max(w.w1, (num_sms - used) & ~1);
+  }
+  if (v2 <= 0) {
+    const int used = cs_sms(true, w.w2);
+    if (used > 0) w.w2 = std::max(w.w2, (num_sms - used) & ~1);
+  }
   return w;
 }
 
@@ -1205,7 +1239,9 @@ int run_step(const lora_proj* projs, int n, int mode, void* ws, const Plan& pl, 
     {
       // sv (and dB where fused) before the event the dx contraction waits for
       ProfScope ps(LORA_KERNEL_ROWPROJ, rs);
-      if ((rc = launch_dy_pass(dys, arena(ws, pl, kPhBwdRows), d, ctas, rs)) != LORA_OK) return rc;
+      if ((rc = launch_dy_pass(dys, arena(ws, pl, kPhBwdRows), d, ctas, pl.dy_cut_device ? d->num_sms : ctas, rs)) !=
+          LORA_OK)
+        return rc;
       if ((rc = launch_rows(rows, arena(ws, pl, kPhBwdRows), d, ctas, rs)) != LORA_OK) return rc;
     }
     // sv is complete: the dx contraction may start (on the main stream: at once, or after this event)
@@ -1394,14 +1430,21 @@ int plan_all(const lora_proj* projs, int n, int mode, Plan* pl, bool allow_split
             gemm_shape(b.prob[b.num_problems], sh.T, sh.d_in, sh.d_out, sh.rank);
           add_problem(b);
         }
-        int sp[kMaxProblems];
-        choose_splits(b, sp, pairs_dir[dir]);
-        if (!allow_split)
-          for (int q = 0; q < b.num_problems; ++q) sp[q] = 1;
-        for (int q = 0; q < b.num_problems; ++q) {
-          const int pi = order[i0 + q];
-          (dir == 0 ? pl->split_f : pl->split_b)[pi] = sp[q];
-          split_need[pi] = std::max(split_need[pi], split_floats(b.prob[q], sp[q]));
+        // the splits for the pairs this call's contraction gets, and the partials sized for the
+        // larger of those splits and the ones on every pair: a forward-and-backward call's workspace,
+        // whose side stream may leave few pairs to a contraction, must also hold a forward or
+        // backward call of the same shapes on all of them
+        for (int pass = 0; pass < 2; ++pass) {
+          if (pass == 1 && pairs_dir[dir] == kPlanPairs) break;
+          int sp[kMaxProblems];
+          choose_splits(b, sp, pass == 0 ? pairs_dir[dir] : kPlanPairs);
+          if (!allow_split)
+            for (int q = 0; q < b.num_problems; ++q) sp[q] = 1;
+          for (int q = 0; q < b.num_problems; ++q) {
+            const int pi = order[i0 + q];
+            if (pass == 0) (dir == 0 ? pl->split_f : pl->split_b)[pi] = sp[q];
+            split_need[pi] = std::max(split_need[pi], split_floats(b.prob[q], sp[q]));
+          }
         }
       }
     }
@@ -1724,8 +1767,19 @@ int lora_stack_workspace_size(const lora_proj* projs, int n_proj, int mode, size
   return rec(LORA_OK);
 }
 
+namespace {
+int stack_step(const lora_proj* projs, int n_proj, int mode, void* workspace, size_t workspace_bytes, void* stream,
+               bool dy_cut_device);
+}
+
 int lora_stack_step(const lora_proj* projs, int n_proj, int mode, void* workspace, size_t workspace_bytes,
                     void* stream) {
+  return stack_step(projs, n_proj, mode, workspace, workspace_bytes, stream, false);
+}
+
+namespace {
+int stack_step(const lora_proj* projs, int n_proj, int mode, void* workspace, size_t workspace_bytes, void* stream,
+               bool dy_cut_device) {
   if (!projs) return rec(LORA_ENULL);
   if (n_proj < 1 || n_proj > 64 || mode < LORA_FWD || mode > LORA_FWD_BWD) return rec(LORA_EINVAL);
   DeviceInfo* d = nullptr;
@@ -1741,8 +1795,10 @@ int lora_stack_step(const lora_proj* projs, int n_proj, int mode, void* workspac
       return rec(LORA_ENULL);  // the backward needs the saved su
   }
   if ((rc = check_ws(workspace, workspace_bytes, need)) != LORA_OK) return rec(rc);
+  pl.dy_cut_device = dy_cut_device;
   return rec(run_step(projs, n_proj, mode, workspace, pl, d, static_cast<cudaStream_t>(stream)));
 }
+}  // namespace
 
 int lora_linear_fwd(const lora_shape* shape, const lora_bf16* x, const lora_bf16* W, const lora_bf16* A,
                     const lora_bf16* B, lora_bf16* y, lora_bf16* su, void* workspace, size_t workspace_bytes,
@@ -1890,7 +1946,7 @@ int lora_stack_ckpt(const lora_proj* projs, int n_layers, int n_per_layer, void*
   // Stage III: from the last layer back, re-run its forward saving su, then its backward
   for (int l = n_layers - 1; l >= 0; --l) {
     layer_copy(projs + (size_t)l * n_per_layer, n_per_layer, su_scratch, &layer);
-    if ((rc = lora_stack_step(layer.data(), n_per_layer, LORA_FWD_BWD, step_ws, wb, stream)) != LORA_OK) return rec(rc);
+    if ((rc = stack_step(layer.data(), n_per_layer, LORA_FWD_BWD, step_ws, wb, stream, true)) != LORA_OK) return rec(rc);
   }
   return rec(LORA_OK);
 }
