@@ -21,11 +21,11 @@
 // outputs, or fp32 partials when a tile's reduction spans several work units
 // (summed in unit order by a second pass, so results never depend on
 // scheduling).  Two accumulators let the read-back of one unit overlap the
-// next unit's loads and MMAs.  The MMAs are tiny (N = rank), but each reads
-// its 4 KB X tile from shared memory, ~64 cycles apiece: with the copies'
-// issue cost that bounds the rate one CTA streams X at (~45-60 GB/s), so
-// these kernels fill the HBM bandwidth only on many SMs.  Every wait is
-// bounded.
+// next unit's loads and MMAs.  The MMAs are tiny (N = rank), and a stream of
+// them from one thread takes ~47 cycles per MMA whatever N up to 64; one CTA
+// streams X at ~45-60 GB/s, bounded by the X bytes its ring keeps in flight
+// (16 KB boxes, 8 stages) against the load latency, so these kernels fill the
+// HBM bandwidth only on many SMs.  Every wait is bounded.
 #include "rank_store.cuh"
 
 namespace lora {
