@@ -1171,6 +1171,9 @@ int run_step(const lora_proj* projs, int n, int mode, void* ws, const Plan& pl, 
   int* counters = at<int>(ws, 0);
   int next_counter = 0;
   if (cudaMemsetAsync(ws, 0, pl.zero_bytes, st) != cudaSuccess) return LORA_ECUDA;
+  // whether a kernel of this call already ran on the main stream: a contraction launched after one may
+  // load its base operands (inputs of the call) before the previous grid ends
+  bool prior_main = false;
   // forward and backward in one call: the backward's rank-r work runs on a side
   // stream with a few SMs while the contractions use the rest; a backward alone
   // computes sv (which the dx contraction reads) first on every SM, then dA (and
@@ -1297,6 +1300,7 @@ int run_step(const lora_proj* projs, int n, int mode, void* ws, const Plan& pl, 
       ProfScope ps(LORA_KERNEL_ROWPROJ, st);
       if ((rc = launch_rows(rows, arena(ws, pl, kPhFwdRows), d, d->num_sms, st)) != LORA_OK) return rc;
     }
+    if (!rows.empty()) prior_main = true;
     // the backward's rank-r work needs su only: it may start now, beside the forward contractions
     if (ov.on && (rc = ov.fork()) != LORA_OK) return rc;
     if (ov.on && (rc = bwd_rank(ov.side, ov.side_ctas, ov.side, ov.side_ctas2)) != LORA_OK) return rc;
@@ -1312,6 +1316,8 @@ int run_step(const lora_proj* projs, int n, int mode, void* ws, const Plan& pl, 
         GemmBatch b;
         init_batch(b, d);
         b.tile_counter = counters + next_counter++;
+        b.early_inputs = prior_main ? 1 : 0;
+        prior_main = true;
         int sp[kMaxProblems];
         float* parts[kMaxProblems];
         for (size_t i = i0; i < order.size() && i < i0 + kMaxProblems; ++i) {
@@ -1332,9 +1338,11 @@ int run_step(const lora_proj* projs, int n, int mode, void* ws, const Plan& pl, 
   }
   if (mode & LORA_BWD) {
     // (a forward-and-backward call without the side stream runs it here too, on every SM)
-    if (!(mode == LORA_FWD_BWD && ov.on) &&
-        (rc = bwd_rank(st, d->num_sms, ov.on ? ov.side : st, ov.on ? ov.side_ctas2 : d->num_sms)) != LORA_OK)
-      return rc;
+    if (!(mode == LORA_FWD_BWD && ov.on)) {
+      if ((rc = bwd_rank(st, d->num_sms, ov.on ? ov.side : st, ov.on ? ov.side_ctas2 : d->num_sms)) != LORA_OK)
+        return rc;
+      if (any_adapter(projs, n)) prior_main = true;  // the pass over dy or the row products ran here
+    }
     // the dx contraction reads sv: when the side stream computed it, wait for it
     if (mode == LORA_FWD_BWD && ov.on && (rc = ov.wait_sv()) != LORA_OK) return rc;
     std::vector<Operands>& ops = bops;
@@ -1348,6 +1356,8 @@ int run_step(const lora_proj* projs, int n, int mode, void* ws, const Plan& pl, 
         GemmBatch b;
         init_batch(b, d);
         b.tile_counter = counters + next_counter++;
+        b.early_inputs = prior_main ? 1 : 0;
+        prior_main = true;
         int sp[kMaxProblems];
         float* parts[kMaxProblems];
         for (size_t i = i0; i < order.size() && i < i0 + kMaxProblems; ++i) {

@@ -311,7 +311,9 @@ __global__ void __launch_bounds__(Cfg<kQ>::kThreads, 1) fused_lora_gemm(const __
   __syncthreads();
   tc_fence_after();
   cluster_sync_all();  // both CTAs' barriers exist before any cross-CTA arrival
-  griddep_wait();      // the previous grid's outputs (su, sv, tile counter) are ready
+  // the previous grid's outputs (su, sv) are ready; with early inputs only the producer waits, before its
+  // first adapter-slab load (the tile counter was cleared before the call's first kernel)
+  if (!b.early_inputs) griddep_wait();
   const uint32_t tmem_base = ctl->tmem_base;
   const uint32_t tile_empty_root = mapa_shared(smem_u32(&ctl->tile_empty[0]), pb);
 
@@ -322,6 +324,7 @@ __global__ void __launch_bounds__(Cfg<kQ>::kThreads, 1) fused_lora_gemm(const __
       int stage = 0;
       uint32_t phase = 0;
       int fills = 0;
+      bool waited = !b.early_inputs;  // this thread has waited for the previous grid
       for (int it = 0;; ++it) {
         const int slot = it % kTileRing;
         const uint32_t par = (uint32_t)((it / kTileRing) & 1);
@@ -374,6 +377,10 @@ __global__ void __launch_bounds__(Cfg<kQ>::kThreads, 1) fused_lora_gemm(const __
           const uint32_t a_dst = a_addr_of(base, stage);
           const uint32_t b_dst = a_dst + kAHalf;
           const int kc = main ? kb * kBK : (kb - Q.kb_main) * kBK;
+          if (!main && !waited) {
+            griddep_wait();  // su or sv comes from the previous grid
+            waited = true;
+          }
           const CUtensorMap* ta = main ? &b.tmA[p] : &b.tmA2[p];
           const CUtensorMap* tb = main ? &b.tmB[p] : &b.tmB2[p];
           if (a_mine) tma_load_2d_pair(a_dst, ta, bar, kc, my_m);
@@ -1120,6 +1127,9 @@ __global__ void __launch_bounds__(Cfg<kQ>::kThreads, 1) fused_lora_gemm(const __
       }
     }
   }
+  // with early inputs a CTA may have loaded no adapter slab: it still leaves only after the previous
+  // grid, so that this grid's completion implies that grid's (the next grid waits for this one only)
+  if (b.early_inputs && threadIdx.x == 0) griddep_wait();
   __syncthreads();
   cluster_sync_all();  // no cross-CTA access is pending in either CTA
   if (warp == 1) {

@@ -129,6 +129,10 @@ struct GemmBatch {
   int* tile_counter;   // zero at launch; hands out tiles in list order
   int* status;
   long long limit_ns;
+  // 1: an earlier kernel of the same call precedes this launch on its stream, so the call's inputs
+  // (the base contraction's operands) were complete before this grid started and its main blocks may
+  // be loaded before the previous grid ends; only the adapter slab's activations (su or sv) wait
+  int early_inputs;
 };
 
 // b_mn_major: the weight operand is contracted over its rows (backward);
