@@ -1414,10 +1414,22 @@ int plan_all(const lora_proj* projs, int n, int mode, Plan* pl, bool allow_split
   // the side stream's SMs are left out of the contractions they run beside: the
   // forward's in a forward-and-backward call, the dx contraction's in any call with a backward
   int pairs_dir[2] = {kPlanPairs, kPlanPairs};
+  // pair counts the partials are also sized for: every pair, and the side widths of the same shapes with
+  // bf16 and with 4-bit weights, so that a size reported from the shapes alone (lora_workspace_size)
+  // covers a call of either weight kind in any mode
+  std::vector<int> pairs_alt[2] = {{kPlanPairs}, {kPlanPairs}};
   if ((mode & LORA_BWD) && overlap_enabled() && any_adapter(projs, n)) {
     const SideWidths w = side_widths(kPlanSms, projs, n);
     if (mode == LORA_FWD_BWD) pairs_dir[0] = (kPlanSms - w.w1) / 2;
     pairs_dir[1] = (kPlanSms - w.w2) / 2;
+    static const uint8_t kAnyCodes = 0;  // a non-null code pointer marks a projection 4-bit for the widths
+    for (int q4 = 0; q4 < 2; ++q4) {
+      std::vector<lora_proj> as(projs, projs + n);
+      for (lora_proj& p : as) p.Wq.codes = q4 ? &kAnyCodes : nullptr;
+      const SideWidths wa = side_widths(kPlanSms, as.data(), n);
+      pairs_alt[0].push_back((kPlanSms - wa.w1) / 2);
+      pairs_alt[1].push_back((kPlanSms - wa.w2) / 2);
+    }
   }
   std::vector<size_t> split_need(n, 0);
   for (int dir = 0; dir < 2; ++dir) {
@@ -1441,13 +1453,14 @@ int plan_all(const lora_proj* projs, int n, int mode, Plan* pl, bool allow_split
           add_problem(b);
         }
         // the splits for the pairs this call's contraction gets, and the partials sized for the
-        // larger of those splits and the ones on every pair: a forward-and-backward call's workspace,
-        // whose side stream may leave few pairs to a contraction, must also hold a forward or
-        // backward call of the same shapes on all of them
-        for (int pass = 0; pass < 2; ++pass) {
-          if (pass == 1 && pairs_dir[dir] == kPlanPairs) break;
+        // largest of those splits and the ones for the other pair counts above: a forward-and-backward
+        // call's workspace, whose side stream may leave few pairs to a contraction, must also hold a
+        // forward or backward call of the same shapes
+        for (size_t pass = 0; pass <= pairs_alt[dir].size(); ++pass) {
+          const int pairs = pass == 0 ? pairs_dir[dir] : pairs_alt[dir][pass - 1];
+          if (pass > 0 && pairs == pairs_dir[dir]) continue;
           int sp[kMaxProblems];
-          choose_splits(b, sp, pass == 0 ? pairs_dir[dir] : kPlanPairs);
+          choose_splits(b, sp, pairs);
           if (!allow_split)
             for (int q = 0; q < b.num_problems; ++q) sp[q] = 1;
           for (int q = 0; q < b.num_problems; ++q) {

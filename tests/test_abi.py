@@ -137,6 +137,29 @@ def test_forward_and_backward_plan_their_splits_for_the_contractions_sms(lib):
     assert fwd > 0 and both > fwd
 
 
+def test_forward_and_backward_workspace_covers_every_call_of_the_shape(lib):
+    """The size a forward-and-backward query reports from the shape alone
+    covers a forward or a backward call of that shape, with bf16 or 4-bit
+    weights: the partials of split contractions are sized for the pairs a
+    contraction gets beside the side stream (whose width depends on the
+    weight kind and, for few output tiles, on the cluster split), and on all
+    pairs."""
+    # (the first three violated it when the partials were sized for the side stream's pairs alone)
+    shapes = [(128, 2048, 8192, 16), (256, 2048, 8192, 16), (128, 4096, 6144, 64), (200, 768, 1024, 24),
+              (512, 3072, 3072, 16), (256, 3072, 8192, 16), (256, 8192, 3072, 16), (2048, 3072, 3072, 16),
+              (256, 1024, 4096, 128), (1000, 2048, 256, 64), (64, 512, 768, 8)]
+    fake_q4 = lora.lora_q4_weight(256, 512)  # sizes only: the pointers are never read
+    for T, K, N, r in shapes:
+        st = lora.make_shape(T, K, N, r, 2.0)
+        both = lora.lora_workspace_size(st, lora.LORA_FWD_BWD)
+        for mode in (lora.LORA_FWD, lora.LORA_BWD, lora.LORA_FWD_BWD):
+            assert lora.lora_workspace_size(st, mode) <= both, (T, K, N, r, mode)
+            if K % 256 == 0:
+                q4 = lora.lora_stack_workspace_size([lora.make_proj(st, Wq=fake_q4)], mode)
+                if mode != lora.LORA_FWD_BWD:
+                    assert q4 <= both, (T, K, N, r, mode, q4, both)
+
+
 def test_last_error_follows_the_threads_latest_call(lib):
     """lora_last_error repeats the code of the calling thread's latest call,
     successes included, and is per thread."""
